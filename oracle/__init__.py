@@ -1,0 +1,208 @@
+"""DQGAN oracle -- TEST INFRASTRUCTURE ONLY.
+
+Python access (ctypes + numpy) to the plain C statement of Algorithm 2 in
+``dqgan_oracle.c`` and to the exact-rational replay in ``exact.py``.  Only the
+tests, ``__graft_entry__.smoke()`` and the CPU-baseline leg of ``bench.py``
+may import this package; the product path never does.
+
+Conventions (restated, not shared, with the CUDA library):
+
+* compressors: 0 scaled sign, 1 top-k, 2 b-bit stochastic quantiser,
+  3 identity;
+* arrays are numpy ``float32`` (gradients, residuals, parameters) and
+  ``uint8`` (messages);
+* ``step`` is the iteration index t of Algorithm 2, starting at 1.
+"""
+from __future__ import annotations
+
+import ctypes
+import dataclasses
+
+import numpy as np
+
+from .build_oracle import build_oracle
+
+SIGN, TOPK, SQUANT, IDENTITY = 0, 1, 2, 3
+COMPRESSOR_NAMES = {"sign": SIGN, "topk": TOPK, "squant": SQUANT, "identity": IDENTITY}
+
+
+class _OrcCfg(ctypes.Structure):
+    _fields_ = [
+        ("d", ctypes.c_int64),
+        ("k", ctypes.c_int64),
+        ("lr", ctypes.c_float),
+        ("M", ctypes.c_int32),
+        ("compressor", ctypes.c_int32),
+        ("bucket", ctypes.c_int32),
+        ("bits", ctypes.c_int32),
+        ("keep_lookahead", ctypes.c_int32),
+        ("seed", ctypes.c_uint64),
+    ]
+
+
+@dataclasses.dataclass
+class Config:
+    d: int
+    M: int
+    compressor: int
+    lr: float = 1e-3
+    bucket: int = 512
+    k: int = 1
+    bits: int = 8
+    seed: int = 0
+    keep_lookahead: bool = False
+
+    def c_struct(self) -> _OrcCfg:
+        return _OrcCfg(d=self.d, k=self.k, lr=self.lr, M=self.M, compressor=self.compressor,
+                       bucket=self.bucket, bits=self.bits,
+                       keep_lookahead=1 if self.keep_lookahead else 0, seed=self.seed)
+
+
+_lib = None
+
+
+def lib() -> ctypes.CDLL:
+    global _lib
+    if _lib is None:
+        path = build_oracle()
+        L = ctypes.CDLL(path)
+        P = ctypes.POINTER
+        f32p, u8p = P(ctypes.c_float), P(ctypes.c_uint8)
+        cfgp = P(_OrcCfg)
+        L.orc_philox4x32_10.argtypes = [P(ctypes.c_uint32), P(ctypes.c_uint32), P(ctypes.c_uint32)]
+        L.orc_philox4x32_10.restype = None
+        L.orc_squant_uniform.argtypes = [ctypes.c_uint64, ctypes.c_int32, ctypes.c_int64, ctypes.c_int64]
+        L.orc_squant_uniform.restype = ctypes.c_float
+        L.orc_layout.argtypes = [cfgp, P(ctypes.c_int64), P(ctypes.c_int64)]
+        L.orc_layout.restype = ctypes.c_int64
+        L.orc_sign_l1.argtypes = [f32p, ctypes.c_int64, ctypes.c_int32]
+        L.orc_sign_l1.restype = ctypes.c_float
+        L.orc_sign_scale.argtypes = [f32p, ctypes.c_int64, ctypes.c_int32]
+        L.orc_sign_scale.restype = ctypes.c_float
+        L.orc_squant_decode.argtypes = [ctypes.c_int32, ctypes.c_float, ctypes.c_int32]
+        L.orc_squant_decode.restype = ctypes.c_float
+        L.orc_topk_select.argtypes = [f32p, ctypes.c_int64, ctypes.c_int64, u8p]
+        L.orc_topk_select.restype = None
+        L.orc_decode.argtypes = [cfgp, u8p, f32p]
+        L.orc_decode.restype = None
+        L.orc_worker_step.argtypes = [cfgp, ctypes.c_int32, ctypes.c_int64, f32p, f32p, f32p, u8p]
+        L.orc_worker_step.restype = None
+        L.orc_server_step.argtypes = [cfgp, u8p, ctypes.c_int64, f32p]
+        L.orc_server_step.restype = None
+        L.orc_lookahead.argtypes = [ctypes.c_int64, f32p, f32p, f32p]
+        L.orc_lookahead.restype = None
+        _lib = L
+    return _lib
+
+
+def _f32(a: np.ndarray):
+    assert a.dtype == np.float32 and a.flags.c_contiguous
+    return a.ctypes.data_as(ctypes.POINTER(ctypes.c_float))
+
+
+def _u8(a: np.ndarray):
+    assert a.dtype == np.uint8 and a.flags.c_contiguous
+    return a.ctypes.data_as(ctypes.POINTER(ctypes.c_uint8))
+
+
+def philox4x32_10(ctr, key) -> np.ndarray:
+    c = (ctypes.c_uint32 * 4)(*[int(x) & 0xFFFFFFFF for x in ctr])
+    k = (ctypes.c_uint32 * 2)(*[int(x) & 0xFFFFFFFF for x in key])
+    o = (ctypes.c_uint32 * 4)()
+    lib().orc_philox4x32_10(c, k, o)
+    return np.array(list(o), dtype=np.uint32)
+
+
+def squant_uniform(seed: int, worker: int, step: int, j: int) -> float:
+    return float(lib().orc_squant_uniform(seed, worker, step, j))
+
+
+def layout(cfg: Config):
+    """(scales offset, payload offset, total bytes) of one message."""
+    a, b = ctypes.c_int64(), ctypes.c_int64()
+    total = lib().orc_layout(ctypes.byref(cfg.c_struct()), ctypes.byref(a), ctypes.byref(b))
+    return a.value, b.value, total
+
+
+def message_bytes(cfg: Config) -> int:
+    return layout(cfg)[2]
+
+
+def sign_l1(x: np.ndarray, bucket: int) -> float:
+    x = np.ascontiguousarray(x, dtype=np.float32)
+    return float(lib().orc_sign_l1(_f32(x), x.size, bucket))
+
+
+def sign_scale(x: np.ndarray, bucket: int) -> float:
+    x = np.ascontiguousarray(x, dtype=np.float32)
+    return float(lib().orc_sign_scale(_f32(x), x.size, bucket))
+
+
+def squant_decode(code: int, s: float, K: int) -> float:
+    return float(lib().orc_squant_decode(code, s, K))
+
+
+def topk_select(p: np.ndarray, k: int) -> np.ndarray:
+    p = np.ascontiguousarray(p, dtype=np.float32)
+    sel = np.zeros(p.size, dtype=np.uint8)
+    lib().orc_topk_select(_f32(p), p.size, k, _u8(sel))
+    return sel.astype(bool)
+
+
+def decode(cfg: Config, msg: np.ndarray) -> np.ndarray:
+    q = np.zeros(cfg.d, dtype=np.float32)
+    lib().orc_decode(ctypes.byref(cfg.c_struct()), _u8(np.ascontiguousarray(msg)), _f32(q))
+    return q
+
+
+def worker_step(cfg: Config, worker: int, step: int, g: np.ndarray, e: np.ndarray,
+                h: np.ndarray | None = None) -> np.ndarray:
+    """One worker step of Algorithm 2; updates e (and h) in place, returns the message."""
+    g = np.ascontiguousarray(g, dtype=np.float32)
+    msg = np.zeros(message_bytes(cfg), dtype=np.uint8)
+    hp = _f32(h) if h is not None else ctypes.POINTER(ctypes.c_float)()
+    lib().orc_worker_step(ctypes.byref(cfg.c_struct()), worker, step, _f32(g), _f32(e), hp, _u8(msg))
+    return msg
+
+
+def server_step(cfg: Config, msgs: np.ndarray, w: np.ndarray) -> None:
+    """Server step of Algorithm 2 on M stacked messages (M x message_bytes); updates w."""
+    msgs = np.ascontiguousarray(msgs, dtype=np.uint8)
+    assert msgs.ndim == 2 and msgs.shape[0] == cfg.M
+    lib().orc_server_step(ctypes.byref(cfg.c_struct()), _u8(msgs), msgs.shape[1], _f32(w))
+
+
+def lookahead(w: np.ndarray, h: np.ndarray) -> np.ndarray:
+    out = np.empty_like(w)
+    lib().orc_lookahead(w.size, _f32(w), _f32(h), _f32(out))
+    return out
+
+
+class State:
+    """Oracle state of Algorithm 2 for M workers: residuals e, lookahead offsets h, step t."""
+
+    def __init__(self, cfg: Config):
+        self.cfg = cfg
+        self.e = np.zeros((cfg.M, cfg.d), dtype=np.float32)
+        self.h = np.zeros((cfg.M, cfg.d), dtype=np.float32) if cfg.keep_lookahead else None
+        self.t = 1
+
+    def compress_all(self, g: np.ndarray, workers=None) -> np.ndarray:
+        """Worker steps for all (or the listed) workers at the current step."""
+        cfg = self.cfg
+        ws = range(cfg.M) if workers is None else workers
+        msgs = np.zeros((cfg.M, message_bytes(cfg)), dtype=np.uint8)
+        for i in ws:
+            e_i = self.e[i]
+            h_i = self.h[i] if self.h is not None else None
+            msgs[i] = worker_step(cfg, i, self.t, g[i], e_i, h_i)
+        return msgs
+
+    def server(self, msgs: np.ndarray, w: np.ndarray) -> None:
+        server_step(self.cfg, msgs, w)
+        self.t += 1
+
+    def step(self, g: np.ndarray, w: np.ndarray) -> np.ndarray:
+        msgs = self.compress_all(g)
+        self.server(msgs, w)
+        return msgs
