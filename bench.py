@@ -1,0 +1,423 @@
+"""Benchmark of the DQGAN hot path (Algorithm 2: worker error-feedback +
+compression of all M workers, then the fused server decode/average/update).
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME]
+                    [--impl reference] [--lookahead]
+
+One step = dqgan_workers_compress_all over all M workers + dqgan_server_
+aggregate_update, on fresh synthetic gradients already resident in HBM.
+Gradient generation and an L2 flush (a 256 MB write) run between timed
+regions and are not timed; each step's timed region is bracketed by CUDA
+events on the stream the kernels run on.  The metric is updated parameters
+per second, d * M per step, over all ranks.
+
+Default workload: the d = 1e8, M = 32, sign-per-4096 stress configuration
+(the largest that fits one GPU).  N > 1 (torchrun, one rank per GPU) runs N
+independent replicas -- the simulated workers share nothing across GPUs --
+and reports the whole-job rate over the max-over-ranks time.
+
+--impl reference times the CPU oracle (single thread, the code as the tests
+use it) on a bounded sample of the same workload and prints the same line
+with "impl": "reference".
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import re
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+from paper_2010_13359_gb300.workloads import SIGN, SQUANT, TOPK, IDENTITY, WORKLOADS  # noqa: E402
+
+METRIC = "updated params/sec (d*M per step) and achieved HBM GB/s vs GB300 roofline"
+UNIT = "params/s"
+FALLBACK_HBM_GBS = 6800.0
+COMPRESSOR_NAME = {SIGN: "sign", TOPK: "topk", SQUANT: "squant", IDENTITY: "identity"}
+KERNEL_SOURCE = {SIGN: "dense_compress.cu", SQUANT: "dense_compress.cu", IDENTITY: "dense_compress.cu",
+                 TOPK: "topk.cu"}
+
+
+def parse_args():
+    ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=20)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--workload", default="stress_sign", choices=sorted(WORKLOADS))
+    ap.add_argument("--impl", default="gpu", choices=["gpu", "reference"])
+    ap.add_argument("--lookahead", action="store_true", help="also keep the lookahead offsets h")
+    ap.add_argument("--no-e2e", action="store_true", help="skip the end-to-end (host buffers) phase")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    return ap.parse_args()
+
+
+# ---------------------------------------------------------------------------
+# bytes per step (algorithmic minimum)
+# ---------------------------------------------------------------------------
+
+def message_payload_bytes(wl) -> int:
+    nb = -(-wl.d // wl.bucket)
+    if wl.compressor == SIGN:
+        return 4 * nb + 4 * (-(-wl.d // 32))
+    if wl.compressor == SQUANT:
+        return 4 * nb + 4 * (-(-wl.d * wl.bits // 32))
+    if wl.compressor == TOPK:
+        return 8 * wl.k
+    return 4 * wl.d
+
+
+def compress_bytes(wl, lookahead: bool) -> int:
+    """Per launch over all M workers: read g and e, write e (+h), write the message."""
+    per_worker = 12 * wl.d + (4 * wl.d if lookahead else 0) + message_payload_bytes(wl)
+    return wl.M * per_worker
+
+
+def server_bytes(wl) -> int:
+    """Read and write w, read all M messages (top-k: read and write only the touched w)."""
+    if wl.compressor == TOPK:
+        return wl.M * 8 * wl.k + 8 * min(wl.d, wl.M * wl.k)
+    return 8 * wl.d + wl.M * message_payload_bytes(wl)
+
+
+# ---------------------------------------------------------------------------
+# environment helpers
+# ---------------------------------------------------------------------------
+
+def dist_env():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+def hbm_peak():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(path) as f:
+            v = float(json.load(f)["hbm_gbs"])
+        return v, "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def source_digest(name: str) -> str:
+    with open(os.path.join(ROOT, "paper_2010_13359_gb300", "csrc", name), "rb") as f:
+        return hashlib.sha256(f.read()).hexdigest()[:16]
+
+
+def profiled_traffic(wl, kernel_file: str, units: int):
+    """DRAM bytes per launch from the committed ncu summary of this workload,
+    scaled to `units` parameters; None if absent or the kernel changed since."""
+    path = os.path.join(ROOT, "profiles", f"ncu_compress_{wl.name}.md")
+    if not os.path.exists(path):
+        return None
+    txt = open(path).read()
+    m_b = re.search(r"dram_bytes_per_param\s*=\s*([0-9.eE+-]+)", txt)
+    m_h = re.search(r"source_sha256_16\s*=\s*([0-9a-f]+)", txt)
+    if not m_b or not m_h or m_h.group(1) != source_digest(kernel_file):
+        return None
+    return float(m_b.group(1)) * units
+
+
+class ClockSampler:
+    """nvidia-smi clocks / throttle reasons sampled every 200 ms while running."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.tmp = tempfile.NamedTemporaryFile("w+", suffix=".csv", delete=False)
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "200"],
+                stdout=self.tmp, stderr=subprocess.DEVNULL)
+            time.sleep(0.3)
+        except Exception:
+            self.proc = None
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            time.sleep(0.25)
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except Exception:
+                self.proc.kill()
+
+    def summary(self):
+        self.tmp.flush()
+        rows = []
+        with open(self.tmp.name) as f:
+            for line in f:
+                parts = [p.strip() for p in line.split(",")]
+                if len(parts) < 9:
+                    continue
+                try:
+                    rows.append((float(parts[1]), float(parts[2]), float(parts[3]), parts[4:9]))
+                except ValueError:
+                    continue
+        os.unlink(self.tmp.name)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["unsampled"], "samples": 0}
+        loaded = [r for r in rows if r[2] > 200.0] or rows
+        names = ["active_mask", "hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown",
+                 "sw_power_cap"]
+        reasons = set()
+        for r in loaded:
+            for name, val in zip(names[1:], r[3][1:]):
+                if val.lower().startswith("active"):
+                    reasons.add(name)
+        return {"sm_mhz": statistics.median(r[0] for r in loaded), "sm_max_mhz": max(r[1] for r in rows),
+                "reasons": sorted(reasons), "samples": len(loaded),
+                "power_w_max": max(r[2] for r in rows)}
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle timing (cpu_baseline leg and the reference arm)
+# ---------------------------------------------------------------------------
+
+def oracle_step_time(wl, worker_fraction: float = 1.0, server_fraction: float = 1 / 64):
+    """Single-thread oracle time for one full step of `wl`, estimated from a
+    bounded sample: one worker step on a bucket-aligned prefix of the vector
+    (`worker_fraction` of d; every worker's step costs the same per
+    parameter) and the server step on a bucket-aligned prefix
+    (`server_fraction` of d), both scaled to all M workers and all of d."""
+    import numpy as np
+
+    import oracle
+
+    def prefix(frac):
+        if wl.compressor in (SIGN, SQUANT):
+            return min(wl.d, max(wl.bucket, int(wl.d * frac) // wl.bucket * wl.bucket))
+        return min(wl.d, max(1, int(wl.d * frac)))
+
+    def cfg_of(n):
+        k = max(1, int(round(wl.k * n / wl.d))) if wl.compressor == TOPK else wl.k
+        return oracle.Config(d=n, M=wl.M, compressor=wl.compressor, lr=wl.lr, bucket=wl.bucket, k=k,
+                             bits=wl.bits, seed=wl.seed)
+
+    rng = np.random.default_rng(1)
+    wd = prefix(worker_fraction)
+    g = (rng.standard_normal(wd, dtype=np.float32) * np.float32(1e-3)).astype(np.float32)
+    e = np.zeros(wd, np.float32)
+    t0 = time.perf_counter()
+    oracle.worker_step(cfg_of(wd), 0, 1, g, e)
+    t_worker = (time.perf_counter() - t0) * (wl.d / wd)
+    sd = prefix(server_fraction)
+    sub = cfg_of(sd)
+    sub_msg = oracle.worker_step(sub, 0, 1, g[:sd].copy() if sd <= wd else
+                                 rng.standard_normal(sd, dtype=np.float32), np.zeros(sd, np.float32))
+    msgs = np.repeat(sub_msg[None, :], wl.M, axis=0)
+    w = np.zeros(sd, np.float32)
+    t0 = time.perf_counter()
+    oracle.server_step(sub, msgs, w)
+    t_server = (time.perf_counter() - t0) * (wl.d / sd)
+    step = wl.M * t_worker + t_server
+    sample = (f"one worker step on {wd} of d = {wl.d} parameters ({t_worker:.2f} s scaled to d, "
+              f"x M = {wl.M}) + the server step on {sd} parameters ({t_server:.2f} s scaled to d); "
+              f"one host thread")
+    return step, sample
+
+
+def run_reference(args, rank, world):
+    if rank != 0:
+        return 0
+    wl = WORKLOADS[args.workload]
+    step_times = []
+    sample = ""
+    for i in range(args.warmup + args.steps):
+        st, sample = oracle_step_time(wl, worker_fraction=1 / 8, server_fraction=1 / 64)
+        if i >= args.warmup:
+            step_times.append(st)
+    total = sum(step_times)
+    value = wl.d * wl.M * len(step_times) / total
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * total / len(step_times),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+        "data": "synthetic", "config": workload_config(wl, args),
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def workload_config(wl, args):
+    c = {"workload": wl.name, "d": wl.d, "M": wl.M, "compressor": COMPRESSOR_NAME[wl.compressor],
+         "lr": wl.lr, "gradients": wl.dist, "lookahead": bool(args.lookahead),
+         "l2": "flushed before every timed step (256 MB write); inputs also exceed L2",
+         "parallelism": f"replicas{args.gpus}" if args.gpus > 1 else "single"}
+    if wl.compressor in (SIGN, SQUANT):
+        c["bucket"] = wl.bucket
+    if wl.compressor == SQUANT:
+        c["bits"] = wl.bits
+    if wl.compressor == TOPK:
+        c["k"] = wl.k
+    return c
+
+
+# ---------------------------------------------------------------------------
+# GPU arm
+# ---------------------------------------------------------------------------
+
+def run_gpu(args, rank, world, local):
+    import torch
+    import torch.distributed as tdist
+
+    import paper_2010_13359_gb300 as P
+
+    wl = WORKLOADS[args.workload]
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if world > 1:
+        tdist.init_process_group("nccl", device_id=dev)
+
+    def barrier():
+        if world > 1:
+            tdist.barrier()
+
+    stream = torch.cuda.current_stream(dev)
+    flags = P.KEEP_LOOKAHEAD if args.lookahead else 0
+    h = P.create(P.make_config(d=wl.d, M=wl.M, compressor=wl.compressor, lr=wl.lr, bucket=wl.bucket,
+                               k=wl.k, bits=wl.bits, seed=wl.seed, flags=flags,
+                               cuda_stream=stream.cuda_stream))
+    mb = h.message_bytes()
+    g = torch.empty((wl.M, wl.d), dtype=torch.float32, device=dev)
+    msgs = torch.empty((wl.M, mb), dtype=torch.uint8, device=dev)
+    w = wl.w0_torch(dev)
+    flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+    std_vec = wl.std_vector_torch(dev) if wl.dist == "gauss" else None
+
+    def one_step(t, ev=None):
+        wl.fill_gradients_torch(g, t, std_vec)
+        flush.zero_()
+        if ev:
+            ev[0].record(stream)
+        h.workers_compress_all(g, wl.d, msgs)
+        if ev:
+            ev[1].record(stream)
+        h.server_aggregate_update(msgs, w)
+        if ev:
+            ev[2].record(stream)
+
+    for t in range(1, args.warmup + 1):
+        one_step(t)
+    torch.cuda.synchronize(dev)
+    barrier()
+    torch.cuda.synchronize(dev)
+    events = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
+    launches0 = h.launch_count()
+    with ClockSampler(local) as clk:
+        for s in range(args.steps):
+            one_step(args.warmup + 1 + s, events[s])
+        torch.cuda.synchronize(dev)
+    barrier()
+    torch.cuda.synchronize(dev)
+    launches = h.launch_count() - launches0
+    comp_ms = [e[0].elapsed_time(e[1]) for e in events]
+    serv_ms = [e[1].elapsed_time(e[2]) for e in events]
+    total_ms = sum(c + s for c, s in zip(comp_ms, serv_ms))
+    if world > 1:
+        tt = torch.tensor([total_ms], dtype=torch.float64, device=dev)
+        tdist.all_reduce(tt, op=tdist.ReduceOp.MAX)
+        total_ms = float(tt.item())
+    units = wl.d * wl.M
+    value = world * units * args.steps / (total_ms / 1e3)
+
+    # end to end: host gradients (pinned) -> device, the two C-ABI calls, params -> host
+    e2e = None
+    if not args.no_e2e:
+        g_host = torch.empty((wl.M, wl.d), dtype=torch.float32, pin_memory=True)
+        w_host = torch.empty(wl.d, dtype=torch.float32, pin_memory=True)
+        g_host.copy_(g)
+        torch.cuda.synchronize(dev)
+        e2e_steps = max(1, min(args.steps, 10))
+
+        def e2e_step():
+            g.copy_(g_host, non_blocking=True)
+            h.workers_compress_all(g, wl.d, msgs)
+            h.server_aggregate_update(msgs, w)
+            w_host.copy_(w, non_blocking=True)
+
+        e2e_step()
+        torch.cuda.synchronize(dev)
+        barrier()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(e2e_steps):
+            e2e_step()
+        b.record(stream)
+        torch.cuda.synchronize(dev)
+        e2e_ms = a.elapsed_time(b)
+        if world > 1:
+            tt = torch.tensor([e2e_ms], dtype=torch.float64, device=dev)
+            tdist.all_reduce(tt, op=tdist.ReduceOp.MAX)
+            e2e_ms = float(tt.item())
+        e2e = {"value": world * units * e2e_steps / (e2e_ms / 1e3), "unit": UNIT,
+               "h2d_bytes_per_step": int(g.numel() * 4), "d2h_bytes_per_step": int(w.numel() * 4),
+               "steps": e2e_steps, "ms_per_step": e2e_ms / e2e_steps}
+        del g_host, w_host
+
+    h.synchronize()
+    h.destroy()
+    if world > 1:
+        tdist.destroy_process_group()
+    if rank != 0:
+        return 0
+
+    peak, peak_kind = hbm_peak()
+    comp_avg = statistics.mean(comp_ms)
+    serv_avg = statistics.mean(serv_ms)
+    cb = compress_bytes(wl, args.lookahead)
+    sb = server_bytes(wl)
+    comp_gbs = cb / (comp_avg / 1e3) / 1e9
+    serv_gbs = sb / (serv_avg / 1e3) / 1e9
+    traffic = profiled_traffic(wl, KERNEL_SOURCE[wl.compressor], units) if not args.lookahead else None
+    roofline = {"bound": "hbm", "kernel": f"{COMPRESSOR_NAME[wl.compressor]}_compress (all M workers)",
+                "achieved": comp_gbs, "peak": peak, "unit": "GB/s", "frac": comp_gbs / peak,
+                "traffic": traffic, "algorithmic_bytes": cb, "ms": comp_avg,
+                "peak_source": f"{peak_kind} hbm_gbs"}
+    roofline_server = {"bound": "hbm", "kernel": f"{COMPRESSOR_NAME[wl.compressor]}_server",
+                       "achieved": serv_gbs, "peak": peak, "unit": "GB/s", "frac": serv_gbs / peak,
+                       "algorithmic_bytes": sb, "ms": serv_avg}
+    cpu = None
+    if world == 1 and not args.no_cpu_baseline:
+        st, sample = oracle_step_time(wl)
+        cpu = {"value": units / st, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample}
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": total_ms / args.steps, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+        "config": workload_config(wl, args), "roofline": roofline, "roofline_server": roofline_server,
+        "cpu_baseline": cpu, "e2e": e2e, "gpu_launches": launches, "clocks": clk.summary(),
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def main():
+    args = parse_args()
+    rank, world, local = dist_env()
+    if args.impl == "reference":
+        return run_reference(args, rank, world)
+    return run_gpu(args, rank, world, local)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,223 @@
+/*
+ * dqgan.h -- C-ABI of the GB300 (sm_103a) DQGAN hot path.
+ *
+ * One iteration of Algorithm 2 (DQGAN) of "A Distributed Training Algorithm
+ * of Generative Adversarial Networks with Quantized Gradients" (Chen, Yang,
+ * Shen, Pang; arXiv 2010.13359) for M workers that live as separate buffers
+ * on ONE GPU:
+ *
+ *   worker m (Algorithm 2, worker part):
+ *     w_{t-1/2} = w_{t-1} - [eta F(w_{t-3/2}) + e_{t-1}]       lookahead
+ *     p_t       = eta F(w_{t-1/2}; xi_t) + e_{t-1}               error feedback
+ *     p_hat_t   = Q(p_t), packed into a message                  compression
+ *     e_t       = p_t - p_hat_t                                  residual
+ *   server (Algorithm 2, server part):
+ *     q_hat_t = (1/M) sum_m p_hat_t^(m);   w_t = w_{t-1} - q_hat_t
+ *
+ * Q is a delta-approximate compressor (Definition 1, Section 3.1): the scaled
+ * sign of Section 2.4 (one l1 scale per bucket), top-k (Theorem 1), or the
+ * b-bit stochastic quantiser of Hou et al. with an l_inf scale per bucket
+ * (Section 2.4, proof of Theorem 2), or the identity.  The caller supplies
+ * the stochastic gradients F(.; xi) -- the GAN forward/backward pass is not
+ * part of this library.
+ *
+ * Conventions for every call:
+ *   - Every call returns a status (DQGAN_OK or a negative DQGAN_ERR_*) and
+ *     never aborts or exits.  On error, dqgan_last_error() describes it.
+ *   - Device pointers are CUDA device (or managed) addresses on the device
+ *     that was current when the handle was created; they must be non-NULL
+ *     and 16-byte aligned unless stated otherwise.
+ *   - Work is enqueued asynchronously on the handle's stream (the
+ *     cuda_stream of the config).  Asynchronous CUDA errors surface at
+ *     dqgan_synchronize() (or at any later call that checks).
+ *   - The library owns the residuals e, the lookahead offsets h, its scratch
+ *     space and the step counter t.  The caller owns gradients, messages and
+ *     parameters.
+ *   - Arithmetic is IEEE binary32 with one rounding per operation (no fused
+ *     multiply-add), so compressed messages and residuals are reproducible
+ *     bit for bit from identical state.
+ *   - A handle may be used from one host thread at a time.
+ */
+#ifndef DQGAN_H_
+#define DQGAN_H_
+
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define DQGAN_API __attribute__((visibility("default")))
+#else
+#define DQGAN_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* Status codes. */
+#define DQGAN_OK 0
+#define DQGAN_ERR_INVALID_ARG (-1) /* bad config, index, size, NULL or misaligned pointer */
+#define DQGAN_ERR_OOM (-2)         /* device allocation failed */
+#define DQGAN_ERR_CUDA (-3)        /* a CUDA runtime call or kernel launch failed */
+#define DQGAN_ERR_UNSUPPORTED (-4) /* valid request this build does not provide */
+#define DQGAN_ERR_TIMEOUT (-5)     /* a bounded device-side wait gave up */
+
+/* Compressors Q (Section 2.4, Section 3.2). */
+#define DQGAN_SIGN 0     /* scaled sign, s_b = ||p_b||_1 / n_b per bucket */
+#define DQGAN_TOPK 1     /* k entries of largest |p_j|, ties to the lower index */
+#define DQGAN_SQUANT 2   /* b-bit stochastic quantiser, s_b = ||p_b||_inf */
+#define DQGAN_IDENTITY 3 /* no compression (uncompressed distributed OMD) */
+
+/* Config flags. */
+#define DQGAN_KEEP_LOOKAHEAD 1u /* keep h = eta F + e per worker for the lookahead */
+
+/*
+ * Problem description.  56 bytes, no implicit padding.
+ *   d           parameters in the flat vector w = [theta, phi] (Section 2.1);
+ *               1 <= d <= 2^32 - 1.
+ *   k           top-k only: entries kept per worker, 1 <= k <= d.
+ *   lr          step size eta of Algorithm 2, finite.
+ *   M           workers, 1 <= M <= 4096.
+ *   compressor  DQGAN_SIGN / TOPK / SQUANT / IDENTITY.
+ *   bucket      sign and squant: elements per scale, a power of two in
+ *               [32, 4096]; the last bucket may be partial.  Ignored otherwise.
+ *   bits        squant only: bits per code b in {2, 4, 8}.
+ *   flags       0 or DQGAN_KEEP_LOOKAHEAD.
+ *   seed        64-bit key of the Philox4x32-10 draws of the squant rounding.
+ *   cuda_stream the cudaStream_t all work is enqueued on (NULL: legacy stream).
+ */
+typedef struct dqgan_config {
+  int64_t d;
+  int64_t k;
+  float lr;
+  int32_t M;
+  int32_t compressor;
+  int32_t bucket;
+  int32_t bits;
+  uint32_t flags;
+  uint64_t seed;
+  void* cuda_stream;
+} dqgan_config;
+
+typedef struct dqgan_handle dqgan_handle;
+
+/*
+ * Message layout (one per worker, `dqgan_message_bytes` bytes, a multiple of
+ * 256; every section starts at a multiple of 256 bytes; nb = ceil(d/bucket)):
+ *   SIGN:     [nb fp32 scales s_b][ceil(d/32) u32 words]; bit (j mod 32) of
+ *             word (j div 32) is 1 iff p_j < 0 (so -0 and +0 send +s_b);
+ *             Q(p)_j = bit ? -s_b : +s_b.  Bits past d are 0.
+ *   SQUANT:   [nb fp32 scales s_b = max |p_j|][ceil(d*b/32) u32 words]; the
+ *             b-bit code of element j sits at bit (j*b) mod 32 of word
+ *             (j*b) div 32; code = K + sign(p_j) * level, K = 2^(b-1) - 1,
+ *             level in [0, K]; Q(p)_j = sign * fl(s_b * fl(level / K)) and +0
+ *             for level 0.  Bits past d*b are 0.
+ *   TOPK:     k records {u32 index j, f32 p_j}, ascending index.
+ *   IDENTITY: d fp32 values p_j.
+ * Bytes between sections are not written by the library.
+ */
+
+/* Host-only (no CUDA call): message size and section offsets for a config.
+ * Returns DQGAN_OK or DQGAN_ERR_INVALID_ARG; any output pointer may be NULL. */
+DQGAN_API int dqgan_message_layout(const dqgan_config* cfg, int64_t* scales_offset,
+                         int64_t* payload_offset, int64_t* total_bytes);
+
+/* Host-only: validate a config without touching the GPU.  DQGAN_OK or
+ * DQGAN_ERR_INVALID_ARG (text in dqgan_last_error(NULL)). */
+DQGAN_API int dqgan_validate_config(const dqgan_config* cfg);
+
+/*
+ * Create a handle for Algorithm 2 with the given config (the problem
+ * statement dqgan_create(d, M, compressor, lr, buckets) plus the fields the
+ * compressors need).  Allocates on the current device: e (M x d fp32, zero:
+ * e_0 = 0), h (M x d fp32, zero, only with DQGAN_KEEP_LOOKAHEAD: F(w_{-1/2})
+ * is taken as 0 so that w_{1/2} = w_0), and top-k scratch.  Sets t = 1.
+ * *out receives the handle; on error *out is NULL and
+ * dqgan_last_error(NULL) holds the reason.
+ */
+DQGAN_API int dqgan_create(const dqgan_config* cfg, dqgan_handle** out);
+
+/* Release everything the handle owns (synchronises its stream first).
+ * NULL is accepted and is a no-op. */
+DQGAN_API int dqgan_destroy(dqgan_handle* h);
+
+/* Bytes of one worker's message (see the layout above); -1 for a NULL handle. */
+DQGAN_API int64_t dqgan_message_bytes(const dqgan_handle* h);
+
+/*
+ * Worker step of Algorithm 2 for worker i at the current step t:
+ *   p = fl(fl(eta * g_j) + e_j); message = pack(Q(p)); e = fl(p - Q(p));
+ *   with DQGAN_KEEP_LOOKAHEAD also h = fl(fl(eta * g_j) + e_j) (new e).
+ * g:       device, d fp32, caller-owned, read only (F(w_{t-1/2}^(i); xi_t^(i))).
+ * out_msg: device, dqgan_message_bytes() bytes, caller-owned, written.
+ * Updates e^(i) (and h^(i)).  0 <= i < M.  Does not advance t.
+ */
+DQGAN_API int dqgan_worker_compress(dqgan_handle* h, int32_t i, const float* g, void* out_msg);
+
+/*
+ * The worker step for all M workers in one launch per kernel stage.
+ * g_all:    device, worker m's gradient at g_all + m * g_stride (floats);
+ *           g_stride >= d and a multiple of 4.
+ * msgs_all: device, worker m's message at msgs_all + m * dqgan_message_bytes().
+ */
+DQGAN_API int dqgan_workers_compress_all(dqgan_handle* h, const float* g_all, int64_t g_stride,
+                               void* msgs_all);
+
+/*
+ * Server step of Algorithm 2, fused: decode the M messages, average them
+ * (q_hat = fl(sum_m Q_m / M); the summation order over m is not specified,
+ * except for TOPK and IDENTITY where it is worker order), and update the
+ * parameters in place, w = fl(w - q_hat).  Then t <- t + 1.
+ * msgs_all: device, M messages back to back (stride dqgan_message_bytes()).
+ * params:   device, d fp32, caller-owned, read and written.
+ */
+DQGAN_API int dqgan_server_aggregate_update(dqgan_handle* h, const void* msgs_all, float* params);
+
+/*
+ * Lookahead of Algorithm 2 for worker i: out = fl(params - h^(i)), i.e.
+ * w_{t-1/2}^(i) = w_{t-1} - [eta F(w_{t-3/2}^(i)) + e_{t-1}^(i)].  Needs
+ * DQGAN_KEEP_LOOKAHEAD (else DQGAN_ERR_UNSUPPORTED).  At t = 1, h = 0 and
+ * the result is params.  params, out_w_half: device, d fp32.
+ */
+DQGAN_API int dqgan_worker_lookahead(dqgan_handle* h, int32_t i, const float* params, float* out_w_half);
+
+/* Wait for the handle's stream; DQGAN_ERR_CUDA if any enqueued work failed. */
+DQGAN_API int dqgan_synchronize(dqgan_handle* h);
+
+/* Copy worker i's residual e^(i) (d fp32) to / from dst / src, which may be a
+ * host or a device pointer (any alignment).  Synchronous. */
+DQGAN_API int dqgan_get_residual(dqgan_handle* h, int32_t i, float* dst);
+DQGAN_API int dqgan_set_residual(dqgan_handle* h, int32_t i, const float* src);
+
+/* Same for the lookahead offset h^(i); DQGAN_ERR_UNSUPPORTED without
+ * DQGAN_KEEP_LOOKAHEAD. */
+DQGAN_API int dqgan_get_lookahead(dqgan_handle* h, int32_t i, float* dst);
+DQGAN_API int dqgan_set_lookahead(dqgan_handle* h, int32_t i, const float* src);
+
+/* Current step t (1-based) and its setter (t >= 1); -1 for a NULL handle. */
+DQGAN_API int64_t dqgan_get_step(const dqgan_handle* h);
+DQGAN_API int dqgan_set_step(dqgan_handle* h, int64_t t);
+
+/*
+ * Checkpoint / resume.  The state is a 64-byte header (magic, d, M,
+ * compressor, flags, t) followed by e (M x d fp32) and, with
+ * DQGAN_KEEP_LOOKAHEAD, h (M x d fp32).  host buffers of at least
+ * dqgan_state_bytes() bytes.  Synchronous.  Loading checks that the header
+ * matches the handle's config (else DQGAN_ERR_INVALID_ARG).
+ */
+DQGAN_API int64_t dqgan_state_bytes(const dqgan_handle* h);
+DQGAN_API int dqgan_save_state(dqgan_handle* h, void* host_dst, int64_t bytes);
+DQGAN_API int dqgan_load_state(dqgan_handle* h, const void* host_src, int64_t bytes);
+
+/* Kernels this handle has launched so far. */
+DQGAN_API uint64_t dqgan_launch_count(const dqgan_handle* h);
+
+/* Text of the last error on this handle, or of the last failed
+ * create / validate / layout call in this thread when h is NULL.
+ * Never NULL; valid until the next call on the same handle / thread. */
+DQGAN_API const char* dqgan_last_error(const dqgan_handle* h);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* DQGAN_H_ */

@@ -1,0 +1,11 @@
+"""GB300-native (sm_103a) hot path of DQGAN (arXiv 2010.13359, Algorithm 2).
+
+The compute lives in ``libdqgan.so`` (CUDA kernels behind the C-ABI of
+``include/dqgan.h``); ``dqgan`` is its ctypes binding and ``workloads`` makes
+the seeded synthetic inputs.
+"""
+from . import dqgan  # noqa: F401
+from .dqgan import (  # noqa: F401
+    IDENTITY, KEEP_LOOKAHEAD, SIGN, SQUANT, TOPK, Config, DqganError, Handle, create, make_config,
+    message_layout, validate_config,
+)

@@ -1,0 +1,459 @@
+// C-ABI of the DQGAN hot path (declared in include/dqgan.h): argument
+// checking, ownership of the per-worker state (residuals e, lookahead offsets
+// h, top-k scratch, step t) and dispatch to the kernels.  Every entry point
+// returns a status and never aborts.
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <new>
+#include <string>
+
+#include "internal.cuh"
+
+struct dqgan_handle {
+  dqgan_config cfg;
+  cudaStream_t stream = nullptr;
+  int device = 0;
+  int64_t ld = 0;  // row stride of e and h, floats
+  int64_t nb = 0;
+  dq::Layout lay{};
+  float* e = nullptr;
+  float* h = nullptr;
+  void* scratch = nullptr;
+  size_t scratch_bytes = 0;
+  int64_t t = 1;
+  uint64_t launches = 0;
+  std::string err;
+};
+
+namespace {
+
+thread_local std::string tl_err;
+
+int set_error(dqgan_handle* h, int code, const char* fmt, ...) {
+  char buf[512];
+  va_list ap;
+  va_start(ap, fmt);
+  vsnprintf(buf, sizeof buf, fmt, ap);
+  va_end(ap);
+  if (h) h->err = buf;
+  else tl_err = buf;
+  return code;
+}
+
+bool is_pow2(int64_t x) { return x > 0 && (x & (x - 1)) == 0; }
+bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
+
+// Returns an empty string for a valid config, else the reason.
+std::string check_config(const dqgan_config* c) {
+  char buf[256];
+  if (!c) return "config is NULL";
+  if (c->d < 1 || c->d > 0xFFFFFFFFll) {
+    snprintf(buf, sizeof buf, "d = %lld outside [1, 2^32 - 1]", (long long)c->d);
+    return buf;
+  }
+  if (c->M < 1 || c->M > 4096) {
+    snprintf(buf, sizeof buf, "M = %d outside [1, 4096]", c->M);
+    return buf;
+  }
+  if (!std::isfinite(c->lr)) return "lr is not finite";
+  if (c->flags & ~DQGAN_KEEP_LOOKAHEAD) return "unknown flag bits";
+  switch (c->compressor) {
+    case DQGAN_SIGN:
+    case DQGAN_SQUANT:
+      if (!is_pow2(c->bucket) || c->bucket < 32 || c->bucket > 4096) {
+        snprintf(buf, sizeof buf, "bucket = %d is not a power of two in [32, 4096]", c->bucket);
+        return buf;
+      }
+      if (c->compressor == DQGAN_SQUANT && c->bits != 2 && c->bits != 4 && c->bits != 8) {
+        snprintf(buf, sizeof buf, "bits = %d not in {2, 4, 8}", c->bits);
+        return buf;
+      }
+      break;
+    case DQGAN_TOPK:
+      if (c->k < 1 || c->k > c->d) {
+        snprintf(buf, sizeof buf, "k = %lld outside [1, d]", (long long)c->k);
+        return buf;
+      }
+      break;
+    case DQGAN_IDENTITY:
+      break;
+    default:
+      snprintf(buf, sizeof buf, "unknown compressor %d", c->compressor);
+      return buf;
+  }
+  return "";
+}
+
+int64_t round_up(int64_t x, int64_t m) { return (x + m - 1) / m * m; }
+
+int cuda_fail(dqgan_handle* h, cudaError_t e, const char* what) {
+  return set_error(h, DQGAN_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+}
+
+dq::CompressArgs compress_args(dqgan_handle* h, const float* g, int64_t g_stride, void* msg,
+                               int64_t msg_stride, int32_t worker0, int32_t nworkers) {
+  dq::CompressArgs a{};
+  a.g = g;
+  a.g_stride = g_stride;
+  a.e = h->e;
+  a.h = h->h;
+  a.ld = h->ld;
+  a.msg = reinterpret_cast<uint8_t*>(msg);
+  a.msg_stride = msg_stride;
+  a.d = h->cfg.d;
+  a.nb = h->nb;
+  a.off_payload = h->lay.off_payload;
+  a.lr = h->cfg.lr;
+  a.bucket = h->cfg.bucket;
+  a.bits = h->cfg.bits;
+  a.worker0 = worker0;
+  a.nworkers = nworkers;
+  a.seed_lo = (uint32_t)(h->cfg.seed & 0xFFFFFFFFu);
+  a.seed_hi = (uint32_t)(h->cfg.seed >> 32);
+  a.step = (uint32_t)h->t;
+  return a;
+}
+
+int run_compress(dqgan_handle* h, const dq::CompressArgs& a) {
+  const bool keep = (h->cfg.flags & DQGAN_KEEP_LOOKAHEAD) != 0;
+  cudaError_t st = cudaSuccess;
+  switch (h->cfg.compressor) {
+    case DQGAN_SIGN: st = dq::launch_sign_compress(a, keep, h->stream, &h->launches); break;
+    case DQGAN_SQUANT: st = dq::launch_squant_compress(a, keep, h->stream, &h->launches); break;
+    case DQGAN_IDENTITY: st = dq::launch_identity_compress(a, keep, h->stream, &h->launches); break;
+    case DQGAN_TOPK: {
+      // scratch rows: one per concurrently compressed worker
+      st = dq::launch_topk_compress(a, h->cfg.k, keep, h->scratch, h->stream, &h->launches);
+      break;
+    }
+  }
+  if (st != cudaSuccess) return cuda_fail(h, st, "compress launch");
+  return DQGAN_OK;
+}
+
+int check_worker(dqgan_handle* h, int32_t i) {
+  if (i < 0 || i >= h->cfg.M)
+    return set_error(h, DQGAN_ERR_INVALID_ARG, "worker %d outside [0, %d)", i, h->cfg.M);
+  return DQGAN_OK;
+}
+
+int copy_rows(dqgan_handle* h, float* base, int32_t i, void* dst, const void* src) {
+  float* row = base + (int64_t)i * h->ld;
+  cudaError_t st;
+  if (dst) st = cudaMemcpyAsync(dst, row, (size_t)h->cfg.d * 4, cudaMemcpyDefault, h->stream);
+  else st = cudaMemcpyAsync(row, src, (size_t)h->cfg.d * 4, cudaMemcpyDefault, h->stream);
+  if (st != cudaSuccess) return cuda_fail(h, st, "copy");
+  st = cudaStreamSynchronize(h->stream);
+  if (st != cudaSuccess) return cuda_fail(h, st, "copy sync");
+  return DQGAN_OK;
+}
+
+struct StateHeader {
+  char magic[8];
+  int64_t d;
+  int64_t k;
+  int64_t t;
+  int32_t M;
+  int32_t compressor;
+  int32_t bucket;
+  int32_t bits;
+  uint32_t flags;
+  uint32_t reserved;
+};
+static_assert(sizeof(StateHeader) == 56, "state header layout");
+constexpr int64_t kHeaderBytes = 64;
+
+}  // namespace
+
+namespace dq {
+
+bool message_layout(const dqgan_config& c, Layout* out) {
+  if (!check_config(&c).empty()) return false;
+  const int64_t nb = (c.compressor == DQGAN_SIGN || c.compressor == DQGAN_SQUANT)
+                         ? (c.d + c.bucket - 1) / c.bucket
+                         : 0;
+  Layout L{0, 0, 0};
+  switch (c.compressor) {
+    case DQGAN_SIGN:
+      L.off_payload = round_up(4 * nb, 256);
+      L.total = round_up(L.off_payload + 4 * ((c.d + 31) / 32), 256);
+      break;
+    case DQGAN_SQUANT:
+      L.off_payload = round_up(4 * nb, 256);
+      L.total = round_up(L.off_payload + 4 * ((c.d * c.bits + 31) / 32), 256);
+      break;
+    case DQGAN_TOPK:
+      L.total = round_up(8 * c.k, 256);
+      break;
+    case DQGAN_IDENTITY:
+      L.total = round_up(4 * c.d, 256);
+      break;
+  }
+  *out = L;
+  return true;
+}
+
+}  // namespace dq
+
+extern "C" {
+
+int dqgan_validate_config(const dqgan_config* cfg) {
+  const std::string why = check_config(cfg);
+  if (!why.empty()) return set_error(nullptr, DQGAN_ERR_INVALID_ARG, "%s", why.c_str());
+  return DQGAN_OK;
+}
+
+int dqgan_message_layout(const dqgan_config* cfg, int64_t* scales_offset, int64_t* payload_offset,
+                         int64_t* total_bytes) {
+  const std::string why = check_config(cfg);
+  if (!why.empty()) return set_error(nullptr, DQGAN_ERR_INVALID_ARG, "%s", why.c_str());
+  dq::Layout L;
+  dq::message_layout(*cfg, &L);
+  if (scales_offset) *scales_offset = L.off_scales;
+  if (payload_offset) *payload_offset = L.off_payload;
+  if (total_bytes) *total_bytes = L.total;
+  return DQGAN_OK;
+}
+
+int dqgan_create(const dqgan_config* cfg, dqgan_handle** out) {
+  if (!out) return set_error(nullptr, DQGAN_ERR_INVALID_ARG, "out is NULL");
+  *out = nullptr;
+  const std::string why = check_config(cfg);
+  if (!why.empty()) return set_error(nullptr, DQGAN_ERR_INVALID_ARG, "%s", why.c_str());
+  dqgan_handle* h = new (std::nothrow) dqgan_handle();
+  if (!h) return set_error(nullptr, DQGAN_ERR_OOM, "host allocation failed");
+  h->cfg = *cfg;
+  h->stream = reinterpret_cast<cudaStream_t>(cfg->cuda_stream);
+  dq::message_layout(*cfg, &h->lay);
+  h->nb = (cfg->d + cfg->bucket - 1) / (cfg->bucket > 0 ? cfg->bucket : 1);
+  h->ld = round_up(cfg->d, 64);
+  cudaError_t st = cudaGetDevice(&h->device);
+  if (st != cudaSuccess) {
+    delete h;
+    return set_error(nullptr, DQGAN_ERR_CUDA, "cudaGetDevice: %s", cudaGetErrorString(st));
+  }
+  const size_t rows_bytes = (size_t)cfg->M * (size_t)h->ld * sizeof(float);
+  auto fail_oom = [&](const char* what, cudaError_t e) {
+    cudaGetLastError();
+    if (h->e) cudaFree(h->e);
+    if (h->h) cudaFree(h->h);
+    if (h->scratch) cudaFree(h->scratch);
+    delete h;
+    return set_error(nullptr, e == cudaErrorMemoryAllocation ? DQGAN_ERR_OOM : DQGAN_ERR_CUDA,
+                     "%s: %s", what, cudaGetErrorString(e));
+  };
+  if ((st = cudaMalloc(&h->e, rows_bytes)) != cudaSuccess) return fail_oom("allocating e", st);
+  if (cfg->flags & DQGAN_KEEP_LOOKAHEAD)
+    if ((st = cudaMalloc(&h->h, rows_bytes)) != cudaSuccess) return fail_oom("allocating h", st);
+  if (cfg->compressor == DQGAN_TOPK) {
+    h->scratch_bytes = dq::topk_scratch_bytes(cfg->d, cfg->M);
+    if ((st = cudaMalloc(&h->scratch, h->scratch_bytes)) != cudaSuccess)
+      return fail_oom("allocating top-k scratch", st);
+  }
+  if ((st = cudaMemsetAsync(h->e, 0, rows_bytes, h->stream)) != cudaSuccess) return fail_oom("zeroing e", st);
+  if (h->h && (st = cudaMemsetAsync(h->h, 0, rows_bytes, h->stream)) != cudaSuccess)
+    return fail_oom("zeroing h", st);
+  if (h->scratch && (st = cudaMemsetAsync(h->scratch, 0, h->scratch_bytes, h->stream)) != cudaSuccess)
+    return fail_oom("zeroing scratch", st);
+  if ((st = cudaStreamSynchronize(h->stream)) != cudaSuccess) return fail_oom("create sync", st);
+  h->t = 1;
+  *out = h;
+  return DQGAN_OK;
+}
+
+int dqgan_destroy(dqgan_handle* h) {
+  if (!h) return DQGAN_OK;
+  cudaStreamSynchronize(h->stream);
+  if (h->e) cudaFree(h->e);
+  if (h->h) cudaFree(h->h);
+  if (h->scratch) cudaFree(h->scratch);
+  const cudaError_t st = cudaGetLastError();
+  delete h;
+  if (st != cudaSuccess) return set_error(nullptr, DQGAN_ERR_CUDA, "destroy: %s", cudaGetErrorString(st));
+  return DQGAN_OK;
+}
+
+int64_t dqgan_message_bytes(const dqgan_handle* h) { return h ? h->lay.total : -1; }
+
+int dqgan_worker_compress(dqgan_handle* h, int32_t i, const float* g, void* out_msg) {
+  if (!h) return set_error(nullptr, DQGAN_ERR_INVALID_ARG, "handle is NULL");
+  if (int r = check_worker(h, i)) return r;
+  if (!g || !out_msg) return set_error(h, DQGAN_ERR_INVALID_ARG, "NULL gradient or message pointer");
+  if (!aligned16(g) || !aligned16(out_msg))
+    return set_error(h, DQGAN_ERR_INVALID_ARG, "gradient and message must be 16-byte aligned");
+  return run_compress(h, compress_args(h, g, 0, out_msg, 0, i, 1));
+}
+
+int dqgan_workers_compress_all(dqgan_handle* h, const float* g_all, int64_t g_stride, void* msgs_all) {
+  if (!h) return set_error(nullptr, DQGAN_ERR_INVALID_ARG, "handle is NULL");
+  if (!g_all || !msgs_all) return set_error(h, DQGAN_ERR_INVALID_ARG, "NULL gradient or message pointer");
+  if (!aligned16(g_all) || !aligned16(msgs_all))
+    return set_error(h, DQGAN_ERR_INVALID_ARG, "gradients and messages must be 16-byte aligned");
+  if (g_stride < h->cfg.d || (g_stride & 3))
+    return set_error(h, DQGAN_ERR_INVALID_ARG, "g_stride = %lld must be >= d and a multiple of 4",
+                     (long long)g_stride);
+  return run_compress(h, compress_args(h, g_all, g_stride, msgs_all, h->lay.total, 0, h->cfg.M));
+}
+
+int dqgan_server_aggregate_update(dqgan_handle* h, const void* msgs_all, float* params) {
+  if (!h) return set_error(nullptr, DQGAN_ERR_INVALID_ARG, "handle is NULL");
+  if (!msgs_all || !params) return set_error(h, DQGAN_ERR_INVALID_ARG, "NULL message or parameter pointer");
+  if (!aligned16(msgs_all) || !aligned16(params))
+    return set_error(h, DQGAN_ERR_INVALID_ARG, "messages and parameters must be 16-byte aligned");
+  dq::ServerArgs s{};
+  s.msgs = reinterpret_cast<const uint8_t*>(msgs_all);
+  s.msg_stride = h->lay.total;
+  s.w = params;
+  s.d = h->cfg.d;
+  s.k = h->cfg.k;
+  s.off_payload = h->lay.off_payload;
+  s.M = h->cfg.M;
+  s.bucket = h->cfg.bucket;
+  s.bits = h->cfg.bits;
+  s.M_pow2 = is_pow2(h->cfg.M) ? 1 : 0;
+  s.inv_M = 1.0f / (float)h->cfg.M;
+  cudaError_t st = cudaSuccess;
+  switch (h->cfg.compressor) {
+    case DQGAN_SIGN: st = dq::launch_sign_server(s, h->stream, &h->launches); break;
+    case DQGAN_SQUANT: st = dq::launch_squant_server(s, h->stream, &h->launches); break;
+    case DQGAN_IDENTITY: st = dq::launch_identity_server(s, h->stream, &h->launches); break;
+    case DQGAN_TOPK: st = dq::launch_topk_server(s, h->stream, &h->launches); break;
+  }
+  if (st != cudaSuccess) return cuda_fail(h, st, "server launch");
+  h->t += 1;
+  return DQGAN_OK;
+}
+
+int dqgan_worker_lookahead(dqgan_handle* h, int32_t i, const float* params, float* out_w_half) {
+  if (!h) return set_error(nullptr, DQGAN_ERR_INVALID_ARG, "handle is NULL");
+  if (!(h->cfg.flags & DQGAN_KEEP_LOOKAHEAD))
+    return set_error(h, DQGAN_ERR_UNSUPPORTED, "lookahead needs DQGAN_KEEP_LOOKAHEAD");
+  if (int r = check_worker(h, i)) return r;
+  if (!params || !out_w_half) return set_error(h, DQGAN_ERR_INVALID_ARG, "NULL pointer");
+  if (!aligned16(params) || !aligned16(out_w_half))
+    return set_error(h, DQGAN_ERR_INVALID_ARG, "pointers must be 16-byte aligned");
+  const cudaError_t st = dq::launch_lookahead(params, h->h + (int64_t)i * h->ld, out_w_half, h->cfg.d,
+                                              h->stream, &h->launches);
+  if (st != cudaSuccess) return cuda_fail(h, st, "lookahead launch");
+  return DQGAN_OK;
+}
+
+int dqgan_synchronize(dqgan_handle* h) {
+  if (!h) return set_error(nullptr, DQGAN_ERR_INVALID_ARG, "handle is NULL");
+  cudaError_t st = cudaStreamSynchronize(h->stream);
+  if (st == cudaSuccess) st = cudaGetLastError();
+  if (st != cudaSuccess) return cuda_fail(h, st, "synchronize");
+  return DQGAN_OK;
+}
+
+int dqgan_get_residual(dqgan_handle* h, int32_t i, float* dst) {
+  if (!h) return set_error(nullptr, DQGAN_ERR_INVALID_ARG, "handle is NULL");
+  if (int r = check_worker(h, i)) return r;
+  if (!dst) return set_error(h, DQGAN_ERR_INVALID_ARG, "dst is NULL");
+  return copy_rows(h, h->e, i, dst, nullptr);
+}
+
+int dqgan_set_residual(dqgan_handle* h, int32_t i, const float* src) {
+  if (!h) return set_error(nullptr, DQGAN_ERR_INVALID_ARG, "handle is NULL");
+  if (int r = check_worker(h, i)) return r;
+  if (!src) return set_error(h, DQGAN_ERR_INVALID_ARG, "src is NULL");
+  return copy_rows(h, h->e, i, nullptr, src);
+}
+
+int dqgan_get_lookahead(dqgan_handle* h, int32_t i, float* dst) {
+  if (!h) return set_error(nullptr, DQGAN_ERR_INVALID_ARG, "handle is NULL");
+  if (!h->h) return set_error(h, DQGAN_ERR_UNSUPPORTED, "lookahead needs DQGAN_KEEP_LOOKAHEAD");
+  if (int r = check_worker(h, i)) return r;
+  if (!dst) return set_error(h, DQGAN_ERR_INVALID_ARG, "dst is NULL");
+  return copy_rows(h, h->h, i, dst, nullptr);
+}
+
+int dqgan_set_lookahead(dqgan_handle* h, int32_t i, const float* src) {
+  if (!h) return set_error(nullptr, DQGAN_ERR_INVALID_ARG, "handle is NULL");
+  if (!h->h) return set_error(h, DQGAN_ERR_UNSUPPORTED, "lookahead needs DQGAN_KEEP_LOOKAHEAD");
+  if (int r = check_worker(h, i)) return r;
+  if (!src) return set_error(h, DQGAN_ERR_INVALID_ARG, "src is NULL");
+  return copy_rows(h, h->h, i, nullptr, src);
+}
+
+int64_t dqgan_get_step(const dqgan_handle* h) { return h ? h->t : -1; }
+
+int dqgan_set_step(dqgan_handle* h, int64_t t) {
+  if (!h) return set_error(nullptr, DQGAN_ERR_INVALID_ARG, "handle is NULL");
+  if (t < 1 || t > 0xFFFFFFFFll) return set_error(h, DQGAN_ERR_INVALID_ARG, "step %lld outside [1, 2^32)", (long long)t);
+  h->t = t;
+  return DQGAN_OK;
+}
+
+int64_t dqgan_state_bytes(const dqgan_handle* h) {
+  if (!h) return -1;
+  const int64_t rows = (int64_t)h->cfg.M * h->cfg.d * 4;
+  return kHeaderBytes + rows * (h->h ? 2 : 1);
+}
+
+int dqgan_save_state(dqgan_handle* h, void* host_dst, int64_t bytes) {
+  if (!h) return set_error(nullptr, DQGAN_ERR_INVALID_ARG, "handle is NULL");
+  if (!host_dst || bytes < dqgan_state_bytes(h))
+    return set_error(h, DQGAN_ERR_INVALID_ARG, "state buffer NULL or smaller than %lld bytes",
+                     (long long)dqgan_state_bytes(h));
+  uint8_t* dst = reinterpret_cast<uint8_t*>(host_dst);
+  StateHeader hd{};
+  memcpy(hd.magic, "DQGANST1", 8);
+  hd.d = h->cfg.d;
+  hd.k = h->cfg.k;
+  hd.t = h->t;
+  hd.M = h->cfg.M;
+  hd.compressor = h->cfg.compressor;
+  hd.bucket = h->cfg.bucket;
+  hd.bits = h->cfg.bits;
+  hd.flags = h->cfg.flags;
+  memset(dst, 0, kHeaderBytes);
+  memcpy(dst, &hd, sizeof hd);
+  const size_t row = (size_t)h->cfg.d * 4;
+  uint8_t* out = dst + kHeaderBytes;
+  for (int which = 0; which < (h->h ? 2 : 1); ++which) {
+    float* base = which == 0 ? h->e : h->h;
+    cudaError_t st = cudaMemcpy2DAsync(out, row, base, (size_t)h->ld * 4, row, (size_t)h->cfg.M,
+                                       cudaMemcpyDefault, h->stream);
+    if (st != cudaSuccess) return cuda_fail(h, st, "save state copy");
+    out += row * (size_t)h->cfg.M;
+  }
+  const cudaError_t st = cudaStreamSynchronize(h->stream);
+  if (st != cudaSuccess) return cuda_fail(h, st, "save state sync");
+  return DQGAN_OK;
+}
+
+int dqgan_load_state(dqgan_handle* h, const void* host_src, int64_t bytes) {
+  if (!h) return set_error(nullptr, DQGAN_ERR_INVALID_ARG, "handle is NULL");
+  if (!host_src || bytes < dqgan_state_bytes(h))
+    return set_error(h, DQGAN_ERR_INVALID_ARG, "state buffer NULL or smaller than %lld bytes",
+                     (long long)dqgan_state_bytes(h));
+  const uint8_t* src = reinterpret_cast<const uint8_t*>(host_src);
+  StateHeader hd;
+  memcpy(&hd, src, sizeof hd);
+  if (memcmp(hd.magic, "DQGANST1", 8) != 0 || hd.d != h->cfg.d || hd.M != h->cfg.M ||
+      hd.compressor != h->cfg.compressor || hd.flags != h->cfg.flags || hd.k != h->cfg.k ||
+      hd.bucket != h->cfg.bucket || hd.bits != h->cfg.bits || hd.t < 1)
+    return set_error(h, DQGAN_ERR_INVALID_ARG, "state header does not match this handle's config");
+  const size_t row = (size_t)h->cfg.d * 4;
+  const uint8_t* in = src + kHeaderBytes;
+  for (int which = 0; which < (h->h ? 2 : 1); ++which) {
+    float* base = which == 0 ? h->e : h->h;
+    cudaError_t st = cudaMemcpy2DAsync(base, (size_t)h->ld * 4, in, row, row, (size_t)h->cfg.M,
+                                       cudaMemcpyDefault, h->stream);
+    if (st != cudaSuccess) return cuda_fail(h, st, "load state copy");
+    in += row * (size_t)h->cfg.M;
+  }
+  const cudaError_t st = cudaStreamSynchronize(h->stream);
+  if (st != cudaSuccess) return cuda_fail(h, st, "load state sync");
+  h->t = hd.t;
+  return DQGAN_OK;
+}
+
+uint64_t dqgan_launch_count(const dqgan_handle* h) { return h ? h->launches : 0; }
+
+const char* dqgan_last_error(const dqgan_handle* h) { return h ? h->err.c_str() : tl_err.c_str(); }
+
+}  // extern "C"

@@ -1,0 +1,435 @@
+// Worker side of Algorithm 2 (DQGAN) for the dense compressors: fused
+//   p = fl(fl(eta * g) + e)            error feedback
+//   Q(p) and its packed message         scaled sign / b-bit stochastic / identity
+//   e = fl(p - Q(p))                    residual, written in place
+//   h = fl(fl(eta * g) + e)             lookahead offset (optional)
+// in one pass over g and e.
+//
+// Mapping: one warp per bucket.  Lane l owns the 4-element chunks
+// c = l, l + 32, l + 64, ... of its bucket, loaded with 128-bit coalesced
+// loads (a warp reads 512 contiguous bytes per load instruction) and held in
+// registers until the bucket's scale is known.  The bucket's l1 sum is taken
+// in the library's fixed order: each lane adds its chunk sums
+// ((|a0|+|a1|)+|a2|)+|a3| in increasing c, then five xor-shuffle rounds with
+// partners 16, 8, 4, 2, 1 combine the 32 lane totals.  The max-abs scale of
+// the stochastic quantiser is exact in any order.
+#include "internal.cuh"
+
+namespace dq {
+namespace {
+
+__host__ __device__ __forceinline__ int64_t min64(int64_t x, int64_t y) { return x < y ? x : y; }
+__host__ __device__ __forceinline__ int64_t max64(int64_t x, int64_t y) { return x > y ? x : y; }
+
+__device__ __forceinline__ float4 ld_stream4(const float* p) {
+  return __ldcs(reinterpret_cast<const float4*>(p));
+}
+__device__ __forceinline__ void st_stream4(float* p, float4 v) {
+  __stcs(reinterpret_cast<float4*>(p), v);
+}
+
+// Spread the low 8 bits of x so that bit r lands on bit 4r.
+__device__ __forceinline__ uint32_t spread_nibbles(uint32_t x) {
+  x &= 0xFFu;
+  x = (x | (x << 12)) & 0x000F000Fu;
+  x = (x | (x << 6)) & 0x03030303u;
+  x = (x | (x << 3)) & 0x11111111u;
+  return x;
+}
+
+// Philox4x32-10 (Salmon et al., SC'11): 10 rounds, multipliers 0xD2511F53 and
+// 0xCD9E8D57, Weyl key increments 0x9E3779B9 and 0xBB67AE85 between rounds.
+__device__ __forceinline__ uint4 philox4x32_10(uint4 x, uint32_t k0, uint32_t k1) {
+#pragma unroll
+  for (int round = 0; round < 10; ++round) {
+    if (round > 0) {
+      k0 += 0x9E3779B9u;
+      k1 += 0xBB67AE85u;
+    }
+    const uint32_t lo_a = 0xD2511F53u * x.x;
+    const uint32_t hi_a = __umulhi(0xD2511F53u, x.x);
+    const uint32_t lo_b = 0xCD9E8D57u * x.z;
+    const uint32_t hi_b = __umulhi(0xCD9E8D57u, x.z);
+    x = make_uint4(hi_b ^ x.y ^ k0, lo_b, hi_a ^ x.w ^ k1, lo_a);
+  }
+  return x;
+}
+
+// Loads the CPL chunks of this lane's share of bucket `b` and forms p.
+// Out-of-bucket or out-of-range elements read as 0 and give p = 0.
+// sg (if HOLD) receives fl(eta * g) for the lookahead offset.
+template <int CPL, bool HOLD>
+__device__ __forceinline__ void load_and_form(const CompressArgs& a, const float* g, const float* e,
+                                              int64_t base, int lane, bool full,
+                                              float (&p)[CPL][4], float (&sg)[HOLD ? CPL : 1][4]) {
+  const int nchunk = a.bucket >> 2;
+  if (full) {
+#pragma unroll
+    for (int i = 0; i < CPL; ++i) {
+      const int c = lane + 32 * i;
+      float4 gv = make_float4(0.f, 0.f, 0.f, 0.f), ev = gv;
+      if (c < nchunk) {
+        gv = ld_stream4(g + base + 4 * c);
+        ev = ld_stream4(e + base + 4 * c);
+      }
+      const float gq[4] = {gv.x, gv.y, gv.z, gv.w};
+      const float eq[4] = {ev.x, ev.y, ev.z, ev.w};
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const float s = __fmul_rn(a.lr, gq[q]);
+        p[i][q] = (c < nchunk) ? __fadd_rn(s, eq[q]) : 0.f;
+        if constexpr (HOLD) sg[i][q] = s;
+      }
+    }
+  } else {
+#pragma unroll
+    for (int i = 0; i < CPL; ++i) {
+      const int c = lane + 32 * i;
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const int64_t j = base + 4 * c + q;
+        const bool ok = (c < nchunk) && (j < a.d);
+        const float gq = ok ? g[j] : 0.f;
+        const float eq = ok ? e[j] : 0.f;
+        const float s = __fmul_rn(a.lr, gq);
+        p[i][q] = ok ? __fadd_rn(s, eq) : 0.f;
+        if constexpr (HOLD) sg[i][q] = s;
+      }
+    }
+  }
+}
+
+// Stores the new residual (and lookahead offset) of one chunk.
+template <bool KEEP_H, bool HOLD, int CPL>
+__device__ __forceinline__ void store_chunk(const CompressArgs& a, const float* g, float* e, float* h,
+                                            int64_t j, bool full, int nvalid, const float (&en)[4],
+                                            const float (&sg)[HOLD ? CPL : 1][4], int i) {
+  if (full) {
+    st_stream4(e + j, make_float4(en[0], en[1], en[2], en[3]));
+    if constexpr (KEEP_H) {
+      float s4[4];
+      if constexpr (HOLD) {
+#pragma unroll
+        for (int q = 0; q < 4; ++q) s4[q] = sg[i][q];
+      } else {
+        const float4 gv = __ldg(reinterpret_cast<const float4*>(g + j));
+        s4[0] = __fmul_rn(a.lr, gv.x);
+        s4[1] = __fmul_rn(a.lr, gv.y);
+        s4[2] = __fmul_rn(a.lr, gv.z);
+        s4[3] = __fmul_rn(a.lr, gv.w);
+      }
+      st_stream4(h + j, make_float4(__fadd_rn(s4[0], en[0]), __fadd_rn(s4[1], en[1]),
+                                    __fadd_rn(s4[2], en[2]), __fadd_rn(s4[3], en[3])));
+    }
+  } else {
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      if (q < nvalid) {
+        e[j + q] = en[q];
+        if constexpr (KEEP_H) {
+          float s;
+          if constexpr (HOLD) s = sg[i][q];
+          else s = __fmul_rn(a.lr, g[j + q]);
+          h[j + q] = __fadd_rn(s, en[q]);
+        }
+      }
+    }
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Scaled sign, s_b = ||p_b||_1 / n_b (Section 2.4; error-feedback sign
+// compressor of Section 3.1).  Bit = (p < 0); Q(p) = bit ? -s_b : s_b.
+// ---------------------------------------------------------------------------
+template <int CPL, bool KEEP_H>
+__global__ void __launch_bounds__(128)
+sign_compress_kernel(const CompressArgs a) {
+  constexpr bool HOLD = KEEP_H && CPL <= 8;
+  const int lane = threadIdx.x & 31;
+  const int64_t b = (int64_t)blockIdx.x * 4 + (threadIdx.x >> 5);
+  if (b >= a.nb) return;  // whole warp leaves together
+  const int row = blockIdx.y;
+  const int worker = a.worker0 + row;
+  const float* g = a.g + (int64_t)row * a.g_stride;
+  float* e = a.e + (int64_t)worker * a.ld;
+  float* h = KEEP_H ? a.h + (int64_t)worker * a.ld : nullptr;
+  uint8_t* msg = a.msg + (int64_t)row * a.msg_stride;
+
+  const int64_t base = b * a.bucket;
+  const int64_t count = min64((int64_t)a.bucket, a.d - base);
+  const bool full = (count == a.bucket);
+  const int nchunk = a.bucket >> 2;
+
+  float p[CPL][4];
+  float sg[HOLD ? CPL : 1][4];
+  load_and_form<CPL, HOLD>(a, g, e, base, lane, full, p, sg);
+
+  // l1 of the bucket in the fixed order
+  float acc = 0.f;
+#pragma unroll
+  for (int i = 0; i < CPL; ++i) {
+    const float cs = __fadd_rn(__fadd_rn(__fadd_rn(fabsf(p[i][0]), fabsf(p[i][1])), fabsf(p[i][2])),
+                               fabsf(p[i][3]));
+    acc = __fadd_rn(acc, cs);
+  }
+#pragma unroll
+  for (int off = 16; off >= 1; off >>= 1) acc = __fadd_rn(acc, __shfl_xor_sync(kFullMask, acc, off));
+  const float s = __fdiv_rn(acc, (float)count);
+  if (lane == 0) reinterpret_cast<float*>(msg)[b] = s;
+
+  uint32_t* words = reinterpret_cast<uint32_t*>(msg + a.off_payload);
+  const int64_t word0 = base >> 5;
+  const int64_t nwords = (a.d + 31) >> 5;
+  const int words_in_bucket = a.bucket >> 5;
+#pragma unroll
+  for (int i = 0; i < CPL; ++i) {
+    const uint32_t B0 = __ballot_sync(kFullMask, p[i][0] < 0.f);
+    const uint32_t B1 = __ballot_sync(kFullMask, p[i][1] < 0.f);
+    const uint32_t B2 = __ballot_sync(kFullMask, p[i][2] < 0.f);
+    const uint32_t B3 = __ballot_sync(kFullMask, p[i][3] < 0.f);
+    // Row i covers chunks 32i..32i+31, i.e. words 4i..4i+3 of the bucket; bit
+    // 4r+q of word 4i+u comes from element q of the chunk in lane 8u+r.
+    if (lane < 4) {
+      const int wib = 4 * i + lane;
+      if (wib < words_in_bucket && word0 + wib < nwords) {
+        const int sh = 8 * lane;
+        const uint32_t wv = spread_nibbles(B0 >> sh) | (spread_nibbles(B1 >> sh) << 1) |
+                            (spread_nibbles(B2 >> sh) << 2) | (spread_nibbles(B3 >> sh) << 3);
+        words[word0 + wib] = wv;
+      }
+    }
+    const int c = lane + 32 * i;
+    if (c < nchunk) {
+      const int64_t j = base + 4 * c;
+      const int nvalid = (int)min64(4, a.d - j);
+      if (nvalid > 0) {
+        float en[4];
+#pragma unroll
+        for (int q = 0; q < 4; ++q) en[q] = __fsub_rn(p[i][q], p[i][q] < 0.f ? -s : s);
+        store_chunk<KEEP_H, HOLD, CPL>(a, g, e, h, j, full, nvalid, en, sg, i);
+      }
+    }
+  }
+}
+
+// ---------------------------------------------------------------------------
+// b-bit stochastic quantiser of Hou et al. (Section 2.4, proof of Theorem 2):
+// s_b = max |p_j|, levels B_r = r / K, K = 2^(b-1) - 1; |p_j| K / s_b rounds
+// up from r = floor(.) iff u < frac(.), u the 24-bit Philox4x32-10 draw of
+// counter (j div 4, worker, step, 0x51) word j mod 4; code = K +- level.
+// ---------------------------------------------------------------------------
+template <int CPL, int BITS, bool KEEP_H>
+__global__ void __launch_bounds__(128)
+squant_compress_kernel(const CompressArgs a) {
+  constexpr int K = (1 << (BITS - 1)) - 1;
+  constexpr bool HOLD = KEEP_H && CPL <= 8;
+  __shared__ float level_value[K + 1];  // fl(r / K)
+  for (int r = threadIdx.x; r <= K; r += blockDim.x) level_value[r] = __fdiv_rn((float)r, (float)K);
+  __syncthreads();
+
+  const int lane = threadIdx.x & 31;
+  const int64_t b = (int64_t)blockIdx.x * 4 + (threadIdx.x >> 5);
+  if (b >= a.nb) return;
+  const int row = blockIdx.y;
+  const int worker = a.worker0 + row;
+  const float* g = a.g + (int64_t)row * a.g_stride;
+  float* e = a.e + (int64_t)worker * a.ld;
+  float* h = KEEP_H ? a.h + (int64_t)worker * a.ld : nullptr;
+  uint8_t* msg = a.msg + (int64_t)row * a.msg_stride;
+
+  const int64_t base = b * a.bucket;
+  const int64_t count = min64((int64_t)a.bucket, a.d - base);
+  const bool full = (count == a.bucket);
+  const int nchunk = a.bucket >> 2;
+
+  float p[CPL][4];
+  float sg[HOLD ? CPL : 1][4];
+  load_and_form<CPL, HOLD>(a, g, e, base, lane, full, p, sg);
+
+  float mx = 0.f;
+#pragma unroll
+  for (int i = 0; i < CPL; ++i)
+#pragma unroll
+    for (int q = 0; q < 4; ++q) mx = fmaxf(mx, fabsf(p[i][q]));
+#pragma unroll
+  for (int off = 16; off >= 1; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(kFullMask, mx, off));
+  const float s = mx;
+  if (lane == 0) reinterpret_cast<float*>(msg)[b] = s;
+  const float inv = (s > 0.f) ? __fdiv_rn((float)K, s) : 0.f;
+
+  uint32_t* words = reinterpret_cast<uint32_t*>(msg + a.off_payload);
+  const int64_t nwords = (a.d * BITS + 31) >> 5;
+#pragma unroll
+  for (int i = 0; i < CPL; ++i) {
+    const int c = lane + 32 * i;
+    const int64_t j = base + 4 * c;
+    const int64_t cg = j >> 2;  // global chunk index = Philox counter word 0
+    const int nvalid = (c < nchunk) ? (int)max64(0, min64(4, a.d - j)) : 0;
+    const uint4 r4 = philox4x32_10(make_uint4((uint32_t)cg, (uint32_t)worker, a.step, kSquantTag),
+                                   a.seed_lo, a.seed_hi);
+    const uint32_t rq[4] = {r4.x, r4.y, r4.z, r4.w};
+    uint32_t chunk_bits = 0;
+    float en[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      const float pv = p[i][q];
+      int code = K;
+      float qv = 0.f;
+      if (s > 0.f) {
+        const float t = fminf(__fmul_rn(fabsf(pv), inv), (float)K);
+        const float r = floorf(t);
+        const float f = __fsub_rn(t, r);
+        const float u = __fmul_rn(__uint2float_rn(rq[q] >> 8), 0x1p-24f);
+        int level = (int)r + (u < f ? 1 : 0);
+        level = min(level, K);
+        const bool neg = pv < 0.f;
+        code = neg ? K - level : K + level;
+        if (level != 0) {
+          const float mag = __fmul_rn(s, level_value[level]);
+          qv = neg ? -mag : mag;
+        }
+      }
+      en[q] = __fsub_rn(pv, qv);
+      if (q < nvalid) chunk_bits |= (uint32_t)code << (q * BITS);
+    }
+    // pack: a chunk is 4*BITS bits; 32 / (4*BITS) neighbouring lanes share a word
+    uint32_t wv = chunk_bits;
+    int64_t widx;
+    bool writer;
+    if constexpr (BITS == 8) {
+      widx = cg;
+      writer = true;
+    } else if constexpr (BITS == 4) {
+      wv <<= 16 * (lane & 1);
+      wv |= __shfl_xor_sync(kFullMask, wv, 1);
+      widx = cg >> 1;
+      writer = (lane & 1) == 0;
+    } else {
+      wv <<= 8 * (lane & 3);
+      wv |= __shfl_xor_sync(kFullMask, wv, 1);
+      wv |= __shfl_xor_sync(kFullMask, wv, 2);
+      widx = cg >> 2;
+      writer = (lane & 3) == 0;
+    }
+    if (writer && c < nchunk && widx < nwords) words[widx] = wv;
+    if (nvalid > 0) store_chunk<KEEP_H, HOLD, CPL>(a, g, e, h, j, full, nvalid, en, sg, i);
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Identity: the message is p itself and e = fl(p - p) = 0.
+// ---------------------------------------------------------------------------
+template <bool KEEP_H>
+__global__ void __launch_bounds__(256)
+identity_compress_kernel(const CompressArgs a) {
+  const int row = blockIdx.y;
+  const int worker = a.worker0 + row;
+  const float* g = a.g + (int64_t)row * a.g_stride;
+  float* e = a.e + (int64_t)worker * a.ld;
+  float* h = KEEP_H ? a.h + (int64_t)worker * a.ld : nullptr;
+  float* vals = reinterpret_cast<float*>(a.msg + (int64_t)row * a.msg_stride);
+  const int64_t nchunks = (a.d + 3) >> 2;
+  for (int64_t c = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; c < nchunks;
+       c += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t j = 4 * c;
+    if (j + 3 < a.d) {
+      const float4 gv = ld_stream4(g + j);
+      const float4 ev = ld_stream4(e + j);
+      const float gq[4] = {gv.x, gv.y, gv.z, gv.w};
+      const float eq[4] = {ev.x, ev.y, ev.z, ev.w};
+      float pv[4], en[4], hv[4];
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const float s = __fmul_rn(a.lr, gq[q]);
+        pv[q] = __fadd_rn(s, eq[q]);
+        en[q] = __fsub_rn(pv[q], pv[q]);
+        hv[q] = __fadd_rn(s, en[q]);
+      }
+      st_stream4(vals + j, make_float4(pv[0], pv[1], pv[2], pv[3]));
+      st_stream4(e + j, make_float4(en[0], en[1], en[2], en[3]));
+      if constexpr (KEEP_H) st_stream4(h + j, make_float4(hv[0], hv[1], hv[2], hv[3]));
+    } else {
+      for (int64_t jj = j; jj < a.d; ++jj) {
+        const float s = __fmul_rn(a.lr, g[jj]);
+        const float pv = __fadd_rn(s, e[jj]);
+        const float en = __fsub_rn(pv, pv);
+        vals[jj] = pv;
+        e[jj] = en;
+        if constexpr (KEEP_H) h[jj] = __fadd_rn(s, en);
+      }
+    }
+  }
+}
+
+template <int CPL>
+cudaError_t sign_dispatch_keep(const CompressArgs& a, bool keep_h, cudaStream_t stream) {
+  const dim3 grid((unsigned)((a.nb + 3) / 4), (unsigned)a.nworkers);
+  if (keep_h) sign_compress_kernel<CPL, true><<<grid, 128, 0, stream>>>(a);
+  else sign_compress_kernel<CPL, false><<<grid, 128, 0, stream>>>(a);
+  return cudaGetLastError();
+}
+
+template <int CPL, int BITS>
+cudaError_t squant_dispatch_keep(const CompressArgs& a, bool keep_h, cudaStream_t stream) {
+  const dim3 grid((unsigned)((a.nb + 3) / 4), (unsigned)a.nworkers);
+  if (keep_h) squant_compress_kernel<CPL, BITS, true><<<grid, 128, 0, stream>>>(a);
+  else squant_compress_kernel<CPL, BITS, false><<<grid, 128, 0, stream>>>(a);
+  return cudaGetLastError();
+}
+
+template <int CPL>
+cudaError_t squant_dispatch_bits(const CompressArgs& a, bool keep_h, cudaStream_t stream) {
+  switch (a.bits) {
+    case 2: return squant_dispatch_keep<CPL, 2>(a, keep_h, stream);
+    case 4: return squant_dispatch_keep<CPL, 4>(a, keep_h, stream);
+    case 8: return squant_dispatch_keep<CPL, 8>(a, keep_h, stream);
+  }
+  return cudaErrorInvalidValue;
+}
+
+}  // namespace
+
+cudaError_t launch_sign_compress(const CompressArgs& a, bool keep_h, cudaStream_t stream,
+                                 uint64_t* launches) {
+  cudaError_t st;
+  switch (a.bucket) {
+    case 32: case 64: case 128: st = sign_dispatch_keep<1>(a, keep_h, stream); break;
+    case 256: st = sign_dispatch_keep<2>(a, keep_h, stream); break;
+    case 512: st = sign_dispatch_keep<4>(a, keep_h, stream); break;
+    case 1024: st = sign_dispatch_keep<8>(a, keep_h, stream); break;
+    case 2048: st = sign_dispatch_keep<16>(a, keep_h, stream); break;
+    case 4096: st = sign_dispatch_keep<32>(a, keep_h, stream); break;
+    default: return cudaErrorInvalidValue;
+  }
+  *launches += 1;
+  return st;
+}
+
+cudaError_t launch_squant_compress(const CompressArgs& a, bool keep_h, cudaStream_t stream,
+                                   uint64_t* launches) {
+  cudaError_t st;
+  switch (a.bucket) {
+    case 32: case 64: case 128: st = squant_dispatch_bits<1>(a, keep_h, stream); break;
+    case 256: st = squant_dispatch_bits<2>(a, keep_h, stream); break;
+    case 512: st = squant_dispatch_bits<4>(a, keep_h, stream); break;
+    case 1024: st = squant_dispatch_bits<8>(a, keep_h, stream); break;
+    case 2048: st = squant_dispatch_bits<16>(a, keep_h, stream); break;
+    case 4096: st = squant_dispatch_bits<32>(a, keep_h, stream); break;
+    default: return cudaErrorInvalidValue;
+  }
+  *launches += 1;
+  return st;
+}
+
+cudaError_t launch_identity_compress(const CompressArgs& a, bool keep_h, cudaStream_t stream,
+                                     uint64_t* launches) {
+  const int64_t nchunks = (a.d + 3) / 4;
+  const int64_t blocks = min64((nchunks + 255) / 256, 152 * 8);
+  const dim3 grid((unsigned)max64(blocks, 1), (unsigned)a.nworkers);
+  if (keep_h) identity_compress_kernel<true><<<grid, 256, 0, stream>>>(a);
+  else identity_compress_kernel<false><<<grid, 256, 0, stream>>>(a);
+  *launches += 1;
+  return cudaGetLastError();
+}
+
+}  // namespace dq

@@ -1,0 +1,94 @@
+// Internal declarations of the sm_103a DQGAN library (not part of the C-ABI).
+//
+// Every kernel computes in IEEE binary32 with explicit round-to-nearest
+// intrinsics (__fmul_rn, __fadd_rn, __fsub_rn, __fdiv_rn), which the compiler
+// never contracts into fused multiply-adds; the library is also built with
+// -fmad=false.  That makes messages and residuals reproducible bit for bit.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "dqgan.h"
+
+namespace dq {
+
+constexpr unsigned kFullMask = 0xffffffffu;
+// Counter word 3 of the Philox4x32-10 draws of the stochastic quantiser.
+constexpr uint32_t kSquantTag = 0x51u;
+
+struct Layout {
+  int64_t off_scales;
+  int64_t off_payload;
+  int64_t total;
+};
+
+// Host-side layout of one message (see dqgan.h); returns false on a bad config.
+bool message_layout(const dqgan_config& cfg, Layout* out);
+
+// Arguments shared by every worker-side (compress) kernel.  One launch covers
+// `nworkers` consecutive workers starting at `worker0`; launch row y (blockIdx.y)
+// is worker worker0 + y.
+struct CompressArgs {
+  const float* g;      // gradient of row y at g + y * g_stride
+  int64_t g_stride;    // floats, multiple of 4
+  float* e;            // residual of worker w at e + w * ld (library-owned)
+  float* h;            // lookahead offset of worker w at h + w * ld, or nullptr
+  int64_t ld;          // floats, multiple of 64
+  uint8_t* msg;        // message of row y at msg + y * msg_stride
+  int64_t msg_stride;  // bytes
+  int64_t d;
+  int64_t nb;          // buckets: ceil(d / bucket)
+  int64_t off_payload; // byte offset of the payload section in a message
+  float lr;
+  int32_t bucket;
+  int32_t bits;
+  int32_t worker0;
+  int32_t nworkers;
+  uint32_t seed_lo, seed_hi;
+  uint32_t step;
+};
+
+// Arguments of the server (decode + average + update) kernels.
+struct ServerArgs {
+  const uint8_t* msgs;  // message m at msgs + m * msg_stride
+  int64_t msg_stride;
+  float* w;             // d parameters, updated in place
+  int64_t d;
+  int64_t k;            // top-k records per message
+  int64_t off_payload;
+  int32_t M;
+  int32_t bucket;
+  int32_t bits;
+  float inv_M;          // exact 1/M when M is a power of two
+  int32_t M_pow2;       // 1 if M is a power of two (then x/M == x * inv_M exactly)
+};
+
+// Scratch of the top-k path for `nworkers` concurrent workers.
+struct TopkScratch {
+  void* base;
+  size_t bytes;
+};
+
+// Kernel launchers: each enqueues its kernels on `stream`, adds the number of
+// kernels it launched to *launches and returns the launch status.
+cudaError_t launch_sign_compress(const CompressArgs& a, bool keep_h, cudaStream_t stream,
+                                 uint64_t* launches);
+cudaError_t launch_squant_compress(const CompressArgs& a, bool keep_h, cudaStream_t stream,
+                                   uint64_t* launches);
+cudaError_t launch_identity_compress(const CompressArgs& a, bool keep_h, cudaStream_t stream,
+                                     uint64_t* launches);
+
+size_t topk_scratch_bytes(int64_t d, int32_t nworkers);
+cudaError_t launch_topk_compress(const CompressArgs& a, int64_t k, bool keep_h, void* scratch,
+                                 cudaStream_t stream, uint64_t* launches);
+
+cudaError_t launch_sign_server(const ServerArgs& s, cudaStream_t stream, uint64_t* launches);
+cudaError_t launch_squant_server(const ServerArgs& s, cudaStream_t stream, uint64_t* launches);
+cudaError_t launch_identity_server(const ServerArgs& s, cudaStream_t stream, uint64_t* launches);
+cudaError_t launch_topk_server(const ServerArgs& s, cudaStream_t stream, uint64_t* launches);
+
+cudaError_t launch_lookahead(const float* w, const float* h, float* out, int64_t d,
+                             cudaStream_t stream, uint64_t* launches);
+
+}  // namespace dq

@@ -1,0 +1,90 @@
+"""Helpers shared by the GPU parity tests: run the CUDA path through the C-ABI
+and the oracle side by side on identical seeded inputs, and compare.
+
+Comparison rules (the tolerances are written here, once):
+
+* packed messages (sign words, quantisation codes, top-k records, scales)
+  and the residuals e and lookahead offsets h are compared bit for bit:
+  both sides form p, the scales and Q(p) with the same rounded fp32
+  operations in the same order;
+* parameters w are compared with the normwise relative error
+  max_j |x_j - y_j| / max_j |y_j| <= 1e-5 per step and <= 1e-4 after a whole
+  run: the server may sum the M decoded messages in any order.
+"""
+from __future__ import annotations
+
+import numpy as np
+
+import oracle
+
+STEP_RTOL = 1e-5
+RUN_RTOL = 1e-4
+
+
+def rel_err(x: np.ndarray, y: np.ndarray) -> float:
+    x = np.asarray(x, np.float64)
+    y = np.asarray(y, np.float64)
+    scale = np.max(np.abs(y)) if y.size else 0.0
+    diff = np.max(np.abs(x - y)) if y.size else 0.0
+    if scale == 0.0:
+        return float(diff)
+    return float(diff / scale)
+
+
+def sections(ocfg: oracle.Config, msg: np.ndarray) -> dict:
+    """The meaningful bytes of a message, by name, as uint32 arrays."""
+    off_s, off_p, total = oracle.layout(ocfg)
+    d = ocfg.d
+    msg = np.asarray(msg, np.uint8)
+    if ocfg.compressor in (oracle.SIGN, oracle.SQUANT):
+        nb = -(-d // ocfg.bucket)
+        nwords = -(-d // 32) if ocfg.compressor == oracle.SIGN else -(-d * ocfg.bits // 32)
+        return {"scales": msg[off_s:off_s + 4 * nb].view(np.uint32),
+                "payload": msg[off_p:off_p + 4 * nwords].view(np.uint32)}
+    if ocfg.compressor == oracle.TOPK:
+        return {"records": msg[:8 * ocfg.k].view(np.uint32)}
+    return {"values": msg[:4 * d].view(np.uint32)}
+
+
+def assert_messages_equal(ocfg: oracle.Config, got: np.ndarray, want: np.ndarray, ctx: str = ""):
+    a, b = sections(ocfg, got), sections(ocfg, want)
+    for name in b:
+        if not np.array_equal(a[name], b[name]):
+            bad = np.flatnonzero(a[name] != b[name])
+            raise AssertionError(f"{ctx}: message section {name} differs at {bad.size} words, "
+                                 f"first {bad[:5].tolist()}: gpu {a[name][bad[:5]].tolist()} "
+                                 f"oracle {b[name][bad[:5]].tolist()}")
+
+
+def assert_bits_equal(got: np.ndarray, want: np.ndarray, ctx: str = ""):
+    g = np.ascontiguousarray(got, np.float32).view(np.uint32)
+    w = np.ascontiguousarray(want, np.float32).view(np.uint32)
+    if not np.array_equal(g, w):
+        bad = np.flatnonzero(g != w)
+        raise AssertionError(f"{ctx}: {bad.size} elements differ, first {bad[:5].tolist()}: "
+                             f"gpu {got[bad[:5]].tolist()} oracle {want[bad[:5]].tolist()}")
+
+
+def oracle_config(d, M, compressor, lr=1e-3, bucket=512, k=1, bits=8, seed=0, keep=False):
+    return oracle.Config(d=d, M=M, compressor=compressor, lr=lr, bucket=bucket, k=k, bits=bits,
+                         seed=seed, keep_lookahead=keep)
+
+
+def slice_messages(ocfg: oracle.Config, msgs: np.ndarray, a: int, b: int):
+    """Sub-messages covering elements [a, b) (bucket- and word-aligned a) and
+    the matching oracle config, so the oracle server can be run on a slice of
+    a full-size problem.  Pure byte slicing: no arithmetic of the method."""
+    assert ocfg.compressor in (oracle.SIGN, oracle.SQUANT)
+    assert a % ocfg.bucket == 0 and (b % ocfg.bucket == 0 or b == ocfg.d)
+    sub = oracle.Config(d=b - a, M=ocfg.M, compressor=ocfg.compressor, lr=ocfg.lr, bucket=ocfg.bucket,
+                        k=ocfg.k, bits=ocfg.bits, seed=ocfg.seed)
+    off_s, off_p, _ = oracle.layout(ocfg)
+    s_off_s, s_off_p, s_total = oracle.layout(sub)
+    bits = 1 if ocfg.compressor == oracle.SIGN else ocfg.bits
+    out = np.zeros((ocfg.M, s_total), np.uint8)
+    b0, b1 = a // ocfg.bucket, -(-b // ocfg.bucket)
+    w0, w1 = a * bits // 32, -(-(b * bits) // 32)
+    for m in range(ocfg.M):
+        out[m, s_off_s:s_off_s + 4 * (b1 - b0)] = msgs[m, off_s + 4 * b0:off_s + 4 * b1]
+        out[m, s_off_p:s_off_p + 4 * (w1 - w0)] = msgs[m, off_p + 4 * w0:off_p + 4 * w1]
+    return sub, out
