@@ -56,7 +56,26 @@ def parse_args():
     ap.add_argument("--lookahead", action="store_true", help="also keep the lookahead offsets h")
     ap.add_argument("--no-e2e", action="store_true", help="skip the end-to-end (host buffers) phase")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--override", action="append", default=[], metavar="FIELD=VALUE",
+                    help="change a workload field (e.g. M=4 for a smaller profiling case)")
     return ap.parse_args()
+
+
+def selected_workload(args):
+    """The named workload, with integer fields changed by --override (for the
+    smaller profiling cases); a changed d keeps the gradient distribution."""
+    wl = WORKLOADS[args.workload]
+    if not args.override:
+        return wl
+    kw = {}
+    for item in args.override:
+        key, val = item.split("=", 1)
+        if key not in ("d", "M", "k", "bits", "bucket"):
+            raise SystemExit(f"--override supports d, M, k, bits, bucket, not {key}")
+        kw[key] = int(float(val))
+    if "d" in kw and wl.segment_sizes is not None:
+        kw.update(n_segments=1, segment_sizes=(kw["d"],), segment_std=wl.segment_std[:1])
+    return wl.replace(name=wl.name + "[" + ",".join(args.override) + "]", **kw)
 
 
 # ---------------------------------------------------------------------------
@@ -237,7 +256,7 @@ def oracle_step_time(wl, worker_fraction: float = 1.0, server_fraction: float = 
 def run_reference(args, rank, world):
     if rank != 0:
         return 0
-    wl = WORKLOADS[args.workload]
+    wl = selected_workload(args)
     step_times = []
     sample = ""
     for i in range(args.warmup + args.steps):
@@ -282,7 +301,7 @@ def run_gpu(args, rank, world, local):
 
     import paper_2010_13359_gb300 as P
 
-    wl = WORKLOADS[args.workload]
+    wl = selected_workload(args)
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
     if world > 1:

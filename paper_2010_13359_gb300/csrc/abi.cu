@@ -22,6 +22,7 @@ struct dqgan_handle {
   float* h = nullptr;
   void* scratch = nullptr;
   size_t scratch_bytes = 0;
+  uint32_t* err_word = nullptr;  // device error word written by bounded waits
   int64_t t = 1;
   uint64_t launches = 0;
   std::string err;
@@ -113,6 +114,7 @@ dq::CompressArgs compress_args(dqgan_handle* h, const float* g, int64_t g_stride
   a.seed_lo = (uint32_t)(h->cfg.seed & 0xFFFFFFFFu);
   a.seed_hi = (uint32_t)(h->cfg.seed >> 32);
   a.step = (uint32_t)h->t;
+  a.err = h->err_word;
   return a;
 }
 
@@ -240,10 +242,13 @@ int dqgan_create(const dqgan_config* cfg, dqgan_handle** out) {
     if (h->e) cudaFree(h->e);
     if (h->h) cudaFree(h->h);
     if (h->scratch) cudaFree(h->scratch);
+    if (h->err_word) cudaFree(h->err_word);
     delete h;
     return set_error(nullptr, e == cudaErrorMemoryAllocation ? DQGAN_ERR_OOM : DQGAN_ERR_CUDA,
                      "%s: %s", what, cudaGetErrorString(e));
   };
+  if ((st = cudaMalloc(&h->err_word, 256)) != cudaSuccess) return fail_oom("allocating the error word", st);
+  if ((st = cudaMemsetAsync(h->err_word, 0, 256, h->stream)) != cudaSuccess) return fail_oom("zeroing the error word", st);
   if ((st = cudaMalloc(&h->e, rows_bytes)) != cudaSuccess) return fail_oom("allocating e", st);
   if (cfg->flags & DQGAN_KEEP_LOOKAHEAD)
     if ((st = cudaMalloc(&h->h, rows_bytes)) != cudaSuccess) return fail_oom("allocating h", st);
@@ -269,6 +274,7 @@ int dqgan_destroy(dqgan_handle* h) {
   if (h->e) cudaFree(h->e);
   if (h->h) cudaFree(h->h);
   if (h->scratch) cudaFree(h->scratch);
+  if (h->err_word) cudaFree(h->err_word);
   const cudaError_t st = cudaGetLastError();
   delete h;
   if (st != cudaSuccess) return set_error(nullptr, DQGAN_ERR_CUDA, "destroy: %s", cudaGetErrorString(st));
@@ -345,6 +351,13 @@ int dqgan_synchronize(dqgan_handle* h) {
   cudaError_t st = cudaStreamSynchronize(h->stream);
   if (st == cudaSuccess) st = cudaGetLastError();
   if (st != cudaSuccess) return cuda_fail(h, st, "synchronize");
+  uint32_t word = 0;
+  st = cudaMemcpy(&word, h->err_word, sizeof word, cudaMemcpyDeviceToHost);
+  if (st != cudaSuccess) return cuda_fail(h, st, "reading the error word");
+  if (word != 0) {
+    cudaMemset(h->err_word, 0, sizeof word);
+    return set_error(h, DQGAN_ERR_TIMEOUT, "a bounded device-side wait gave up (error word 0x%x)", word);
+  }
   return DQGAN_OK;
 }
 

@@ -5,68 +5,31 @@
 //   h = fl(fl(eta * g) + e)             lookahead offset (optional)
 // in one pass over g and e.
 //
-// Mapping: one warp per bucket.  Lane l owns the 4-element chunks
-// c = l, l + 32, l + 64, ... of its bucket, loaded with 128-bit coalesced
-// loads (a warp reads 512 contiguous bytes per load instruction) and held in
-// registers until the bucket's scale is known.  The bucket's l1 sum is taken
-// in the library's fixed order: each lane adds its chunk sums
-// ((|a0|+|a1|)+|a2|)+|a3| in increasing c, then five xor-shuffle rounds with
+// Mapping: a bucket is cut into 4-element chunks; a warp reads rows of 32
+// consecutive chunks (512 contiguous bytes) with 128-bit loads and keeps them
+// in registers until the bucket's scale is known, so g and e are read once
+// and e is written once.  The bucket's l1 sum is taken in the library's fixed
+// order: lane l adds the chunk sums ((|a0|+|a1|)+|a2|)+|a3| of chunks
+// l, l+32, l+64, ... in increasing order, then five xor-shuffle rounds with
 // partners 16, 8, 4, 2, 1 combine the 32 lane totals.  The max-abs scale of
 // the stochastic quantiser is exact in any order.
-#include "internal.cuh"
+#include "device_common.cuh"
 
 namespace dq {
 namespace {
 
-__host__ __device__ __forceinline__ int64_t min64(int64_t x, int64_t y) { return x < y ? x : y; }
-__host__ __device__ __forceinline__ int64_t max64(int64_t x, int64_t y) { return x > y ? x : y; }
-
-__device__ __forceinline__ float4 ld_stream4(const float* p) {
-  return __ldcs(reinterpret_cast<const float4*>(p));
-}
-__device__ __forceinline__ void st_stream4(float* p, float4 v) {
-  __stcs(reinterpret_cast<float4*>(p), v);
-}
-
-// Spread the low 8 bits of x so that bit r lands on bit 4r.
-__device__ __forceinline__ uint32_t spread_nibbles(uint32_t x) {
-  x &= 0xFFu;
-  x = (x | (x << 12)) & 0x000F000Fu;
-  x = (x | (x << 6)) & 0x03030303u;
-  x = (x | (x << 3)) & 0x11111111u;
-  return x;
-}
-
-// Philox4x32-10 (Salmon et al., SC'11): 10 rounds, multipliers 0xD2511F53 and
-// 0xCD9E8D57, Weyl key increments 0x9E3779B9 and 0xBB67AE85 between rounds.
-__device__ __forceinline__ uint4 philox4x32_10(uint4 x, uint32_t k0, uint32_t k1) {
-#pragma unroll
-  for (int round = 0; round < 10; ++round) {
-    if (round > 0) {
-      k0 += 0x9E3779B9u;
-      k1 += 0xBB67AE85u;
-    }
-    const uint32_t lo_a = 0xD2511F53u * x.x;
-    const uint32_t hi_a = __umulhi(0xD2511F53u, x.x);
-    const uint32_t lo_b = 0xCD9E8D57u * x.z;
-    const uint32_t hi_b = __umulhi(0xCD9E8D57u, x.z);
-    x = make_uint4(hi_b ^ x.y ^ k0, lo_b, hi_a ^ x.w ^ k1, lo_a);
-  }
-  return x;
-}
-
-// Loads the CPL chunks of this lane's share of bucket `b` and forms p.
-// Out-of-bucket or out-of-range elements read as 0 and give p = 0.
-// sg (if HOLD) receives fl(eta * g) for the lookahead offset.
+// Loads this thread's CPL chunks c = c0 + 32 i of the bucket starting at
+// element `base` and forms p.  Out-of-bucket or out-of-range elements read as
+// 0 and give p = 0.  sg (if HOLD) receives fl(eta * g) for the lookahead.
 template <int CPL, bool HOLD>
 __device__ __forceinline__ void load_and_form(const CompressArgs& a, const float* g, const float* e,
-                                              int64_t base, int lane, bool full,
+                                              int64_t base, int c0, bool full,
                                               float (&p)[CPL][4], float (&sg)[HOLD ? CPL : 1][4]) {
   const int nchunk = a.bucket >> 2;
   if (full) {
 #pragma unroll
     for (int i = 0; i < CPL; ++i) {
-      const int c = lane + 32 * i;
+      const int c = c0 + 32 * i;
       float4 gv = make_float4(0.f, 0.f, 0.f, 0.f), ev = gv;
       if (c < nchunk) {
         gv = ld_stream4(g + base + 4 * c);
@@ -84,7 +47,7 @@ __device__ __forceinline__ void load_and_form(const CompressArgs& a, const float
   } else {
 #pragma unroll
     for (int i = 0; i < CPL; ++i) {
-      const int c = lane + 32 * i;
+      const int c = c0 + 32 * i;
 #pragma unroll
       for (int q = 0; q < 4; ++q) {
         const int64_t j = base + 4 * c + q;
@@ -140,14 +103,31 @@ __device__ __forceinline__ void store_chunk(const CompressArgs& a, const float* 
 // ---------------------------------------------------------------------------
 // Scaled sign, s_b = ||p_b||_1 / n_b (Section 2.4; error-feedback sign
 // compressor of Section 3.1).  Bit = (p < 0); Q(p) = bit ? -s_b : s_b.
+//
+// WPB warps share a bucket (4 for 4096, 2 for 2048, 1 up to 1024); each
+// thread holds CPT chunks in registers.  Warp w of a bucket owns the chunk
+// rows w*CPT .. w*CPT+CPT-1 (row r = chunks 32r .. 32r+31, contiguous in
+// memory), so lane l holds the chunk sums of positions r of the l1 chain
+// "lane l adds chunks l, l+32, l+64, ... in order".  With one warp the chain
+// runs in registers; with several, the chunk sums go through shared memory
+// and warp 0 runs the chains, so the sum is the same whatever WPB is.
 // ---------------------------------------------------------------------------
-template <int CPL, bool KEEP_H>
-__global__ void __launch_bounds__(128)
+
+template <int CPT, int WPB, bool KEEP_H>
+__global__ void __launch_bounds__(32 * WPB * (WPB < 4 ? 4 / WPB : 1))
 sign_compress_kernel(const CompressArgs a) {
-  constexpr bool HOLD = KEEP_H && CPL <= 8;
+  constexpr bool HOLD = KEEP_H && CPT <= 8;
+  constexpr int BPC = WPB < 4 ? 4 / WPB : 1;  // buckets per CTA (CTA = max(4, WPB) warps)
+  constexpr int CHAIN = 32 * CPT * WPB;
+  __shared__ float chain[WPB > 1 ? BPC * CHAIN : 1];
+  __shared__ float scale_sh[BPC];
   const int lane = threadIdx.x & 31;
-  const int64_t b = (int64_t)blockIdx.x * 4 + (threadIdx.x >> 5);
-  if (b >= a.nb) return;  // whole warp leaves together
+  const int warp = threadIdx.x >> 5;
+  const int slot = warp / WPB;  // bucket within the CTA
+  const int wib = warp % WPB;   // warp within the bucket
+  const int64_t b = (int64_t)blockIdx.x * BPC + slot;
+  const bool valid = b < a.nb;
+  if (WPB == 1 && !valid) return;  // no barriers below for a single warp per bucket
   const int row = blockIdx.y;
   const int worker = a.worker0 + row;
   const float* g = a.g + (int64_t)row * a.g_stride;
@@ -156,49 +136,65 @@ sign_compress_kernel(const CompressArgs a) {
   uint8_t* msg = a.msg + (int64_t)row * a.msg_stride;
 
   const int64_t base = b * a.bucket;
-  const int64_t count = min64((int64_t)a.bucket, a.d - base);
+  const int64_t count = valid ? min64((int64_t)a.bucket, a.d - base) : 0;
   const bool full = (count == a.bucket);
   const int nchunk = a.bucket >> 2;
+  const int row0 = wib * CPT;  // first chunk row of this warp
 
-  float p[CPL][4];
-  float sg[HOLD ? CPL : 1][4];
-  load_and_form<CPL, HOLD>(a, g, e, base, lane, full, p, sg);
-
-  // l1 of the bucket in the fixed order
-  float acc = 0.f;
+  float p[CPT][4];
+  float sg[HOLD ? CPT : 1][4];
+  if (valid) {
+    load_and_form<CPT, HOLD>(a, g, e, base, 32 * row0 + lane, full, p, sg);
+  } else {
 #pragma unroll
-  for (int i = 0; i < CPL; ++i) {
-    const float cs = __fadd_rn(__fadd_rn(__fadd_rn(fabsf(p[i][0]), fabsf(p[i][1])), fabsf(p[i][2])),
-                               fabsf(p[i][3]));
-    acc = __fadd_rn(acc, cs);
+    for (int i = 0; i < CPT; ++i)
+#pragma unroll
+      for (int q = 0; q < 4; ++q) p[i][q] = 0.f;
   }
+
+  float s;
+  if constexpr (WPB == 1) {
+    float acc = 0.f;
 #pragma unroll
-  for (int off = 16; off >= 1; off >>= 1) acc = __fadd_rn(acc, __shfl_xor_sync(kFullMask, acc, off));
-  const float s = __fdiv_rn(acc, (float)count);
-  if (lane == 0) reinterpret_cast<float*>(msg)[b] = s;
+    for (int i = 0; i < CPT; ++i)
+      acc = __fadd_rn(acc, __fadd_rn(__fadd_rn(__fadd_rn(fabsf(p[i][0]), fabsf(p[i][1])), fabsf(p[i][2])),
+                                     fabsf(p[i][3])));
+#pragma unroll
+    for (int off = 16; off >= 1; off >>= 1) acc = __fadd_rn(acc, __shfl_xor_sync(kFullMask, acc, off));
+    s = __fdiv_rn(acc, (float)count);
+  } else {
+    float* ch = chain + slot * CHAIN;
+#pragma unroll
+    for (int i = 0; i < CPT; ++i)
+      ch[(row0 + i) * 32 + lane] =
+          __fadd_rn(__fadd_rn(__fadd_rn(fabsf(p[i][0]), fabsf(p[i][1])), fabsf(p[i][2])), fabsf(p[i][3]));
+    __syncthreads();
+    if (wib == 0) {
+      float acc = 0.f;
+#pragma unroll 8
+      for (int r = 0; r < CPT * WPB; ++r) acc = __fadd_rn(acc, ch[r * 32 + lane]);
+#pragma unroll
+      for (int off = 16; off >= 1; off >>= 1) acc = __fadd_rn(acc, __shfl_xor_sync(kFullMask, acc, off));
+      if (lane == 0) scale_sh[slot] = valid ? __fdiv_rn(acc, (float)count) : 0.f;
+    }
+    __syncthreads();
+    s = scale_sh[slot];
+    if (!valid) return;
+  }
+  if (wib == 0 && lane == 0) reinterpret_cast<float*>(msg)[b] = s;
 
   uint32_t* words = reinterpret_cast<uint32_t*>(msg + a.off_payload);
   const int64_t word0 = base >> 5;
   const int64_t nwords = (a.d + 31) >> 5;
   const int words_in_bucket = a.bucket >> 5;
 #pragma unroll
-  for (int i = 0; i < CPL; ++i) {
-    const uint32_t B0 = __ballot_sync(kFullMask, p[i][0] < 0.f);
-    const uint32_t B1 = __ballot_sync(kFullMask, p[i][1] < 0.f);
-    const uint32_t B2 = __ballot_sync(kFullMask, p[i][2] < 0.f);
-    const uint32_t B3 = __ballot_sync(kFullMask, p[i][3] < 0.f);
-    // Row i covers chunks 32i..32i+31, i.e. words 4i..4i+3 of the bucket; bit
-    // 4r+q of word 4i+u comes from element q of the chunk in lane 8u+r.
-    if (lane < 4) {
-      const int wib = 4 * i + lane;
-      if (wib < words_in_bucket && word0 + wib < nwords) {
-        const int sh = 8 * lane;
-        const uint32_t wv = spread_nibbles(B0 >> sh) | (spread_nibbles(B1 >> sh) << 1) |
-                            (spread_nibbles(B2 >> sh) << 2) | (spread_nibbles(B3 >> sh) << 3);
-        words[word0 + wib] = wv;
-      }
+  for (int i = 0; i < CPT; ++i) {
+    const uint32_t wv = pack_sign_row(p[i][0], p[i][1], p[i][2], p[i][3], lane);
+    if ((lane & 3) == 0 && lane < 16) {
+      const int wib_word = 4 * (row0 + i) + (lane >> 2);
+      if (wib_word < words_in_bucket && word0 + wib_word < nwords) words[word0 + wib_word] = wv;
     }
-    const int c = lane + 32 * i;
+    const int c = 32 * (row0 + i) + lane;
     if (c < nchunk) {
       const int64_t j = base + 4 * c;
       const int nvalid = (int)min64(4, a.d - j);
@@ -206,7 +202,7 @@ sign_compress_kernel(const CompressArgs a) {
         float en[4];
 #pragma unroll
         for (int q = 0; q < 4; ++q) en[q] = __fsub_rn(p[i][q], p[i][q] < 0.f ? -s : s);
-        store_chunk<KEEP_H, HOLD, CPL>(a, g, e, h, j, full, nvalid, en, sg, i);
+        store_chunk<KEEP_H, HOLD, CPT>(a, g, e, h, j, full, nvalid, en, sg, i);
       }
     }
   }
@@ -218,18 +214,24 @@ sign_compress_kernel(const CompressArgs a) {
 // up from r = floor(.) iff u < frac(.), u the 24-bit Philox4x32-10 draw of
 // counter (j div 4, worker, step, 0x51) word j mod 4; code = K +- level.
 // ---------------------------------------------------------------------------
-template <int CPL, int BITS, bool KEEP_H>
-__global__ void __launch_bounds__(128)
+template <int CPT, int WPB, int BITS, bool KEEP_H>
+__global__ void __launch_bounds__(32 * WPB * (WPB < 4 ? 4 / WPB : 1))
 squant_compress_kernel(const CompressArgs a) {
   constexpr int K = (1 << (BITS - 1)) - 1;
-  constexpr bool HOLD = KEEP_H && CPL <= 8;
-  __shared__ float level_value[K + 1];  // fl(r / K)
+  constexpr bool HOLD = KEEP_H && CPT <= 8;
+  constexpr int BPC = WPB < 4 ? 4 / WPB : 1;  // buckets per CTA (CTA = max(4, WPB) warps)
+  __shared__ float level_value[K + 1];        // fl(r / K)
+  __shared__ float warp_max[BPC * WPB];
   for (int r = threadIdx.x; r <= K; r += blockDim.x) level_value[r] = __fdiv_rn((float)r, (float)K);
   __syncthreads();
 
   const int lane = threadIdx.x & 31;
-  const int64_t b = (int64_t)blockIdx.x * 4 + (threadIdx.x >> 5);
-  if (b >= a.nb) return;
+  const int warp = threadIdx.x >> 5;
+  const int slot = warp / WPB;  // bucket within the CTA
+  const int wib = warp % WPB;   // warp within the bucket
+  const int64_t b = (int64_t)blockIdx.x * BPC + slot;
+  const bool valid = b < a.nb;
+  if (WPB == 1 && !valid) return;
   const int row = blockIdx.y;
   const int worker = a.worker0 + row;
   const float* g = a.g + (int64_t)row * a.g_stride;
@@ -238,30 +240,46 @@ squant_compress_kernel(const CompressArgs a) {
   uint8_t* msg = a.msg + (int64_t)row * a.msg_stride;
 
   const int64_t base = b * a.bucket;
-  const int64_t count = min64((int64_t)a.bucket, a.d - base);
+  const int64_t count = valid ? min64((int64_t)a.bucket, a.d - base) : 0;
   const bool full = (count == a.bucket);
   const int nchunk = a.bucket >> 2;
+  const int row0 = wib * CPT;  // first chunk row of this warp
 
-  float p[CPL][4];
-  float sg[HOLD ? CPL : 1][4];
-  load_and_form<CPL, HOLD>(a, g, e, base, lane, full, p, sg);
+  float p[CPT][4];
+  float sg[HOLD ? CPT : 1][4];
+  if (valid) {
+    load_and_form<CPT, HOLD>(a, g, e, base, 32 * row0 + lane, full, p, sg);
+  } else {
+#pragma unroll
+    for (int i = 0; i < CPT; ++i)
+#pragma unroll
+      for (int q = 0; q < 4; ++q) p[i][q] = 0.f;
+  }
 
+  // s = max |p| over the bucket (exact in any order)
   float mx = 0.f;
 #pragma unroll
-  for (int i = 0; i < CPL; ++i)
+  for (int i = 0; i < CPT; ++i)
 #pragma unroll
     for (int q = 0; q < 4; ++q) mx = fmaxf(mx, fabsf(p[i][q]));
 #pragma unroll
   for (int off = 16; off >= 1; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(kFullMask, mx, off));
+  if constexpr (WPB > 1) {
+    if (lane == 0) warp_max[warp] = mx;
+    __syncthreads();
+#pragma unroll
+    for (int w = 0; w < WPB; ++w) mx = fmaxf(mx, warp_max[slot * WPB + w]);
+    if (!valid) return;
+  }
   const float s = mx;
-  if (lane == 0) reinterpret_cast<float*>(msg)[b] = s;
+  if (wib == 0 && lane == 0) reinterpret_cast<float*>(msg)[b] = s;
   const float inv = (s > 0.f) ? __fdiv_rn((float)K, s) : 0.f;
 
   uint32_t* words = reinterpret_cast<uint32_t*>(msg + a.off_payload);
   const int64_t nwords = (a.d * BITS + 31) >> 5;
 #pragma unroll
-  for (int i = 0; i < CPL; ++i) {
-    const int c = lane + 32 * i;
+  for (int i = 0; i < CPT; ++i) {
+    const int c = 32 * (row0 + i) + lane;
     const int64_t j = base + 4 * c;
     const int64_t cg = j >> 2;  // global chunk index = Philox counter word 0
     const int nvalid = (c < nchunk) ? (int)max64(0, min64(4, a.d - j)) : 0;
@@ -272,24 +290,10 @@ squant_compress_kernel(const CompressArgs a) {
     float en[4];
 #pragma unroll
     for (int q = 0; q < 4; ++q) {
-      const float pv = p[i][q];
       int code = K;
       float qv = 0.f;
-      if (s > 0.f) {
-        const float t = fminf(__fmul_rn(fabsf(pv), inv), (float)K);
-        const float r = floorf(t);
-        const float f = __fsub_rn(t, r);
-        const float u = __fmul_rn(__uint2float_rn(rq[q] >> 8), 0x1p-24f);
-        int level = (int)r + (u < f ? 1 : 0);
-        level = min(level, K);
-        const bool neg = pv < 0.f;
-        code = neg ? K - level : K + level;
-        if (level != 0) {
-          const float mag = __fmul_rn(s, level_value[level]);
-          qv = neg ? -mag : mag;
-        }
-      }
-      en[q] = __fsub_rn(pv, qv);
+      if (s > 0.f) squant_element<K>(p[i][q], s, inv, rq[q], level_value, &code, &qv);
+      en[q] = __fsub_rn(p[i][q], qv);
       if (q < nvalid) chunk_bits |= (uint32_t)code << (q * BITS);
     }
     // pack: a chunk is 4*BITS bits; 32 / (4*BITS) neighbouring lanes share a word
@@ -312,7 +316,7 @@ squant_compress_kernel(const CompressArgs a) {
       writer = (lane & 3) == 0;
     }
     if (writer && c < nchunk && widx < nwords) words[widx] = wv;
-    if (nvalid > 0) store_chunk<KEEP_H, HOLD, CPL>(a, g, e, h, j, full, nvalid, en, sg, i);
+    if (nvalid > 0) store_chunk<KEEP_H, HOLD, CPT>(a, g, e, h, j, full, nvalid, en, sg, i);
   }
 }
 
@@ -361,28 +365,32 @@ identity_compress_kernel(const CompressArgs a) {
   }
 }
 
-template <int CPL>
+template <int CPT, int WPB>
 cudaError_t sign_dispatch_keep(const CompressArgs& a, bool keep_h, cudaStream_t stream) {
-  const dim3 grid((unsigned)((a.nb + 3) / 4), (unsigned)a.nworkers);
-  if (keep_h) sign_compress_kernel<CPL, true><<<grid, 128, 0, stream>>>(a);
-  else sign_compress_kernel<CPL, false><<<grid, 128, 0, stream>>>(a);
+  constexpr int BPC = WPB < 4 ? 4 / WPB : 1;
+  constexpr int THREADS = 32 * WPB * BPC;
+  const dim3 grid((unsigned)((a.nb + BPC - 1) / BPC), (unsigned)a.nworkers);
+  if (keep_h) sign_compress_kernel<CPT, WPB, true><<<grid, THREADS, 0, stream>>>(a);
+  else sign_compress_kernel<CPT, WPB, false><<<grid, THREADS, 0, stream>>>(a);
   return cudaGetLastError();
 }
 
-template <int CPL, int BITS>
+template <int CPT, int WPB, int BITS>
 cudaError_t squant_dispatch_keep(const CompressArgs& a, bool keep_h, cudaStream_t stream) {
-  const dim3 grid((unsigned)((a.nb + 3) / 4), (unsigned)a.nworkers);
-  if (keep_h) squant_compress_kernel<CPL, BITS, true><<<grid, 128, 0, stream>>>(a);
-  else squant_compress_kernel<CPL, BITS, false><<<grid, 128, 0, stream>>>(a);
+  constexpr int BPC = WPB < 4 ? 4 / WPB : 1;
+  constexpr int THREADS = 32 * WPB * BPC;
+  const dim3 grid((unsigned)((a.nb + BPC - 1) / BPC), (unsigned)a.nworkers);
+  if (keep_h) squant_compress_kernel<CPT, WPB, BITS, true><<<grid, THREADS, 0, stream>>>(a);
+  else squant_compress_kernel<CPT, WPB, BITS, false><<<grid, THREADS, 0, stream>>>(a);
   return cudaGetLastError();
 }
 
-template <int CPL>
+template <int CPT, int WPB>
 cudaError_t squant_dispatch_bits(const CompressArgs& a, bool keep_h, cudaStream_t stream) {
   switch (a.bits) {
-    case 2: return squant_dispatch_keep<CPL, 2>(a, keep_h, stream);
-    case 4: return squant_dispatch_keep<CPL, 4>(a, keep_h, stream);
-    case 8: return squant_dispatch_keep<CPL, 8>(a, keep_h, stream);
+    case 2: return squant_dispatch_keep<CPT, WPB, 2>(a, keep_h, stream);
+    case 4: return squant_dispatch_keep<CPT, WPB, 4>(a, keep_h, stream);
+    case 8: return squant_dispatch_keep<CPT, WPB, 8>(a, keep_h, stream);
   }
   return cudaErrorInvalidValue;
 }
@@ -393,12 +401,12 @@ cudaError_t launch_sign_compress(const CompressArgs& a, bool keep_h, cudaStream_
                                  uint64_t* launches) {
   cudaError_t st;
   switch (a.bucket) {
-    case 32: case 64: case 128: st = sign_dispatch_keep<1>(a, keep_h, stream); break;
-    case 256: st = sign_dispatch_keep<2>(a, keep_h, stream); break;
-    case 512: st = sign_dispatch_keep<4>(a, keep_h, stream); break;
-    case 1024: st = sign_dispatch_keep<8>(a, keep_h, stream); break;
-    case 2048: st = sign_dispatch_keep<16>(a, keep_h, stream); break;
-    case 4096: st = sign_dispatch_keep<32>(a, keep_h, stream); break;
+    case 32: case 64: case 128: st = sign_dispatch_keep<1, 1>(a, keep_h, stream); break;
+    case 256: st = sign_dispatch_keep<2, 1>(a, keep_h, stream); break;
+    case 512: st = sign_dispatch_keep<4, 1>(a, keep_h, stream); break;
+    case 1024: st = sign_dispatch_keep<2, 4>(a, keep_h, stream); break;
+    case 2048: st = sign_dispatch_keep<2, 8>(a, keep_h, stream); break;
+    case 4096: st = sign_dispatch_keep<2, 16>(a, keep_h, stream); break;
     default: return cudaErrorInvalidValue;
   }
   *launches += 1;
@@ -409,12 +417,12 @@ cudaError_t launch_squant_compress(const CompressArgs& a, bool keep_h, cudaStrea
                                    uint64_t* launches) {
   cudaError_t st;
   switch (a.bucket) {
-    case 32: case 64: case 128: st = squant_dispatch_bits<1>(a, keep_h, stream); break;
-    case 256: st = squant_dispatch_bits<2>(a, keep_h, stream); break;
-    case 512: st = squant_dispatch_bits<4>(a, keep_h, stream); break;
-    case 1024: st = squant_dispatch_bits<8>(a, keep_h, stream); break;
-    case 2048: st = squant_dispatch_bits<16>(a, keep_h, stream); break;
-    case 4096: st = squant_dispatch_bits<32>(a, keep_h, stream); break;
+    case 32: case 64: case 128: st = squant_dispatch_bits<1, 1>(a, keep_h, stream); break;
+    case 256: st = squant_dispatch_bits<2, 1>(a, keep_h, stream); break;
+    case 512: st = squant_dispatch_bits<4, 1>(a, keep_h, stream); break;
+    case 1024: st = squant_dispatch_bits<8, 1>(a, keep_h, stream); break;
+    case 2048: st = squant_dispatch_bits<2, 8>(a, keep_h, stream); break;
+    case 4096: st = squant_dispatch_bits<2, 16>(a, keep_h, stream); break;
     default: return cudaErrorInvalidValue;
   }
   *launches += 1;

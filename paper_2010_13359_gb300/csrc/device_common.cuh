@@ -1,0 +1,157 @@
+// Device helpers shared by the compress kernels: fp32 element rules of the
+// method, Philox4x32-10, sign bit packing, and the TMA / mbarrier primitives
+// of the staged (shared-memory pipelined) kernels.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "internal.cuh"
+
+namespace dq {
+
+__host__ __device__ __forceinline__ int64_t min64(int64_t x, int64_t y) { return x < y ? x : y; }
+__host__ __device__ __forceinline__ int64_t max64(int64_t x, int64_t y) { return x > y ? x : y; }
+
+__device__ __forceinline__ float4 ld_stream4(const float* p) {
+  return __ldcs(reinterpret_cast<const float4*>(p));
+}
+__device__ __forceinline__ void st_stream4(float* p, float4 v) {
+  __stcs(reinterpret_cast<float4*>(p), v);
+}
+
+// p = fl(fl(eta * g) + e): error feedback of Algorithm 2, two roundings.
+__device__ __forceinline__ float ef_p(float lr, float g, float e) { return __fadd_rn(__fmul_rn(lr, g), e); }
+
+// ((|a0| + |a1|) + |a2|) + |a3|: one chunk's share of the bucket l1 sum.
+__device__ __forceinline__ float chunk_abs_sum(float a0, float a1, float a2, float a3) {
+  return __fadd_rn(__fadd_rn(__fadd_rn(fabsf(a0), fabsf(a1)), fabsf(a2)), fabsf(a3));
+}
+
+// Spread the low 8 bits of x so that bit r lands on bit 4r.
+__device__ __forceinline__ uint32_t spread_nibbles(uint32_t x) {
+  x &= 0xFFu;
+  x = (x | (x << 12)) & 0x000F000Fu;
+  x = (x | (x << 6)) & 0x03030303u;
+  x = (x | (x << 3)) & 0x11111111u;
+  return x;
+}
+
+// Packs the signs of one row of 32 chunks (128 elements, 4 words) with four
+// ballots.  Bit 4r+k of word u of the row is element k of the chunk in lane
+// 8u+r: lane 4u+k spreads byte u of ballot k onto bits 4r+k and lanes
+// 4u..4u+3 OR their parts together.  Returns the word in lanes 0, 4, 8, 12.
+__device__ __forceinline__ uint32_t pack_sign_row(float p0, float p1, float p2, float p3, int lane) {
+  const uint32_t B0 = __ballot_sync(kFullMask, p0 < 0.f);
+  const uint32_t B1 = __ballot_sync(kFullMask, p1 < 0.f);
+  const uint32_t B2 = __ballot_sync(kFullMask, p2 < 0.f);
+  const uint32_t B3 = __ballot_sync(kFullMask, p3 < 0.f);
+  const int k = lane & 3, u = (lane >> 2) & 3;
+  const uint32_t Bk = (k == 0) ? B0 : (k == 1) ? B1 : (k == 2) ? B2 : B3;
+  uint32_t v = spread_nibbles(Bk >> (8 * u)) << k;
+  v |= __shfl_xor_sync(kFullMask, v, 1);
+  v |= __shfl_xor_sync(kFullMask, v, 2);
+  return v;
+}
+
+// Philox4x32-10 (Salmon et al., SC'11): 10 rounds, multipliers 0xD2511F53 and
+// 0xCD9E8D57, Weyl key increments 0x9E3779B9 and 0xBB67AE85 between rounds.
+__device__ __forceinline__ uint4 philox4x32_10(uint4 x, uint32_t k0, uint32_t k1) {
+#pragma unroll
+  for (int round = 0; round < 10; ++round) {
+    if (round > 0) {
+      k0 += 0x9E3779B9u;
+      k1 += 0xBB67AE85u;
+    }
+    const uint32_t lo_a = 0xD2511F53u * x.x;
+    const uint32_t hi_a = __umulhi(0xD2511F53u, x.x);
+    const uint32_t lo_b = 0xCD9E8D57u * x.z;
+    const uint32_t hi_b = __umulhi(0xCD9E8D57u, x.z);
+    x = make_uint4(hi_b ^ x.y ^ k0, lo_b, hi_a ^ x.w ^ k1, lo_a);
+  }
+  return x;
+}
+
+// One element of the b-bit stochastic quantiser (s > 0): code and Q(p).
+// t = min(fl(|p| * inv), K); r = floor(t); rounds up iff u < t - r, u the top
+// 24 bits of the Philox word; code = K -+ level; Q = sign * fl(s * fl(level/K)).
+template <int K>
+__device__ __forceinline__ void squant_element(float p, float s, float inv, uint32_t rnd,
+                                               const float* level_value, int* code, float* q) {
+  const float t = fminf(__fmul_rn(fabsf(p), inv), (float)K);
+  const float r = floorf(t);
+  const float f = __fsub_rn(t, r);
+  const float u = __fmul_rn(__uint2float_rn(rnd >> 8), 0x1p-24f);
+  int level = (int)r + (u < f ? 1 : 0);
+  level = level < K ? level : K;
+  const bool neg = p < 0.f;
+  *code = neg ? K - level : K + level;
+  float qv = 0.f;
+  if (level != 0) {
+    const float mag = __fmul_rn(s, level_value[level]);
+    qv = neg ? -mag : mag;
+  }
+  *q = qv;
+}
+
+// ---------------------------------------------------------------------------
+// mbarrier + 1-D TMA bulk copy (cp.async.bulk) primitives.  Every wait is
+// bounded: after kSpinLimit polls (each may sleep up to kSuspendNs) it sets
+// kErrTimeout in the launch's error word and returns false.
+// ---------------------------------------------------------------------------
+constexpr uint32_t kErrTimeout = 1u;
+constexpr uint32_t kSpinLimit = 1u << 21;
+constexpr uint32_t kSuspendNs = 500u;
+
+__device__ __forceinline__ uint32_t smem_addr(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(smem_addr(bar)), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void mbar_fence_init() {
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(smem_addr(bar)) : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_addr(bar)), "r"(bytes)
+               : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(smem_addr(bar)), "r"(parity), "r"(kSuspendNs)
+      : "memory");
+  return ok != 0;
+}
+
+__device__ __forceinline__ bool mbar_wait_bounded(uint64_t* bar, uint32_t parity, uint32_t* err) {
+  for (uint32_t it = 0; it < kSpinLimit; ++it)
+    if (mbar_try_wait(bar, parity)) return true;
+  atomicOr(err, kErrTimeout);
+  return false;
+}
+
+// Global -> shared bulk copy of `bytes` (multiple of 16, both addresses
+// 16-byte aligned); completion counted on `bar`.
+__device__ __forceinline__ void tma_load_1d(void* dst_smem, const void* src_gmem, uint32_t bytes,
+                                            uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+          smem_addr(dst_smem)),
+      "l"(src_gmem), "r"(bytes), "r"(smem_addr(bar))
+      : "memory");
+}
+
+}  // namespace dq

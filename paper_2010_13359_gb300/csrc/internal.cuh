@@ -47,6 +47,7 @@ struct CompressArgs {
   int32_t nworkers;
   uint32_t seed_lo, seed_hi;
   uint32_t step;
+  uint32_t* err;       // device error word (bit 0: a bounded wait timed out)
 };
 
 // Arguments of the server (decode + average + update) kernels.

@@ -2,10 +2,11 @@
 //   decode the M messages, q_hat = fl(sum_m Q_m / M), w = fl(w - q_hat).
 // and the worker lookahead w_{t-1/2} = fl(w - h).
 //
-// Dense compressors: one thread per 4-element chunk of w; the thread walks
-// the M messages in worker order and keeps 4 fp32 accumulators.  Message
-// bytes per chunk are a word (or part of one) and one scale per worker, read
-// with plain coalesced loads; w is read and written once with 128-bit loads.
+// Stochastic quantiser, identity, and sign with buckets < 512: one thread per
+// 4-element chunk of w walks the M messages in worker order with 4 fp32
+// accumulators, fetching the message words of 8 (4) workers before using
+// them.  Sign with buckets >= 512: bit-transposed table decode (below).
+// w is read and written once.
 #include "internal.cuh"
 
 namespace dq {
@@ -13,6 +14,13 @@ namespace {
 
 __device__ __forceinline__ float average(float acc, const ServerArgs& s) {
   return s.M_pow2 ? __fmul_rn(acc, s.inv_M) : __fdiv_rn(acc, (float)s.M);
+}
+
+// q_hat = acc / M; with M a power of two the product by the exact 1/M.
+template <bool POW2>
+__device__ __forceinline__ float average_t(float acc, const ServerArgs& s) {
+  if constexpr (POW2) return __fmul_rn(acc, s.inv_M);
+  else return __fdiv_rn(acc, (float)s.M);
 }
 
 // Applies w_j = fl(w_j - acc_j / M) for the chunk at element j.
@@ -29,7 +37,8 @@ __device__ __forceinline__ void apply_chunk(const ServerArgs& s, int64_t j, cons
   }
 }
 
-// Scaled sign: Q_m(p)_j = bit ? -s_m : s_m.
+// Scaled sign, any bucket: Q_m(p)_j = bit ? -s_m : s_m summed in worker
+// order, message words and scales fetched 8 workers at a time.
 __global__ void __launch_bounds__(256) sign_server_kernel(const ServerArgs s) {
   const int64_t c = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   const int64_t j = 4 * c;
@@ -38,66 +47,352 @@ __global__ void __launch_bounds__(256) sign_server_kernel(const ServerArgs s) {
   const int64_t word = j >> 5;
   const int shift = (int)(j & 31);
   float acc[4] = {0.f, 0.f, 0.f, 0.f};
-  for (int m = 0; m < s.M; ++m) {
-    const uint8_t* msg = s.msgs + (int64_t)m * s.msg_stride;
-    const float sc = __ldg(reinterpret_cast<const float*>(msg) + bkt);
-    const uint32_t bits = __ldg(reinterpret_cast<const uint32_t*>(msg + s.off_payload) + word) >> shift;
+  for (int m0 = 0; m0 < s.M; m0 += 8) {
+    float sc[8];
+    uint32_t bits[8];
 #pragma unroll
-    for (int q = 0; q < 4; ++q) acc[q] = __fadd_rn(acc[q], ((bits >> q) & 1u) ? -sc : sc);
+    for (int u = 0; u < 8; ++u) {
+      sc[u] = 0.f;
+      bits[u] = 0;
+      if (m0 + u < s.M) {
+        const uint8_t* msg = s.msgs + (int64_t)(m0 + u) * s.msg_stride;
+        sc[u] = __ldg(reinterpret_cast<const float*>(msg) + bkt);
+        bits[u] = __ldg(reinterpret_cast<const uint32_t*>(msg + s.off_payload) + word) >> shift;
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < 8; ++u)
+      if (m0 + u < s.M)
+#pragma unroll
+        for (int q = 0; q < 4; ++q) acc[q] = __fadd_rn(acc[q], ((bits[u] >> q) & 1u) ? -sc[u] : sc[u]);
   }
   apply_chunk(s, j, acc);
 }
 
-// b-bit stochastic quantiser: Q_m(p)_j = sign * fl(s_m * fl(level / K)), +0 at level 0.
-template <int BITS>
+// 32x32 bit transpose across a warp: on entry lane m holds row m; on exit
+// lane l holds column l (bit m = bit l of row m).  Five block-swap stages;
+// each is a shuffle, a rotate and a bit-select.  The per-lane masks and
+// rotate amounts do not depend on the data and are computed once.
+struct TransposeLane {
+  uint32_t keep[5];
+  uint32_t rot[5];
+  __device__ __forceinline__ explicit TransposeLane(int lane) {
+    const uint32_t masks[5] = {0x0000FFFFu, 0x00FF00FFu, 0x0F0F0F0Fu, 0x33333333u, 0x55555555u};
+#pragma unroll
+    for (int st = 0; st < 5; ++st) {
+      const int jj = 16 >> st;
+      const bool lower = (lane & jj) == 0;
+      keep[st] = lower ? masks[st] : ~masks[st];
+      rot[st] = lower ? jj : 32 - jj;
+    }
+  }
+};
+
+__device__ __forceinline__ uint32_t warp_transpose32(uint32_t x, const TransposeLane& tl) {
+#pragma unroll
+  for (int st = 0; st < 5; ++st) {
+    const uint32_t y = __shfl_xor_sync(kFullMask, x, 16 >> st);
+    const uint32_t t = __funnelshift_l(y, y, tl.rot[st]);
+    x = (x & tl.keep[st]) | (t & ~tl.keep[st]);
+  }
+  return x;
+}
+
+// Scaled sign, buckets of 512..4096.  One warp per (bucket, slice of up to 32
+// message words = 1024 elements), no shared memory and no block barriers.
+// Lane m loads worker m's words of the slice (32 contiguous bytes at a time)
+// and a warp transpose gives lane l the M sign bits of one element.  The sum
+// over workers comes from per-bucket tables of partial sums over groups of
+// five workers, T_g[v] = sum_{r<5} (bit r of v ? -s_{5g+r} : s_{5g+r}) (in
+// r order), held in registers: lane l keeps T_g[l], and a lookup is one
+// shuffle whose source lane is the 5-bit field (shuffles use the lane index
+// mod 32).  Up to 32 workers the group values are added pairwise,
+// ((T_0 + T_1) + (T_2 + T_3)) + ((T_4 + T_5) + T_6); beyond 32, slab after
+// slab and group after group.  Neither is worker order.
+constexpr int kSliceWords = 32;
+
+// T_g[lane] for the 7 groups of five workers of one 32-worker slab.
+__device__ __forceinline__ void build_group_tables(float my_scale, int in_slab, int lane, float (&T)[7]) {
+#pragma unroll
+  for (int grp = 0; grp < 7; ++grp) {
+    float t = 0.f;
+#pragma unroll
+    for (int r = 0; r < 5; ++r) {
+      const int wk = 5 * grp + r;
+      if (wk < 32) {
+        const float sc = __shfl_sync(kFullMask, my_scale, wk);
+        if (wk < in_slab) t = __fadd_rn(t, ((lane >> r) & 1) ? -sc : sc);
+      }
+    }
+    T[grp] = t;
+  }
+}
+
+// This lane's 8 message words starting at word w0 (zero past the message).
+__device__ __forceinline__ void load_words8(const uint32_t* wp, int64_t w0, int64_t nwords, bool active,
+                                            uint32_t (&wd)[8]) {
+#pragma unroll
+  for (int k = 0; k < 8; ++k) wd[k] = 0;
+  if (!active) return;
+  if (w0 + 7 < nwords) {
+    const uint4 lo = __ldcs(reinterpret_cast<const uint4*>(wp));
+    const uint4 hi = __ldcs(reinterpret_cast<const uint4*>(wp) + 1);
+    wd[0] = lo.x; wd[1] = lo.y; wd[2] = lo.z; wd[3] = lo.w;
+    wd[4] = hi.x; wd[5] = hi.y; wd[6] = hi.z; wd[7] = hi.w;
+  } else {
+#pragma unroll
+    for (int k = 0; k < 8; ++k)
+      if (w0 + k < nwords) wd[k] = wp[k];
+  }
+}
+
+// Sum over the NG five-worker groups of one element's transposed sign mask x:
+// the lookups are added pairwise, ((v0 + v1) + (v2 + v3)) + ((v4 + v5) + v6).
+template <int NG>
+__device__ __forceinline__ float group_sum(uint32_t x, const float (&T)[7]) {
+  float v[NG];
+#pragma unroll
+  for (int grp = 0; grp < NG; ++grp) v[grp] = __shfl_sync(kFullMask, T[grp], (int)(x >> (5 * grp)));
+#pragma unroll
+  for (int width = 1; width < NG; width *= 2)
+#pragma unroll
+    for (int i = 0; i + width < NG; i += 2 * width) v[i] = __fadd_rn(v[i], v[i + width]);
+  return v[0];
+}
+
+// The table sums of 8 transposed words.
+template <int NG>
+__device__ __forceinline__ void sums8(const uint32_t (&wd)[8], const float (&T)[7], const TransposeLane& tl,
+                                      float (&out)[8]) {
+#pragma unroll
+  for (int k = 0; k < 8; ++k) out[k] = group_sum<NG>(warp_transpose32(wd[k], tl), T);
+}
+
+template <int NG>
+__device__ __forceinline__ void accumulate8_dyn(const uint32_t (&wd)[8], const float (&T)[7], int ngroups,
+                                                const TransposeLane& tl, float* acc) {
+#pragma unroll
+  for (int k = 0; k < 8; ++k) {
+    const uint32_t x = warp_transpose32(wd[k], tl);
+    float a = acc[k];
+#pragma unroll
+    for (int grp = 0; grp < 7; ++grp)
+      if (grp < ngroups) a = __fadd_rn(a, __shfl_sync(kFullMask, T[grp], (int)(x >> (5 * grp))));
+    acc[k] = a;
+  }
+}
+
+// M <= 32 workers in NG = ceil(M / 5) groups; w updated after every 8 words.
+// The next 8 words and parameters are fetched before the current ones are
+// decoded.
+template <int NG, bool POW2>
+__global__ void __launch_bounds__(256) sign_server_shfl_kernel(const ServerArgs s) {
+  const int lane = threadIdx.x & 31;
+  const int64_t gw = (int64_t)blockIdx.x * 8 + (threadIdx.x >> 5);
+  const int words_per_bucket = s.bucket >> 5;
+  const int sw = words_per_bucket < kSliceWords ? words_per_bucket : kSliceWords;  // 16 or 32
+  const int spb = words_per_bucket / sw;  // slices per bucket
+  const int64_t nb = (s.d + s.bucket - 1) / s.bucket;
+  const int64_t b = gw / spb;
+  if (b >= nb) return;
+  const int64_t wbase = b * words_per_bucket + (gw % spb) * sw;
+  const int64_t nwords = (s.d + 31) >> 5;
+  const TransposeLane tl(lane);
+  const uint8_t* my_msg = s.msgs + (int64_t)lane * s.msg_stride;
+  const bool active = lane < s.M;
+  const float my_scale = active ? __ldg(reinterpret_cast<const float*>(my_msg) + b) : 0.f;
+  float T[7];
+  build_group_tables(my_scale, s.M, lane, T);
+  const uint32_t* wp = reinterpret_cast<const uint32_t*>(my_msg + s.off_payload) + wbase;
+  float* wl = s.w + 32 * wbase + lane;
+  const int64_t jmax = s.d - 32 * wbase - lane;  // wl[32 i] is a parameter iff 32 i < jmax
+  const int iters = sw / 8;
+  uint32_t wd[8];
+  float wv[8];
+  load_words8(wp, wbase, nwords, active, wd);
+#pragma unroll
+  for (int k = 0; k < 8; ++k) wv[k] = (32 * k < jmax) ? __ldcs(wl + 32 * k) : 0.f;
+#pragma unroll 1
+  for (int it = 0; it < iters; ++it) {
+    uint32_t wd_next[8];
+    float wv_next[8];
+    const bool more = it + 1 < iters;
+    if (more) {
+      load_words8(wp + 8 * (it + 1), wbase + 8 * (it + 1), nwords, active, wd_next);
+#pragma unroll
+      for (int k = 0; k < 8; ++k) {
+        const int64_t off = 32 * (8 * (it + 1) + k);
+        wv_next[k] = (off < jmax) ? __ldcs(wl + off) : 0.f;
+      }
+    }
+    float sum[8];
+    sums8<NG>(wd, T, tl, sum);
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+      const int64_t off = 32 * (8 * it + k);
+      if (off < jmax) __stcs(wl + off, __fsub_rn(wv[k], average_t<POW2>(sum[k], s)));
+    }
+    if (more) {
+#pragma unroll
+      for (int k = 0; k < 8; ++k) {
+        wd[k] = wd_next[k];
+        wv[k] = wv_next[k];
+      }
+    }
+  }
+}
+
+// Any M: workers taken 32 at a time, groups added in order, w updated at the end.
+__global__ void __launch_bounds__(256) sign_server_slabs_kernel(const ServerArgs s) {
+  const int lane = threadIdx.x & 31;
+  const int64_t gw = (int64_t)blockIdx.x * 8 + (threadIdx.x >> 5);
+  const int words_per_bucket = s.bucket >> 5;
+  const int sw = words_per_bucket < kSliceWords ? words_per_bucket : kSliceWords;
+  const int spb = words_per_bucket / sw;
+  const int64_t nb = (s.d + s.bucket - 1) / s.bucket;
+  const int64_t b = gw / spb;
+  if (b >= nb) return;
+  const int64_t wbase = b * words_per_bucket + (gw % spb) * sw;
+  const int64_t nwords = (s.d + 31) >> 5;
+  const TransposeLane tl(lane);
+  float acc[kSliceWords];
+#pragma unroll
+  for (int i = 0; i < kSliceWords; ++i) acc[i] = 0.f;
+  for (int slab = 0; slab * 32 < s.M; ++slab) {
+    const int in_slab = min(32, s.M - slab * 32);
+    const uint8_t* my_msg = s.msgs + (int64_t)(slab * 32 + lane) * s.msg_stride;
+    const float my_scale = (lane < in_slab) ? __ldg(reinterpret_cast<const float*>(my_msg) + b) : 0.f;
+    float T[7];
+    build_group_tables(my_scale, in_slab, lane, T);
+    const int ngroups = (in_slab + 4) / 5;
+    const uint32_t* wp = reinterpret_cast<const uint32_t*>(my_msg + s.off_payload) + wbase;
+#pragma unroll
+    for (int it = 0; it < kSliceWords / 8; ++it) {
+      if (it * 8 < sw) {
+        uint32_t wd[8];
+        load_words8(wp + 8 * it, wbase + 8 * it, nwords, lane < in_slab, wd);
+        accumulate8_dyn<7>(wd, T, ngroups, tl, acc + 8 * it);
+      }
+    }
+  }
+#pragma unroll
+  for (int i = 0; i < kSliceWords; ++i) {
+    const int64_t j = 32 * (wbase + i) + lane;
+    if (i < sw && j < s.d) __stcs(s.w + j, __fsub_rn(__ldcs(s.w + j), average(acc[i], s)));
+  }
+}
+
+// b-bit stochastic quantiser: Q_m(p)_j = fl(s_m * V[code]) with
+// V[code] = sign(code - K) * fl(|code - K| / K) (so V[K] = +0), summed in
+// worker order.  One thread per 4-element chunk (a fixed grid strides over
+// the chunks), code words of 8 workers fetched before they are decoded.  For
+// b = 4, 8 V lives in shared memory replicated once per bank (entry c of lane
+// l at [c][l]), so the random code lookups of a warp never conflict; for
+// b = 2 (V in {-1, 0, +1}) the value is a select.
+template <int BITS, bool POW2>
 __global__ void __launch_bounds__(256) squant_server_kernel(const ServerArgs s) {
   constexpr int K = (1 << (BITS - 1)) - 1;
   constexpr uint32_t MASK = (1u << BITS) - 1u;
-  __shared__ float level_value[K + 1];
-  for (int r = threadIdx.x; r <= K; r += blockDim.x) level_value[r] = __fdiv_rn((float)r, (float)K);
-  __syncthreads();
-  const int64_t c = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-  const int64_t j = 4 * c;
-  if (j >= s.d) return;
-  const int64_t bkt = j / s.bucket;
-  const int64_t bitpos = j * BITS;  // a chunk's 4*BITS bits never straddle a word
-  const int64_t word = bitpos >> 5;
-  const int shift = (int)(bitpos & 31);
-  float acc[4] = {0.f, 0.f, 0.f, 0.f};
-  for (int m = 0; m < s.M; ++m) {
-    const uint8_t* msg = s.msgs + (int64_t)m * s.msg_stride;
-    const float sc = __ldg(reinterpret_cast<const float*>(msg) + bkt);
-    const uint32_t bits = __ldg(reinterpret_cast<const uint32_t*>(msg + s.off_payload) + word) >> shift;
-#pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      const int level = (int)((bits >> (q * BITS)) & MASK) - K;
+  constexpr int CODES = (BITS == 2) ? 1 : (1 << BITS);
+  __shared__ float V[CODES * 32];
+  if constexpr (BITS != 2) {
+    for (int t = threadIdx.x; t < CODES * 32; t += blockDim.x) {
+      const int code = t >> 5;
+      const int level = code - K;
       float v = 0.f;
-      if (level != 0) {
-        const float mag = __fmul_rn(sc, level_value[level < 0 ? -level : level]);
+      if (code <= 2 * K && level != 0) {
+        const float mag = __fdiv_rn((float)(level < 0 ? -level : level), (float)K);
         v = level < 0 ? -mag : mag;
       }
-      acc[q] = __fadd_rn(acc[q], v);
+      V[t] = v;
+    }
+    __syncthreads();
+  }
+  const float* Vl = V + (threadIdx.x & 31);
+  const int64_t nchunks = (s.d + 3) >> 2;
+  for (int64_t c = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; c < nchunks;
+       c += (int64_t)gridDim.x * blockDim.x) {
+    const int64_t j = 4 * c;
+    const int64_t bkt = j / s.bucket;
+    const int64_t bitpos = j * BITS;  // a chunk's 4*BITS bits never straddle a word
+    const int64_t word = bitpos >> 5;
+    const int shift = (int)(bitpos & 31);
+    const uint8_t* m_scale = s.msgs + 4 * bkt;
+    const uint8_t* m_word = s.msgs + s.off_payload + 4 * word;
+    float acc[4] = {0.f, 0.f, 0.f, 0.f};
+    for (int m0 = 0; m0 < s.M; m0 += 8) {
+      uint32_t bits[8];
+      float sc[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const bool ok = m0 + u < s.M;
+        const int64_t off = (int64_t)(m0 + u) * s.msg_stride;
+        bits[u] = ok ? __ldcs(reinterpret_cast<const uint32_t*>(m_word + off)) >> shift : 0u;
+        sc[u] = ok ? __ldg(reinterpret_cast<const float*>(m_scale + off)) : 0.f;
+      }
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        if (m0 + u < s.M) {
+#pragma unroll
+          for (int q = 0; q < 4; ++q) {
+            float v;
+            if constexpr (BITS == 2) {
+              const uint32_t code = (bits[u] >> (2 * q)) & 3u;
+              v = (code == 0) ? -sc[u] : (code == 2 ? sc[u] : 0.f);  // fl(s * 1) = s
+            } else if constexpr (BITS == 8) {
+              v = __fmul_rn(sc[u], Vl[__byte_perm(bits[u], 0, 0x4440 | q) << 5]);
+            } else {
+              v = __fmul_rn(sc[u], Vl[((bits[u] >> (q * BITS)) & MASK) << 5]);
+            }
+            acc[q] = __fadd_rn(acc[q], v);
+          }
+        }
+      }
+    }
+    if (j + 3 < s.d) {
+      float4 wv = __ldcs(reinterpret_cast<const float4*>(s.w + j));
+      wv.x = __fsub_rn(wv.x, average_t<POW2>(acc[0], s));
+      wv.y = __fsub_rn(wv.y, average_t<POW2>(acc[1], s));
+      wv.z = __fsub_rn(wv.z, average_t<POW2>(acc[2], s));
+      wv.w = __fsub_rn(wv.w, average_t<POW2>(acc[3], s));
+      __stcs(reinterpret_cast<float4*>(s.w + j), wv);
+    } else {
+      for (int q = 0; q < 4 && j + q < s.d; ++q) s.w[j + q] = __fsub_rn(s.w[j + q], average_t<POW2>(acc[q], s));
     }
   }
-  apply_chunk(s, j, acc);
 }
 
-// Identity: the messages are the p vectors themselves.
+// Identity: the messages are the p vectors themselves (worker order).
 __global__ void __launch_bounds__(256) identity_server_kernel(const ServerArgs s) {
   const int64_t c = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   const int64_t j = 4 * c;
   if (j >= s.d) return;
   float acc[4] = {0.f, 0.f, 0.f, 0.f};
-  for (int m = 0; m < s.M; ++m) {
-    const float* vals = reinterpret_cast<const float*>(s.msgs + (int64_t)m * s.msg_stride);
-    if (j + 3 < s.d) {
-      const float4 v = __ldcs(reinterpret_cast<const float4*>(vals + j));
-      acc[0] = __fadd_rn(acc[0], v.x);
-      acc[1] = __fadd_rn(acc[1], v.y);
-      acc[2] = __fadd_rn(acc[2], v.z);
-      acc[3] = __fadd_rn(acc[3], v.w);
-    } else {
-      for (int q = 0; q < 4 && j + q < s.d; ++q) acc[q] = __fadd_rn(acc[q], vals[j + q]);
+  const bool vec = j + 3 < s.d;
+  for (int m0 = 0; m0 < s.M; m0 += 4) {
+    float4 v[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      v[u] = make_float4(0.f, 0.f, 0.f, 0.f);
+      if (m0 + u < s.M) {
+        const float* vals = reinterpret_cast<const float*>(s.msgs + (int64_t)(m0 + u) * s.msg_stride);
+        if (vec) {
+          v[u] = __ldcs(reinterpret_cast<const float4*>(vals + j));
+        } else {
+          v[u].x = vals[j];
+          if (j + 1 < s.d) v[u].y = vals[j + 1];
+          if (j + 2 < s.d) v[u].z = vals[j + 2];
+        }
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      if (m0 + u < s.M) {
+        acc[0] = __fadd_rn(acc[0], v[u].x);
+        acc[1] = __fadd_rn(acc[1], v[u].y);
+        acc[2] = __fadd_rn(acc[2], v[u].z);
+        acc[3] = __fadd_rn(acc[3], v[u].w);
+      }
     }
   }
   apply_chunk(s, j, acc);
@@ -170,17 +465,48 @@ unsigned chunk_blocks(int64_t d, int threads) {
 }  // namespace
 
 cudaError_t launch_sign_server(const ServerArgs& s, cudaStream_t stream, uint64_t* launches) {
-  sign_server_kernel<<<chunk_blocks(s.d, 256), 256, 0, stream>>>(s);
+  if (s.bucket >= 512) {
+    const int64_t nb = (s.d + s.bucket - 1) / s.bucket;
+    const int64_t wpb = s.bucket >= 1024 ? s.bucket / 1024 : 1;  // warps per bucket
+    const int64_t warps = nb * wpb;
+    const unsigned blocks = (unsigned)((warps + 7) / 8);
+    if (s.M > 32) {
+      sign_server_slabs_kernel<<<blocks, 256, 0, stream>>>(s);
+    } else {
+      const int ng = (s.M + 4) / 5;
+      const bool p2 = s.M_pow2 != 0;
+#define DQ_SIGN_SERVER(NG) \
+      (p2 ? sign_server_shfl_kernel<NG, true><<<blocks, 256, 0, stream>>>(s) \
+          : sign_server_shfl_kernel<NG, false><<<blocks, 256, 0, stream>>>(s))
+      switch (ng) {
+        case 1: DQ_SIGN_SERVER(1); break;
+        case 2: DQ_SIGN_SERVER(2); break;
+        case 3: DQ_SIGN_SERVER(3); break;
+        case 4: DQ_SIGN_SERVER(4); break;
+        case 5: DQ_SIGN_SERVER(5); break;
+        case 6: DQ_SIGN_SERVER(6); break;
+        default: DQ_SIGN_SERVER(7); break;
+      }
+#undef DQ_SIGN_SERVER
+    }
+  } else {
+    sign_server_kernel<<<chunk_blocks(s.d, 256), 256, 0, stream>>>(s);
+  }
   *launches += 1;
   return cudaGetLastError();
 }
 
 cudaError_t launch_squant_server(const ServerArgs& s, cudaStream_t stream, uint64_t* launches) {
-  const unsigned blocks = chunk_blocks(s.d, 256);
+  const unsigned chunk_grid = chunk_blocks(s.d, 256);
+  const unsigned blocks = chunk_grid < 152u * 6u ? chunk_grid : 152u * 6u;  // V is built once per block
+  const bool p2 = s.M_pow2 != 0;
   switch (s.bits) {
-    case 2: squant_server_kernel<2><<<blocks, 256, 0, stream>>>(s); break;
-    case 4: squant_server_kernel<4><<<blocks, 256, 0, stream>>>(s); break;
-    case 8: squant_server_kernel<8><<<blocks, 256, 0, stream>>>(s); break;
+    case 2: p2 ? squant_server_kernel<2, true><<<blocks, 256, 0, stream>>>(s)
+               : squant_server_kernel<2, false><<<blocks, 256, 0, stream>>>(s); break;
+    case 4: p2 ? squant_server_kernel<4, true><<<blocks, 256, 0, stream>>>(s)
+               : squant_server_kernel<4, false><<<blocks, 256, 0, stream>>>(s); break;
+    case 8: p2 ? squant_server_kernel<8, true><<<blocks, 256, 0, stream>>>(s)
+               : squant_server_kernel<8, false><<<blocks, 256, 0, stream>>>(s); break;
     default: return cudaErrorInvalidValue;
   }
   *launches += 1;

@@ -150,10 +150,15 @@ def test_per_worker_calls_match_batched(P, case):
     run_parity(P, ocfg, T=2, batched=False, seed=3)
 
 
-@pytest.mark.parametrize("M", [1, 5, 8])
-def test_worker_counts(P, M):
-    ocfg = oracle_config(50_000, M, oracle.SIGN, lr=1e-2, bucket=512)
-    run_parity(P, ocfg, T=4, seed=M)
+@pytest.mark.parametrize("M,comp,bucket", [
+    (1, oracle.SIGN, 512), (5, oracle.SIGN, 512), (8, oracle.SIGN, 1024), (32, oracle.SIGN, 2048),
+    (33, oracle.SIGN, 4096), (70, oracle.SIGN, 1024), (3, oracle.SIGN, 256), (40, oracle.SIGN, 64),
+    (20, oracle.SQUANT, 512), (33, oracle.IDENTITY, 512), (9, oracle.TOPK, 512)])
+def test_worker_counts(P, M, comp, bucket):
+    """Non-power-of-two M, M above 32 (several 32-worker slabs in the sign
+    server), every server path."""
+    ocfg = oracle_config(50_000 + 3, M, comp, lr=1e-2, bucket=bucket, bits=8, k=777)
+    run_parity(P, ocfg, T=3, seed=M)
 
 
 def test_multi_tile_topk_many_steps(P):
