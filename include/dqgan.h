@@ -211,6 +211,35 @@ DQGAN_API int dqgan_load_state(dqgan_handle* h, const void* host_src, int64_t by
 /* Kernels this handle has launched so far. */
 DQGAN_API uint64_t dqgan_launch_count(const dqgan_handle* h);
 
+/*
+ * Top-k worker step without any device allocation.  The paper has no
+ * counterpart: this entry point exists for callers that cannot allocate
+ * device memory (code inside a host framework that owns all device memory
+ * under a fixed plan, or a hot path that must not risk an allocation), which
+ * rules out dqgan_create.  It computes exactly what dqgan_worker_compress
+ * does for DQGAN_TOPK (same kernels, same bits):
+ *   p = fl(fl(lr * g_j) + e_j); out_msg = the k records {u32 j, f32 p_j} of
+ *   the k largest |p_j| (ties to the lower index), ascending index;
+ *   e_j = +0 at the kept entries and p_j elsewhere.
+ * g:       device, d fp32, read only.
+ * e:       device, d fp32, caller-owned residual, read and written.
+ * out_msg: device, at least 8*k bytes, written.
+ * All three 16-byte aligned.  1 <= d <= 1,048,576 (2^20); 1 <= k <= d.
+ * cuda_stream: the cudaStream_t to enqueue on (NULL: legacy stream).
+ * Scratch: a fixed 4.25 MiB array in this library's device memory, reserved
+ * on every GPU that loads the library until the process exits.  Nothing is
+ * allocated or freed.  The first call on a device looks up the array's
+ * device address (cudaGetSymbolAddress); make that first call before any
+ * stream capture.  Every call clears the part of the array it uses, and all
+ * calls share the array: calls whose work overlaps on the GPU (other
+ * streams, other host threads) race and give wrong results.
+ * Returns DQGAN_OK, DQGAN_ERR_INVALID_ARG (sizes beyond the limit, NULL or
+ * misaligned pointers) or DQGAN_ERR_CUDA; the reason is in
+ * dqgan_last_error(NULL).
+ */
+DQGAN_API int dqgan_topk_compress_noalloc(const float* g, float* e, void* out_msg, int64_t d, int64_t k,
+                                          float lr, void* cuda_stream);
+
 /* Text of the last error on this handle, or of the last failed
  * create / validate / layout call in this thread when h is NULL.
  * Never NULL; valid until the next call on the same handle / thread. */

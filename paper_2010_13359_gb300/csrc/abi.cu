@@ -171,6 +171,8 @@ constexpr int64_t kHeaderBytes = 64;
 
 namespace dq {
 
+int set_thread_error(int code, const char* msg) { return set_error(nullptr, code, "%s", msg); }
+
 bool message_layout(const dqgan_config& c, Layout* out) {
   if (!check_config(&c).empty()) return false;
   const int64_t nb = (c.compressor == DQGAN_SIGN || c.compressor == DQGAN_SQUANT)

@@ -26,6 +26,9 @@ struct Layout {
 // Host-side layout of one message (see dqgan.h); returns false on a bad config.
 bool message_layout(const dqgan_config& cfg, Layout* out);
 
+// Records `msg` as this thread's last error (dqgan_last_error(NULL)); returns code.
+int set_thread_error(int code, const char* msg);
+
 // Arguments shared by every worker-side (compress) kernel.  One launch covers
 // `nworkers` consecutive workers starting at `worker0`; launch row y (blockIdx.y)
 // is worker worker0 + y.

@@ -88,6 +88,7 @@ def load_library(path: str = LIBRARY) -> ctypes.CDLL:
         "dqgan_load_state": (ctypes.c_int, [H, P, i64]),
         "dqgan_launch_count": (u64, [H]),
         "dqgan_last_error": (ctypes.c_char_p, [H]),
+        "dqgan_topk_compress_noalloc": (ctypes.c_int, [P, P, P, i64, i64, ctypes.c_float, P]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(L, name)
@@ -222,3 +223,10 @@ class Handle:
 
 def create(cfg: Config) -> Handle:
     return Handle(cfg)
+
+
+def topk_compress_noalloc(g, e, out_msg, d: int, k: int, lr: float, cuda_stream: int | None = None) -> None:
+    """dqgan_topk_compress_noalloc: top-k worker step on a caller-owned residual,
+    with no device allocation (scratch is a fixed array in the library)."""
+    _check(load_library().dqgan_topk_compress_noalloc(_ptr(g), _ptr(e), _ptr(out_msg), d, k, lr,
+                                                      cuda_stream))
