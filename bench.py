@@ -55,6 +55,10 @@ def parse_args():
     ap.add_argument("--impl", default="gpu", choices=["gpu", "reference"])
     ap.add_argument("--lookahead", action="store_true", help="also keep the lookahead offsets h")
     ap.add_argument("--no-e2e", action="store_true", help="skip the end-to-end (host buffers) phase")
+    ap.add_argument("--e2e-mode", default="zerocopy", choices=["copy", "pipelined", "zerocopy"],
+                    help="how host gradients reach the kernels: one bulk copy then compute; per-worker "
+                         "copies on a second stream overlapped with per-worker compress; or the compress "
+                         "kernels reading the pinned host buffer directly (NVLink-C2C)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--override", action="append", default=[], metavar="FIELD=VALUE",
                     help="change a workload field (e.g. M=4 for a smaller profiling case)")
@@ -109,6 +113,22 @@ def server_bytes(wl) -> int:
 # ---------------------------------------------------------------------------
 # environment helpers
 # ---------------------------------------------------------------------------
+
+def max_over_ranks(x: float, world: int, device=None) -> float:
+    """The largest x over all ranks (all_reduce MAX; NCCL on GPUs, gloo on CPU)."""
+    if world <= 1:
+        return x
+    import torch
+    import torch.distributed as tdist
+    t = torch.tensor([x], dtype=torch.float64, device=device)
+    tdist.all_reduce(t, op=tdist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def whole_job_rate(units_per_rank: int, steps: int, world: int, max_ms: float) -> float:
+    """Units processed by all ranks per second, timed by the slowest rank."""
+    return world * units_per_rank * steps / (max_ms / 1e3)
+
 
 def dist_env():
     rank = int(os.environ.get("RANK", "0"))
@@ -351,15 +371,11 @@ def run_gpu(args, rank, world, local):
     launches = h.launch_count() - launches0
     comp_ms = [e[0].elapsed_time(e[1]) for e in events]
     serv_ms = [e[1].elapsed_time(e[2]) for e in events]
-    total_ms = sum(c + s for c, s in zip(comp_ms, serv_ms))
-    if world > 1:
-        tt = torch.tensor([total_ms], dtype=torch.float64, device=dev)
-        tdist.all_reduce(tt, op=tdist.ReduceOp.MAX)
-        total_ms = float(tt.item())
+    total_ms = max_over_ranks(sum(c + s for c, s in zip(comp_ms, serv_ms)), world, dev)
     units = wl.d * wl.M
-    value = world * units * args.steps / (total_ms / 1e3)
+    value = whole_job_rate(units, args.steps, world, total_ms)
 
-    # end to end: host gradients (pinned) -> device, the two C-ABI calls, params -> host
+    # end to end: host gradients (pinned) -> the C-ABI calls -> params -> host
     e2e = None
     if not args.no_e2e:
         g_host = torch.empty((wl.M, wl.d), dtype=torch.float32, pin_memory=True)
@@ -367,10 +383,24 @@ def run_gpu(args, rank, world, local):
         g_host.copy_(g)
         torch.cuda.synchronize(dev)
         e2e_steps = max(1, min(args.steps, 10))
+        copy_stream = torch.cuda.Stream(dev)
+        copied = [torch.cuda.Event() for _ in range(wl.M)]
 
         def e2e_step():
-            g.copy_(g_host, non_blocking=True)
-            h.workers_compress_all(g, wl.d, msgs)
+            if args.e2e_mode == "copy":
+                g.copy_(g_host, non_blocking=True)
+                h.workers_compress_all(g, wl.d, msgs)
+            elif args.e2e_mode == "pipelined":
+                copy_stream.wait_stream(stream)
+                with torch.cuda.stream(copy_stream):
+                    for i in range(wl.M):
+                        g[i].copy_(g_host[i], non_blocking=True)
+                        copied[i].record(copy_stream)
+                for i in range(wl.M):
+                    stream.wait_event(copied[i])
+                    h.worker_compress(i, g[i], msgs[i])
+            else:  # the kernels read the pinned host gradients in place
+                h.workers_compress_all(g_host, wl.d, msgs)
             h.server_aggregate_update(msgs, w)
             w_host.copy_(w, non_blocking=True)
 
@@ -383,14 +413,10 @@ def run_gpu(args, rank, world, local):
             e2e_step()
         b.record(stream)
         torch.cuda.synchronize(dev)
-        e2e_ms = a.elapsed_time(b)
-        if world > 1:
-            tt = torch.tensor([e2e_ms], dtype=torch.float64, device=dev)
-            tdist.all_reduce(tt, op=tdist.ReduceOp.MAX)
-            e2e_ms = float(tt.item())
-        e2e = {"value": world * units * e2e_steps / (e2e_ms / 1e3), "unit": UNIT,
+        e2e_ms = max_over_ranks(a.elapsed_time(b), world, dev)
+        e2e = {"value": whole_job_rate(units, e2e_steps, world, e2e_ms), "unit": UNIT,
                "h2d_bytes_per_step": int(g.numel() * 4), "d2h_bytes_per_step": int(w.numel() * 4),
-               "steps": e2e_steps, "ms_per_step": e2e_ms / e2e_steps}
+               "steps": e2e_steps, "ms_per_step": e2e_ms / e2e_steps, "mode": args.e2e_mode}
         del g_host, w_host
 
     h.synchronize()

@@ -147,7 +147,9 @@ DQGAN_API int64_t dqgan_message_bytes(const dqgan_handle* h);
  * Worker step of Algorithm 2 for worker i at the current step t:
  *   p = fl(fl(eta * g_j) + e_j); message = pack(Q(p)); e = fl(p - Q(p));
  *   with DQGAN_KEEP_LOOKAHEAD also h = fl(fl(eta * g_j) + e_j) (new e).
- * g:       device, d fp32, caller-owned, read only (F(w_{t-1/2}^(i); xi_t^(i))).
+ * g:       d fp32, caller-owned, read only (F(w_{t-1/2}^(i); xi_t^(i))): device
+ *          memory, or pinned host memory (cudaHostAlloc / cudaMallocHost), which
+ *          the kernels then read in place over the host link.
  * out_msg: device, dqgan_message_bytes() bytes, caller-owned, written.
  * Updates e^(i) (and h^(i)).  0 <= i < M.  Does not advance t.
  */
@@ -155,8 +157,9 @@ DQGAN_API int dqgan_worker_compress(dqgan_handle* h, int32_t i, const float* g, 
 
 /*
  * The worker step for all M workers in one launch per kernel stage.
- * g_all:    device, worker m's gradient at g_all + m * g_stride (floats);
- *           g_stride >= d and a multiple of 4.
+ * g_all:    worker m's gradient at g_all + m * g_stride (floats), device or
+ *           pinned host memory as for dqgan_worker_compress; g_stride >= d and a
+ *           multiple of 4.
  * msgs_all: device, worker m's message at msgs_all + m * dqgan_message_bytes().
  */
 DQGAN_API int dqgan_workers_compress_all(dqgan_handle* h, const float* g_all, int64_t g_stride,

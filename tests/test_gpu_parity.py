@@ -254,3 +254,37 @@ def test_error_conventions(P):
     with pytest.raises(P.DqganError) as ei:
         P.create(P.make_config(d=0, M=2, compressor=P.SIGN))
     assert ei.value.status == P.dqgan.ERR_INVALID_ARG
+
+
+@pytest.mark.parametrize("case", [(oracle.SIGN, dict(bucket=4096)), (oracle.SQUANT, dict(bucket=512, bits=8)),
+                                  (oracle.TOPK, dict(k=999))], ids=_case_id)
+def test_pinned_host_gradients_read_in_place(P, case):
+    """Gradients in pinned host memory are read in place by the kernels (over
+    the host link) and give the same bits as the same gradients in HBM."""
+    comp, kw = case
+    dev = torch.device("cuda:0")
+    stream = torch.cuda.current_stream(dev)
+    ocfg = oracle_config(100_003, 3, comp, lr=0.01, seed=5, **kw)
+    ld = (ocfg.d + 3) // 4 * 4
+    rng = np.random.default_rng(1)
+    g_host = torch.zeros((ocfg.M, ld), dtype=torch.float32).pin_memory()
+    g_host[:, :ocfg.d] = torch.from_numpy(grads("gauss", ocfg.M, ocfg.d, rng))
+    g_dev = g_host.to(dev)
+    a = P.create(gpu_config(P, ocfg, stream))
+    b = P.create(gpu_config(P, ocfg, stream))
+    mb = a.message_bytes()
+    ma = torch.zeros((ocfg.M, mb), dtype=torch.uint8, device=dev)
+    mbuf = torch.zeros((ocfg.M, mb), dtype=torch.uint8, device=dev)
+    for _ in range(2):
+        a.workers_compress_all(g_dev, ld, ma)
+        b.workers_compress_all(g_host, ld, mbuf)
+        a.synchronize()
+        b.synchronize()
+        assert torch.equal(ma, mbuf)
+        for i in range(ocfg.M):
+            ea, eb = np.empty(ocfg.d, np.float32), np.empty(ocfg.d, np.float32)
+            a.get_residual(i, ea)
+            b.get_residual(i, eb)
+            assert_bits_equal(eb, ea, f"residual worker {i}")
+    a.destroy()
+    b.destroy()
