@@ -23,6 +23,9 @@ struct dqgan_handle {
   void* scratch = nullptr;
   size_t scratch_bytes = 0;
   uint32_t* err_word = nullptr;  // device error word written by bounded waits
+  CUtensorMap sign_map;          // TMA map of the last message buffer the sign server saw
+  const void* sign_map_msgs = nullptr;
+  bool sign_map_ok = false;
   int64_t t = 1;
   uint64_t launches = 0;
   std::string err;
@@ -322,6 +325,15 @@ int dqgan_server_aggregate_update(dqgan_handle* h, const void* msgs_all, float* 
   s.bits = h->cfg.bits;
   s.M_pow2 = is_pow2(h->cfg.M) ? 1 : 0;
   s.inv_M = 1.0f / (float)h->cfg.M;
+  s.err = h->err_word;
+  s.sign_words_map = nullptr;
+  if (h->cfg.compressor == DQGAN_SIGN && h->cfg.bucket >= 1024 && h->cfg.M <= 32) {
+    if (h->sign_map_msgs != msgs_all) {
+      h->sign_map_ok = dq::encode_sign_words_map(s.msgs, s.msg_stride, s.off_payload, s.d, s.M, &h->sign_map);
+      h->sign_map_msgs = msgs_all;
+    }
+    if (h->sign_map_ok) s.sign_words_map = &h->sign_map;
+  }
   cudaError_t st = cudaSuccess;
   switch (h->cfg.compressor) {
     case DQGAN_SIGN: st = dq::launch_sign_server(s, h->stream, &h->launches); break;

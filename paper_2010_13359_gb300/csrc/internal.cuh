@@ -9,6 +9,8 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <cuda.h>
+
 #include "dqgan.h"
 
 namespace dq {
@@ -66,7 +68,16 @@ struct ServerArgs {
   int32_t bits;
   float inv_M;          // exact 1/M when M is a power of two
   int32_t M_pow2;       // 1 if M is a power of two (then x/M == x * inv_M exactly)
+  uint32_t* err;        // device error word (bit 0: a bounded wait timed out)
+  const CUtensorMap* sign_words_map;  // TMA map of the M messages' sign words, or nullptr
 };
+
+// TMA tensor map over the sign words of M messages: a 2-D array of u32, rows
+// = workers (M), columns = message words up to the end of the payload;
+// boxes of 32 words x 32 workers, 128-byte swizzle, zero fill outside.
+// Returns false if the driver entry point or the encoding is unavailable.
+bool encode_sign_words_map(const uint8_t* msgs, int64_t msg_stride, int64_t off_payload, int64_t d, int32_t M,
+                           CUtensorMap* out);
 
 // Scratch of the top-k path for `nworkers` concurrent workers.
 struct TopkScratch {

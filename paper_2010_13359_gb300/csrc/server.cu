@@ -7,7 +7,7 @@
 // accumulators, fetching the message words of 8 (4) workers before using
 // them.  Sign with buckets >= 512: bit-transposed table decode (below).
 // w is read and written once.
-#include "internal.cuh"
+#include "device_common.cuh"
 
 namespace dq {
 namespace {
@@ -242,6 +242,121 @@ __global__ void __launch_bounds__(256) sign_server_shfl_kernel(const ServerArgs 
   }
 }
 
+// Buckets of 1024..4096 with M <= 32: the same decode, with the message
+// words staged in shared memory by TMA instead of read by the lanes.  A 2-D
+// tensor map views the M messages as rows of u32 words; one box is 32 words
+// of every worker (M rows of 128 bytes, 128-byte swizzle: the 16-byte chunk c
+// of row r sits at chunk c ^ (r mod 8)), so lane m reads its worker's words
+// with conflict-free 128-bit shared loads.  Each warp owns two box buffers
+// and one mbarrier per buffer: while it decodes slice i it has the copy of
+// slice i + 1 in flight.  Waits are bounded (error word on time-out).
+constexpr int kTmaWarps = 8;
+constexpr int kTmaBoxBytes = 32 * 32 * 4;
+constexpr int kTmaSmemBytes = kTmaWarps * 2 * kTmaBoxBytes + 1024;  // + alignment slack
+
+template <int NG, bool POW2>
+__global__ void __launch_bounds__(32 * kTmaWarps)
+sign_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap tmap) {
+  extern __shared__ uint8_t smem_raw[];
+  __shared__ uint64_t bars[kTmaWarps][2];
+  const int lane = threadIdx.x & 31;
+  const int warp = threadIdx.x >> 5;
+  // 1024-byte aligned buffers (required by the 128-byte swizzle)
+  const uint32_t raw = smem_addr(smem_raw);
+  uint8_t* base = smem_raw + ((1024u - (raw & 1023u)) & 1023u);
+  uint8_t* const buf0 = base + warp * 2 * kTmaBoxBytes;  // buffer i at buf0 + i * kTmaBoxBytes
+  uint64_t* bar = bars[warp];
+  if (lane == 0) {
+    mbar_init(&bar[0], 1);
+    mbar_init(&bar[1], 1);
+    mbar_fence_init();
+  }
+  __syncwarp();
+
+  const int words_per_bucket = s.bucket >> 5;  // 32..128
+  const int spb = words_per_bucket >> 5;       // 32-word slices per bucket
+  const int64_t nb = (s.d + s.bucket - 1) / s.bucket;
+  const int64_t nslices = nb * spb;
+  const int64_t stride = (int64_t)gridDim.x * kTmaWarps;
+  const int32_t x0 = (int32_t)(s.off_payload >> 2);
+  const uint32_t box_bytes = (uint32_t)(s.M < 32 ? s.M : 32) * 128u;
+  const bool active = lane < s.M;
+  const TransposeLane tl(lane);
+
+  int64_t sl = (int64_t)blockIdx.x * kTmaWarps + warp;
+  auto wbase_of = [&](int64_t slice) {
+    const int64_t b = slice / spb;
+    return b * words_per_bucket + (slice - b * spb) * 32;
+  };
+  if (sl < nslices && lane == 0) {
+    mbar_arrive_expect_tx(&bar[0], box_bytes);
+    tma_load_2d(buf0, &tmap, x0 + (int32_t)wbase_of(sl), 0, &bar[0]);
+  }
+  uint32_t it = 0;
+  bool ok = true;
+  for (; sl < nslices; sl += stride, ++it) {
+    const int cur = (int)(it & 1u);
+    const int64_t nxt = sl + stride;
+    if (nxt < nslices && lane == 0) {
+      fence_proxy_async_shared();  // this warp's reads of that buffer came before
+      mbar_arrive_expect_tx(&bar[cur ^ 1], box_bytes);
+      tma_load_2d(buf0 + (cur ^ 1) * kTmaBoxBytes, &tmap, x0 + (int32_t)wbase_of(nxt), 0, &bar[cur ^ 1]);
+    }
+    const int64_t b = sl / spb;
+    const int64_t wbase = wbase_of(sl);
+    float* wl = s.w + 32 * wbase + lane;
+    const int64_t jmax = s.d - 32 * wbase - lane;  // wl[32 i] is a parameter iff 32 i < jmax
+    float wv[8];
+#pragma unroll
+    for (int k = 0; k < 8; ++k) wv[k] = (32 * k < jmax) ? __ldcs(wl + 32 * k) : 0.f;
+    const float my_scale =
+        active ? __ldg(reinterpret_cast<const float*>(s.msgs + (int64_t)lane * s.msg_stride) + b) : 0.f;
+    float T[7];
+    build_group_tables(my_scale, s.M, lane, T);
+    ok = mbar_wait_bounded(&bar[cur], (it >> 1) & 1u, s.err);
+    ok = __all_sync(kFullMask, ok);
+    if (!ok) break;
+    const uint8_t* row = buf0 + cur * kTmaBoxBytes + lane * 128;
+    const int sw = lane & 7;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      uint32_t wd[8];
+      if (active) {
+        const uint4 lo = *reinterpret_cast<const uint4*>(row + (((2 * q) ^ sw) << 4));
+        const uint4 hi = *reinterpret_cast<const uint4*>(row + (((2 * q + 1) ^ sw) << 4));
+        wd[0] = lo.x; wd[1] = lo.y; wd[2] = lo.z; wd[3] = lo.w;
+        wd[4] = hi.x; wd[5] = hi.y; wd[6] = hi.z; wd[7] = hi.w;
+      } else {
+#pragma unroll
+        for (int k = 0; k < 8; ++k) wd[k] = 0u;
+      }
+      float wv_next[8];
+      if (q < 3) {
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+          const int64_t off = 32 * (8 * (q + 1) + k);
+          wv_next[k] = (off < jmax) ? __ldcs(wl + off) : 0.f;
+        }
+      }
+      float sum[8];
+      sums8<NG>(wd, T, tl, sum);
+#pragma unroll
+      for (int k = 0; k < 8; ++k) {
+        const int64_t off = 32 * (8 * q + k);
+        if (off < jmax) __stcs(wl + off, __fsub_rn(wv[k], average_t<POW2>(sum[k], s)));
+      }
+      if (q < 3) {
+#pragma unroll
+        for (int k = 0; k < 8; ++k) wv[k] = wv_next[k];
+      }
+    }
+    __syncwarp();
+  }
+  // after a time-out the copy of the next slice may still be in flight
+  if (!ok && lane == 0 && sl + stride < nslices)
+    mbar_wait_bounded(&bar[(it & 1u) ^ 1u], ((it + 1) >> 1) & 1u, s.err);
+}
+
 // Any M: workers taken 32 at a time, groups added in order, w updated at the end.
 __global__ void __launch_bounds__(256) sign_server_slabs_kernel(const ServerArgs s) {
   const int lane = threadIdx.x & 31;
@@ -457,6 +572,33 @@ lookahead_kernel(const float* __restrict__ w, const float* __restrict__ h, float
   }
 }
 
+template <int NG, bool POW2>
+cudaError_t launch_sign_tma(const ServerArgs& s, cudaStream_t stream) {
+  auto kern = sign_server_tma_kernel<NG, POW2>;
+  int dev = 0;
+  cudaError_t st = cudaGetDevice(&dev);
+  if (st != cudaSuccess) return st;
+  static int blocks_for[64] = {0};
+  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+  if (blocks_for[dev] == 0) {
+    if ((st = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kTmaSmemBytes)) !=
+        cudaSuccess)
+      return st;
+    int sms = 0, per_sm = 0;
+    if ((st = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return st;
+    if ((st = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, 32 * kTmaWarps, kTmaSmemBytes)) !=
+        cudaSuccess)
+      return st;
+    blocks_for[dev] = sms * (per_sm > 0 ? per_sm : 1);
+  }
+  const int64_t nb = (s.d + s.bucket - 1) / s.bucket;
+  const int64_t warps = nb * (s.bucket / 1024);
+  const int64_t need = (warps + kTmaWarps - 1) / kTmaWarps;
+  const unsigned blocks = (unsigned)(need < blocks_for[dev] ? need : blocks_for[dev]);
+  kern<<<blocks, 32 * kTmaWarps, kTmaSmemBytes, stream>>>(s, *s.sign_words_map);
+  return cudaGetLastError();
+}
+
 unsigned chunk_blocks(int64_t d, int threads) {
   const int64_t chunks = (d + 3) / 4;
   return (unsigned)((chunks + threads - 1) / threads);
@@ -465,6 +607,23 @@ unsigned chunk_blocks(int64_t d, int threads) {
 }  // namespace
 
 cudaError_t launch_sign_server(const ServerArgs& s, cudaStream_t stream, uint64_t* launches) {
+  if (s.bucket >= 1024 && s.M <= 32 && s.sign_words_map != nullptr) {
+    const bool p2 = s.M_pow2 != 0;
+    cudaError_t st;
+#define DQ_SIGN_TMA(NG) st = (p2 ? launch_sign_tma<NG, true>(s, stream) : launch_sign_tma<NG, false>(s, stream))
+    switch ((s.M + 4) / 5) {
+      case 1: DQ_SIGN_TMA(1); break;
+      case 2: DQ_SIGN_TMA(2); break;
+      case 3: DQ_SIGN_TMA(3); break;
+      case 4: DQ_SIGN_TMA(4); break;
+      case 5: DQ_SIGN_TMA(5); break;
+      case 6: DQ_SIGN_TMA(6); break;
+      default: DQ_SIGN_TMA(7); break;
+    }
+#undef DQ_SIGN_TMA
+    *launches += 1;
+    return st;
+  }
   if (s.bucket >= 512) {
     const int64_t nb = (s.d + s.bucket - 1) / s.bucket;
     const int64_t wpb = s.bucket >= 1024 ? s.bucket / 1024 : 1;  // warps per bucket
@@ -531,6 +690,36 @@ cudaError_t launch_lookahead(const float* w, const float* h, float* out, int64_t
   lookahead_kernel<<<chunk_blocks(d, 256), 256, 0, stream>>>(w, h, out, d);
   *launches += 1;
   return cudaGetLastError();
+}
+
+}  // namespace dq
+
+namespace dq {
+
+bool encode_sign_words_map(const uint8_t* msgs, int64_t msg_stride, int64_t off_payload, int64_t d, int32_t M,
+                           CUtensorMap* out) {
+  using EncodeFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+  static EncodeFn encode = nullptr;
+  static bool looked_up = false;
+  if (!looked_up) {
+    looked_up = true;
+    void* fn = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      encode = reinterpret_cast<EncodeFn>(fn);
+  }
+  if (!encode || M < 1) return false;
+  const cuuint64_t dims[2] = {(cuuint64_t)(off_payload / 4 + (d + 31) / 32), (cuuint64_t)M};
+  const cuuint64_t strides[1] = {(cuuint64_t)msg_stride};
+  const cuuint32_t box[2] = {32u, (cuuint32_t)(M < 32 ? M : 32)};
+  const cuuint32_t elem[2] = {1u, 1u};
+  return encode(out, CU_TENSOR_MAP_DATA_TYPE_UINT32, 2, const_cast<uint8_t*>(msgs), dims, strides, box, elem,
+                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
+                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
 }  // namespace dq
