@@ -23,9 +23,9 @@ struct dqgan_handle {
   void* scratch = nullptr;
   size_t scratch_bytes = 0;
   uint32_t* err_word = nullptr;  // device error word written by bounded waits
-  CUtensorMap sign_map;          // TMA map of the last message buffer the sign server saw
-  const void* sign_map_msgs = nullptr;
-  bool sign_map_ok = false;
+  CUtensorMap words_map;         // TMA map of the last message buffer the server saw
+  const void* words_map_msgs = nullptr;
+  bool words_map_ok = false;
   int64_t t = 1;
   uint64_t launches = 0;
   std::string err;
@@ -327,12 +327,18 @@ int dqgan_server_aggregate_update(dqgan_handle* h, const void* msgs_all, float* 
   s.inv_M = 1.0f / (float)h->cfg.M;
   s.err = h->err_word;
   s.sign_words_map = nullptr;
-  if (h->cfg.compressor == DQGAN_SIGN && h->cfg.bucket >= 1024 && h->cfg.M <= 32) {
-    if (h->sign_map_msgs != msgs_all) {
-      h->sign_map_ok = dq::encode_sign_words_map(s.msgs, s.msg_stride, s.off_payload, s.d, s.M, &h->sign_map);
-      h->sign_map_msgs = msgs_all;
+  s.squant_words_map = nullptr;
+  const bool tma_sign = h->cfg.compressor == DQGAN_SIGN && h->cfg.bucket >= 1024 && h->cfg.M <= 32;
+  const bool tma_squant = h->cfg.compressor == DQGAN_SQUANT && h->cfg.M <= 32 &&
+                          h->cfg.bucket >= 32 * (32 / h->cfg.bits);
+  if (tma_sign || tma_squant) {
+    if (h->words_map_msgs != msgs_all) {
+      const int64_t payload_words = tma_sign ? (s.d + 31) / 32 : (s.d * s.bits + 31) / 32;
+      h->words_map_ok = dq::encode_words_map(s.msgs, s.msg_stride, s.off_payload, payload_words, s.M, tma_sign,
+                                             &h->words_map);
+      h->words_map_msgs = msgs_all;
     }
-    if (h->sign_map_ok) s.sign_words_map = &h->sign_map;
+    if (h->words_map_ok) (tma_sign ? s.sign_words_map : s.squant_words_map) = &h->words_map;
   }
   cudaError_t st = cudaSuccess;
   switch (h->cfg.compressor) {

@@ -69,15 +69,16 @@ struct ServerArgs {
   float inv_M;          // exact 1/M when M is a power of two
   int32_t M_pow2;       // 1 if M is a power of two (then x/M == x * inv_M exactly)
   uint32_t* err;        // device error word (bit 0: a bounded wait timed out)
-  const CUtensorMap* sign_words_map;  // TMA map of the M messages' sign words, or nullptr
+  const CUtensorMap* sign_words_map;    // TMA map of the M messages' sign words, or nullptr
+  const CUtensorMap* squant_words_map;  // TMA map of the M messages' code words, or nullptr
 };
 
-// TMA tensor map over the sign words of M messages: a 2-D array of u32, rows
-// = workers (M), columns = message words up to the end of the payload;
-// boxes of 32 words x 32 workers, 128-byte swizzle, zero fill outside.
-// Returns false if the driver entry point or the encoding is unavailable.
-bool encode_sign_words_map(const uint8_t* msgs, int64_t msg_stride, int64_t off_payload, int64_t d, int32_t M,
-                           CUtensorMap* out);
+// TMA tensor map over the payload words of M messages: a 2-D array of u32,
+// rows = workers (M), columns = message words up to the end of the payload;
+// boxes of 32 words x min(M, 32) workers, 128-byte swizzle or none, zero fill
+// outside.  Returns false if the driver entry point or the encoding fails.
+bool encode_words_map(const uint8_t* msgs, int64_t msg_stride, int64_t off_payload, int64_t payload_words,
+                      int32_t M, bool swizzle128, CUtensorMap* out);
 
 // Scratch of the top-k path for `nworkers` concurrent workers.
 struct TopkScratch {

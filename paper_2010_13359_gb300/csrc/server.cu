@@ -477,6 +477,140 @@ __global__ void __launch_bounds__(256) squant_server_kernel(const ServerArgs s) 
   }
 }
 
+// b-bit stochastic quantiser with M <= 32 and buckets of at least 32*32/b
+// elements: the code words are staged by TMA like the sign words above (a
+// box is 32 words of every worker, M rows of 128 bytes, no swizzle: lane l
+// reads word l of row m, one conflict-free 128-byte row per worker).  Lane l
+// owns the 32/b consecutive elements of its word; per worker, in worker
+// order, it decodes them with the worker's scale (broadcast by shuffle from
+// the lane that loaded it) and V[code] (b = 8: the bank-replicated table;
+// b = 4: 15 entries in a register, looked up by shuffle; b = 2: a select).
+// Worker-order sums from +0, so the result equals the oracle's bit for bit.
+template <int BITS, bool POW2>
+__global__ void __launch_bounds__(32 * kTmaWarps)
+squant_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap tmap) {
+  constexpr int K = (1 << (BITS - 1)) - 1;
+  constexpr uint32_t MASK = (1u << BITS) - 1u;
+  constexpr int EPL = 32 / BITS;  // elements per lane (one code word)
+  constexpr int SLICE = 32 * EPL; // elements per slice
+  extern __shared__ uint8_t smem_raw[];
+  __shared__ uint64_t bars[kTmaWarps][2];
+  __shared__ float V8[BITS == 8 ? 256 * 32 : 1];
+  const int lane = threadIdx.x & 31;
+  const int warp = threadIdx.x >> 5;
+  const uint32_t box_bytes = (uint32_t)s.M * 128u;
+  const uint32_t raw = smem_addr(smem_raw);  // 128-byte aligned boxes
+  uint8_t* const buf0 = smem_raw + ((128u - (raw & 127u)) & 127u) + warp * 2 * box_bytes;  // buffer i at + i*box
+  uint64_t* bar = bars[warp];
+  if constexpr (BITS == 8) {
+    for (int t = threadIdx.x; t < 256 * 32; t += blockDim.x) {
+      const int code = t >> 5;
+      const int level = code - K;
+      float v = 0.f;
+      if (code <= 2 * K && level != 0) {
+        const float mag = __fdiv_rn((float)(level < 0 ? -level : level), (float)K);
+        v = level < 0 ? -mag : mag;
+      }
+      V8[t] = v;
+    }
+  }
+  float V4 = 0.f;  // b = 4: lane c holds V[c]
+  if constexpr (BITS == 4) {
+    const int level = lane - K;
+    if (lane <= 2 * K && level != 0) {
+      const float mag = __fdiv_rn((float)(level < 0 ? -level : level), (float)K);
+      V4 = level < 0 ? -mag : mag;
+    }
+  }
+  if (lane == 0) {
+    mbar_init(&bar[0], 1);
+    mbar_init(&bar[1], 1);
+    mbar_fence_init();
+  }
+  __syncthreads();
+
+  const int spb = s.bucket / SLICE;  // slices per bucket
+  const int64_t nb = (s.d + s.bucket - 1) / s.bucket;
+  const int64_t nslices = nb * spb;
+  const int64_t stride = (int64_t)gridDim.x * kTmaWarps;
+  const int32_t x0 = (int32_t)(s.off_payload >> 2);
+  const bool active = lane < s.M;
+  int64_t sl = (int64_t)blockIdx.x * kTmaWarps + warp;
+  // slice sl covers code words [32 sl, 32 sl + 32): buckets hold whole slices
+  if (sl < nslices && lane == 0) {
+    mbar_arrive_expect_tx(&bar[0], box_bytes);
+    tma_load_2d(buf0, &tmap, x0 + (int32_t)(32 * sl), 0, &bar[0]);
+  }
+  uint32_t it = 0;
+  bool ok = true;
+  for (; sl < nslices; sl += stride, ++it) {
+    const int cur = (int)(it & 1u);
+    const int64_t nxt = sl + stride;
+    if (nxt < nslices && lane == 0) {
+      fence_proxy_async_shared();
+      mbar_arrive_expect_tx(&bar[cur ^ 1], box_bytes);
+      tma_load_2d(buf0 + (cur ^ 1) * box_bytes, &tmap, x0 + (int32_t)(32 * nxt), 0, &bar[cur ^ 1]);
+    }
+    const int64_t b = sl / spb;
+    const int64_t j0 = SLICE * sl + EPL * lane;  // this lane's first element
+    float wv[EPL];
+#pragma unroll
+    for (int q = 0; q < EPL / 4; ++q) {
+      const int64_t j = j0 + 4 * q;
+      if (j + 3 < s.d) {
+        const float4 x = __ldcs(reinterpret_cast<const float4*>(s.w + j));
+        wv[4 * q] = x.x; wv[4 * q + 1] = x.y; wv[4 * q + 2] = x.z; wv[4 * q + 3] = x.w;
+      } else {
+#pragma unroll
+        for (int r = 0; r < 4; ++r) wv[4 * q + r] = (j + r < s.d) ? s.w[j + r] : 0.f;
+      }
+    }
+    const float my_scale =
+        active ? __ldg(reinterpret_cast<const float*>(s.msgs + (int64_t)lane * s.msg_stride) + b) : 0.f;
+    ok = mbar_wait_bounded(&bar[cur], (it >> 1) & 1u, s.err);
+    ok = __all_sync(kFullMask, ok);
+    if (!ok) break;
+    const uint32_t* words = reinterpret_cast<const uint32_t*>(buf0 + cur * box_bytes) + lane;
+    float acc[EPL];
+#pragma unroll
+    for (int e = 0; e < EPL; ++e) acc[e] = 0.f;
+    for (int m = 0; m < s.M; ++m) {
+      const uint32_t word = words[32 * m];
+      const float sc = __shfl_sync(kFullMask, my_scale, m);
+#pragma unroll
+      for (int e = 0; e < EPL; ++e) {
+        const uint32_t code = (word >> (BITS * e)) & MASK;
+        float v;
+        if constexpr (BITS == 2) {
+          v = (code == 0) ? -sc : (code == 2 ? sc : 0.f);  // fl(s * 1) = s
+        } else if constexpr (BITS == 4) {
+          v = __fmul_rn(sc, __shfl_sync(kFullMask, V4, (int)code));
+        } else {
+          v = __fmul_rn(sc, V8[(code << 5) + lane]);
+        }
+        acc[e] = __fadd_rn(acc[e], v);
+      }
+    }
+#pragma unroll
+    for (int q = 0; q < EPL / 4; ++q) {
+      const int64_t j = j0 + 4 * q;
+      float o[4];
+#pragma unroll
+      for (int r = 0; r < 4; ++r) o[r] = __fsub_rn(wv[4 * q + r], average_t<POW2>(acc[4 * q + r], s));
+      if (j + 3 < s.d) {
+        __stcs(reinterpret_cast<float4*>(s.w + j), make_float4(o[0], o[1], o[2], o[3]));
+      } else {
+#pragma unroll
+        for (int r = 0; r < 4; ++r)
+          if (j + r < s.d) s.w[j + r] = o[r];
+      }
+    }
+    __syncwarp();
+  }
+  if (!ok && lane == 0 && sl + stride < nslices)
+    mbar_wait_bounded(&bar[(it & 1u) ^ 1u], ((it + 1) >> 1) & 1u, s.err);
+}
+
 // Identity: the messages are the p vectors themselves (worker order).
 __global__ void __launch_bounds__(256) identity_server_kernel(const ServerArgs s) {
   const int64_t c = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
@@ -599,6 +733,25 @@ cudaError_t launch_sign_tma(const ServerArgs& s, cudaStream_t stream) {
   return cudaGetLastError();
 }
 
+template <int BITS, bool POW2>
+cudaError_t launch_squant_tma(const ServerArgs& s, cudaStream_t stream) {
+  auto kern = squant_server_tma_kernel<BITS, POW2>;
+  const int smem = kTmaWarps * 2 * s.M * 128 + 128;  // + alignment slack
+  int dev = 0;
+  cudaError_t st = cudaGetDevice(&dev);
+  if (st != cudaSuccess) return st;
+  if ((st = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem)) != cudaSuccess) return st;
+  int sms = 0, per_sm = 0;
+  if ((st = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return st;
+  if ((st = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, 32 * kTmaWarps, smem)) != cudaSuccess)
+    return st;
+  const int64_t nslices = ((s.d + s.bucket - 1) / s.bucket) * (s.bucket / (32 * (32 / BITS)));
+  const int64_t need = (nslices + kTmaWarps - 1) / kTmaWarps;
+  const int64_t cap = (int64_t)sms * (per_sm > 0 ? per_sm : 1);
+  kern<<<(unsigned)(need < cap ? need : cap), 32 * kTmaWarps, smem, stream>>>(s, *s.squant_words_map);
+  return cudaGetLastError();
+}
+
 unsigned chunk_blocks(int64_t d, int threads) {
   const int64_t chunks = (d + 3) / 4;
   return (unsigned)((chunks + threads - 1) / threads);
@@ -656,6 +809,17 @@ cudaError_t launch_sign_server(const ServerArgs& s, cudaStream_t stream, uint64_
 }
 
 cudaError_t launch_squant_server(const ServerArgs& s, cudaStream_t stream, uint64_t* launches) {
+  if (s.squant_words_map != nullptr && s.M <= 32 && s.bucket >= 32 * (32 / s.bits)) {
+    const bool p2 = s.M_pow2 != 0;
+    cudaError_t st = cudaErrorInvalidValue;
+    switch (s.bits) {
+      case 2: st = p2 ? launch_squant_tma<2, true>(s, stream) : launch_squant_tma<2, false>(s, stream); break;
+      case 4: st = p2 ? launch_squant_tma<4, true>(s, stream) : launch_squant_tma<4, false>(s, stream); break;
+      case 8: st = p2 ? launch_squant_tma<8, true>(s, stream) : launch_squant_tma<8, false>(s, stream); break;
+    }
+    *launches += 1;
+    return st;
+  }
   const unsigned chunk_grid = chunk_blocks(s.d, 256);
   const unsigned blocks = chunk_grid < 152u * 6u ? chunk_grid : 152u * 6u;  // V is built once per block
   const bool p2 = s.M_pow2 != 0;
@@ -696,8 +860,8 @@ cudaError_t launch_lookahead(const float* w, const float* h, float* out, int64_t
 
 namespace dq {
 
-bool encode_sign_words_map(const uint8_t* msgs, int64_t msg_stride, int64_t off_payload, int64_t d, int32_t M,
-                           CUtensorMap* out) {
+bool encode_words_map(const uint8_t* msgs, int64_t msg_stride, int64_t off_payload, int64_t payload_words,
+                      int32_t M, bool swizzle128, CUtensorMap* out) {
   using EncodeFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
                                 const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
                                 CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
@@ -713,12 +877,13 @@ bool encode_sign_words_map(const uint8_t* msgs, int64_t msg_stride, int64_t off_
       encode = reinterpret_cast<EncodeFn>(fn);
   }
   if (!encode || M < 1) return false;
-  const cuuint64_t dims[2] = {(cuuint64_t)(off_payload / 4 + (d + 31) / 32), (cuuint64_t)M};
+  const cuuint64_t dims[2] = {(cuuint64_t)(off_payload / 4 + payload_words), (cuuint64_t)M};
   const cuuint64_t strides[1] = {(cuuint64_t)msg_stride};
   const cuuint32_t box[2] = {32u, (cuuint32_t)(M < 32 ? M : 32)};
   const cuuint32_t elem[2] = {1u, 1u};
   return encode(out, CU_TENSOR_MAP_DATA_TYPE_UINT32, 2, const_cast<uint8_t*>(msgs), dims, strides, box, elem,
-                CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
+                CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle128 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE,
+                CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
                 CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
