@@ -60,6 +60,9 @@ def parse_args():
                          "copies on a second stream overlapped with per-worker compress; or the compress "
                          "kernels reading the pinned host buffer directly (NVLink-C2C)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--sweep", action="store_true",
+                    help="instead of the one-line result, print one line per d = 2^16 .. 2^27 "
+                         "(M = 8, sign per 1024, DCGAN gradient law): the roofline curve")
     ap.add_argument("--override", action="append", default=[], metavar="FIELD=VALUE",
                     help="change a workload field (e.g. M=4 for a smaller profiling case)")
     return ap.parse_args()
@@ -456,11 +459,56 @@ def run_gpu(args, rank, world, local):
     return 0
 
 
+def run_sweep(args):
+    """Device-resident step time over d = 2^16 .. 2^27 (M = 8, sign per 1024)."""
+    import torch
+
+    import paper_2010_13359_gb300 as P
+    from paper_2010_13359_gb300.workloads import sweep_workload
+
+    dev = torch.device("cuda", 0)
+    stream = torch.cuda.current_stream(dev)
+    peak, peak_kind = hbm_peak()
+    for log2_d in range(16, 28):
+        wl = sweep_workload(log2_d)
+        h = P.create(P.make_config(d=wl.d, M=wl.M, compressor=wl.compressor, lr=wl.lr, bucket=wl.bucket,
+                                   seed=wl.seed, cuda_stream=stream.cuda_stream))
+        g = torch.empty((wl.M, wl.d), dtype=torch.float32, device=dev)
+        msgs = torch.empty((wl.M, h.message_bytes()), dtype=torch.uint8, device=dev)
+        w = wl.w0_torch(dev)
+        flush = torch.empty(256 << 20, dtype=torch.uint8, device=dev)
+        std_vec = wl.std_vector_torch(dev)
+        comp, serv = [], []
+        for t in range(1, args.warmup + args.steps + 1):
+            wl.fill_gradients_torch(g, t, std_vec)
+            flush.zero_()
+            ev = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
+            ev[0].record(stream)
+            h.workers_compress_all(g, wl.d, msgs)
+            ev[1].record(stream)
+            h.server_aggregate_update(msgs, w)
+            ev[2].record(stream)
+            torch.cuda.synchronize(dev)
+            if t > args.warmup:
+                comp.append(ev[0].elapsed_time(ev[1]))
+                serv.append(ev[1].elapsed_time(ev[2]))
+        h.destroy()
+        c_ms, s_ms = statistics.median(comp), statistics.median(serv)
+        cb, sb = compress_bytes(wl, False), server_bytes(wl)
+        print(json.dumps({"sweep": "sign_1024_M8", "d": wl.d, "M": wl.M, "params_per_s": wl.d * wl.M / ((c_ms + s_ms) / 1e3),
+                          "compress_ms": c_ms, "compress_gbs": cb / c_ms / 1e6, "compress_frac": cb / c_ms / 1e6 / peak,
+                          "server_ms": s_ms, "server_gbs": sb / s_ms / 1e6, "server_frac": sb / s_ms / 1e6 / peak,
+                          "peak": peak, "peak_source": peak_kind}), flush=True)
+    return 0
+
+
 def main():
     args = parse_args()
     rank, world, local = dist_env()
     if args.impl == "reference":
         return run_reference(args, rank, world)
+    if args.sweep:
+        return run_sweep(args)
     return run_gpu(args, rank, world, local)
 
 

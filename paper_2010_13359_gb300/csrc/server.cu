@@ -571,26 +571,38 @@ squant_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap
     ok = __all_sync(kFullMask, ok);
     if (!ok) break;
     const uint32_t* words = reinterpret_cast<const uint32_t*>(buf0 + cur * box_bytes) + lane;
+    const float* V8l = V8 + lane;
     float acc[EPL];
 #pragma unroll
     for (int e = 0; e < EPL; ++e) acc[e] = 0.f;
-    for (int m = 0; m < s.M; ++m) {
-      const uint32_t word = words[32 * m];
-      const float sc = __shfl_sync(kFullMask, my_scale, m);
+    // one worker's contribution, added in worker order
+    auto add_worker = [&](uint32_t word, float sc) {
 #pragma unroll
       for (int e = 0; e < EPL; ++e) {
-        const uint32_t code = (word >> (BITS * e)) & MASK;
         float v;
         if constexpr (BITS == 2) {
+          const uint32_t code = (word >> (2 * e)) & 3u;
           v = (code == 0) ? -sc : (code == 2 ? sc : 0.f);  // fl(s * 1) = s
         } else if constexpr (BITS == 4) {
-          v = __fmul_rn(sc, __shfl_sync(kFullMask, V4, (int)code));
+          v = __fmul_rn(sc, __shfl_sync(kFullMask, V4, (int)((word >> (4 * e)) & MASK)));
         } else {
-          v = __fmul_rn(sc, V8[(code << 5) + lane]);
+          v = __fmul_rn(sc, V8l[__byte_perm(word, 0u, 0x4440u | (uint32_t)e) * 32u]);
         }
         acc[e] = __fadd_rn(acc[e], v);
       }
+    };
+    int m = 0;
+    for (; m + 4 <= s.M; m += 4) {
+      const uint32_t w0 = words[32 * m], w1 = words[32 * (m + 1)];
+      const uint32_t w2 = words[32 * (m + 2)], w3 = words[32 * (m + 3)];
+      const float s0 = __shfl_sync(kFullMask, my_scale, m), s1 = __shfl_sync(kFullMask, my_scale, m + 1);
+      const float s2 = __shfl_sync(kFullMask, my_scale, m + 2), s3 = __shfl_sync(kFullMask, my_scale, m + 3);
+      add_worker(w0, s0);
+      add_worker(w1, s1);
+      add_worker(w2, s2);
+      add_worker(w3, s3);
     }
+    for (; m < s.M; ++m) add_worker(words[32 * m], __shfl_sync(kFullMask, my_scale, m));
 #pragma unroll
     for (int q = 0; q < EPL / 4; ++q) {
       const int64_t j = j0 + 4 * q;
@@ -650,7 +662,8 @@ __global__ void __launch_bounds__(256) identity_server_kernel(const ServerArgs s
 // Top-k: every worker's records are sorted by index, so whether an index
 // appears in worker m's list is a binary search.  The thread holding the
 // first occurrence (lowest worker) of an index sums that index's values over
-// all workers in worker order and applies the update; the others do nothing.
+// all workers in worker order and applies the update; the others stop at the
+// first earlier worker that holds their index.
 __device__ __forceinline__ bool find_index(const uint2* rec, int64_t k, uint32_t idx, float* val) {
   int64_t lo = 0, hi = k;  // search [lo, hi)
   while (lo < hi) {

@@ -252,7 +252,9 @@ __global__ void __launch_bounds__(kThreads) topk_filter_kernel(const CompressArg
     for (int q = 0; q < 4; ++q)
       if (cmask & (1u << q)) rs.cand[pos++] = (uint32_t)(j + q);
   }
-  atomicAdd(&tile_above, above);
+#pragma unroll
+  for (int off = 16; off >= 1; off >>= 1) above += __shfl_xor_sync(kFullMask, above, off);
+  if (lane == 0 && above) atomicAdd(&tile_above, above);
   __syncthreads();
   for (int i = threadIdx.x; i < kBins1; i += kThreads)
     if (hist[i]) atomicAdd(&rs.hist1[i], hist[i]);
@@ -333,9 +335,15 @@ __global__ void __launch_bounds__(kThreads) topk_offsets_kernel(int64_t d, void*
 }
 
 // 9. write the kept records of each tile in index order; e = +0 there.
+// Element order in a tile is row-major: row i (1024 elements) is split over
+// the 8 warps, 128 elements each, 4 per lane.  Each lane counts its keys
+// above T and equal to T, packed as (above | ties << 16) (a tile holds at
+// most 4096 of either), a warp shuffle scan ranks the lanes and one block
+// exchange of the 32 warp-row totals ranks the warps: one barrier per tile.
 template <bool KEEP_H>
 __global__ void __launch_bounds__(kThreads)
 topk_compact_kernel(const CompressArgs a, int64_t k, void* scratch) {
+  __shared__ uint32_t totals[kRows][kThreads / 32];
   const int row = blockIdx.y;
   const int worker = a.worker0 + row;
   float* e = a.e + (int64_t)worker * a.ld;
@@ -344,50 +352,78 @@ topk_compact_kernel(const CompressArgs a, int64_t k, void* scratch) {
   uint2* rec = reinterpret_cast<uint2*>(a.msg + (int64_t)row * a.msg_stride);
   RowScratch rs = row_scratch(scratch, a.d, row);
   const uint32_t T = rs.state[ST_T], need = rs.state[ST_NEED];
-  uint32_t tie_rank = rs.ties_before[blockIdx.x];
-  uint32_t out = rs.out_off[blockIdx.x];
+  const uint32_t tie_rank0 = rs.ties_before[blockIdx.x];
+  const uint32_t out0 = rs.out_off[blockIdx.x];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int64_t tile0 = (int64_t)blockIdx.x * kTile;
+  float v[kRows][4];
+  uint32_t gmask[kRows], tmask[kRows], excl[kRows];
+#pragma unroll
   for (int i = 0; i < kRows; ++i) {
     const int64_t j = tile0 + 4 * ((int64_t)i * kThreads + threadIdx.x);
-    float v[4] = {0.f, 0.f, 0.f, 0.f};
     int nvalid = 0;
     if (j + 3 < a.d) {
       const float4 x = __ldcs(reinterpret_cast<const float4*>(e + j));
-      v[0] = x.x; v[1] = x.y; v[2] = x.z; v[3] = x.w;
+      v[i][0] = x.x; v[i][1] = x.y; v[i][2] = x.z; v[i][3] = x.w;
       nvalid = 4;
     } else {
-      for (int q = 0; q < 4 && j + q < a.d; ++q) { v[q] = e[j + q]; nvalid = q + 1; }
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        v[i][q] = (j + q < a.d) ? e[j + q] : 0.f;
+        if (j + q < a.d) nvalid = q + 1;
+      }
     }
-    uint32_t tmask = 0, gmask = 0;
+    gmask[i] = 0;
+    tmask[i] = 0;
 #pragma unroll
     for (int q = 0; q < 4; ++q) {
       if (q < nvalid) {
-        const uint32_t key = key_of(v[q]);
-        if (key > T) gmask |= 1u << q;
-        else if (key == T) tmask |= 1u << q;
+        const uint32_t key = key_of(v[i][q]);
+        if (key > T) gmask[i] |= 1u << q;
+        else if (key == T) tmask[i] |= 1u << q;
       }
     }
-    uint32_t tie_total;
-    const uint32_t my_tie0 = tie_rank + block_exclusive_scan(__popc(tmask), &tie_total);
-    uint32_t smask = gmask, r = my_tie0;
+    const uint32_t packed = (uint32_t)__popc(gmask[i]) | ((uint32_t)__popc(tmask[i]) << 16);
+    uint32_t incl = packed;
 #pragma unroll
-    for (int q = 0; q < 4; ++q)
-      if (tmask & (1u << q)) {
-        if (r < need) smask |= 1u << q;
-        ++r;
-      }
-    uint32_t sel_total;
-    uint32_t pos = out + block_exclusive_scan(__popc(smask), &sel_total);
+    for (int off = 1; off < 32; off <<= 1) {
+      const uint32_t y = __shfl_up_sync(kFullMask, incl, off);
+      if (lane >= off) incl += y;
+    }
+    excl[i] = incl - packed;
+    if (lane == 31) totals[i][warp] = incl;
+  }
+  __syncthreads();
+  uint32_t before = 0;  // packed counts of the tile's earlier warp-rows
+#pragma unroll
+  for (int i = 0; i < kRows; ++i) {
+    uint32_t row_before = 0, row_total = 0;
+#pragma unroll
+    for (int w = 0; w < kThreads / 32; ++w) {
+      const uint32_t t = totals[i][w];
+      if (w < warp) row_before += t;
+      row_total += t;
+    }
+    const uint32_t pre = before + row_before + excl[i];
+    before += row_total;
+    if ((gmask[i] | tmask[i]) == 0) continue;
+    uint32_t R = tie_rank0 + (pre >> 16);  // global rank of this lane's first tie
+    const uint32_t sel_ties_before = min(R, need) - min(tie_rank0, need);
+    uint32_t pos = out0 + (pre & 0xFFFFu) + sel_ties_before;
+    const int64_t j = tile0 + 4 * ((int64_t)i * kThreads + threadIdx.x);
 #pragma unroll
     for (int q = 0; q < 4; ++q) {
-      if ((smask & (1u << q)) && pos < k) {  // pos < k always holds; the guard keeps writes in the message
-        rec[pos++] = make_uint2((uint32_t)(j + q), __float_as_uint(v[q]));
-        e[j + q] = __fsub_rn(v[q], v[q]);
+      bool take = (gmask[i] >> q) & 1u;
+      if ((tmask[i] >> q) & 1u) {
+        take = R < need;
+        ++R;
+      }
+      if (take && pos < k) {  // pos < k always holds; the guard keeps writes in the message
+        rec[pos++] = make_uint2((uint32_t)(j + q), __float_as_uint(v[i][q]));
+        e[j + q] = __fsub_rn(v[i][q], v[i][q]);
         if constexpr (KEEP_H) h[j + q] = __fadd_rn(__fmul_rn(a.lr, g[j + q]), e[j + q]);
       }
     }
-    tie_rank += tie_total;
-    out += sel_total;
   }
 }
 
