@@ -36,14 +36,14 @@ import time
 ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
-from paper_2010_13359_gb300.workloads import SIGN, SQUANT, TOPK, IDENTITY, WORKLOADS  # noqa: E402
+from paper_2010_13359_gb300.workloads import SIGN, SQUANT, TOPK, IDENTITY, QSGD, WORKLOADS  # noqa: E402
 
 METRIC = "updated params/sec (d*M per step) and achieved HBM GB/s vs GB300 roofline"
 UNIT = "params/s"
 FALLBACK_HBM_GBS = 6800.0
-COMPRESSOR_NAME = {SIGN: "sign", TOPK: "topk", SQUANT: "squant", IDENTITY: "identity"}
+COMPRESSOR_NAME = {SIGN: "sign", TOPK: "topk", SQUANT: "squant", IDENTITY: "identity", QSGD: "qsgd"}
 KERNEL_SOURCE = {SIGN: "dense_compress.cu", SQUANT: "dense_compress.cu", IDENTITY: "dense_compress.cu",
-                 TOPK: "topk.cu"}
+                 TOPK: "topk.cu", QSGD: "dense_compress.cu"}
 
 
 def parse_args():
@@ -93,7 +93,7 @@ def message_payload_bytes(wl) -> int:
     nb = -(-wl.d // wl.bucket)
     if wl.compressor == SIGN:
         return 4 * nb + 4 * (-(-wl.d // 32))
-    if wl.compressor == SQUANT:
+    if wl.compressor in (SQUANT, QSGD):
         return 4 * nb + 4 * (-(-wl.d * wl.bits // 32))
     if wl.compressor == TOPK:
         return 8 * wl.k
@@ -244,7 +244,7 @@ def oracle_step_time(wl, worker_fraction: float = 1.0, server_fraction: float = 
     import oracle
 
     def prefix(frac):
-        if wl.compressor in (SIGN, SQUANT):
+        if wl.compressor in (SIGN, SQUANT, QSGD):
             return min(wl.d, max(wl.bucket, int(wl.d * frac) // wl.bucket * wl.bucket))
         return min(wl.d, max(1, int(wl.d * frac)))
 
@@ -305,9 +305,9 @@ def workload_config(wl, args):
          "lr": wl.lr, "gradients": wl.dist, "lookahead": bool(args.lookahead),
          "l2": "flushed before every timed step (256 MB write); inputs also exceed L2",
          "parallelism": f"replicas{args.gpus}" if args.gpus > 1 else "single"}
-    if wl.compressor in (SIGN, SQUANT):
+    if wl.compressor in (SIGN, SQUANT, QSGD):
         c["bucket"] = wl.bucket
-    if wl.compressor == SQUANT:
+    if wl.compressor in (SQUANT, QSGD):
         c["bits"] = wl.bits
     if wl.compressor == TOPK:
         c["k"] = wl.k

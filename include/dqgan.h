@@ -15,9 +15,10 @@
  *     q_hat_t = (1/M) sum_m p_hat_t^(m);   w_t = w_{t-1} - q_hat_t
  *
  * Q is a delta-approximate compressor (Definition 1, Section 3.1): the scaled
- * sign of Section 2.4 (one l1 scale per bucket), top-k (Theorem 1), or the
- * b-bit stochastic quantiser of Hou et al. with an l_inf scale per bucket
- * (Section 2.4, proof of Theorem 2), or the identity.  The caller supplies
+ * sign of Section 2.4 (one l1 scale per bucket), top-k (Theorem 1), the b-bit
+ * stochastic quantiser of Hou et al. with an l_inf scale per bucket (Section
+ * 2.4, proof of Theorem 2), the same quantiser with QSGD's l2 scale (Eq.
+ * (qsgd)), or the identity.  The caller supplies
  * the stochastic gradients F(.; xi) -- the GAN forward/backward pass is not
  * part of this library.
  *
@@ -66,6 +67,7 @@ extern "C" {
 #define DQGAN_TOPK 1     /* k entries of largest |p_j|, ties to the lower index */
 #define DQGAN_SQUANT 2   /* b-bit stochastic quantiser, s_b = ||p_b||_inf */
 #define DQGAN_IDENTITY 3 /* no compression (uncompressed distributed OMD) */
+#define DQGAN_QSGD 4     /* b-bit stochastic quantiser, s_b = ||p_b||_2 (Eq. (qsgd)) */
 
 /* Config flags. */
 #define DQGAN_KEEP_LOOKAHEAD 1u /* keep h = eta F + e per worker for the lookahead */
@@ -77,10 +79,10 @@ extern "C" {
  *   k           top-k only: entries kept per worker, 1 <= k <= d.
  *   lr          step size eta of Algorithm 2, finite.
  *   M           workers, 1 <= M <= 4096.
- *   compressor  DQGAN_SIGN / TOPK / SQUANT / IDENTITY.
- *   bucket      sign and squant: elements per scale, a power of two in
+ *   compressor  DQGAN_SIGN / TOPK / SQUANT / IDENTITY / QSGD.
+ *   bucket      sign, squant, qsgd: elements per scale, a power of two in
  *               [32, 4096]; the last bucket may be partial.  Ignored otherwise.
- *   bits        squant only: bits per code b in {2, 4, 8}.
+ *   bits        squant, qsgd: bits per code b in {2, 4, 8}.
  *   flags       0 or DQGAN_KEEP_LOOKAHEAD.
  *   seed        64-bit key of the Philox4x32-10 draws of the squant rounding.
  *   cuda_stream the cudaStream_t all work is enqueued on (NULL: legacy stream).
@@ -111,6 +113,10 @@ typedef struct dqgan_handle dqgan_handle;
  *             (j*b) div 32; code = K + sign(p_j) * level, K = 2^(b-1) - 1,
  *             level in [0, K]; Q(p)_j = sign * fl(s_b * fl(level / K)) and +0
  *             for level 0.  Bits past d*b are 0.
+ *   QSGD:     as SQUANT with s_b = fl(sqrt(sum_j p_j^2)), the sum of squares
+ *             taken in the same fixed order as the SIGN l1 sum (chunks of 4,
+ *             ((x0^2+x1^2)+x2^2)+x3^2; lane l of 32 adds chunks l, l+32, ...;
+ *             xor rounds 16, 8, 4, 2, 1).
  *   TOPK:     k records {u32 index j, f32 p_j}, ascending index.
  *   IDENTITY: d fp32 values p_j.
  * Bytes between sections are not written by the library.

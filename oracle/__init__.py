@@ -7,8 +7,9 @@ may import this package; the product path never does.
 
 Conventions (restated, not shared, with the CUDA library):
 
-* compressors: 0 scaled sign, 1 top-k, 2 b-bit stochastic quantiser,
-  3 identity;
+* compressors: 0 scaled sign, 1 top-k, 2 b-bit stochastic quantiser with
+  the l_inf scale (Hou et al.), 3 identity, 4 b-bit stochastic quantiser
+  with the l2 scale (QSGD);
 * arrays are numpy ``float32`` (gradients, residuals, parameters) and
   ``uint8`` (messages);
 * ``step`` is the iteration index t of Algorithm 2, starting at 1.
@@ -22,8 +23,8 @@ import numpy as np
 
 from .build_oracle import build_oracle
 
-SIGN, TOPK, SQUANT, IDENTITY = 0, 1, 2, 3
-COMPRESSOR_NAMES = {"sign": SIGN, "topk": TOPK, "squant": SQUANT, "identity": IDENTITY}
+SIGN, TOPK, SQUANT, IDENTITY, QSGD = 0, 1, 2, 3, 4
+COMPRESSOR_NAMES = {"sign": SIGN, "topk": TOPK, "squant": SQUANT, "identity": IDENTITY, "qsgd": QSGD}
 
 
 class _OrcCfg(ctypes.Structure):
@@ -79,6 +80,10 @@ def lib() -> ctypes.CDLL:
         L.orc_sign_l1.restype = ctypes.c_float
         L.orc_sign_scale.argtypes = [f32p, ctypes.c_int64, ctypes.c_int32]
         L.orc_sign_scale.restype = ctypes.c_float
+        L.orc_qsgd_sumsq.argtypes = [f32p, ctypes.c_int64, ctypes.c_int32]
+        L.orc_qsgd_sumsq.restype = ctypes.c_float
+        L.orc_qsgd_scale.argtypes = [f32p, ctypes.c_int64, ctypes.c_int32]
+        L.orc_qsgd_scale.restype = ctypes.c_float
         L.orc_squant_decode.argtypes = [ctypes.c_int32, ctypes.c_float, ctypes.c_int32]
         L.orc_squant_decode.restype = ctypes.c_float
         L.orc_topk_select.argtypes = [f32p, ctypes.c_int64, ctypes.c_int64, u8p]
@@ -136,6 +141,16 @@ def sign_l1(x: np.ndarray, bucket: int) -> float:
 def sign_scale(x: np.ndarray, bucket: int) -> float:
     x = np.ascontiguousarray(x, dtype=np.float32)
     return float(lib().orc_sign_scale(_f32(x), x.size, bucket))
+
+
+def qsgd_sumsq(x: np.ndarray, bucket: int) -> float:
+    x = np.ascontiguousarray(x, dtype=np.float32)
+    return float(lib().orc_qsgd_sumsq(_f32(x), x.size, bucket))
+
+
+def qsgd_scale(x: np.ndarray, bucket: int) -> float:
+    x = np.ascontiguousarray(x, dtype=np.float32)
+    return float(lib().orc_qsgd_scale(_f32(x), x.size, bucket))
 
 
 def squant_decode(code: int, s: float, K: int) -> float:

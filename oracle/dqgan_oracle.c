@@ -31,7 +31,7 @@
 #error "the oracle must not be compiled with -ffast-math"
 #endif
 
-enum { ORC_SIGN = 0, ORC_TOPK = 1, ORC_SQUANT = 2, ORC_IDENTITY = 3 };
+enum { ORC_SIGN = 0, ORC_TOPK = 1, ORC_SQUANT = 2, ORC_IDENTITY = 3, ORC_QSGD = 4 };
 
 /* Counter word 3 of every Philox draw made by the stochastic quantiser. */
 #define ORC_TAG_SQUANT 0x51u
@@ -90,7 +90,7 @@ float orc_squant_uniform(uint64_t seed, int32_t worker, int64_t step, int64_t j)
 /* whole message is padded to a multiple of 256 bytes; padding is zero.      */
 /*   sign:     [nb fp32 scales][ceil(d/32) u32 words]                        */
 /*             bit (j mod 32) of word (j div 32) is 1 iff p_j < 0            */
-/*   squant:   [nb fp32 scales][ceil(d*b/32) u32 words]                      */
+/*   squant, qsgd: [nb fp32 scales][ceil(d*b/32) u32 words]                  */
 /*             code j sits in bits [(j*b) mod 32, +b) of word (j*b) div 32   */
 /*   top-k:    k records {u32 index, f32 value}, ascending index             */
 /*   identity: d fp32 values                                                 */
@@ -106,7 +106,8 @@ int64_t orc_layout(const orc_cfg* c, int64_t* off_scales, int64_t* off_payload) 
       *off_payload = round256(4 * nb);
       return round256(*off_payload + 4 * words);
     }
-    case ORC_SQUANT: {
+    case ORC_SQUANT:
+    case ORC_QSGD: {
       int64_t words = (c->d * c->bits + 31) / 32;
       *off_payload = round256(4 * nb);
       return round256(*off_payload + 4 * words);
@@ -162,6 +163,39 @@ float orc_sign_scale(const float* x, int64_t count, int32_t bucket) {
 }
 
 /* ------------------------------------------------------------------------ */
+/* QSGD scale (Section 2.4, Eq. (qsgd) of Alistarh et al.): the l2 norm of  */
+/* the bucket, s = fl(sqrt(sum_j x_j^2)).  The sum of squares is taken in    */
+/* the same fixed order as the scaled sign's l1 sum: a chunk's share is      */
+/* ((x0*x0 + x1*x1) + x2*x2) + x3*x3, lane l adds chunks l, l+32, ... in     */
+/* increasing order, then the five exchange rounds 16, 8, 4, 2, 1.          */
+/* ------------------------------------------------------------------------ */
+float orc_qsgd_sumsq(const float* x, int64_t count, int32_t bucket) {
+  float lane[32];
+  for (int l = 0; l < 32; ++l) lane[l] = 0.0f;
+  int64_t chunks = bucket / 4;
+  for (int64_t c = 0; c < chunks; ++c) {
+    float sq[4];
+    for (int q = 0; q < 4; ++q) {
+      int64_t j = 4 * c + q;
+      float v = (j < count) ? x[j] : 0.0f;
+      sq[q] = v * v;
+    }
+    float chunk_sum = ((sq[0] + sq[1]) + sq[2]) + sq[3];
+    lane[c % 32] = lane[c % 32] + chunk_sum;
+  }
+  for (int off = 16; off >= 1; off /= 2) {
+    float next[32];
+    for (int l = 0; l < 32; ++l) next[l] = lane[l] + lane[l ^ off];
+    for (int l = 0; l < 32; ++l) lane[l] = next[l];
+  }
+  return lane[0];
+}
+
+float orc_qsgd_scale(const float* x, int64_t count, int32_t bucket) {
+  return sqrtf(orc_qsgd_sumsq(x, count, bucket));
+}
+
+/* ------------------------------------------------------------------------ */
 /* m-bit stochastic quantiser of Hou et al. (Section 2.4, Appendix A proof   */
 /* of Theorem 2) with s = ||v_b||_inf per bucket and uniform levels          */
 /* B_r = r / K, K = 2^(b-1) - 1.  A code is the signed level shifted by K,   */
@@ -174,13 +208,19 @@ float orc_squant_decode(int32_t code, float s, int32_t K) {
   return level < 0 ? -mag : mag;
 }
 
+/* The b-bit stochastic rounding of one bucket with scale s: the l_inf norm
+ * for Hou et al.'s quantiser, the l2 norm for QSGD (Section 2.4). */
 static void squant_bucket(const orc_cfg* c, int32_t worker, int64_t step, int64_t start,
                           int64_t count, const float* p, float* s_out, int32_t* codes) {
   int32_t K = (1 << (c->bits - 1)) - 1;
   float s = 0.0f;
-  for (int64_t j = 0; j < count; ++j) {
-    float a = fabsf(p[j]);
-    if (a > s) s = a;
+  if (c->compressor == ORC_QSGD) {
+    s = orc_qsgd_scale(p, count, c->bucket);
+  } else {
+    for (int64_t j = 0; j < count; ++j) {
+      float a = fabsf(p[j]);
+      if (a > s) s = a;
+    }
   }
   *s_out = s;
   if (s == 0.0f) {
@@ -252,7 +292,8 @@ void orc_decode(const orc_cfg* c, const uint8_t* msg, float* q) {
       }
       break;
     }
-    case ORC_SQUANT: {
+    case ORC_SQUANT:
+    case ORC_QSGD: {
       const float* scales = (const float*)(msg + off_s);
       const uint32_t* words = (const uint32_t*)(msg + off_p);
       int32_t K = (1 << (c->bits - 1)) - 1;
@@ -321,7 +362,8 @@ void orc_worker_step(const orc_cfg* c, int32_t worker, int64_t step, const float
       }
       break;
     }
-    case ORC_SQUANT: {
+    case ORC_SQUANT:
+    case ORC_QSGD: {
       float* scales = (float*)(msg + off_s);
       uint32_t* words = (uint32_t*)(msg + off_p);
       int32_t K = (1 << (c->bits - 1)) - 1;

@@ -54,16 +54,17 @@ def q_topk(p: Vec, k: int) -> Vec:
     return [p[j] if j in keep else Fraction(0) for j in range(len(p))]
 
 
-def q_squant(p: Vec, bucket: int, bits: int, uniforms: Sequence[Fraction]) -> Vec:
-    """b-bit stochastic quantiser, s = max |p| per bucket, levels B_r = r/K.
+def q_squant(p: Vec, bucket: int, bits: int, uniforms: Sequence[Fraction], scales=None) -> Vec:
+    """b-bit stochastic quantiser, s = max |p| per bucket (or the given
+    per-bucket scales, e.g. QSGD's l2 norms), levels B_r = r/K.
 
     Element j rounds |p_j|/s * K up from level r = floor(.) with the draw
     uniforms[j]: up iff u < frac(|p_j| K / s)."""
     K = 2 ** (bits - 1) - 1
     out = []
-    for start in range(0, len(p), bucket):
+    for bi, start in enumerate(range(0, len(p), bucket)):
         blk = p[start:start + bucket]
-        s = max((abs(x) for x in blk), default=Fraction(0))
+        s = max((abs(x) for x in blk), default=Fraction(0)) if scales is None else scales[bi]
         for off, x in enumerate(blk):
             if s == 0:
                 out.append(Fraction(0))

@@ -6,6 +6,6 @@ the seeded synthetic inputs.
 """
 from . import dqgan  # noqa: F401
 from .dqgan import (  # noqa: F401
-    IDENTITY, KEEP_LOOKAHEAD, SIGN, SQUANT, TOPK, Config, DqganError, Handle, create, make_config,
+    IDENTITY, KEEP_LOOKAHEAD, QSGD, SIGN, SQUANT, TOPK, Config, DqganError, Handle, create, make_config,
     message_layout, validate_config,
 )

@@ -66,11 +66,12 @@ std::string check_config(const dqgan_config* c) {
   switch (c->compressor) {
     case DQGAN_SIGN:
     case DQGAN_SQUANT:
+    case DQGAN_QSGD:
       if (!is_pow2(c->bucket) || c->bucket < 32 || c->bucket > 4096) {
         snprintf(buf, sizeof buf, "bucket = %d is not a power of two in [32, 4096]", c->bucket);
         return buf;
       }
-      if (c->compressor == DQGAN_SQUANT && c->bits != 2 && c->bits != 4 && c->bits != 8) {
+      if (c->compressor != DQGAN_SIGN && c->bits != 2 && c->bits != 4 && c->bits != 8) {
         snprintf(buf, sizeof buf, "bits = %d not in {2, 4, 8}", c->bits);
         return buf;
       }
@@ -126,7 +127,8 @@ int run_compress(dqgan_handle* h, const dq::CompressArgs& a) {
   cudaError_t st = cudaSuccess;
   switch (h->cfg.compressor) {
     case DQGAN_SIGN: st = dq::launch_sign_compress(a, keep, h->stream, &h->launches); break;
-    case DQGAN_SQUANT: st = dq::launch_squant_compress(a, keep, h->stream, &h->launches); break;
+    case DQGAN_SQUANT: st = dq::launch_squant_compress(a, keep, false, h->stream, &h->launches); break;
+    case DQGAN_QSGD: st = dq::launch_squant_compress(a, keep, true, h->stream, &h->launches); break;
     case DQGAN_IDENTITY: st = dq::launch_identity_compress(a, keep, h->stream, &h->launches); break;
     case DQGAN_TOPK: {
       // scratch rows: one per concurrently compressed worker
@@ -178,7 +180,7 @@ int set_thread_error(int code, const char* msg) { return set_error(nullptr, code
 
 bool message_layout(const dqgan_config& c, Layout* out) {
   if (!check_config(&c).empty()) return false;
-  const int64_t nb = (c.compressor == DQGAN_SIGN || c.compressor == DQGAN_SQUANT)
+  const int64_t nb = (c.compressor == DQGAN_SIGN || c.compressor == DQGAN_SQUANT || c.compressor == DQGAN_QSGD)
                          ? (c.d + c.bucket - 1) / c.bucket
                          : 0;
   Layout L{0, 0, 0};
@@ -188,6 +190,7 @@ bool message_layout(const dqgan_config& c, Layout* out) {
       L.total = round_up(L.off_payload + 4 * ((c.d + 31) / 32), 256);
       break;
     case DQGAN_SQUANT:
+    case DQGAN_QSGD:
       L.off_payload = round_up(4 * nb, 256);
       L.total = round_up(L.off_payload + 4 * ((c.d * c.bits + 31) / 32), 256);
       break;
@@ -329,7 +332,7 @@ int dqgan_server_aggregate_update(dqgan_handle* h, const void* msgs_all, float* 
   s.sign_words_map = nullptr;
   s.squant_words_map = nullptr;
   const bool tma_sign = h->cfg.compressor == DQGAN_SIGN && h->cfg.bucket >= 1024 && h->cfg.M <= 32;
-  const bool tma_squant = h->cfg.compressor == DQGAN_SQUANT && h->cfg.M <= 32 &&
+  const bool tma_squant = (h->cfg.compressor == DQGAN_SQUANT || h->cfg.compressor == DQGAN_QSGD) && h->cfg.M <= 32 &&
                           h->cfg.bucket >= 32 * (32 / h->cfg.bits);
   if (tma_sign || tma_squant) {
     if (h->words_map_msgs != msgs_all) {
@@ -343,7 +346,8 @@ int dqgan_server_aggregate_update(dqgan_handle* h, const void* msgs_all, float* 
   cudaError_t st = cudaSuccess;
   switch (h->cfg.compressor) {
     case DQGAN_SIGN: st = dq::launch_sign_server(s, h->stream, &h->launches); break;
-    case DQGAN_SQUANT: st = dq::launch_squant_server(s, h->stream, &h->launches); break;
+    case DQGAN_SQUANT:
+    case DQGAN_QSGD: st = dq::launch_squant_server(s, h->stream, &h->launches); break;
     case DQGAN_IDENTITY: st = dq::launch_identity_server(s, h->stream, &h->launches); break;
     case DQGAN_TOPK: st = dq::launch_topk_server(s, h->stream, &h->launches); break;
   }

@@ -209,19 +209,24 @@ sign_compress_kernel(const CompressArgs a) {
 }
 
 // ---------------------------------------------------------------------------
-// b-bit stochastic quantiser of Hou et al. (Section 2.4, proof of Theorem 2):
-// s_b = max |p_j|, levels B_r = r / K, K = 2^(b-1) - 1; |p_j| K / s_b rounds
+// b-bit stochastic quantiser of Hou et al. (Section 2.4, proof of Theorem 2),
+// and QSGD's variant with the l2 scale (Eq. (qsgd)):
+// s_b = max |p_j| (or ||p_b||_2), levels B_r = r / K, K = 2^(b-1) - 1; |p_j| K / s_b rounds
 // up from r = floor(.) iff u < frac(.), u the 24-bit Philox4x32-10 draw of
 // counter (j div 4, worker, step, 0x51) word j mod 4; code = K +- level.
 // ---------------------------------------------------------------------------
-template <int CPT, int WPB, int BITS, bool KEEP_H>
+// L2 = false: s_b = max |p_j| (Hou et al.); L2 = true: s_b = fl(sqrt(sum p_j^2))
+// (QSGD), the sum of squares in the fixed chain order of the scaled sign.
+template <int CPT, int WPB, int BITS, bool KEEP_H, bool L2>
 __global__ void __launch_bounds__(32 * WPB * (WPB < 4 ? 4 / WPB : 1))
 squant_compress_kernel(const CompressArgs a) {
   constexpr int K = (1 << (BITS - 1)) - 1;
   constexpr bool HOLD = KEEP_H && CPT <= 8;
   constexpr int BPC = WPB < 4 ? 4 / WPB : 1;  // buckets per CTA (CTA = max(4, WPB) warps)
+  constexpr int CHAIN = 32 * CPT * WPB;
   __shared__ float level_value[K + 1];        // fl(r / K)
   __shared__ float warp_max[BPC * WPB];
+  __shared__ float chain[(L2 && WPB > 1) ? BPC * CHAIN : 1];
   for (int r = threadIdx.x; r <= K; r += blockDim.x) level_value[r] = __fdiv_rn((float)r, (float)K);
   __syncthreads();
 
@@ -256,20 +261,53 @@ squant_compress_kernel(const CompressArgs a) {
       for (int q = 0; q < 4; ++q) p[i][q] = 0.f;
   }
 
-  // s = max |p| over the bucket (exact in any order)
   float mx = 0.f;
+  if constexpr (!L2) {
+    // s = max |p| over the bucket (exact in any order)
 #pragma unroll
-  for (int i = 0; i < CPT; ++i)
+    for (int i = 0; i < CPT; ++i)
 #pragma unroll
-    for (int q = 0; q < 4; ++q) mx = fmaxf(mx, fabsf(p[i][q]));
+      for (int q = 0; q < 4; ++q) mx = fmaxf(mx, fabsf(p[i][q]));
 #pragma unroll
-  for (int off = 16; off >= 1; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(kFullMask, mx, off));
-  if constexpr (WPB > 1) {
-    if (lane == 0) warp_max[warp] = mx;
-    __syncthreads();
+    for (int off = 16; off >= 1; off >>= 1) mx = fmaxf(mx, __shfl_xor_sync(kFullMask, mx, off));
+    if constexpr (WPB > 1) {
+      if (lane == 0) warp_max[warp] = mx;
+      __syncthreads();
 #pragma unroll
-    for (int w = 0; w < WPB; ++w) mx = fmaxf(mx, warp_max[slot * WPB + w]);
-    if (!valid) return;
+      for (int w = 0; w < WPB; ++w) mx = fmaxf(mx, warp_max[slot * WPB + w]);
+      if (!valid) return;
+    }
+  } else {
+    // s = sqrt of the sum of squares in the chain order
+    float cs[CPT];
+#pragma unroll
+    for (int i = 0; i < CPT; ++i)
+      cs[i] = __fadd_rn(__fadd_rn(__fadd_rn(__fmul_rn(p[i][0], p[i][0]), __fmul_rn(p[i][1], p[i][1])),
+                                  __fmul_rn(p[i][2], p[i][2])),
+                        __fmul_rn(p[i][3], p[i][3]));
+    float acc = 0.f;
+    if constexpr (WPB == 1) {
+#pragma unroll
+      for (int i = 0; i < CPT; ++i) acc = __fadd_rn(acc, cs[i]);
+#pragma unroll
+      for (int off = 16; off >= 1; off >>= 1) acc = __fadd_rn(acc, __shfl_xor_sync(kFullMask, acc, off));
+      mx = __fsqrt_rn(acc);
+    } else {
+      float* ch = chain + slot * CHAIN;
+#pragma unroll
+      for (int i = 0; i < CPT; ++i) ch[(row0 + i) * 32 + lane] = cs[i];
+      __syncthreads();
+      if (wib == 0) {
+#pragma unroll 8
+        for (int r = 0; r < CPT * WPB; ++r) acc = __fadd_rn(acc, ch[r * 32 + lane]);
+#pragma unroll
+        for (int off = 16; off >= 1; off >>= 1) acc = __fadd_rn(acc, __shfl_xor_sync(kFullMask, acc, off));
+        if (lane == 0) warp_max[slot * WPB] = __fsqrt_rn(acc);
+      }
+      __syncthreads();
+      mx = warp_max[slot * WPB];
+      if (!valid) return;
+    }
   }
   const float s = mx;
   if (wib == 0 && lane == 0) reinterpret_cast<float*>(msg)[b] = s;
@@ -375,22 +413,25 @@ cudaError_t sign_dispatch_keep(const CompressArgs& a, bool keep_h, cudaStream_t 
   return cudaGetLastError();
 }
 
-template <int CPT, int WPB, int BITS>
+template <int CPT, int WPB, int BITS, bool L2>
 cudaError_t squant_dispatch_keep(const CompressArgs& a, bool keep_h, cudaStream_t stream) {
   constexpr int BPC = WPB < 4 ? 4 / WPB : 1;
   constexpr int THREADS = 32 * WPB * BPC;
   const dim3 grid((unsigned)((a.nb + BPC - 1) / BPC), (unsigned)a.nworkers);
-  if (keep_h) squant_compress_kernel<CPT, WPB, BITS, true><<<grid, THREADS, 0, stream>>>(a);
-  else squant_compress_kernel<CPT, WPB, BITS, false><<<grid, THREADS, 0, stream>>>(a);
+  if (keep_h) squant_compress_kernel<CPT, WPB, BITS, true, L2><<<grid, THREADS, 0, stream>>>(a);
+  else squant_compress_kernel<CPT, WPB, BITS, false, L2><<<grid, THREADS, 0, stream>>>(a);
   return cudaGetLastError();
 }
 
 template <int CPT, int WPB>
-cudaError_t squant_dispatch_bits(const CompressArgs& a, bool keep_h, cudaStream_t stream) {
+cudaError_t squant_dispatch_bits(const CompressArgs& a, bool keep_h, bool l2, cudaStream_t stream) {
   switch (a.bits) {
-    case 2: return squant_dispatch_keep<CPT, WPB, 2>(a, keep_h, stream);
-    case 4: return squant_dispatch_keep<CPT, WPB, 4>(a, keep_h, stream);
-    case 8: return squant_dispatch_keep<CPT, WPB, 8>(a, keep_h, stream);
+    case 2: return l2 ? squant_dispatch_keep<CPT, WPB, 2, true>(a, keep_h, stream)
+                      : squant_dispatch_keep<CPT, WPB, 2, false>(a, keep_h, stream);
+    case 4: return l2 ? squant_dispatch_keep<CPT, WPB, 4, true>(a, keep_h, stream)
+                      : squant_dispatch_keep<CPT, WPB, 4, false>(a, keep_h, stream);
+    case 8: return l2 ? squant_dispatch_keep<CPT, WPB, 8, true>(a, keep_h, stream)
+                      : squant_dispatch_keep<CPT, WPB, 8, false>(a, keep_h, stream);
   }
   return cudaErrorInvalidValue;
 }
@@ -413,16 +454,16 @@ cudaError_t launch_sign_compress(const CompressArgs& a, bool keep_h, cudaStream_
   return st;
 }
 
-cudaError_t launch_squant_compress(const CompressArgs& a, bool keep_h, cudaStream_t stream,
+cudaError_t launch_squant_compress(const CompressArgs& a, bool keep_h, bool l2, cudaStream_t stream,
                                    uint64_t* launches) {
   cudaError_t st;
   switch (a.bucket) {
-    case 32: case 64: case 128: st = squant_dispatch_bits<1, 1>(a, keep_h, stream); break;
-    case 256: st = squant_dispatch_bits<2, 1>(a, keep_h, stream); break;
-    case 512: st = squant_dispatch_bits<4, 1>(a, keep_h, stream); break;
-    case 1024: st = squant_dispatch_bits<8, 1>(a, keep_h, stream); break;
-    case 2048: st = squant_dispatch_bits<2, 8>(a, keep_h, stream); break;
-    case 4096: st = squant_dispatch_bits<2, 16>(a, keep_h, stream); break;
+    case 32: case 64: case 128: st = squant_dispatch_bits<1, 1>(a, keep_h, l2, stream); break;
+    case 256: st = squant_dispatch_bits<2, 1>(a, keep_h, l2, stream); break;
+    case 512: st = squant_dispatch_bits<4, 1>(a, keep_h, l2, stream); break;
+    case 1024: st = squant_dispatch_bits<8, 1>(a, keep_h, l2, stream); break;
+    case 2048: st = squant_dispatch_bits<2, 8>(a, keep_h, l2, stream); break;
+    case 4096: st = squant_dispatch_bits<2, 16>(a, keep_h, l2, stream); break;
     default: return cudaErrorInvalidValue;
   }
   *launches += 1;

@@ -90,7 +90,8 @@ struct TopkScratch {
 // kernels it launched to *launches and returns the launch status.
 cudaError_t launch_sign_compress(const CompressArgs& a, bool keep_h, cudaStream_t stream,
                                  uint64_t* launches);
-cudaError_t launch_squant_compress(const CompressArgs& a, bool keep_h, cudaStream_t stream,
+// l2_scale = false: Hou et al.'s max-abs scale; true: QSGD's l2 scale.
+cudaError_t launch_squant_compress(const CompressArgs& a, bool keep_h, bool l2_scale, cudaStream_t stream,
                                    uint64_t* launches);
 cudaError_t launch_identity_compress(const CompressArgs& a, bool keep_h, cudaStream_t stream,
                                      uint64_t* launches);

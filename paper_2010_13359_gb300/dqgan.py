@@ -21,7 +21,7 @@ ERR_CUDA = -3
 ERR_UNSUPPORTED = -4
 ERR_TIMEOUT = -5
 
-SIGN, TOPK, SQUANT, IDENTITY = 0, 1, 2, 3
+SIGN, TOPK, SQUANT, IDENTITY, QSGD = 0, 1, 2, 3, 4
 KEEP_LOOKAHEAD = 1
 
 

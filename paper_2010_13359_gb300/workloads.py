@@ -25,7 +25,7 @@ import math
 
 import numpy as np
 
-SIGN, TOPK, SQUANT, IDENTITY = 0, 1, 2, 3
+SIGN, TOPK, SQUANT, IDENTITY, QSGD = 0, 1, 2, 3, 4
 
 
 @dataclasses.dataclass(frozen=True)
@@ -149,8 +149,8 @@ def _dcgan(name, compressor, **kw):
                     n_segments=16, std_range=(1e-4, 1e-1), **kw)
 
 
-def _resnet(name, bits):
-    return Workload(name=name, d=25_000_000, M=16, compressor=SQUANT, bucket=512, bits=bits,
+def _resnet(name, bits, compressor=SQUANT):
+    return Workload(name=name, d=25_000_000, M=16, compressor=compressor, bucket=512, bits=bits,
                     steps=50, n_segments=64, std_range=(1e-5, 1e-1))
 
 
@@ -166,6 +166,8 @@ WORKLOADS = {
     "resnet_squant_b2": _resnet("resnet_squant_b2", 2),
     "resnet_squant_b4": _resnet("resnet_squant_b4", 4),
     "resnet_squant_b8": _resnet("resnet_squant_b8", 8),
+    # Same vector with QSGD's l2-scaled quantiser (Eq. (qsgd)), 8 bits.
+    "resnet_qsgd_b8": _resnet("resnet_qsgd_b8", 8, QSGD),
     # Heavy-tailed stress case: d = 1e8, M = 32, sign per 4096, Student-t(3) * 1e-3.
     "stress_sign": Workload(name="stress_sign", d=100_000_000, M=32, compressor=SIGN, bucket=4096,
                             steps=20, n_segments=1, segment_sizes=(100_000_000,),

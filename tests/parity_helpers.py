@@ -36,7 +36,7 @@ def sections(ocfg: oracle.Config, msg: np.ndarray) -> dict:
     off_s, off_p, total = oracle.layout(ocfg)
     d = ocfg.d
     msg = np.asarray(msg, np.uint8)
-    if ocfg.compressor in (oracle.SIGN, oracle.SQUANT):
+    if ocfg.compressor in (oracle.SIGN, oracle.SQUANT, oracle.QSGD):
         nb = -(-d // ocfg.bucket)
         nwords = -(-d // 32) if ocfg.compressor == oracle.SIGN else -(-d * ocfg.bits // 32)
         return {"scales": msg[off_s:off_s + 4 * nb].view(np.uint32),
@@ -74,7 +74,7 @@ def slice_messages(ocfg: oracle.Config, msgs: np.ndarray, a: int, b: int):
     """Sub-messages covering elements [a, b) (bucket- and word-aligned a) and
     the matching oracle config, so the oracle server can be run on a slice of
     a full-size problem.  Pure byte slicing: no arithmetic of the method."""
-    assert ocfg.compressor in (oracle.SIGN, oracle.SQUANT)
+    assert ocfg.compressor in (oracle.SIGN, oracle.SQUANT, oracle.QSGD)
     assert a % ocfg.bucket == 0 and (b % ocfg.bucket == 0 or b == ocfg.d)
     sub = oracle.Config(d=b - a, M=ocfg.M, compressor=ocfg.compressor, lr=ocfg.lr, bucket=ocfg.bucket,
                         k=ocfg.k, bits=ocfg.bits, seed=ocfg.seed)

@@ -108,6 +108,9 @@ EDGE_CASES = [
     (oracle.SQUANT, dict(bucket=64, bits=2)),
     (oracle.SQUANT, dict(bucket=512, bits=4)),
     (oracle.SQUANT, dict(bucket=4096, bits=8)),
+    (oracle.QSGD, dict(bucket=32, bits=4)),
+    (oracle.QSGD, dict(bucket=512, bits=8)),
+    (oracle.QSGD, dict(bucket=4096, bits=2)),
     (oracle.TOPK, dict(k=1)),
     (oracle.TOPK, dict(k=7)),
     (oracle.TOPK, dict(k=-1)),  # k = d
@@ -117,7 +120,7 @@ EDGE_CASES = [
 
 def _case_id(c):
     comp, kw = c
-    name = {0: "sign", 1: "topk", 2: "squant", 3: "identity"}[comp]
+    name = {0: "sign", 1: "topk", 2: "squant", 3: "identity", 4: "qsgd"}[comp]
     return name + "".join(f"-{k}{v}" for k, v in kw.items())
 
 
@@ -134,6 +137,7 @@ def test_edge_sizes(P, case, d):
 
 @pytest.mark.parametrize("kind", ["ties", "zeros"])
 @pytest.mark.parametrize("case", [(oracle.SIGN, dict(bucket=256)), (oracle.SQUANT, dict(bucket=256, bits=4)),
+                                  (oracle.QSGD, dict(bucket=1024, bits=8)),
                                   (oracle.TOPK, dict(k=300)), (oracle.TOPK, dict(k=5000))], ids=_case_id)
 def test_degenerate_values(P, case, kind):
     comp, kw = case
@@ -142,6 +146,7 @@ def test_degenerate_values(P, case, kind):
 
 
 @pytest.mark.parametrize("case", [(oracle.SIGN, dict(bucket=1024)), (oracle.SQUANT, dict(bucket=512, bits=8)),
+                                  (oracle.QSGD, dict(bucket=2048, bits=4)),
                                   (oracle.TOPK, dict(k=2000)), (oracle.IDENTITY, dict())], ids=_case_id)
 def test_per_worker_calls_match_batched(P, case):
     """dqgan_worker_compress per worker gives the same as the batched call."""
@@ -153,7 +158,8 @@ def test_per_worker_calls_match_batched(P, case):
 @pytest.mark.parametrize("M,comp,bucket", [
     (1, oracle.SIGN, 512), (5, oracle.SIGN, 512), (8, oracle.SIGN, 1024), (32, oracle.SIGN, 2048),
     (33, oracle.SIGN, 4096), (70, oracle.SIGN, 1024), (3, oracle.SIGN, 256), (40, oracle.SIGN, 64),
-    (20, oracle.SQUANT, 512), (33, oracle.IDENTITY, 512), (9, oracle.TOPK, 512)])
+    (20, oracle.SQUANT, 512), (33, oracle.IDENTITY, 512), (9, oracle.TOPK, 512), (6, oracle.QSGD, 512),
+    (40, oracle.QSGD, 1024)])
 def test_worker_counts(P, M, comp, bucket):
     """Non-power-of-two M, M above 32 (several 32-worker slabs in the sign
     server), every server path."""

@@ -147,6 +147,13 @@ def test_resnet_squant_sampled(P, bits):
                 locked_steps={wl.steps})
 
 
+def test_resnet_qsgd_sampled(P):
+    wl = WORKLOADS["resnet_qsgd_b8"]
+    d = wl.d
+    slices = [(0, 512 * 4096), ((d - 1_000_000) // 512 * 512, d)]
+    sampled_run(P, wl, steps=10, free_steps=2, sample=[0, wl.M - 1], slices=slices, locked_steps={10})
+
+
 def test_stress_sign_sampled(P):
     wl = WORKLOADS["stress_sign"]
     d = wl.d

@@ -610,3 +610,102 @@ def test_bilinear_game_lookahead_converges_where_plain_step_spirals():
     assert run(False, oracle.SIGN) > 5 * n0
     assert run(True, oracle.IDENTITY) < 0.25 * n0
     assert run(True, oracle.SIGN) < 0.25 * n0
+
+
+# ---------------------------------------------------------------------------
+# QSGD: the b-bit stochastic quantiser with the l2 scale (Section 2.4, Eq. (qsgd))
+# ---------------------------------------------------------------------------
+
+@pytest.mark.parametrize("bucket", [32, 512, 4096])
+@pytest.mark.parametrize("count_frac", [1.0, 0.41])
+def test_qsgd_scale_is_the_l2_norm(bucket, count_frac):
+    count = max(1, int(bucket * count_frac))
+    x = (rng(bucket * 7 + count).standard_normal(count) * np.exp(rng(count + 1).uniform(-6, 2, count)))
+    x = x.astype(np.float32)
+    got = Fraction(oracle.qsgd_sumsq(x, bucket))
+    want = exact.sq_norm(exact.frac_vec(x))
+    # every square rounds once and every addition once: (n + 1) u relative
+    assert abs(got - want) <= Fraction(count + 1) * Fraction(U32) * want * Fraction(11, 10)
+    s = oracle.qsgd_scale(x, bucket)
+    assert s == np.float32(np.sqrt(np.float32(oracle.qsgd_sumsq(x, bucket))))
+    assert abs(s - math.sqrt(float(want))) <= 4 * U32 * s
+    for j in [0, count // 3, count - 1]:
+        y = x.copy()
+        y[j] = np.float32(1e5)
+        assert oracle.qsgd_sumsq(y, bucket) >= 1e10
+
+
+@pytest.mark.parametrize("bits", [2, 4, 8])
+def test_qsgd_moments_by_exact_enumeration(bits):
+    """With the l2 scale (>= every |v_i|) the quantiser is unbiased and has the
+    second moment of the proof of Theorem 2, element by element."""
+    K = 2 ** (bits - 1) - 1
+    n = 10
+    v32 = rng(40 + bits).standard_normal(n).astype(np.float32)
+    s = Fraction(oracle.qsgd_scale(v32, 16))
+    v = exact.frac_vec(v32)
+    assert all(abs(x) <= s for x in v)
+    q_up = exact.q_squant(v, n, bits, [Fraction(0)] * n, scales=[s])
+    q_dn = exact.q_squant(v, n, bits, [Fraction(1)] * n, scales=[s])
+    for i, x in enumerate(v):
+        t = abs(x) * K / s
+        r = t.numerator // t.denominator
+        f = t - r
+        B_r, B_r1 = Fraction(r, K), Fraction(min(r + 1, K), K)
+        mean = f * q_up[i] + (1 - f) * q_dn[i]
+        second = f * q_up[i] ** 2 + (1 - f) * q_dn[i] ** 2
+        assert mean == x
+        assert second == abs(x) * s * (B_r + B_r1) - B_r * B_r1 * s * s
+
+
+@pytest.mark.parametrize("bits", [2, 4, 8])
+def test_qsgd_oracle_codes_match_exact_rule(bits):
+    d, bucket, seed = 2000, 256, 9
+    cfg = oracle.Config(d=d, M=1, compressor=oracle.QSGD, lr=1.0, bucket=bucket, bits=bits, seed=seed)
+    x = (rng(bits + 50).standard_normal(d) * np.exp(rng(51).uniform(-3, 1, d))).astype(np.float32)
+    e = np.zeros(d, np.float32)
+    msg = oracle.worker_step(cfg, 2, 6, x, e)
+    off_s, off_p, _ = oracle.layout(cfg)
+    K = 2 ** (bits - 1) - 1
+    nb = -(-d // bucket)
+    scales = msg[off_s:off_s + 4 * nb].view(np.float32)
+    words = msg[off_p:].view(np.uint32)
+    mismatches = 0
+    for b in range(nb):
+        blk = x[b * bucket:(b + 1) * bucket]
+        assert scales[b] == np.float32(oracle.qsgd_scale(blk, bucket))
+        s = Fraction(float(scales[b]))
+        for off, xv in enumerate(blk):
+            j = b * bucket + off
+            code = (int(words[(j * bits) >> 5]) >> ((j * bits) & 31)) & ((1 << bits) - 1)
+            u = Fraction(oracle.squant_uniform(seed, 2, 6, j))
+            t = abs(Fraction(float(xv))) * K / s
+            r = t.numerator // t.denominator
+            level = min(r + (1 if u < t - r else 0), K)
+            want = K - level if xv < 0 else K + level
+            if code != want:
+                mismatches += 1
+                assert abs(code - want) == 1
+    assert mismatches <= max(2, d // 500)
+    np.testing.assert_array_equal(e, x - oracle.decode(cfg, msg))
+
+
+@pytest.mark.parametrize("bits", [4, 8])
+def test_qsgd_unbiased_and_variance_bound_over_philox_streams(bits):
+    """Monte Carlo over 2048 steps: mean of Q(v) is v, and the expected residual
+    respects QSGD's variance bound min(n/K^2, sqrt(n)/K) ||v||^2 (Alistarh et
+    al., the compressor Eq. (qsgd) cites) and is below ||v||^2 (delta > 0)."""
+    n = 64
+    cfg = oracle.Config(d=n, M=1, compressor=oracle.QSGD, lr=1.0, bucket=n, bits=bits, seed=321)
+    v = rng(60 + bits).standard_normal(n).astype(np.float32)
+    T = 2048
+    qs = np.empty((T, n), np.float64)
+    for t in range(T):
+        qs[t] = oracle.decode(cfg, oracle.worker_step(cfg, 0, t + 1, v, np.zeros(n, np.float32)))
+    K = 2 ** (bits - 1) - 1
+    s = float(np.linalg.norm(v.astype(np.float64)))
+    assert np.all(np.abs(qs.mean(0) - v) <= 5 * (s / K / 2) / math.sqrt(T) + 1e-6)
+    resid = np.sum((qs - v) ** 2, 1).mean()
+    vv = np.sum(v.astype(np.float64) ** 2)
+    assert resid <= min(n / K ** 2, math.sqrt(n) / K) * vv * 1.1
+    assert resid < vv
