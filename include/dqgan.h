@@ -189,8 +189,26 @@ DQGAN_API int dqgan_server_aggregate_update(dqgan_handle* h, const void* msgs_al
  */
 DQGAN_API int dqgan_worker_lookahead(dqgan_handle* h, int32_t i, const float* params, float* out_w_half);
 
-/* Wait for the handle's stream; DQGAN_ERR_CUDA if any enqueued work failed. */
+/* Wait for the handle's stream.  DQGAN_ERR_CUDA if any enqueued work failed;
+ * DQGAN_ERR_TIMEOUT if a bounded device-side wait of an enqueued kernel gave
+ * up since the last call (the error word is then cleared, the handle and the
+ * CUDA context stay usable, and the results of the steps since the last
+ * successful synchronize are undefined). */
 DQGAN_API int dqgan_synchronize(dqgan_handle* h);
+
+/*
+ * Failure-detection self-test.  The paper has no counterpart: it checks the
+ * library's own fault handling.  Enqueues on the handle's stream one kernel
+ * that initialises an mbarrier expecting one arrival, polls it `polls` times
+ * (each poll may sleep up to 0.5 us; 0 means the limit every library wait
+ * uses, 2^21 polls, about a second) while nothing arrives, then sets the
+ * time-out bit of the handle's error word and returns -- the same path every
+ * bounded wait in the library takes when a transfer never completes.  The
+ * next dqgan_synchronize returns DQGAN_ERR_TIMEOUT and clears the word; the
+ * residuals, lookahead offsets and step counter are untouched.
+ * Returns DQGAN_OK, DQGAN_ERR_INVALID_ARG (polls above 2^21) or DQGAN_ERR_CUDA.
+ */
+DQGAN_API int dqgan_selftest_wait_timeout(dqgan_handle* h, uint32_t polls);
 
 /* Copy worker i's residual e^(i) (d fp32) to / from dst / src, which may be a
  * host or a device pointer (any alignment).  Synchronous. */

@@ -385,6 +385,17 @@ int dqgan_synchronize(dqgan_handle* h) {
   return DQGAN_OK;
 }
 
+int dqgan_selftest_wait_timeout(dqgan_handle* h, uint32_t polls) {
+  if (!h) return set_error(nullptr, DQGAN_ERR_INVALID_ARG, "handle is NULL");
+  const uint32_t max_polls = dq::wait_selftest_max_polls();
+  if (polls > max_polls)
+    return set_error(h, DQGAN_ERR_INVALID_ARG, "polls must be at most %u", max_polls);
+  if (polls == 0) polls = max_polls;
+  const cudaError_t st = dq::launch_wait_selftest(polls, h->err_word, h->stream, &h->launches);
+  if (st != cudaSuccess) return cuda_fail(h, st, "self-test launch");
+  return DQGAN_OK;
+}
+
 int dqgan_get_residual(dqgan_handle* h, int32_t i, float* dst) {
   if (!h) return set_error(nullptr, DQGAN_ERR_INVALID_ARG, "handle is NULL");
   if (int r = check_worker(h, i)) return r;

@@ -105,6 +105,11 @@ cudaError_t launch_squant_server(const ServerArgs& s, cudaStream_t stream, uint6
 cudaError_t launch_identity_server(const ServerArgs& s, cudaStream_t stream, uint64_t* launches);
 cudaError_t launch_topk_server(const ServerArgs& s, cudaStream_t stream, uint64_t* launches);
 
+// Enqueues one kernel that polls an mbarrier nobody arrives on `polls` times
+// and then sets kErrTimeout in *err (the bounded-wait path, on demand).
+cudaError_t launch_wait_selftest(uint32_t polls, uint32_t* err, cudaStream_t stream, uint64_t* launches);
+uint32_t wait_selftest_max_polls();
+
 cudaError_t launch_lookahead(const float* w, const float* h, float* out, int64_t d,
                              cudaStream_t stream, uint64_t* launches);
 

@@ -89,6 +89,7 @@ def load_library(path: str = LIBRARY) -> ctypes.CDLL:
         "dqgan_launch_count": (u64, [H]),
         "dqgan_last_error": (ctypes.c_char_p, [H]),
         "dqgan_topk_compress_noalloc": (ctypes.c_int, [P, P, P, i64, i64, ctypes.c_float, P]),
+        "dqgan_selftest_wait_timeout": (ctypes.c_int, [H, ctypes.c_uint32]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(L, name)
@@ -185,6 +186,11 @@ class Handle:
 
     def synchronize(self) -> None:
         _check(load_library().dqgan_synchronize(self._h), self._h)
+
+    def selftest_wait_timeout(self, polls: int = 0) -> None:
+        """Enqueue the bounded-wait self-test; the next synchronize() raises
+        DqganError with status ERR_TIMEOUT."""
+        _check(load_library().dqgan_selftest_wait_timeout(self._h, polls), self._h)
 
     # -- state ----------------------------------------------------------------
     def get_residual(self, i: int, dst) -> None:

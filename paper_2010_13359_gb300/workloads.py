@@ -175,6 +175,20 @@ WORKLOADS = {
 }
 
 
+def game_diag_np(d: int, seed: int, lo: float = 0.5, hi: float = 1.5) -> np.ndarray:
+    """The positive diagonal D (length d/2) of the bilinear game x^T D y."""
+    rng = np.random.Generator(np.random.Philox(key=seed))
+    return rng.uniform(lo, hi, size=d // 2).astype(np.float32)
+
+
+def game_noise_np(d: int, seed: int, step: int, worker: int, std: float) -> np.ndarray:
+    """The operator noise sigma * xi of worker `worker` at step `step`."""
+    if std == 0.0:
+        return np.zeros(d, np.float32)
+    rng = np.random.Generator(np.random.Philox(key=(seed * 7919 + step * 131 + worker) & 0xFFFFFFFF))
+    return (rng.standard_normal(d, dtype=np.float32) * np.float32(std)).astype(np.float32)
+
+
 def sweep_workload(log2_d: int) -> Workload:
     """d = 2^log2_d, M = 8, sign per 1024, DCGAN gradient distribution."""
     return _dcgan(f"sweep_2^{log2_d}", SIGN, bucket=1024).replace(
