@@ -131,7 +131,7 @@ int run_compress(dqgan_handle* h, const dq::CompressArgs& a) {
     case DQGAN_QSGD: st = dq::launch_squant_compress(a, keep, true, h->stream, &h->launches); break;
     case DQGAN_IDENTITY: st = dq::launch_identity_compress(a, keep, h->stream, &h->launches); break;
     case DQGAN_TOPK: {
-      // scratch rows: one per concurrently compressed worker
+      // scratch rows: one per worker
       st = dq::launch_topk_compress(a, h->cfg.k, keep, h->scratch, h->stream, &h->launches);
       break;
     }
@@ -349,7 +349,7 @@ int dqgan_server_aggregate_update(dqgan_handle* h, const void* msgs_all, float* 
     case DQGAN_SQUANT:
     case DQGAN_QSGD: st = dq::launch_squant_server(s, h->stream, &h->launches); break;
     case DQGAN_IDENTITY: st = dq::launch_identity_server(s, h->stream, &h->launches); break;
-    case DQGAN_TOPK: st = dq::launch_topk_server(s, h->stream, &h->launches); break;
+    case DQGAN_TOPK: st = dq::launch_topk_server(s, h->scratch, h->stream, &h->launches); break;
   }
   if (st != cudaSuccess) return cuda_fail(h, st, "server launch");
   h->t += 1;

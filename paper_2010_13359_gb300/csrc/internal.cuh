@@ -80,12 +80,6 @@ struct ServerArgs {
 bool encode_words_map(const uint8_t* msgs, int64_t msg_stride, int64_t off_payload, int64_t payload_words,
                       int32_t M, bool swizzle128, CUtensorMap* out);
 
-// Scratch of the top-k path for `nworkers` concurrent workers.
-struct TopkScratch {
-  void* base;
-  size_t bytes;
-};
-
 // Kernel launchers: each enqueues its kernels on `stream`, adds the number of
 // kernels it launched to *launches and returns the launch status.
 cudaError_t launch_sign_compress(const CompressArgs& a, bool keep_h, cudaStream_t stream,
@@ -96,14 +90,20 @@ cudaError_t launch_squant_compress(const CompressArgs& a, bool keep_h, bool l2_s
 cudaError_t launch_identity_compress(const CompressArgs& a, bool keep_h, cudaStream_t stream,
                                      uint64_t* launches);
 
+// Scratch of the top-k path: one row per worker (kept across calls: the
+// candidate threshold carried from call to call lives there) and the
+// server's record-range table for `nworkers` messages.
 size_t topk_scratch_bytes(int64_t d, int32_t nworkers);
+// Leading bytes of a row that must be zero before a first call; the rest of
+// the row needs no clearing.
+size_t topk_scratch_clear_bytes(int64_t d);
 cudaError_t launch_topk_compress(const CompressArgs& a, int64_t k, bool keep_h, void* scratch,
                                  cudaStream_t stream, uint64_t* launches);
 
 cudaError_t launch_sign_server(const ServerArgs& s, cudaStream_t stream, uint64_t* launches);
 cudaError_t launch_squant_server(const ServerArgs& s, cudaStream_t stream, uint64_t* launches);
 cudaError_t launch_identity_server(const ServerArgs& s, cudaStream_t stream, uint64_t* launches);
-cudaError_t launch_topk_server(const ServerArgs& s, cudaStream_t stream, uint64_t* launches);
+cudaError_t launch_topk_server(const ServerArgs& s, void* scratch, cudaStream_t stream, uint64_t* launches);
 
 // Enqueues one kernel that polls an mbarrier nobody arrives on `polls` times
 // and then sets kErrTimeout in *err (the bounded-wait path, on demand).

@@ -21,10 +21,10 @@
 namespace dq {
 namespace {
 
-// Largest d the fixed scratch supports, and the scratch itself (4.25 MiB;
-// one worker's top-k scratch at that d needs just under 4.02 MiB).
+// Largest d the fixed scratch supports, and the scratch itself (8.75 MiB;
+// one worker's top-k scratch at that d needs just under 8.02 MiB).
 constexpr int64_t kNoAllocMaxD = 1 << 20;
-constexpr size_t kNoAllocScratchBytes = (size_t)17 << 18;
+constexpr size_t kNoAllocScratchBytes = (size_t)35 << 18;
 constexpr int kMaxDevices = 64;
 
 static __device__ __align__(256) unsigned char noalloc_scratch[kNoAllocScratchBytes];
@@ -82,8 +82,11 @@ extern "C" int dqgan_topk_compress_noalloc(const float* g, float* e, void* out_m
   }
 
   cudaStream_t stream = reinterpret_cast<cudaStream_t>(cuda_stream);
-  // the histograms and counters of the top-k stages must start at zero
-  st = cudaMemsetAsync(scratch, 0, need, stream);
+  // the histogram and counters of the top-k stages must start at zero (the
+  // kernels return them to zero; clearing makes each call independent of how
+  // an earlier one ended).  The candidate threshold carried from the previous
+  // call stays: it only decides how much work the first pass does.
+  st = cudaMemsetAsync(scratch, 0, dq::topk_scratch_clear_bytes(d), stream);
   if (st != cudaSuccess) {
     snprintf(why, sizeof why, "clearing the scratch: %s", cudaGetErrorString(st));
     return dq::set_thread_error(DQGAN_ERR_CUDA, why);

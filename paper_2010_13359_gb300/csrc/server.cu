@@ -659,50 +659,6 @@ __global__ void __launch_bounds__(256) identity_server_kernel(const ServerArgs s
   apply_chunk(s, j, acc);
 }
 
-// Top-k: every worker's records are sorted by index, so whether an index
-// appears in worker m's list is a binary search.  The thread holding the
-// first occurrence (lowest worker) of an index sums that index's values over
-// all workers in worker order and applies the update; the others stop at the
-// first earlier worker that holds their index.
-__device__ __forceinline__ bool find_index(const uint2* rec, int64_t k, uint32_t idx, float* val) {
-  int64_t lo = 0, hi = k;  // search [lo, hi)
-  while (lo < hi) {
-    const int64_t mid = (lo + hi) >> 1;
-    const uint32_t v = __ldg(&rec[mid].x);
-    if (v < idx) lo = mid + 1;
-    else hi = mid;
-  }
-  if (lo < k) {
-    const uint2 r = __ldg(&rec[lo]);
-    if (r.x == idx) {
-      *val = __uint_as_float(r.y);
-      return true;
-    }
-  }
-  return false;
-}
-
-__global__ void __launch_bounds__(256) topk_server_kernel(const ServerArgs s) {
-  const int64_t tid = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-  if (tid >= (int64_t)s.M * s.k) return;
-  const int m = (int)(tid / s.k);
-  const int64_t r = tid - (int64_t)m * s.k;
-  const uint2 mine = __ldg(reinterpret_cast<const uint2*>(s.msgs + (int64_t)m * s.msg_stride) + r);
-  const uint32_t idx = mine.x;
-  if (idx >= s.d) return;  // records come from the compressor and are < d; never write past w
-  float v;
-  for (int m2 = 0; m2 < m; ++m2) {
-    const uint2* rec = reinterpret_cast<const uint2*>(s.msgs + (int64_t)m2 * s.msg_stride);
-    if (find_index(rec, s.k, idx, &v)) return;  // an earlier worker owns this index
-  }
-  float acc = __fadd_rn(0.f, __uint_as_float(mine.y));
-  for (int m2 = m + 1; m2 < s.M; ++m2) {
-    const uint2* rec = reinterpret_cast<const uint2*>(s.msgs + (int64_t)m2 * s.msg_stride);
-    if (find_index(rec, s.k, idx, &v)) acc = __fadd_rn(acc, v);
-  }
-  s.w[idx] = __fsub_rn(s.w[idx], average(acc, s));
-}
-
 __global__ void __launch_bounds__(256)
 lookahead_kernel(const float* __restrict__ w, const float* __restrict__ h, float* __restrict__ out,
                  int64_t d) {
@@ -855,12 +811,6 @@ cudaError_t launch_identity_server(const ServerArgs& s, cudaStream_t stream, uin
   return cudaGetLastError();
 }
 
-cudaError_t launch_topk_server(const ServerArgs& s, cudaStream_t stream, uint64_t* launches) {
-  const int64_t n = (int64_t)s.M * s.k;
-  topk_server_kernel<<<(unsigned)((n + 255) / 256), 256, 0, stream>>>(s);
-  *launches += 1;
-  return cudaGetLastError();
-}
 
 cudaError_t launch_lookahead(const float* w, const float* h, float* out, int64_t d,
                              cudaStream_t stream, uint64_t* launches) {

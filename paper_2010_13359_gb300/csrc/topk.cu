@@ -1,85 +1,108 @@
-// Worker side of Algorithm 2 with the top-k compressor (Section 2.4, Theorem 1):
-// keep the k entries of p = fl(fl(eta*g) + e) with the largest |p_j| (ties to
-// the lower index), send them as (u32 index, f32 value) records in ascending
-// index order, and keep e_j = +0 at the kept entries and e_j = p_j elsewhere.
+// Top-k compressor of Algorithm 2 (Section 2.4, Theorem 1), worker and server.
 //
-// |p_j| is ordered by its bit pattern with the sign cleared (a 31-bit key),
-// so the k-th largest key is found by a three-digit radix select (11 + 10 +
-// 10 bits) without sorting:
-//   1. pass over g, e (tiles of 4096): p -> e in place, h (optional), and a
-//      block-shared histogram of the top 11 key bits, merged into global;
-//   2. one block finds the digit b0 holding the k-th largest key;
-//   3. pass over p: per tile, count keys with digit > b0 (all kept) and append
-//      the indices with digit == b0 to a candidate list, histogramming their
-//      middle digit;
-//   4-6. the middle and low digits are selected on the (short) candidate list,
-//      giving the threshold key T and the number `need` of keys equal to T
-//      that are kept (the lowest indices among them);
-//   7. per-tile counts of candidates above T and equal to T;
-//   8. one block scans the tiles: output offset of every tile;
-//   9. pass over p: each tile writes its kept records in index order (block
-//      scan) and zeroes e at the kept entries.
-// Every histogram and counter is returned to zero by the stage that consumes
-// it, so the scratch needs no clearing between calls.
+// Worker: keep the k entries of p = fl(fl(eta*g) + e) with the largest |p_j|
+// (ties to the lower index), send them as (u32 index, f32 value) records in
+// ascending index order, and keep e_j = p_j - p_j (+0) at the kept entries
+// and e_j = p_j elsewhere.  |p_j| is ordered by its bit pattern with the sign
+// cleared (a 31-bit key), so the k-th largest key T is found by a three-digit
+// radix select (11 + 10 + 10 bits) without sorting.
+//
+// Two kernels per call, one pass over the dense vectors:
+//   1. form (tiles of 4096 elements): p -> e in place, h (optional), a
+//      histogram of the top key digit, and the tile's candidates -- the
+//      elements whose key is at least a threshold tau carried over from the
+//      worker's previous call (15/16 of its T) -- written in index order to
+//      the tile's slot, with the tile's count.
+//   2. select-and-compact, one cluster of 8 CTAs per worker.  Every CTA
+//      selects the top digit b0 of T from the histogram.  The candidates are
+//      split evenly over the 8 CTAs (by their index order, through a prefix
+//      of the tile counts), each CTA histograms the middle and then the low
+//      digit of its share, the cluster sums the histograms through
+//      distributed shared memory, and T and the number `need` of keys equal
+//      to T that are kept (the lowest indices) follow.  If T >= tau, every
+//      key >= T was a candidate and T is exact; otherwise (first call, or T
+//      fell below the carried threshold) each CTA re-extracts its tiles'
+//      elements with top digit >= b0 from p and the selection is repeated.
+//      Kept records are then written at position (number of keys > T before
+//      it) + min(number of keys == T before it, need).
+// The carried threshold only decides how much work the first pass saves the
+// second; the result is the same bit for bit either way.
+//
+// Server: w_j -= (sum over workers, in worker order, of the value recorded
+// for j) / M at the indices some worker sent; elsewhere w is unchanged (the
+// absent +0 terms leave the sum and w as they are).  A first kernel finds, for
+// each worker and each tile of 4096 indices, where the tile's records start;
+// a second kernel sums each tile's records in shared memory, worker by
+// worker, and updates the touched parameters.
+#include <cooperative_groups.h>
+
+#include "device_common.cuh"
 #include "internal.cuh"
 
 namespace dq {
 namespace {
 
-constexpr int kTile = 4096;          // elements per tile
-constexpr int kThreads = 256;        // threads per tile block
-constexpr int kRows = kTile / (4 * kThreads);  // 4 rows of 256 chunks
-constexpr int kBins0 = 2048, kBins1 = 1024, kBins2 = 1024;
+namespace cg = cooperative_groups;
+
+constexpr int kTile = 4096;                                   // elements per tile
+constexpr int kFormThreads = 256;                             // threads of a form block
+constexpr int kFormRows = kTile / (4 * kFormThreads);         // float4 rows per form thread
+constexpr int kCluster = 8;                                   // CTAs per worker in the select kernel
+constexpr int kSelThreads = 512;                              // threads of a select CTA
+constexpr int kSelRows = kTile / (4 * kSelThreads);           // float4 rows per select thread
+constexpr int kBins0 = 2048, kBins1 = 1024;                   // 11-bit, then 10-bit digits
 constexpr int kStateWords = 32;
+constexpr int kChunkTiles = 2048;                             // tile prefixes a select CTA holds at once
+constexpr int kCacheCap = 20480;                              // candidates a select CTA keeps on chip
+constexpr int kBatch = 8;                                     // candidate loads in flight per thread
+constexpr int kSrvTile = 256;                                 // indices per server tile
+constexpr int kSrvThreads = 256;
+constexpr int kSrvWarpMaxM = 64;                              // workers the warp-per-tile server takes
+constexpr int kSrvWarpBuf = 512;                              // records a server warp stages at once
+constexpr uint32_t kTauValid = 0x80000000u;                   // flag bit of the carried threshold word
 
-// state words
-enum : int { ST_B0 = 0, ST_KREM0, ST_CAND, ST_B1, ST_KREM1, ST_T, ST_NEED };
+// State words.  ST_TAU (the carried threshold: kTauValid | key, or 0 for
+// none) is the last word, so that a caller may clear the others and keep it.
+enum : int { ST_TAU = kStateWords - 1 };
 
-__host__ __device__ __forceinline__ int64_t tiles_of(int64_t d) { return (d + kTile - 1) / kTile; }
+__host__ __device__ constexpr int64_t tiles_of(int64_t d) { return (d + kTile - 1) / kTile; }
+__host__ __device__ constexpr int64_t round64(int64_t x) { return (x + 63) / 64 * 64; }
 
-// Per-worker scratch, in u32 words.
+// Per-worker scratch, in u32 words: hist0 | state | tile counts | the 8
+// CTAs' private tile-prefix arrays (nt + 1 each) | candidate slots (kTile
+// uint2 per tile).
+__host__ __device__ constexpr int64_t head_words(int64_t d) {
+  return round64(kBins0 + kStateWords + tiles_of(d) + kCluster * (tiles_of(d) + 1));
+}
+__host__ __device__ constexpr int64_t row_words(int64_t d) { return head_words(d) + 2 * tiles_of(d) * kTile; }
+__host__ __device__ constexpr int64_t srv_tiles(int64_t d) { return (d + kSrvTile - 1) / kSrvTile; }
+
 struct RowScratch {
   uint32_t* hist0;
-  uint32_t* hist1;
-  uint32_t* hist2;
   uint32_t* state;
-  uint32_t* tile_above;
-  uint32_t* gt_count;
-  uint32_t* tie_count;
-  uint32_t* ties_before;
-  uint32_t* out_off;
-  uint32_t* cand;
+  uint32_t* cnt;
+  uint32_t* gpre;  // kCluster arrays of nt + 1 words
+  uint2* cand;
 };
-
-__host__ __device__ __forceinline__ int64_t row_words(int64_t d) {
-  const int64_t nt = tiles_of(d);
-  const int64_t w = kBins0 + kBins1 + kBins2 + kStateWords + 5 * nt + d;
-  return (w + 63) / 64 * 64;
-}
 
 __device__ __forceinline__ RowScratch row_scratch(void* base, int64_t d, int row) {
   uint32_t* p = reinterpret_cast<uint32_t*>(base) + (int64_t)row * row_words(d);
-  const int64_t nt = tiles_of(d);
   RowScratch r;
   r.hist0 = p;
-  r.hist1 = r.hist0 + kBins0;
-  r.hist2 = r.hist1 + kBins1;
-  r.state = r.hist2 + kBins2;
-  r.tile_above = r.state + kStateWords;
-  r.gt_count = r.tile_above + nt;
-  r.tie_count = r.gt_count + nt;
-  r.ties_before = r.tie_count + nt;
-  r.out_off = r.ties_before + nt;
-  r.cand = r.out_off + nt;
+  r.state = p + kBins0;
+  r.cnt = r.state + kStateWords;
+  r.gpre = r.cnt + tiles_of(d);
+  r.cand = reinterpret_cast<uint2*>(p + head_words(d));
   return r;
 }
 
 __device__ __forceinline__ uint32_t key_of(float v) { return __float_as_uint(v) & 0x7FFFFFFFu; }
+__device__ __forceinline__ uint32_t key_bits(uint32_t bits) { return bits & 0x7FFFFFFFu; }
 
-// Block-wide exclusive scan of one value per thread (kThreads threads).
-// Returns the exclusive prefix; *total receives the block sum.
-__device__ __forceinline__ uint32_t block_exclusive_scan(uint32_t v, uint32_t* total) {
-  __shared__ uint32_t warp_sums[kThreads / 32];
+// Block-wide exclusive scan of one value per thread; *total gets the sum.
+// `warp_sums` is shared memory of NT/32 words.  Two barriers.
+template <int NT>
+__device__ __forceinline__ uint32_t block_exclusive_scan(uint32_t v, uint32_t* total, uint32_t* warp_sums) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   uint32_t x = v;
 #pragma unroll
@@ -89,369 +112,936 @@ __device__ __forceinline__ uint32_t block_exclusive_scan(uint32_t v, uint32_t* t
   }
   if (lane == 31) warp_sums[warp] = x;
   __syncthreads();
-  uint32_t warp_prefix = 0, sum = 0;
+  uint32_t before = 0, sum = 0;
 #pragma unroll
-  for (int w = 0; w < kThreads / 32; ++w) {
+  for (int w = 0; w < NT / 32; ++w) {
     const uint32_t s = warp_sums[w];
-    if (w < warp) warp_prefix += s;
+    if (w < warp) before += s;
     sum += s;
   }
   __syncthreads();
   *total = sum;
-  return warp_prefix + x - v;
+  return before + x - v;
+}
+
+// Block-wide sum of one value per thread (two barriers).
+template <int NT>
+__device__ __forceinline__ uint32_t block_sum(uint32_t v, uint32_t* warp_sums) {
+  uint32_t total;
+  block_exclusive_scan<NT>(v, &total, warp_sums);
+  return total;
+}
+
+// Digit selection in a shared-memory histogram of BINS counts: the digit b
+// with count(> b) < k_rem <= count(>= b); *digit = b, *krem = k_rem -
+// count(> b) (shared-memory outputs, valid after the call for all threads;
+// left as they were when no digit qualifies).
+template <int NT, int BINS>
+__device__ void block_select(const uint32_t* hist, uint32_t k_rem, uint32_t* digit, uint32_t* krem,
+                             uint32_t* warp_sums) {
+  constexpr int kPer = BINS / NT;  // bins per thread, taken in descending digit order
+  static_assert(kPer >= 1 && kPer * NT == BINS, "bins must be a multiple of the block size");
+  uint32_t cnt[kPer];
+  uint32_t local = 0;
+#pragma unroll
+  for (int q = 0; q < kPer; ++q) {
+    cnt[q] = hist[BINS - 1 - ((int)threadIdx.x * kPer + q)];
+    local += cnt[q];
+  }
+  uint32_t total;
+  uint32_t cum = block_exclusive_scan<NT>(local, &total, warp_sums);
+#pragma unroll
+  for (int q = 0; q < kPer; ++q) {
+    if (cum < k_rem && k_rem <= cum + cnt[q]) {
+      *digit = (uint32_t)(BINS - 1 - ((int)threadIdx.x * kPer + q));
+      *krem = k_rem - cum;
+    }
+    cum += cnt[q];
+  }
+  __syncthreads();
+}
+
+// Writes one tile's flagged elements to its candidate slot in index order.
+// Element order in the tile: row i, thread t, component q is tile offset
+// 4 * (i * NT + t) + q.  Per lane and row at most 4 flags, per warp and row
+// at most 128, so the R <= 4 row counts share one 32-bit warp scan (8 bits
+// each).  `totals` is shared memory of NT/32 words.  Returns the tile's
+// count (in every thread); one barrier, two when `reuse` (the caller writes
+// `totals` again afterwards).
+template <int NT, int R, bool REUSE>
+__device__ __forceinline__ uint32_t write_tile_candidates(const float (&v)[R][4], const uint32_t (&cmask)[R],
+                                                          int64_t tile0, uint2* slot, uint32_t* totals) {
+  static_assert(R <= 4, "four 8-bit row counts per word");
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  uint32_t packed = 0;
+#pragma unroll
+  for (int i = 0; i < R; ++i) packed |= (uint32_t)__popc(cmask[i]) << (8 * i);
+  uint32_t incl = packed;
+#pragma unroll
+  for (int off = 1; off < 32; off <<= 1) {
+    const uint32_t y = __shfl_up_sync(kFullMask, incl, off);
+    if (lane >= off) incl += y;
+  }
+  const uint32_t excl = incl - packed;
+  if (lane == 31) totals[warp] = incl;
+  __syncthreads();
+  uint32_t done = 0;
+#pragma unroll
+  for (int i = 0; i < R; ++i) {
+    uint32_t row_before = 0, row_total = 0;
+#pragma unroll
+    for (int w = 0; w < NT / 32; ++w) {
+      const uint32_t f = (totals[w] >> (8 * i)) & 0xFFu;
+      if (w < warp) row_before += f;
+      row_total += f;
+    }
+    uint32_t pos = done + row_before + ((excl >> (8 * i)) & 0xFFu);
+    done += row_total;
+    if (cmask[i]) {
+      const int64_t j = tile0 + 4 * ((int64_t)i * NT + threadIdx.x);
+#pragma unroll
+      for (int q = 0; q < 4; ++q)
+        if ((cmask[i] >> q) & 1u) slot[pos++] = make_uint2((uint32_t)(j + q), __float_as_uint(v[i][q]));
+    }
+  }
+  if constexpr (REUSE) __syncthreads();
+  return done;
 }
 
 // ---------------------------------------------------------------------------
-// 1. p = fl(fl(eta g) + e) into e; h = fl(fl(eta g) + p) (fixed up at the kept
-// entries in stage 9); histogram of the top key digit.
+// 1. p = fl(fl(eta g) + e) into e; h = fl(fl(eta g) + p) (corrected at the kept
+// entries by the second kernel); top-digit histogram; candidates with key >=
+// the carried threshold (none without one).
 // ---------------------------------------------------------------------------
 template <bool KEEP_H>
-__global__ void __launch_bounds__(kThreads) topk_form_kernel(const CompressArgs a, void* scratch) {
+__global__ void __launch_bounds__(kFormThreads, 5) topk_form_kernel(const CompressArgs a, void* scratch) {
   __shared__ uint32_t hist[kBins0];
-  for (int i = threadIdx.x; i < kBins0; i += kThreads) hist[i] = 0;
-  __syncthreads();
+  __shared__ uint32_t totals[kFormThreads / 32];
+  for (int i = threadIdx.x; i < kBins0; i += kFormThreads) hist[i] = 0;
   const int row = blockIdx.y;
   const int worker = a.worker0 + row;
   const float* g = a.g + (int64_t)row * a.g_stride;
   float* e = a.e + (int64_t)worker * a.ld;
   float* h = KEEP_H ? a.h + (int64_t)worker * a.ld : nullptr;
-  const int64_t tile0 = (int64_t)blockIdx.x * kTile;
+  RowScratch rs = row_scratch(scratch, a.d, worker);
+  const uint32_t tau_word = rs.state[ST_TAU];
+  const bool has_tau = (tau_word & kTauValid) != 0;
+  const uint32_t tau = tau_word & 0x7FFFFFFFu;
+  const int64_t tile = blockIdx.x;
+  const int64_t tile0 = tile * kTile;
+  __syncthreads();
+  float v[kFormRows][4];
+  uint32_t cmask[kFormRows];
 #pragma unroll
-  for (int i = 0; i < kRows; ++i) {
-    const int64_t j = tile0 + 4 * ((int64_t)i * kThreads + threadIdx.x);
+  for (int i = 0; i < kFormRows; ++i) {
+    const int64_t j = tile0 + 4 * ((int64_t)i * kFormThreads + threadIdx.x);
+    int nvalid = 0;
     if (j + 3 < a.d) {
       const float4 gv = __ldcs(reinterpret_cast<const float4*>(g + j));
       const float4 ev = __ldcs(reinterpret_cast<const float4*>(e + j));
       const float gq[4] = {gv.x, gv.y, gv.z, gv.w};
       const float eq[4] = {ev.x, ev.y, ev.z, ev.w};
-      float pv[4], hv[4];
+      float hv[4];
 #pragma unroll
       for (int q = 0; q < 4; ++q) {
         const float s = __fmul_rn(a.lr, gq[q]);
-        pv[q] = __fadd_rn(s, eq[q]);
-        hv[q] = __fadd_rn(s, pv[q]);
-        atomicAdd(&hist[key_of(pv[q]) >> 20], 1u);
+        v[i][q] = __fadd_rn(s, eq[q]);
+        hv[q] = __fadd_rn(s, v[i][q]);
       }
-      __stcs(reinterpret_cast<float4*>(e + j), make_float4(pv[0], pv[1], pv[2], pv[3]));
+      __stcs(reinterpret_cast<float4*>(e + j), make_float4(v[i][0], v[i][1], v[i][2], v[i][3]));
       if constexpr (KEEP_H) __stcs(reinterpret_cast<float4*>(h + j), make_float4(hv[0], hv[1], hv[2], hv[3]));
+      nvalid = 4;
     } else {
-      for (int64_t jj = j; jj < a.d && jj < j + 4; ++jj) {
-        const float s = __fmul_rn(a.lr, g[jj]);
-        const float pv = __fadd_rn(s, e[jj]);
-        e[jj] = pv;
-        if constexpr (KEEP_H) h[jj] = __fadd_rn(s, pv);
-        atomicAdd(&hist[key_of(pv) >> 20], 1u);
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        v[i][q] = 0.f;
+        if (j + q < a.d) {
+          const float s = __fmul_rn(a.lr, g[j + q]);
+          v[i][q] = __fadd_rn(s, e[j + q]);
+          e[j + q] = v[i][q];
+          if constexpr (KEEP_H) h[j + q] = __fadd_rn(s, v[i][q]);
+          nvalid = q + 1;
+        }
+      }
+    }
+    cmask[i] = 0;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      if (q < nvalid) {
+        const uint32_t key = key_of(v[i][q]);
+        atomicAdd(&hist[key >> 20], 1u);
+        if (has_tau && key >= tau) cmask[i] |= 1u << q;
       }
     }
   }
-  __syncthreads();
-  RowScratch rs = row_scratch(scratch, a.d, row);
-  for (int i = threadIdx.x; i < kBins0; i += kThreads)
+  const uint32_t ncand =
+      write_tile_candidates<kFormThreads, kFormRows, false>(v, cmask, tile0, rs.cand + tile * kTile, totals);
+  if (threadIdx.x == 0) rs.cnt[tile] = ncand;
+  for (int i = threadIdx.x; i < kBins0; i += kFormThreads)
     if (hist[i]) atomicAdd(&rs.hist0[i], hist[i]);
 }
 
 // ---------------------------------------------------------------------------
-// Digit selection: in a histogram of `bins` counts, find the digit b with
-// count(> b) < k_rem <= count(>= b); store b and k_rem - count(> b); zero the
-// histogram.  One block of 1024 threads per worker row.
+// 2. Select T over the candidates and write the kept records (a cluster of
+// kCluster CTAs per worker).
 // ---------------------------------------------------------------------------
-__device__ void select_digit(uint32_t* hist, int bins, uint32_t k_rem, uint32_t* out_digit,
-                             uint32_t* out_krem) {
-  __shared__ uint32_t warp_sums[32];
-  const int per = bins / 1024;  // 1 or 2 bins per thread, taken in descending digit order
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  uint32_t cnt[2] = {0, 0};
-  uint32_t local = 0;
-  for (int q = 0; q < per; ++q) {
-    const int pos = threadIdx.x * per + q;  // position in descending order
-    cnt[q] = hist[bins - 1 - pos];
-    local += cnt[q];
+struct SelectSmem {
+  uint32_t hist_a[kBins1];          // this CTA's middle-digit histogram (read by the cluster)
+  uint32_t hist_b[kBins1];          // this CTA's low-digit histogram (read by the cluster)
+  uint32_t full[kBins0];            // a whole histogram (top digit; then the cluster's sums)
+  uint32_t tpre[kChunkTiles + 1];   // candidate prefix at the chunk's tiles
+  uint32_t warp_sums[kSelThreads / 32];
+  uint32_t sel[6];
+  uint32_t cta_tot[2];              // keys > T and == T in this CTA's share (read by the cluster)
+  uint32_t span[2];                 // first and last tile overlapping this CTA's share
+  uint2 cache[kCacheCap];           // this CTA's share of the candidates, when it fits
+};
+
+// Tile counts a select thread holds in registers (all tiles, when nt fits).
+constexpr int kRegTiles = 4;
+
+// Candidate f (prefix coordinates of tpre) of the chunk starting at tile tc0.
+__device__ __forceinline__ uint2 chunk_candidate(const uint2* cand, const uint32_t* tpre, int n, int64_t tc0,
+                                                 uint32_t f) {
+  int lo = 0, hi = n;  // tpre[lo] <= f < tpre[hi]
+  while (hi - lo > 1) {
+    const int mid = (lo + hi) >> 1;
+    if (tpre[mid] <= f) lo = mid;
+    else hi = mid;
   }
-  uint32_t x = local;
-  for (int off = 1; off < 32; off <<= 1) {
-    const uint32_t y = __shfl_up_sync(kFullMask, x, off);
-    if (lane >= off) x += y;
-  }
-  if (lane == 31) warp_sums[warp] = x;
-  __syncthreads();
-  uint32_t before = 0;
-  for (int w = 0; w < warp; ++w) before += warp_sums[w];
-  uint32_t cum = before + x - local;  // count of digits above this thread's first
-  for (int q = 0; q < per; ++q) {
-    const int pos = threadIdx.x * per + q;
-    if (cum < k_rem && k_rem <= cum + cnt[q]) {
-      *out_digit = (uint32_t)(bins - 1 - pos);
-      *out_krem = k_rem - cum;
-    }
-    cum += cnt[q];
-  }
-  __syncthreads();
-  for (int q = 0; q < per; ++q) hist[bins - 1 - (threadIdx.x * per + q)] = 0;
+  return cand[(tc0 + lo) * kTile + (f - tpre[lo])];
 }
 
-__global__ void __launch_bounds__(1024) topk_select0_kernel(int64_t d, int64_t k, void* scratch) {
-  RowScratch rs = row_scratch(scratch, d, blockIdx.y);
-  select_digit(rs.hist0, kBins0, (uint32_t)k, &rs.state[ST_B0], &rs.state[ST_KREM0]);
-}
-
-// ---------------------------------------------------------------------------
-// 3. Per tile: count digit0 > b0, append digit0 == b0 to the candidates and
-// histogram their middle digit.
-// ---------------------------------------------------------------------------
-__global__ void __launch_bounds__(kThreads) topk_filter_kernel(const CompressArgs a, void* scratch) {
-  __shared__ uint32_t hist[kBins1];
-  __shared__ uint32_t tile_above;
-  for (int i = threadIdx.x; i < kBins1; i += kThreads) hist[i] = 0;
-  if (threadIdx.x == 0) tile_above = 0;
-  __syncthreads();
-  const int row = blockIdx.y;
-  const int worker = a.worker0 + row;
-  const float* p = a.e + (int64_t)worker * a.ld;
-  RowScratch rs = row_scratch(scratch, a.d, row);
-  const uint32_t b0 = rs.state[ST_B0];
-  const int lane = threadIdx.x & 31;
-  const int64_t tile0 = (int64_t)blockIdx.x * kTile;
-  uint32_t above = 0;
+// Sums the cluster's copies of one histogram into sm.full[0, kBins1).  The
+// cluster barrier publishes every CTA's counts; each histogram buffer is
+// written once per selection round, so no barrier is needed after the reads.
+__device__ __forceinline__ void cluster_sum(cg::cluster_group& cluster, uint32_t* local, SelectSmem& sm) {
+  cluster.sync();
+  for (int i = threadIdx.x; i < kBins1; i += kSelThreads) {
+    uint32_t s = 0;
 #pragma unroll
-  for (int i = 0; i < kRows; ++i) {
-    const int64_t j = tile0 + 4 * ((int64_t)i * kThreads + threadIdx.x);
-    uint32_t keys[4] = {0, 0, 0, 0};
-    int nvalid = 0;
-    if (j + 3 < a.d) {
-      const float4 v = __ldcs(reinterpret_cast<const float4*>(p + j));
-      keys[0] = key_of(v.x); keys[1] = key_of(v.y); keys[2] = key_of(v.z); keys[3] = key_of(v.w);
-      nvalid = 4;
-    } else {
-      for (int q = 0; q < 4 && j + q < a.d; ++q) { keys[q] = key_of(p[j + q]); nvalid = q + 1; }
-    }
-    uint32_t cmask = 0;
-#pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      if (q < nvalid) {
-        const uint32_t dg = keys[q] >> 20;
-        above += (dg > b0);
-        if (dg == b0) {
-          cmask |= 1u << q;
-          atomicAdd(&hist[(keys[q] >> 10) & 1023u], 1u);
-        }
-      }
-    }
-    // warp-aggregated append of the candidates
-    const uint32_t n = __popc(cmask);
-    uint32_t incl = n;
-    for (int off = 1; off < 32; off <<= 1) {
-      const uint32_t y = __shfl_up_sync(kFullMask, incl, off);
-      if (lane >= off) incl += y;
-    }
-    const uint32_t wtotal = __shfl_sync(kFullMask, incl, 31);
-    uint32_t wbase = 0;
-    if (lane == 31 && wtotal) wbase = atomicAdd(&rs.state[ST_CAND], wtotal);
-    wbase = __shfl_sync(kFullMask, wbase, 31);
-    uint32_t pos = wbase + incl - n;
-#pragma unroll
-    for (int q = 0; q < 4; ++q)
-      if (cmask & (1u << q)) rs.cand[pos++] = (uint32_t)(j + q);
-  }
-#pragma unroll
-  for (int off = 16; off >= 1; off >>= 1) above += __shfl_xor_sync(kFullMask, above, off);
-  if (lane == 0 && above) atomicAdd(&tile_above, above);
-  __syncthreads();
-  for (int i = threadIdx.x; i < kBins1; i += kThreads)
-    if (hist[i]) atomicAdd(&rs.hist1[i], hist[i]);
-  if (threadIdx.x == 0) rs.tile_above[blockIdx.x] = tile_above;
-}
-
-__global__ void __launch_bounds__(1024) topk_select1_kernel(int64_t d, void* scratch) {
-  RowScratch rs = row_scratch(scratch, d, blockIdx.y);
-  select_digit(rs.hist1, kBins1, rs.state[ST_KREM0], &rs.state[ST_B1], &rs.state[ST_KREM1]);
-}
-
-// 5. histogram of the low digit over candidates whose middle digit is b1.
-__global__ void __launch_bounds__(kThreads) topk_cand_hist_kernel(const CompressArgs a, void* scratch) {
-  __shared__ uint32_t hist[kBins2];
-  for (int i = threadIdx.x; i < kBins2; i += kThreads) hist[i] = 0;
-  __syncthreads();
-  const int row = blockIdx.y;
-  const float* p = a.e + (int64_t)(a.worker0 + row) * a.ld;
-  RowScratch rs = row_scratch(scratch, a.d, row);
-  const uint32_t ncand = rs.state[ST_CAND], b1 = rs.state[ST_B1];
-  for (uint32_t c = blockIdx.x * kThreads + threadIdx.x; c < ncand; c += gridDim.x * kThreads) {
-    const uint32_t key = key_of(p[rs.cand[c]]);
-    if (((key >> 10) & 1023u) == b1) atomicAdd(&hist[key & 1023u], 1u);
+    for (int r = 0; r < kCluster; ++r) s += cluster.map_shared_rank(local, r)[i];
+    sm.full[i] = s;
   }
   __syncthreads();
-  for (int i = threadIdx.x; i < kBins2; i += kThreads)
-    if (hist[i]) atomicAdd(&rs.hist2[i], hist[i]);
 }
 
-__global__ void __launch_bounds__(1024) topk_select2_kernel(int64_t d, void* scratch) {
-  RowScratch rs = row_scratch(scratch, d, blockIdx.y);
-  __shared__ uint32_t b2;
-  select_digit(rs.hist2, kBins2, rs.state[ST_KREM1], &b2, &rs.state[ST_NEED]);
-  __syncthreads();
-  if (threadIdx.x == 0) rs.state[ST_T] = (rs.state[ST_B0] << 20) | (rs.state[ST_B1] << 10) | b2;
-}
-
-// 7. per-tile counts of candidates above the threshold and equal to it.
-__global__ void __launch_bounds__(kThreads) topk_cand_count_kernel(const CompressArgs a, void* scratch) {
-  const int row = blockIdx.y;
-  const float* p = a.e + (int64_t)(a.worker0 + row) * a.ld;
-  RowScratch rs = row_scratch(scratch, a.d, row);
-  const uint32_t ncand = rs.state[ST_CAND], T = rs.state[ST_T];
-  for (uint32_t c = blockIdx.x * kThreads + threadIdx.x; c < ncand; c += gridDim.x * kThreads) {
-    const uint32_t j = rs.cand[c];
-    const uint32_t key = key_of(p[j]);
-    if (key > T) atomicAdd(&rs.gt_count[j / kTile], 1u);
-    else if (key == T) atomicAdd(&rs.tie_count[j / kTile], 1u);
-  }
-}
-
-// 8. tile offsets: ties before each tile, kept records before each tile.
-__global__ void __launch_bounds__(kThreads) topk_offsets_kernel(int64_t d, void* scratch) {
-  RowScratch rs = row_scratch(scratch, d, blockIdx.y);
-  const int64_t nt = tiles_of(d);
-  const uint32_t need = rs.state[ST_NEED];
-  uint32_t ties_run = 0, out_run = 0;
-  for (int64_t t0 = 0; t0 < nt; t0 += kThreads) {
-    const int64_t t = t0 + threadIdx.x;
-    const uint32_t tie = (t < nt) ? rs.tie_count[t] : 0u;
-    uint32_t tie_total;
-    const uint32_t tie_before = ties_run + block_exclusive_scan(tie, &tie_total);
-    uint32_t taken = 0;
-    if (tie_before < need) taken = min(tie, need - tie_before);
-    const uint32_t sel = (t < nt) ? rs.tile_above[t] + rs.gt_count[t] + taken : 0u;
-    uint32_t sel_total;
-    const uint32_t off = out_run + block_exclusive_scan(sel, &sel_total);
-    if (t < nt) {
-      rs.ties_before[t] = tie_before;
-      rs.out_off[t] = off;
-      rs.gt_count[t] = 0;
-      rs.tie_count[t] = 0;
-    }
-    ties_run += tie_total;
-    out_run += sel_total;
-  }
-  if (threadIdx.x == 0) rs.state[ST_CAND] = 0;
-}
-
-// 9. write the kept records of each tile in index order; e = +0 there.
-// Element order in a tile is row-major: row i (1024 elements) is split over
-// the 8 warps, 128 elements each, 4 per lane.  Each lane counts its keys
-// above T and equal to T, packed as (above | ties << 16) (a tile holds at
-// most 4096 of either), a warp shuffle scan ranks the lanes and one block
-// exchange of the 32 warp-row totals ranks the warps: one barrier per tile.
 template <bool KEEP_H>
-__global__ void __launch_bounds__(kThreads)
-topk_compact_kernel(const CompressArgs a, int64_t k, void* scratch) {
-  __shared__ uint32_t totals[kRows][kThreads / 32];
+__global__ void __cluster_dims__(kCluster, 1, 1) __launch_bounds__(kSelThreads, 1)
+topk_select_kernel(const CompressArgs a, int64_t k, void* scratch) {
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  SelectSmem& sm = *reinterpret_cast<SelectSmem*>(smem_raw);
+  cg::cluster_group cluster = cg::this_cluster();
+  const int rank = (int)cluster.block_rank();
   const int row = blockIdx.y;
   const int worker = a.worker0 + row;
   float* e = a.e + (int64_t)worker * a.ld;
   float* h = KEEP_H ? a.h + (int64_t)worker * a.ld : nullptr;
   const float* g = a.g + (int64_t)row * a.g_stride;
   uint2* rec = reinterpret_cast<uint2*>(a.msg + (int64_t)row * a.msg_stride);
-  RowScratch rs = row_scratch(scratch, a.d, row);
-  const uint32_t T = rs.state[ST_T], need = rs.state[ST_NEED];
-  const uint32_t tie_rank0 = rs.ties_before[blockIdx.x];
-  const uint32_t out0 = rs.out_off[blockIdx.x];
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const int64_t tile0 = (int64_t)blockIdx.x * kTile;
-  float v[kRows][4];
-  uint32_t gmask[kRows], tmask[kRows], excl[kRows];
+  RowScratch rs = row_scratch(scratch, a.d, worker);
+  const int64_t nt = tiles_of(a.d);
+  uint32_t* gpre = rs.gpre + (int64_t)rank * (nt + 1);  // this CTA's private prefix array
+  const uint32_t tau_word = rs.state[ST_TAU];
+  const uint32_t tau = tau_word & 0x7FFFFFFFu;
+  bool fast = (tau_word & kTauValid) != 0;
+  const bool reg_tiles = nt <= (int64_t)kSelThreads * kRegTiles;
+
+  // Top digit b0 from the first pass's histogram (every CTA alike); the
+  // tile counts are fetched alongside.
+  for (int i = threadIdx.x; i < kBins0; i += kSelThreads) sm.full[i] = __ldcg(&rs.hist0[i]);
+  uint32_t cnt_r[kRegTiles];
 #pragma unroll
-  for (int i = 0; i < kRows; ++i) {
-    const int64_t j = tile0 + 4 * ((int64_t)i * kThreads + threadIdx.x);
-    int nvalid = 0;
-    if (j + 3 < a.d) {
-      const float4 x = __ldcs(reinterpret_cast<const float4*>(e + j));
-      v[i][0] = x.x; v[i][1] = x.y; v[i][2] = x.z; v[i][3] = x.w;
-      nvalid = 4;
-    } else {
-#pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        v[i][q] = (j + q < a.d) ? e[j + q] : 0.f;
-        if (j + q < a.d) nvalid = q + 1;
-      }
-    }
-    gmask[i] = 0;
-    tmask[i] = 0;
-#pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      if (q < nvalid) {
-        const uint32_t key = key_of(v[i][q]);
-        if (key > T) gmask[i] |= 1u << q;
-        else if (key == T) tmask[i] |= 1u << q;
-      }
-    }
-    const uint32_t packed = (uint32_t)__popc(gmask[i]) | ((uint32_t)__popc(tmask[i]) << 16);
-    uint32_t incl = packed;
-#pragma unroll
-    for (int off = 1; off < 32; off <<= 1) {
-      const uint32_t y = __shfl_up_sync(kFullMask, incl, off);
-      if (lane >= off) incl += y;
-    }
-    excl[i] = incl - packed;
-    if (lane == 31) totals[i][warp] = incl;
+  for (int q = 0; q < kRegTiles; ++q) {
+    const int64_t t = (int64_t)threadIdx.x * kRegTiles + q;
+    cnt_r[q] = (reg_tiles && t < nt) ? rs.cnt[t] : 0u;
+  }
+  if (threadIdx.x == 0) {
+    sm.sel[0] = 0;
+    sm.sel[1] = (uint32_t)k;
   }
   __syncthreads();
-  uint32_t before = 0;  // packed counts of the tile's earlier warp-rows
+  block_select<kSelThreads, kBins0>(sm.full, (uint32_t)k, &sm.sel[0], &sm.sel[1], sm.warp_sums);
+  const uint32_t b0 = sm.sel[0], krem0 = sm.sel[1];
+
+  // This CTA's share: candidates [F0, F1) in prefix coordinates, lying in
+  // tiles [ta, tb).  With one chunk, sm.tpre[i] is the prefix at tile ta + i.
+  int64_t ta = 0, tb = 0;
+  uint32_t F0 = 0, F1 = 0;
+  bool one_chunk = true, cached = false;
+  uint32_t lo1 = 0, hi1 = 0;  // the share's bounds when it is one chunk
+
+  // Loads the prefix of tiles [tc0, tc0 + n] from gpre into sm.tpre.
+  auto load_chunk = [&](int64_t tc0, int n) {
+    for (int i = threadIdx.x; i <= n; i += kSelThreads) sm.tpre[i] = gpre[tc0 + i];
+    __syncthreads();
+  };
+
+  auto set_up = [&]() {
+    const int64_t t0 = nt * rank / kCluster, t1 = nt * (rank + 1) / kCluster;
+    if (fast && reg_tiles) {
+      // the tile counts are in registers: one scan gives every prefix
+      uint32_t local = 0;
 #pragma unroll
-  for (int i = 0; i < kRows; ++i) {
-    uint32_t row_before = 0, row_total = 0;
+      for (int q = 0; q < kRegTiles; ++q) local += cnt_r[q];
+      uint32_t N;
+      const uint32_t ex = block_exclusive_scan<kSelThreads>(local, &N, sm.warp_sums);
+      F0 = (uint32_t)((uint64_t)N * rank / kCluster);
+      F1 = (uint32_t)((uint64_t)N * (rank + 1) / kCluster);
+      if (threadIdx.x == 0) {
+        sm.span[0] = 0xFFFFFFFFu;
+        sm.span[1] = 0;
+      }
+      __syncthreads();
+      uint32_t p = ex;
 #pragma unroll
-    for (int w = 0; w < kThreads / 32; ++w) {
-      const uint32_t t = totals[i][w];
-      if (w < warp) row_before += t;
-      row_total += t;
+      for (int q = 0; q < kRegTiles; ++q) {
+        const uint32_t t = threadIdx.x * kRegTiles + q;
+        if (cnt_r[q] > 0 && p < F1 && p + cnt_r[q] > F0) {
+          atomicMin(&sm.span[0], t);
+          atomicMax(&sm.span[1], t);
+        }
+        p += cnt_r[q];
+      }
+      __syncthreads();
+      if (F0 < F1) {
+        ta = sm.span[0];
+        tb = (int64_t)sm.span[1] + 1;
+      } else {
+        ta = tb = 0;
+      }
+      p = ex;
+#pragma unroll
+      for (int q = 0; q < kRegTiles; ++q) {
+        const int64_t t = (int64_t)threadIdx.x * kRegTiles + q;
+        if (t >= ta && t < tb) sm.tpre[t - ta] = p;
+        p += cnt_r[q];
+        if (t + 1 == tb) sm.tpre[tb - ta] = p;
+      }
+      __syncthreads();
+      one_chunk = true;
+    } else if (fast) {
+      // all tiles' prefix through this CTA's private array in global memory
+      uint32_t N = 0;
+      for (int64_t base = 0; base < nt; base += kSelThreads) {
+        const int64_t t = base + threadIdx.x;
+        N += block_sum<kSelThreads>(t < nt ? rs.cnt[t] : 0u, sm.warp_sums);
+      }
+      F0 = (uint32_t)((uint64_t)N * rank / kCluster);
+      F1 = (uint32_t)((uint64_t)N * (rank + 1) / kCluster);
+      if (threadIdx.x == 0) {
+        sm.span[0] = 0xFFFFFFFFu;
+        sm.span[1] = 0;
+      }
+      __syncthreads();
+      uint32_t run = 0;
+      for (int64_t base = 0; base < nt; base += kSelThreads) {
+        const int64_t t = base + threadIdx.x;
+        const uint32_t c = t < nt ? rs.cnt[t] : 0u;
+        uint32_t total;
+        const uint32_t p = run + block_exclusive_scan<kSelThreads>(c, &total, sm.warp_sums);
+        if (t < nt) {
+          gpre[t] = p;
+          if (c > 0 && p < F1 && p + c > F0) {
+            atomicMin(&sm.span[0], (uint32_t)t);
+            atomicMax(&sm.span[1], (uint32_t)t);
+          }
+        }
+        run += total;
+      }
+      if (threadIdx.x == 0) gpre[nt] = run;
+      __syncthreads();
+      if (F0 < F1) {
+        ta = sm.span[0];
+        tb = (int64_t)sm.span[1] + 1;
+      } else {
+        ta = tb = 0;
+      }
+      one_chunk = (tb - ta) <= kChunkTiles;
+      if (one_chunk && tb > ta) load_chunk(ta, (int)(tb - ta));
+    } else {
+      // re-extract this CTA's tiles: every element with top digit >= b0
+      for (int64_t t = t0; t < t1; ++t) {
+        const int64_t tile0 = t * kTile;
+        float v[kSelRows][4];
+        uint32_t cmask[kSelRows];
+#pragma unroll
+        for (int i = 0; i < kSelRows; ++i) {
+          const int64_t j = tile0 + 4 * ((int64_t)i * kSelThreads + threadIdx.x);
+          cmask[i] = 0;
+          if (j + 3 < a.d) {
+            const float4 x = *reinterpret_cast<const float4*>(e + j);
+            v[i][0] = x.x; v[i][1] = x.y; v[i][2] = x.z; v[i][3] = x.w;
+#pragma unroll
+            for (int q = 0; q < 4; ++q)
+              if ((key_of(v[i][q]) >> 20) >= b0) cmask[i] |= 1u << q;
+          } else {
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+              v[i][q] = (j + q < a.d) ? e[j + q] : 0.f;
+              if (j + q < a.d && (key_of(v[i][q]) >> 20) >= b0) cmask[i] |= 1u << q;
+            }
+          }
+        }
+        const uint32_t n = write_tile_candidates<kSelThreads, kSelRows, true>(v, cmask, tile0,
+                                                                              rs.cand + t * kTile, sm.warp_sums);
+        if (threadIdx.x == 0) rs.cnt[t] = n;
+      }
+      __syncthreads();
+      // prefix of this CTA's own tiles, from 0
+      uint32_t run = 0;
+      for (int64_t base = t0; base < t1; base += kSelThreads) {
+        const int64_t t = base + threadIdx.x;
+        const uint32_t c = t < t1 ? rs.cnt[t] : 0u;
+        uint32_t total;
+        const uint32_t p = run + block_exclusive_scan<kSelThreads>(c, &total, sm.warp_sums);
+        if (t < t1) gpre[t] = p;
+        run += total;
+      }
+      if (threadIdx.x == 0) gpre[t1] = run;
+      __syncthreads();
+      ta = t0;
+      tb = t1;
+      F0 = 0;
+      F1 = run;
+      one_chunk = (tb - ta) <= kChunkTiles;
+      if (one_chunk && tb > ta) load_chunk(ta, (int)(tb - ta));
     }
-    const uint32_t pre = before + row_before + excl[i];
-    before += row_total;
-    if ((gmask[i] | tmask[i]) == 0) continue;
-    uint32_t R = tie_rank0 + (pre >> 16);  // global rank of this lane's first tie
-    const uint32_t sel_ties_before = min(R, need) - min(tie_rank0, need);
-    uint32_t pos = out0 + (pre & 0xFFFFu) + sel_ties_before;
-    const int64_t j = tile0 + 4 * ((int64_t)i * kThreads + threadIdx.x);
+    cached = false;
+    lo1 = hi1 = 0;
+    if (one_chunk && tb > ta) {
+      lo1 = max(F0, sm.tpre[0]);
+      hi1 = min(F1, sm.tpre[tb - ta]);
+      cached = hi1 - lo1 <= (uint32_t)kCacheCap;
+    }
+  };
+
+  // Runs body(candidate) over this CTA's share, kBatch loads in flight per
+  // thread; with `fill`, also keeps the share on chip.
+  // (body(candidate, valid) is called by every thread of the block the same
+  // number of times, so it may use warp collectives.)
+  auto for_each = [&](auto&& body, bool fill) {
+    if (cached && !fill) {
+      for (uint32_t base = lo1; base < hi1; base += kSelThreads) {
+        const uint32_t f = base + threadIdx.x;
+        body(f < hi1 ? sm.cache[f - lo1] : make_uint2(0u, 0u), f < hi1);
+      }
+      return;
+    }
+    for (int64_t tc0 = ta; tc0 < tb; tc0 += kChunkTiles) {
+      const int n = (int)min64(kChunkTiles, tb - tc0);
+      if (!one_chunk) load_chunk(tc0, n);
+      const uint32_t lo = max(F0, sm.tpre[0]), hi = min(F1, sm.tpre[n]);
+      for (uint32_t base = lo; base < hi; base += kSelThreads * kBatch) {
+        uint2 c[kBatch];
 #pragma unroll
-    for (int q = 0; q < 4; ++q) {
-      bool take = (gmask[i] >> q) & 1u;
-      if ((tmask[i] >> q) & 1u) {
-        take = R < need;
-        ++R;
+        for (int u = 0; u < kBatch; ++u) {
+          const uint32_t f = base + u * kSelThreads + threadIdx.x;
+          c[u] = (f < hi) ? chunk_candidate(rs.cand, sm.tpre, n, tc0, f) : make_uint2(0u, 0u);
+        }
+#pragma unroll
+        for (int u = 0; u < kBatch; ++u) {
+          const uint32_t f = base + u * kSelThreads + threadIdx.x;
+          if (fill && f < hi) sm.cache[f - lo] = c[u];
+          body(c[u], f < hi);
+        }
       }
-      if (take && pos < k) {  // pos < k always holds; the guard keeps writes in the message
-        rec[pos++] = make_uint2((uint32_t)(j + q), __float_as_uint(v[i][q]));
-        e[j + q] = __fsub_rn(v[i][q], v[i][q]);
-        if constexpr (KEEP_H) h[j + q] = __fadd_rn(__fmul_rn(a.lr, g[j + q]), e[j + q]);
-      }
+      if (!one_chunk) __syncthreads();  // sm.tpre is reloaded for the next chunk
+    }
+    if (fill) __syncthreads();
+  };
+
+  uint32_t T = 0, need = 0, my_above = 0;
+  for (int attempt = 0; attempt < 2; ++attempt) {
+    if (attempt > 0) cluster.sync();  // every CTA is done reading the first round's histograms
+    set_up();
+    // middle digit
+    for (int i = threadIdx.x; i < kBins1; i += kSelThreads) {
+      sm.hist_a[i] = 0;
+      sm.hist_b[i] = 0;
+    }
+    __syncthreads();
+    my_above = 0;  // keys whose top digit is above b0
+    for_each(
+        [&](uint2 c, bool valid) {
+          const uint32_t key = key_bits(c.y);
+          if (valid && (key >> 20) == b0) atomicAdd(&sm.hist_a[(key >> 10) & 1023u], 1u);
+          my_above += valid && (key >> 20) > b0;
+        },
+        cached);
+    cluster_sum(cluster, sm.hist_a, sm);
+    if (threadIdx.x == 0) {
+      sm.sel[2] = 0;
+      sm.sel[3] = krem0;
+    }
+    __syncthreads();
+    block_select<kSelThreads, kBins1>(sm.full, krem0, &sm.sel[2], &sm.sel[3], sm.warp_sums);
+    const uint32_t hi21 = (b0 << 10) | sm.sel[2];
+    const uint32_t krem1 = sm.sel[3];
+    // low digit
+    for_each(
+        [&](uint2 c, bool valid) {
+          const uint32_t key = key_bits(c.y);
+          if (valid && (key >> 10) == hi21) atomicAdd(&sm.hist_b[key & 1023u], 1u);
+        },
+        false);
+    cluster_sum(cluster, sm.hist_b, sm);
+    if (threadIdx.x == 0) {
+      sm.sel[4] = 0;
+      sm.sel[5] = krem1;
+    }
+    __syncthreads();
+    block_select<kSelThreads, kBins1>(sm.full, krem1, &sm.sel[4], &sm.sel[5], sm.warp_sums);
+    T = (hi21 << 10) | sm.sel[4];
+    need = sm.sel[5];
+    // T is exact when every key >= T was a candidate, i.e. T >= tau (the
+    // same decision in every CTA of the cluster).
+    if (!fast || T >= tau) break;
+    fast = false;
+  }
+
+  // Keys above and equal to T in this CTA's share, from its own histograms:
+  // top digit above b0, or middle digit above T's, or low digit above T's.
+  {
+    const uint32_t b1 = (T >> 10) & 1023u, b2 = T & 1023u;
+    uint32_t part = my_above;
+    for (int i = threadIdx.x; i < kBins1; i += kSelThreads) {
+      if ((uint32_t)i > b1) part += sm.hist_a[i];
+      if ((uint32_t)i > b2) part += sm.hist_b[i];
+    }
+    const uint32_t cta_gt = block_sum<kSelThreads>(part, sm.warp_sums);
+    if (threadIdx.x == 0) {
+      sm.cta_tot[0] = cta_gt;
+      sm.cta_tot[1] = sm.hist_b[b2];
     }
   }
+  cluster.sync();
+  uint32_t gt_before = 0, tie_before = 0;
+  for (int r = 0; r < rank; ++r) {
+    const uint32_t* tot = cluster.map_shared_rank(sm.cta_tot, r);
+    gt_before += tot[0];
+    tie_before += tot[1];
+  }
+  cluster.sync();  // no CTA leaves while another may still read its shared memory
+
+  // Kept records: position = (keys > T before) + min(keys == T before, need).
+  auto keep = [&](uint2 c) {
+    const uint32_t j = c.x;
+    const float p = __uint_as_float(c.y);
+    const float ej = __fsub_rn(p, p);
+    e[j] = ej;
+    if constexpr (KEEP_H) h[j] = __fadd_rn(__fmul_rn(a.lr, g[j]), ej);
+  };
+  if (cached) {
+    // Each warp takes kEmitRows rows of 32 consecutive candidates; ballots
+    // rank the lanes, one exchange of the warps' counts ranks the warps.
+    constexpr int kEmitRows = 8;
+    constexpr int kWarps = kSelThreads / 32;
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const uint32_t lt = (1u << lane) - 1u;
+    for (uint32_t base = lo1; base < hi1; base += kWarps * kEmitRows * 32) {
+      const uint32_t seg = base + (uint32_t)warp * kEmitRows * 32;
+      uint2 c[kEmitRows];
+      uint32_t gtb[kEmitRows], tieb[kEmitRows];
+      uint32_t wg = 0, wt = 0;
+#pragma unroll
+      for (int u = 0; u < kEmitRows; ++u) {
+        const uint32_t f = seg + 32u * u + lane;
+        const bool valid = f < hi1;
+        c[u] = valid ? sm.cache[f - lo1] : make_uint2(0u, 0u);
+        const uint32_t key = key_bits(c[u].y);
+        gtb[u] = __ballot_sync(kFullMask, valid && key > T);
+        tieb[u] = __ballot_sync(kFullMask, valid && key == T);
+        wg += __popc(gtb[u]);
+        wt += __popc(tieb[u]);
+      }
+      if (lane == 0) sm.warp_sums[warp] = wg | (wt << 16);
+      __syncthreads();
+      uint32_t before = 0, total = 0;
+#pragma unroll
+      for (int w = 0; w < kWarps; ++w) {
+        const uint32_t v = sm.warp_sums[w];
+        if (w < warp) before += v;
+        total += v;
+      }
+      __syncthreads();
+      uint32_t rg = gt_before + (before & 0xFFFFu), rt = tie_before + (before >> 16);
+#pragma unroll
+      for (int u = 0; u < kEmitRows; ++u) {
+        const uint32_t my_g = rg + __popc(gtb[u] & lt), my_t = rt + __popc(tieb[u] & lt);
+        const bool is_gt = (gtb[u] >> lane) & 1u, is_tie = (tieb[u] >> lane) & 1u;
+        if (is_gt || (is_tie && my_t < need)) {
+          const uint32_t pos = my_g + min(my_t, need);
+          if (pos < (uint64_t)k) {  // always true; keeps the write inside the message
+            rec[pos] = c[u];
+            keep(c[u]);
+          }
+        }
+        rg += __popc(gtb[u]);
+        rt += __popc(tieb[u]);
+      }
+      gt_before += total & 0xFFFFu;
+      tie_before += total >> 16;
+    }
+  } else {
+    auto emit = [&](uint2 c, bool valid) {
+      const uint32_t key = key_bits(c.y);
+      const bool is_gt = valid && key > T;
+      const bool is_tie = valid && key == T;
+      uint32_t total;
+      const uint32_t ex = block_exclusive_scan<kSelThreads>((uint32_t)is_gt | ((uint32_t)is_tie << 16), &total,
+                                                            sm.warp_sums);
+      const uint32_t ties = tie_before + (ex >> 16);
+      if (is_gt || (is_tie && ties < need)) {
+        const uint32_t pos = gt_before + (ex & 0xFFFFu) + min(ties, need);
+        if (pos < (uint64_t)k) {  // always true; keeps the write inside the message
+          rec[pos] = c;
+          keep(c);
+        }
+      }
+      gt_before += total & 0xFFFFu;
+      tie_before += total >> 16;
+    };
+    for (int64_t tc0 = ta; tc0 < tb; tc0 += kChunkTiles) {
+      const int n = (int)min64(kChunkTiles, tb - tc0);
+      if (!one_chunk) load_chunk(tc0, n);
+      const uint32_t lo = max(F0, sm.tpre[0]), hi = min(F1, sm.tpre[n]);
+      for (uint32_t base = lo; base < hi; base += kSelThreads * kBatch) {
+        uint2 c[kBatch];
+#pragma unroll
+        for (int u = 0; u < kBatch; ++u) {
+          const uint32_t f = base + u * kSelThreads + threadIdx.x;
+          c[u] = (f < hi) ? chunk_candidate(rs.cand, sm.tpre, n, tc0, f) : make_uint2(0u, 0u);
+        }
+#pragma unroll
+        for (int u = 0; u < kBatch; ++u) emit(c[u], base + u * kSelThreads + threadIdx.x < hi);
+      }
+      __syncthreads();
+    }
+  }
+
+  // For the next call: the histogram back to zero, the threshold 15/16 of T.
+  if (rank == 0) {
+    for (int i = threadIdx.x; i < kBins0; i += kSelThreads) rs.hist0[i] = 0;
+    if (threadIdx.x == 0) {
+      const float t_next = __fmul_rn(__uint_as_float(T), 0.9375f);
+      rs.state[ST_TAU] = kTauValid | key_of(t_next);
+    }
+  }
+}
+
+// ---------------------------------------------------------------------------
+// Server.  starts[m][t] = first record of worker m whose index is in tile t
+// or later (t in [0, nts]); record r writes the tiles (tile(r-1), tile(r)],
+// and the last record also (tile(k-1), nts].
+// ---------------------------------------------------------------------------
+__global__ void __launch_bounds__(256) topk_server_starts_kernel(const ServerArgs s, uint32_t* starts) {
+  const int m = blockIdx.y;
+  const int64_t r = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  const int lane = threadIdx.x & 31;
+  const int64_t nts = srv_tiles(s.d);
+  const uint2* msg = reinterpret_cast<const uint2*>(s.msgs + (int64_t)m * s.msg_stride);
+  uint32_t* st = starts + (int64_t)m * (nts + 1);
+  // this record fills the tiles [t_a, t_b] with r (empty range: t_a > t_b)
+  int64_t t_a = 1, t_b = 0;
+  if (r < s.k) {
+    const int64_t tile = min64(msg[r].x / kSrvTile, nts - 1);
+    const int64_t prev = (r == 0) ? -1 : min64(msg[r - 1].x / kSrvTile, nts - 1);
+    t_a = prev + 1;
+    t_b = tile;
+  }
+  for (int64_t t = t_a; t <= t_b && t < t_a + 32; ++t) st[t] = (uint32_t)r;
+  // long runs (sparse stretches of the index range) are written by the whole warp
+  uint32_t longs = __ballot_sync(kFullMask, t_b - t_a >= 32);
+  while (longs) {
+    const int src = __ffs(longs) - 1;
+    longs &= longs - 1;
+    const int64_t a = __shfl_sync(kFullMask, t_a, src), bnd = __shfl_sync(kFullMask, t_b, src);
+    const uint32_t val = (uint32_t)__shfl_sync(kFullMask, r, src);
+    for (int64_t t = a + 32 + lane; t <= bnd; t += 32) st[t] = val;
+  }
+  // after the last record: the tiles up to nts point past the end
+  const uint32_t last = __ballot_sync(kFullMask, r == s.k - 1);
+  if (last) {
+    const int src = __ffs(last) - 1;
+    const int64_t a = __shfl_sync(kFullMask, t_b, src) + 1;
+    for (int64_t t = a + lane; t <= nts; t += 32) st[t] = (uint32_t)s.k;
+  }
+}
+
+template <bool POW2>
+__device__ __forceinline__ float srv_average(float acc, const ServerArgs& s) {
+  if constexpr (POW2) return __fmul_rn(acc, s.inv_M);
+  else return __fdiv_rn(acc, (float)s.M);
+}
+
+// One warp per tile of kSrvTile indices (M <= kSrvWarpMaxM).  The warp
+// stages the tile's records of all workers in shared memory (one flat,
+// worker-ordered batch of loads), adds them into the tile's sums worker by
+// worker -- program order within the warp keeps worker order, so no block
+// barrier is needed -- and updates the touched w_j (all loads of w issued
+// before the stores).
+struct SrvWarpSmem {
+  float acc[kSrvTile];
+  uint32_t touched[kSrvTile / 32];
+  uint2 buf[kSrvWarpBuf];
+  uint32_t first[kSrvWarpMaxM];
+  uint32_t pre[kSrvWarpMaxM + 1];
+};
+constexpr int kSrvWarps = kSrvThreads / 32;
+
+template <bool POW2>
+__global__ void __launch_bounds__(kSrvThreads) topk_server_warp_kernel(const ServerArgs s, const uint32_t* starts) {
+  extern __shared__ __align__(16) unsigned char smem_raw[];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+  SrvWarpSmem& sm = reinterpret_cast<SrvWarpSmem*>(smem_raw)[warp];
+  const int64_t nts = srv_tiles(s.d);
+  const int64_t t = (int64_t)blockIdx.x * kSrvWarps + warp;
+  if (t >= nts) return;  // the whole warp
+  const int64_t tile0 = t * kSrvTile;
+  const int M = s.M;
+  if (lane < kSrvTile / 32) sm.touched[lane] = 0;
+  // this tile's record range of every worker, and the flat prefix
+  uint32_t run = 0;
+  for (int base = 0; base < M; base += 32) {
+    const int m = base + lane;
+    uint32_t n = 0;
+    if (m < M) {
+      const uint32_t* st = starts + (int64_t)m * (nts + 1);
+      const uint32_t a0 = (uint32_t)min64(st[t], s.k), a1 = (uint32_t)min64(st[t + 1], s.k);
+      n = a1 > a0 ? a1 - a0 : 0u;
+      sm.first[m] = a0;
+    }
+    uint32_t x = n;
+#pragma unroll
+    for (int off = 1; off < 32; off <<= 1) {
+      const uint32_t y = __shfl_up_sync(kFullMask, x, off);
+      if (lane >= off) x += y;
+    }
+    if (m < M) sm.pre[m] = run + x - n;
+    run += __shfl_sync(kFullMask, x, 31);
+  }
+  if (lane == 0) sm.pre[M] = run;
+  __syncwarp();
+  const uint32_t N = run;
+  for (uint32_t b = 0; b < N; b += kSrvWarpBuf) {
+    const uint32_t nb = (uint32_t)min64(kSrvWarpBuf, N - b);
+    // kStage loads in flight per lane, then their shared-memory stores
+    constexpr int kStage = 8;
+    for (uint32_t i0 = 0; i0 < nb; i0 += 32 * kStage) {
+      uint2 v[kStage];
+#pragma unroll
+      for (int u = 0; u < kStage; ++u) {
+        const uint32_t i = i0 + u * 32 + lane;
+        v[u] = make_uint2(0u, 0u);
+        if (i < nb) {
+          const uint32_t f = b + i;
+          int lo = 0, hi = M;  // pre[lo] <= f < pre[hi]
+          while (hi - lo > 1) {
+            const int mid = (lo + hi) >> 1;
+            if (sm.pre[mid] <= f) lo = mid;
+            else hi = mid;
+          }
+          const uint2* msg = reinterpret_cast<const uint2*>(s.msgs + (int64_t)lo * s.msg_stride);
+          v[u] = msg[sm.first[lo] + (f - sm.pre[lo])];
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < kStage; ++u) {
+        const uint32_t i = i0 + u * 32 + lane;
+        if (i < nb) sm.buf[i] = v[u];
+      }
+    }
+    __syncwarp();
+    for (int m = 0; m < M; ++m) {
+      const uint32_t f0 = max64(sm.pre[m], b), f1 = min64(sm.pre[m + 1], b + nb);
+      // a worker's indices are distinct: its records update distinct sums,
+      // four per lane at a time
+      for (uint32_t fb = f0; fb < f1; fb += 4 * 32) {
+        uint2 r[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          const uint32_t f = fb + u * 32 + lane;
+          r[u] = f < f1 ? sm.buf[f - b] : make_uint2(0xFFFFFFFFu, 0u);
+        }
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          const int64_t off = (int64_t)r[u].x - tile0;
+          if (fb + u * 32 + lane < f1 && off >= 0 && off < kSrvTile && (int64_t)r[u].x < s.d) {
+            const uint32_t bit = 1u << (off & 31);
+            const bool seen = (sm.touched[off >> 5] & bit) != 0;
+            // the sum starts at +0 (as a dense sum over all workers would)
+            sm.acc[off] = __fadd_rn(seen ? sm.acc[off] : 0.f, __uint_as_float(r[u].y));
+            if (!seen) atomicOr(&sm.touched[off >> 5], bit);
+          }
+        }
+      }
+      __syncwarp();
+    }
+  }
+  constexpr int kPer = kSrvTile / 32;
+  constexpr int kHalf = kPer / 2;
+#pragma unroll
+  for (int half = 0; half < 2; ++half) {
+    float wv[kHalf];
+#pragma unroll
+    for (int q = 0; q < kHalf; ++q) {
+      const int i = (half * kHalf + q) * 32 + lane;
+      wv[q] = ((sm.touched[i >> 5] >> (i & 31)) & 1u) ? s.w[tile0 + i] : 0.f;
+    }
+#pragma unroll
+    for (int q = 0; q < kHalf; ++q) {
+      const int i = (half * kHalf + q) * 32 + lane;
+      if ((sm.touched[i >> 5] >> (i & 31)) & 1u) s.w[tile0 + i] = __fsub_rn(wv[q], srv_average<POW2>(sm.acc[i], s));
+    }
+  }
+}
+
+// One thread per record of every worker.  The record of the lowest worker
+// holding index j owns j: it sums the values recorded for j over the
+// workers in worker order (the sum starts at +0, as a dense sum over all
+// workers would) and applies w_j -= sum / M; the others find an earlier
+// worker holding j and stop.  Each search looks only at the other worker's
+// records in j's tile of kSrvTile indices (the starts table), and the
+// searches in kSrvGroup workers' lists advance in lockstep so that their
+// loads are in flight together.
+constexpr int kSrvGroup = 8;
+
+template <bool POW2>
+__global__ void __launch_bounds__(kSrvThreads) topk_server_owner_kernel(const ServerArgs s, const uint32_t* starts) {
+  const int64_t id = (int64_t)blockIdx.x * kSrvThreads + threadIdx.x;
+  if (id >= (int64_t)s.M * s.k) return;
+  const int m = (int)(id / s.k);
+  const int64_t r = id - (int64_t)m * s.k;
+  const uint2 mine = reinterpret_cast<const uint2*>(s.msgs + (int64_t)m * s.msg_stride)[r];
+  const uint32_t j = mine.x;
+  if ((int64_t)j >= s.d) return;  // records come from the compressor and are < d
+  const int64_t nts = srv_tiles(s.d);
+  const int64_t t = j / kSrvTile;
+  float acc = __fadd_rn(0.f, __uint_as_float(mine.y));
+  for (int m0 = 0; m0 < s.M; m0 += kSrvGroup) {
+    uint32_t lo[kSrvGroup], hi[kSrvGroup], end[kSrvGroup];
+#pragma unroll
+    for (int u = 0; u < kSrvGroup; ++u) {
+      const int m2 = m0 + u;
+      lo[u] = hi[u] = 0;
+      if (m2 < s.M && m2 != m) {
+        const uint32_t* st = starts + (int64_t)m2 * (nts + 1);
+        lo[u] = (uint32_t)min64(st[t], s.k);
+        hi[u] = (uint32_t)min64(st[t + 1], s.k);
+      }
+      end[u] = hi[u];
+    }
+    // lower bound of j in every range, one halving step for all at a time
+    bool active = true;
+    while (active) {
+      uint32_t x[kSrvGroup];
+#pragma unroll
+      for (int u = 0; u < kSrvGroup; ++u) {
+        x[u] = 0;
+        if (lo[u] < hi[u]) {
+          const uint2* rec = reinterpret_cast<const uint2*>(s.msgs + (int64_t)(m0 + u) * s.msg_stride);
+          x[u] = rec[lo[u] + ((hi[u] - lo[u]) >> 1)].x;
+        }
+      }
+      active = false;
+#pragma unroll
+      for (int u = 0; u < kSrvGroup; ++u) {
+        if (lo[u] < hi[u]) {
+          const uint32_t mid = lo[u] + ((hi[u] - lo[u]) >> 1);
+          if (x[u] < j) lo[u] = mid + 1;
+          else hi[u] = mid;
+          active |= lo[u] < hi[u];
+        }
+      }
+    }
+    float val[kSrvGroup];
+    bool has[kSrvGroup];
+#pragma unroll
+    for (int u = 0; u < kSrvGroup; ++u) {
+      has[u] = false;
+      val[u] = 0.f;
+      if (lo[u] < end[u]) {
+        const uint2* rec = reinterpret_cast<const uint2*>(s.msgs + (int64_t)(m0 + u) * s.msg_stride);
+        const uint2 x = rec[lo[u]];
+        has[u] = x.x == j;
+        val[u] = __uint_as_float(x.y);
+      }
+    }
+#pragma unroll
+    for (int u = 0; u < kSrvGroup; ++u) {
+      if (!has[u]) continue;
+      if (m0 + u < m) return;  // an earlier worker owns j
+      acc = __fadd_rn(acc, val[u]);
+    }
+  }
+  s.w[j] = __fsub_rn(s.w[j], srv_average<POW2>(acc, s));
 }
 
 }  // namespace
 
 size_t topk_scratch_bytes(int64_t d, int32_t nworkers) {
-  return (size_t)row_words(d) * 4u * (size_t)nworkers;
+  const int64_t server_words = round64((int64_t)nworkers * (srv_tiles(d) + 1));
+  return (size_t)(row_words(d) * nworkers + server_words) * 4u;
+}
+
+size_t topk_scratch_clear_bytes(int64_t d) {
+  (void)d;
+  return (size_t)(kBins0 + ST_TAU) * 4u;
+}
+
+// Raises a kernel's dynamic shared memory limit when its static plus dynamic
+// shared memory exceeds the default 48 KB (the value only grows; the
+// attribute is per function, for every device).
+template <typename K>
+cudaError_t ensure_smem(K kernel, size_t bytes, size_t static_bytes, size_t* done) {
+  if (bytes + static_bytes <= 48u * 1024u || bytes <= *done) return cudaSuccess;
+  const cudaError_t st = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
+  if (st == cudaSuccess) *done = bytes;
+  return st;
 }
 
 cudaError_t launch_topk_compress(const CompressArgs& a, int64_t k, bool keep_h, void* scratch,
                                  cudaStream_t stream, uint64_t* launches) {
+  static size_t smem_done[2] = {0, 0};
   const unsigned rows = (unsigned)a.nworkers;
   const dim3 tiles((unsigned)tiles_of(a.d), rows);
-  const dim3 one(1, rows);
-  // candidate-list kernels: a fixed grid that strides over the device-side count
-  const dim3 cgrid((unsigned)((tiles_of(a.d) + 3) / 4 < 1184 ? (tiles_of(a.d) + 3) / 4 : 1184), rows);
-  if (keep_h) topk_form_kernel<true><<<tiles, kThreads, 0, stream>>>(a, scratch);
-  else topk_form_kernel<false><<<tiles, kThreads, 0, stream>>>(a, scratch);
-  topk_select0_kernel<<<one, 1024, 0, stream>>>(a.d, k, scratch);
-  topk_filter_kernel<<<tiles, kThreads, 0, stream>>>(a, scratch);
-  topk_select1_kernel<<<one, 1024, 0, stream>>>(a.d, scratch);
-  topk_cand_hist_kernel<<<cgrid, kThreads, 0, stream>>>(a, scratch);
-  topk_select2_kernel<<<one, 1024, 0, stream>>>(a.d, scratch);
-  topk_cand_count_kernel<<<cgrid, kThreads, 0, stream>>>(a, scratch);
-  topk_offsets_kernel<<<one, kThreads, 0, stream>>>(a.d, scratch);
-  if (keep_h) topk_compact_kernel<true><<<tiles, kThreads, 0, stream>>>(a, k, scratch);
-  else topk_compact_kernel<false><<<tiles, kThreads, 0, stream>>>(a, k, scratch);
-  *launches += 9;
+  const dim3 clusters(kCluster, rows);
+  const size_t smem = sizeof(SelectSmem);
+  cudaError_t st;
+  if (keep_h) {
+    if ((st = ensure_smem(topk_select_kernel<true>, smem, 0, &smem_done[1])) != cudaSuccess) return st;
+    topk_form_kernel<true><<<tiles, kFormThreads, 0, stream>>>(a, scratch);
+    topk_select_kernel<true><<<clusters, kSelThreads, smem, stream>>>(a, k, scratch);
+  } else {
+    if ((st = ensure_smem(topk_select_kernel<false>, smem, 0, &smem_done[0])) != cudaSuccess) return st;
+    topk_form_kernel<false><<<tiles, kFormThreads, 0, stream>>>(a, scratch);
+    topk_select_kernel<false><<<clusters, kSelThreads, smem, stream>>>(a, k, scratch);
+  }
+  *launches += 2;
+  return cudaGetLastError();
+}
+
+cudaError_t launch_topk_server(const ServerArgs& s, void* scratch, cudaStream_t stream, uint64_t* launches) {
+  uint32_t* starts = reinterpret_cast<uint32_t*>(scratch) + row_words(s.d) * s.M;
+  const int64_t n = (int64_t)s.M * s.k;
+  topk_server_starts_kernel<<<dim3((unsigned)((s.k + 255) / 256), (unsigned)s.M), 256, 0, stream>>>(s, starts);
+  if (s.M <= kSrvWarpMaxM) {
+    static size_t smem_done[2] = {0, 0};
+    const size_t smem = sizeof(SrvWarpSmem) * kSrvWarps;
+    const unsigned blocks = (unsigned)((srv_tiles(s.d) + kSrvWarps - 1) / kSrvWarps);
+    cudaError_t st;
+    if (s.M_pow2) st = ensure_smem(topk_server_warp_kernel<true>, smem, 0, &smem_done[1]);
+    else st = ensure_smem(topk_server_warp_kernel<false>, smem, 0, &smem_done[0]);
+    if (st != cudaSuccess) return st;
+    if (s.M_pow2) topk_server_warp_kernel<true><<<blocks, kSrvThreads, smem, stream>>>(s, starts);
+    else topk_server_warp_kernel<false><<<blocks, kSrvThreads, smem, stream>>>(s, starts);
+  } else {
+    const unsigned blocks = (unsigned)((n + kSrvThreads - 1) / kSrvThreads);
+    if (s.M_pow2) topk_server_owner_kernel<true><<<blocks, kSrvThreads, 0, stream>>>(s, starts);
+    else topk_server_owner_kernel<false><<<blocks, kSrvThreads, 0, stream>>>(s, starts);
+  }
+  *launches += 2;
   return cudaGetLastError();
 }
 

@@ -4,8 +4,11 @@ The no-allocation entry point serves callers that cannot allocate device
 memory (and so cannot create a handle): it keeps its scratch in a fixed
 array inside the library and works on a residual the caller owns.  It must
 produce exactly the messages and residuals of dqgan_worker_compress with the
-top-k compressor.  Two calls in a row check that the shared scratch is
-cleared between calls and that the caller's residual carries over.
+top-k compressor.  Four calls in a row, the last two with the gradient
+scale dropped by 1e4 and then raised by 1e8, check that the shared scratch
+is cleared between calls, that the caller's residual carries over, and that
+the candidate threshold carried from call to call (also across the
+parametrised cases, which share the array) never changes a result.
 """
 from __future__ import annotations
 
@@ -35,9 +38,10 @@ def test_noalloc_topk_matches_handle_path(P, d, k):
     pad = (d + 3) // 4 * 4
     e_caller = torch.zeros(pad, dtype=torch.float32, device=dev)
     rng = np.random.default_rng(d)
-    for call in range(2):
+    for call, scale in enumerate([1.0, 1.0, 1e-4, 1e4]):
         g = torch.zeros(pad, dtype=torch.float32, device=dev)
-        g[:d] = torch.from_numpy((rng.standard_normal(d) * np.exp(rng.uniform(-3, 1, d))).astype(np.float32))
+        g[:d] = torch.from_numpy((rng.standard_normal(d) * np.exp(rng.uniform(-3, 1, d)) * scale)
+                                 .astype(np.float32))
         msg_ref = torch.zeros(mb, dtype=torch.uint8, device=dev)
         msg_new = torch.zeros(mb, dtype=torch.uint8, device=dev)
         h.worker_compress(0, g, msg_ref)
