@@ -68,17 +68,16 @@ enum : int { ST_TAU = kStateWords - 1 };
 __host__ __device__ constexpr int64_t tiles_of(int64_t d) { return (d + kTile - 1) / kTile; }
 __host__ __device__ constexpr int64_t round64(int64_t x) { return (x + 63) / 64 * 64; }
 
-// Per-worker scratch, in u32 words: hist0 | state | tile counts | the 8
-// CTAs' private tile-prefix arrays (nt + 1 each) | candidate slots (kTile
-// uint2 per tile).
+// Per-worker scratch, in u32 words: state | tile counts | the 8 CTAs'
+// private tile-prefix arrays (nt + 1 each) | candidate slots (kTile uint2
+// per tile).
 __host__ __device__ constexpr int64_t head_words(int64_t d) {
-  return round64(kBins0 + kStateWords + tiles_of(d) + kCluster * (tiles_of(d) + 1));
+  return round64(kStateWords + tiles_of(d) + kCluster * (tiles_of(d) + 1));
 }
 __host__ __device__ constexpr int64_t row_words(int64_t d) { return head_words(d) + 2 * tiles_of(d) * kTile; }
 __host__ __device__ constexpr int64_t srv_tiles(int64_t d) { return (d + kSrvTile - 1) / kSrvTile; }
 
 struct RowScratch {
-  uint32_t* hist0;
   uint32_t* state;
   uint32_t* cnt;
   uint32_t* gpre;  // kCluster arrays of nt + 1 words
@@ -88,8 +87,7 @@ struct RowScratch {
 __device__ __forceinline__ RowScratch row_scratch(void* base, int64_t d, int row) {
   uint32_t* p = reinterpret_cast<uint32_t*>(base) + (int64_t)row * row_words(d);
   RowScratch r;
-  r.hist0 = p;
-  r.state = p + kBins0;
+  r.state = p;
   r.cnt = r.state + kStateWords;
   r.gpre = r.cnt + tiles_of(d);
   r.cand = reinterpret_cast<uint2*>(p + head_words(d));
@@ -210,14 +208,20 @@ __device__ __forceinline__ uint32_t write_tile_candidates(const float (&v)[R][4]
 
 // ---------------------------------------------------------------------------
 // 1. p = fl(fl(eta g) + e) into e; h = fl(fl(eta g) + p) (corrected at the kept
-// entries by the second kernel); top-digit histogram; candidates with key >=
-// the carried threshold (none without one).
+// entries by the second kernel); candidates with key >= the carried
+// threshold (none without one).  Element order in a tile: row i,
+// thread t, component q is tile offset 4 * (i * 256 + t) + q, so warp w of
+// row i covers the 128 consecutive offsets of group g = 8 i + w.  Candidate
+// values wait in shared memory (flagged in a bitmask) until the block's one
+// barrier; then each warp writes its groups' candidates to the tile's slot
+// in index order.
 // ---------------------------------------------------------------------------
 template <bool KEEP_H>
-__global__ void __launch_bounds__(kFormThreads, 5) topk_form_kernel(const CompressArgs a, void* scratch) {
-  __shared__ uint32_t hist[kBins0];
-  __shared__ uint32_t totals[kFormThreads / 32];
-  for (int i = threadIdx.x; i < kBins0; i += kFormThreads) hist[i] = 0;
+__global__ void __launch_bounds__(kFormThreads, 6) topk_form_kernel(const CompressArgs a, void* scratch) {
+  constexpr int kGroups = kTile / 128;
+  __shared__ float vstage[kTile];
+  __shared__ uint32_t flags[kTile / 32];
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   const int row = blockIdx.y;
   const int worker = a.worker0 + row;
   const float* g = a.g + (int64_t)row * a.g_stride;
@@ -229,12 +233,11 @@ __global__ void __launch_bounds__(kFormThreads, 5) topk_form_kernel(const Compre
   const uint32_t tau = tau_word & 0x7FFFFFFFu;
   const int64_t tile = blockIdx.x;
   const int64_t tile0 = tile * kTile;
-  __syncthreads();
-  float v[kFormRows][4];
-  uint32_t cmask[kFormRows];
 #pragma unroll
   for (int i = 0; i < kFormRows; ++i) {
-    const int64_t j = tile0 + 4 * ((int64_t)i * kFormThreads + threadIdx.x);
+    const int off = 4 * (i * kFormThreads + (int)threadIdx.x);
+    const int64_t j = tile0 + off;
+    float v[4];
     int nvalid = 0;
     if (j + 3 < a.d) {
       const float4 gv = __ldcs(reinterpret_cast<const float4*>(g + j));
@@ -245,40 +248,79 @@ __global__ void __launch_bounds__(kFormThreads, 5) topk_form_kernel(const Compre
 #pragma unroll
       for (int q = 0; q < 4; ++q) {
         const float s = __fmul_rn(a.lr, gq[q]);
-        v[i][q] = __fadd_rn(s, eq[q]);
-        hv[q] = __fadd_rn(s, v[i][q]);
+        v[q] = __fadd_rn(s, eq[q]);
+        hv[q] = __fadd_rn(s, v[q]);
       }
-      __stcs(reinterpret_cast<float4*>(e + j), make_float4(v[i][0], v[i][1], v[i][2], v[i][3]));
+      __stcs(reinterpret_cast<float4*>(e + j), make_float4(v[0], v[1], v[2], v[3]));
       if constexpr (KEEP_H) __stcs(reinterpret_cast<float4*>(h + j), make_float4(hv[0], hv[1], hv[2], hv[3]));
       nvalid = 4;
     } else {
 #pragma unroll
       for (int q = 0; q < 4; ++q) {
-        v[i][q] = 0.f;
+        v[q] = 0.f;
         if (j + q < a.d) {
           const float s = __fmul_rn(a.lr, g[j + q]);
-          v[i][q] = __fadd_rn(s, e[j + q]);
-          e[j + q] = v[i][q];
-          if constexpr (KEEP_H) h[j + q] = __fadd_rn(s, v[i][q]);
+          v[q] = __fadd_rn(s, e[j + q]);
+          e[j + q] = v[q];
+          if constexpr (KEEP_H) h[j + q] = __fadd_rn(s, v[q]);
           nvalid = q + 1;
         }
       }
     }
-    cmask[i] = 0;
+    uint32_t bits = 0;
 #pragma unroll
     for (int q = 0; q < 4; ++q) {
       if (q < nvalid) {
-        const uint32_t key = key_of(v[i][q]);
-        atomicAdd(&hist[key >> 20], 1u);
-        if (has_tau && key >= tau) cmask[i] |= 1u << q;
+        const uint32_t key = key_of(v[q]);
+        if (has_tau && key >= tau) {
+          bits |= 1u << q;
+          vstage[off + q] = v[q];
+        }
+      }
+    }
+    // 8 lanes' 4 flag bits form one 32-bit word of the tile's bitmask
+    uint32_t word = bits << (4 * (lane & 7));
+    word |= __shfl_xor_sync(kFullMask, word, 1);
+    word |= __shfl_xor_sync(kFullMask, word, 2);
+    word |= __shfl_xor_sync(kFullMask, word, 4);
+    if ((lane & 7) == 0) flags[off >> 5] = word;
+  }
+  __syncthreads();
+  // group offsets: every warp scans the 32 groups' counts (group = lane)
+  uint32_t gc = 0;
+#pragma unroll
+  for (int q = 0; q < 4; ++q) gc += __popc(flags[lane * 4 + q]);
+  uint32_t incl = gc;
+#pragma unroll
+  for (int o = 1; o < 32; o <<= 1) {
+    const uint32_t y = __shfl_up_sync(kFullMask, incl, o);
+    if (lane >= o) incl += y;
+  }
+  const uint32_t total = __shfl_sync(kFullMask, incl, 31);
+  uint2* slot = rs.cand + tile * kTile;
+  static_assert(kGroups == kFormRows * (kFormThreads / 32), "one group per warp and row");
+#pragma unroll
+  for (int i = 0; i < kFormRows; ++i) {
+    const int grp = i * (kFormThreads / 32) + warp;
+    const uint32_t gbase = __shfl_sync(kFullMask, incl - gc, grp);
+    const uint32_t lane_bits = (flags[grp * 4 + (lane >> 3)] >> (4 * (lane & 7))) & 0xFu;
+    const uint32_t n = __popc(lane_bits);
+    uint32_t x = n;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const uint32_t y = __shfl_up_sync(kFullMask, x, o);
+      if (lane >= o) x += y;
+    }
+    uint32_t pos = gbase + x - n;
+#pragma unroll
+    for (int q = 0; q < 4; ++q) {
+      if ((lane_bits >> q) & 1u) {
+        const int off = grp * 128 + lane * 4 + q;
+        slot[pos++] = make_uint2((uint32_t)(tile0 + off), __float_as_uint(vstage[off]));
       }
     }
   }
-  const uint32_t ncand =
-      write_tile_candidates<kFormThreads, kFormRows, false>(v, cmask, tile0, rs.cand + tile * kTile, totals);
-  if (threadIdx.x == 0) rs.cnt[tile] = ncand;
-  for (int i = threadIdx.x; i < kBins0; i += kFormThreads)
-    if (hist[i]) atomicAdd(&rs.hist0[i], hist[i]);
+  if (threadIdx.x == 0) rs.cnt[tile] = total;
 }
 
 // ---------------------------------------------------------------------------
@@ -286,6 +328,7 @@ __global__ void __launch_bounds__(kFormThreads, 5) topk_form_kernel(const Compre
 // kCluster CTAs per worker).
 // ---------------------------------------------------------------------------
 struct SelectSmem {
+  uint32_t hist_t[kBins0];          // this CTA's top-digit histogram (read by the cluster)
   uint32_t hist_a[kBins1];          // this CTA's middle-digit histogram (read by the cluster)
   uint32_t hist_b[kBins1];          // this CTA's low-digit histogram (read by the cluster)
   uint32_t full[kBins0];            // a whole histogram (top digit; then the cluster's sums)
@@ -312,12 +355,13 @@ __device__ __forceinline__ uint2 chunk_candidate(const uint2* cand, const uint32
   return cand[(tc0 + lo) * kTile + (f - tpre[lo])];
 }
 
-// Sums the cluster's copies of one histogram into sm.full[0, kBins1).  The
+// Sums the cluster's copies of one histogram into sm.full[0, BINS).  The
 // cluster barrier publishes every CTA's counts; each histogram buffer is
 // written once per selection round, so no barrier is needed after the reads.
+template <int BINS>
 __device__ __forceinline__ void cluster_sum(cg::cluster_group& cluster, uint32_t* local, SelectSmem& sm) {
   cluster.sync();
-  for (int i = threadIdx.x; i < kBins1; i += kSelThreads) {
+  for (int i = threadIdx.x; i < BINS; i += kSelThreads) {
     uint32_t s = 0;
 #pragma unroll
     for (int r = 0; r < kCluster; ++r) s += cluster.map_shared_rank(local, r)[i];
@@ -347,22 +391,14 @@ topk_select_kernel(const CompressArgs a, int64_t k, void* scratch) {
   bool fast = (tau_word & kTauValid) != 0;
   const bool reg_tiles = nt <= (int64_t)kSelThreads * kRegTiles;
 
-  // Top digit b0 from the first pass's histogram (every CTA alike); the
-  // tile counts are fetched alongside.
-  for (int i = threadIdx.x; i < kBins0; i += kSelThreads) sm.full[i] = __ldcg(&rs.hist0[i]);
+  // the first pass's tile counts
   uint32_t cnt_r[kRegTiles];
 #pragma unroll
   for (int q = 0; q < kRegTiles; ++q) {
     const int64_t t = (int64_t)threadIdx.x * kRegTiles + q;
-    cnt_r[q] = (reg_tiles && t < nt) ? rs.cnt[t] : 0u;
+    cnt_r[q] = (fast && reg_tiles && t < nt) ? rs.cnt[t] : 0u;
   }
-  if (threadIdx.x == 0) {
-    sm.sel[0] = 0;
-    sm.sel[1] = (uint32_t)k;
-  }
-  __syncthreads();
-  block_select<kSelThreads, kBins0>(sm.full, (uint32_t)k, &sm.sel[0], &sm.sel[1], sm.warp_sums);
-  const uint32_t b0 = sm.sel[0], krem0 = sm.sel[1];
+  uint32_t b0 = 0;  // top digit of T
 
   // This CTA's share: candidates [F0, F1) in prefix coordinates, lying in
   // tiles [ta, tb).  With one chunk, sm.tpre[i] is the prefix at tile ta + i.
@@ -377,8 +413,9 @@ topk_select_kernel(const CompressArgs a, int64_t k, void* scratch) {
     __syncthreads();
   };
 
+  const int64_t t0 = nt * rank / kCluster, t1 = nt * (rank + 1) / kCluster;  // this CTA's tiles
+
   auto set_up = [&]() {
-    const int64_t t0 = nt * rank / kCluster, t1 = nt * (rank + 1) / kCluster;
     if (fast && reg_tiles) {
       // the tile counts are in registers: one scan gives every prefix
       uint32_t local = 0;
@@ -460,7 +497,7 @@ topk_select_kernel(const CompressArgs a, int64_t k, void* scratch) {
       one_chunk = (tb - ta) <= kChunkTiles;
       if (one_chunk && tb > ta) load_chunk(ta, (int)(tb - ta));
     } else {
-      // re-extract this CTA's tiles: every element with top digit >= b0
+      // re-extract this CTA's tiles from p: every element with top digit >= b0
       for (int64_t t = t0; t < t1; ++t) {
         const int64_t tile0 = t * kTile;
         float v[kSelRows][4];
@@ -551,25 +588,66 @@ topk_select_kernel(const CompressArgs a, int64_t k, void* scratch) {
     if (fill) __syncthreads();
   };
 
-  uint32_t T = 0, need = 0, my_above = 0;
+  // Histogram of the top digit over all of p in this CTA's tiles.
+  auto histogram_p = [&]() {
+    for (int64_t t = t0; t < t1; ++t) {
+#pragma unroll
+      for (int i = 0; i < kSelRows; ++i) {
+        const int64_t j = t * kTile + 4 * ((int64_t)i * kSelThreads + threadIdx.x);
+        if (j + 3 < a.d) {
+          const float4 x = *reinterpret_cast<const float4*>(e + j);
+          atomicAdd(&sm.hist_t[key_of(x.x) >> 20], 1u);
+          atomicAdd(&sm.hist_t[key_of(x.y) >> 20], 1u);
+          atomicAdd(&sm.hist_t[key_of(x.z) >> 20], 1u);
+          atomicAdd(&sm.hist_t[key_of(x.w) >> 20], 1u);
+        } else {
+          for (int64_t jj = j; jj < a.d && jj < j + 4; ++jj) atomicAdd(&sm.hist_t[key_of(e[jj]) >> 20], 1u);
+        }
+      }
+    }
+    __syncthreads();
+  };
+
+  uint32_t T = 0, need = 0;
   for (int attempt = 0; attempt < 2; ++attempt) {
     if (attempt > 0) cluster.sync();  // every CTA is done reading the first round's histograms
-    set_up();
-    // middle digit
+    for (int i = threadIdx.x; i < kBins0; i += kSelThreads) sm.hist_t[i] = 0;
     for (int i = threadIdx.x; i < kBins1; i += kSelThreads) {
       sm.hist_a[i] = 0;
       sm.hist_b[i] = 0;
     }
     __syncthreads();
-    my_above = 0;  // keys whose top digit is above b0
+    // top digit: over the candidates, or over all of p
+    bool filled = false;
+    if (fast) {
+      set_up();
+      for_each(
+          [&](uint2 c, bool valid) {
+            if (valid) atomicAdd(&sm.hist_t[key_bits(c.y) >> 20], 1u);
+          },
+          cached);
+      filled = cached;
+    } else {
+      histogram_p();
+    }
+    cluster_sum<kBins0>(cluster, sm.hist_t, sm);
+    if (threadIdx.x == 0) {
+      sm.sel[0] = 0;
+      sm.sel[1] = (uint32_t)k;
+    }
+    __syncthreads();
+    block_select<kSelThreads, kBins0>(sm.full, (uint32_t)k, &sm.sel[0], &sm.sel[1], sm.warp_sums);
+    b0 = sm.sel[0];
+    const uint32_t krem0 = sm.sel[1];
+    if (!fast) set_up();  // candidates: every element with top digit >= b0
+    // middle digit
     for_each(
         [&](uint2 c, bool valid) {
           const uint32_t key = key_bits(c.y);
           if (valid && (key >> 20) == b0) atomicAdd(&sm.hist_a[(key >> 10) & 1023u], 1u);
-          my_above += valid && (key >> 20) > b0;
         },
-        cached);
-    cluster_sum(cluster, sm.hist_a, sm);
+        cached && !filled);
+    cluster_sum<kBins1>(cluster, sm.hist_a, sm);
     if (threadIdx.x == 0) {
       sm.sel[2] = 0;
       sm.sel[3] = krem0;
@@ -585,7 +663,7 @@ topk_select_kernel(const CompressArgs a, int64_t k, void* scratch) {
           if (valid && (key >> 10) == hi21) atomicAdd(&sm.hist_b[key & 1023u], 1u);
         },
         false);
-    cluster_sum(cluster, sm.hist_b, sm);
+    cluster_sum<kBins1>(cluster, sm.hist_b, sm);
     if (threadIdx.x == 0) {
       sm.sel[4] = 0;
       sm.sel[5] = krem1;
@@ -604,7 +682,9 @@ topk_select_kernel(const CompressArgs a, int64_t k, void* scratch) {
   // top digit above b0, or middle digit above T's, or low digit above T's.
   {
     const uint32_t b1 = (T >> 10) & 1023u, b2 = T & 1023u;
-    uint32_t part = my_above;
+    uint32_t part = 0;
+    for (int i = threadIdx.x; i < kBins0; i += kSelThreads)
+      if ((uint32_t)i > b0) part += sm.hist_t[i];
     for (int i = threadIdx.x; i < kBins1; i += kSelThreads) {
       if ((uint32_t)i > b1) part += sm.hist_a[i];
       if ((uint32_t)i > b2) part += sm.hist_b[i];
@@ -720,13 +800,10 @@ topk_select_kernel(const CompressArgs a, int64_t k, void* scratch) {
     }
   }
 
-  // For the next call: the histogram back to zero, the threshold 15/16 of T.
-  if (rank == 0) {
-    for (int i = threadIdx.x; i < kBins0; i += kSelThreads) rs.hist0[i] = 0;
-    if (threadIdx.x == 0) {
-      const float t_next = __fmul_rn(__uint_as_float(T), 0.9375f);
-      rs.state[ST_TAU] = kTauValid | key_of(t_next);
-    }
+  // For the next call: the candidate threshold, 15/16 of T.
+  if (rank == 0 && threadIdx.x == 0) {
+    const float t_next = __fmul_rn(__uint_as_float(T), 0.9375f);
+    rs.state[ST_TAU] = kTauValid | key_of(t_next);
   }
 }
 
@@ -987,7 +1064,7 @@ size_t topk_scratch_bytes(int64_t d, int32_t nworkers) {
 
 size_t topk_scratch_clear_bytes(int64_t d) {
   (void)d;
-  return (size_t)(kBins0 + ST_TAU) * 4u;
+  return (size_t)ST_TAU * 4u;
 }
 
 // Raises a kernel's dynamic shared memory limit when its static plus dynamic
