@@ -484,7 +484,8 @@ __global__ void __launch_bounds__(256) squant_server_kernel(const ServerArgs s) 
 // owns the 32/b consecutive elements of its word; per worker, in worker
 // order, it decodes them with the worker's scale (broadcast by shuffle from
 // the lane that loaded it) and V[code] (b = 8: the bank-replicated table;
-// b = 4: 15 entries in a register, looked up by shuffle; b = 2: a select).
+// b = 4: the worker's 15 products fl(s * V[c]), one per lane, looked up by
+// shuffle; b = 2: two bit tests, level-0 codes skipped).
 // Worker-order sums from +0, so the result equals the oracle's bit for bit.
 template <int BITS, bool POW2>
 __global__ void __launch_bounds__(32 * kTmaWarps)
@@ -577,14 +578,29 @@ squant_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap
     for (int e = 0; e < EPL; ++e) acc[e] = 0.f;
     // one worker's contribution, added in worker order
     auto add_worker = [&](uint32_t word, float sc) {
+      if constexpr (BITS == 2) {
+        // code 0: -s, 1: +0, 2: +s (fl(s * 1) = s).  Adding +0 never changes
+        // the sum (it starts at +0 and so is never -0), so level-0 codes are
+        // skipped: per element one bit test picks the sign, one the add.
+        const float nsc = -sc;
+#pragma unroll
+        for (int e = 0; e < EPL; ++e) {
+          const bool zero = (word >> (2 * e)) & 1u;
+          const float v = ((word >> (2 * e + 1)) & 1u) ? sc : nsc;
+          acc[e] = zero ? acc[e] : __fadd_rn(acc[e], v);
+        }
+        return;
+      }
+      // b = 4: lane c first forms this worker's decoded value of code c,
+      // fl(s * V[c]); each element then fetches its value with one shuffle
+      const float T4 = (BITS == 4) ? __fmul_rn(sc, V4) : 0.f;
 #pragma unroll
       for (int e = 0; e < EPL; ++e) {
         float v;
         if constexpr (BITS == 2) {
-          const uint32_t code = (word >> (2 * e)) & 3u;
-          v = (code == 0) ? -sc : (code == 2 ? sc : 0.f);  // fl(s * 1) = s
+          v = 0.f;
         } else if constexpr (BITS == 4) {
-          v = __fmul_rn(sc, __shfl_sync(kFullMask, V4, (int)((word >> (4 * e)) & MASK)));
+          v = __shfl_sync(kFullMask, T4, (int)((word >> (4 * e)) & MASK));
         } else {
           v = __fmul_rn(sc, V8l[__byte_perm(word, 0u, 0x4440u | (uint32_t)e) * 32u]);
         }
@@ -602,7 +618,24 @@ squant_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap
       add_worker(w2, s2);
       add_worker(w3, s3);
     }
-    for (; m < s.M; ++m) add_worker(words[32 * m], __shfl_sync(kFullMask, my_scale, m));
+    if constexpr (BITS == 2) {
+      // the last M mod 4 workers as one more group of four: the missing
+      // workers read as all-level-0 words, which add nothing
+      if (m < s.M) {
+        uint32_t wq[4];
+        float sq[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          const bool ok = m + u < s.M;
+          wq[u] = ok ? words[32 * (m + u)] : 0x55555555u;
+          sq[u] = __shfl_sync(kFullMask, my_scale, (m + u) & 31);
+        }
+#pragma unroll
+        for (int u = 0; u < 4; ++u) add_worker(wq[u], sq[u]);
+      }
+    } else {
+      for (; m < s.M; ++m) add_worker(words[32 * m], __shfl_sync(kFullMask, my_scale, m));
+    }
 #pragma unroll
     for (int q = 0; q < EPL / 4; ++q) {
       const int64_t j = j0 + 4 * q;
