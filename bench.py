@@ -89,8 +89,15 @@ def selected_workload(args):
 # bytes per step (algorithmic minimum)
 # ---------------------------------------------------------------------------
 
+def bucket_count(wl) -> int:
+    if wl.layer_buckets:
+        offs = wl.segment_offsets()
+        return sum(-(-(b - a) // wl.bucket) for a, b in zip(offs[:-1], offs[1:]))
+    return -(-wl.d // wl.bucket)
+
+
 def message_payload_bytes(wl) -> int:
-    nb = -(-wl.d // wl.bucket)
+    nb = bucket_count(wl)
     if wl.compressor == SIGN:
         return 4 * nb + 4 * (-(-wl.d // 32))
     if wl.compressor in (SQUANT, QSGD):
@@ -307,6 +314,7 @@ def workload_config(wl, args):
          "parallelism": f"replicas{args.gpus}" if args.gpus > 1 else "single"}
     if wl.compressor in (SIGN, SQUANT, QSGD):
         c["bucket"] = wl.bucket
+        c["buckets"] = "per layer segment" if wl.layer_buckets else "flat"
     if wl.compressor in (SQUANT, QSGD):
         c["bits"] = wl.bits
     if wl.compressor == TOPK:
@@ -339,6 +347,8 @@ def run_gpu(args, rank, world, local):
     h = P.create(P.make_config(d=wl.d, M=wl.M, compressor=wl.compressor, lr=wl.lr, bucket=wl.bucket,
                                k=wl.k, bits=wl.bits, seed=wl.seed, flags=flags,
                                cuda_stream=stream.cuda_stream))
+    if wl.layer_buckets:
+        h.set_segments(wl.segment_offsets())
     mb = h.message_bytes()
     g = torch.empty((wl.M, wl.d), dtype=torch.float32, device=dev)
     msgs = torch.empty((wl.M, mb), dtype=torch.uint8, device=dev)

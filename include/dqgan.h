@@ -235,6 +235,25 @@ DQGAN_API int64_t dqgan_state_bytes(const dqgan_handle* h);
 DQGAN_API int dqgan_save_state(dqgan_handle* h, void* host_dst, int64_t bytes);
 DQGAN_API int dqgan_load_state(dqgan_handle* h, const void* host_src, int64_t bytes);
 
+/*
+ * Per-layer bucketing (the layer-wise variant of Section 2.4's bucketed
+ * compressors): buckets restart at every layer boundary instead of tiling
+ * the flat vector w = [theta, phi].  offsets: host array of nseg + 1
+ * int64, 0 = offsets[0] < offsets[1] < ... < offsets[nseg] = d, the inner
+ * ones multiples of 32; segment i is [offsets[i], offsets[i+1]) and is cut
+ * into buckets of `bucket` elements from its own start, its last bucket
+ * partial.  Buckets are numbered in element order, so a message holds one
+ * scale per bucket of every segment, then the same payload as without
+ * segments; dqgan_message_bytes() reflects the new size (the config-only
+ * dqgan_message_layout() describes the flat layout).  nseg = 0 with
+ * offsets = NULL returns to flat buckets.  Only for DQGAN_SIGN, SQUANT and
+ * QSGD (else DQGAN_ERR_UNSUPPORTED), and only before the first step
+ * (step counter 1; else DQGAN_ERR_INVALID_ARG).  Synchronous; allocates two
+ * small device tables (nb + 1 int64 bucket starts, one u32 per 32 elements).
+ * With segments the servers take their per-element scale-lookup paths.
+ */
+DQGAN_API int dqgan_set_segments(dqgan_handle* h, const int64_t* offsets, int32_t nseg);
+
 /* Kernels this handle has launched so far. */
 DQGAN_API uint64_t dqgan_launch_count(const dqgan_handle* h);
 

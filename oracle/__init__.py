@@ -38,6 +38,8 @@ class _OrcCfg(ctypes.Structure):
         ("bits", ctypes.c_int32),
         ("keep_lookahead", ctypes.c_int32),
         ("seed", ctypes.c_uint64),
+        ("nseg", ctypes.c_int32),
+        ("seg", ctypes.POINTER(ctypes.c_int64)),
     ]
 
 
@@ -52,11 +54,20 @@ class Config:
     bits: int = 8
     seed: int = 0
     keep_lookahead: bool = False
+    segments: tuple | None = None  # layer segment offsets 0 = s_0 < ... < s_n = d, or None
 
     def c_struct(self) -> _OrcCfg:
-        return _OrcCfg(d=self.d, k=self.k, lr=self.lr, M=self.M, compressor=self.compressor,
-                       bucket=self.bucket, bits=self.bits,
-                       keep_lookahead=1 if self.keep_lookahead else 0, seed=self.seed)
+        c = _OrcCfg(d=self.d, k=self.k, lr=self.lr, M=self.M, compressor=self.compressor,
+                    bucket=self.bucket, bits=self.bits,
+                    keep_lookahead=1 if self.keep_lookahead else 0, seed=self.seed)
+        if self.segments is not None:
+            offs = np.ascontiguousarray(self.segments, dtype=np.int64)
+            assert offs.ndim == 1 and offs.size >= 2 and offs[0] == 0 and offs[-1] == self.d
+            assert np.all(np.diff(offs) > 0)
+            c.nseg = offs.size - 1
+            c.seg = offs.ctypes.data_as(ctypes.POINTER(ctypes.c_int64))
+            c._keep = offs  # the offsets must outlive the struct
+        return c
 
 
 _lib = None
@@ -96,6 +107,10 @@ def lib() -> ctypes.CDLL:
         L.orc_server_step.restype = None
         L.orc_lookahead.argtypes = [ctypes.c_int64, f32p, f32p, f32p]
         L.orc_lookahead.restype = None
+        L.orc_bucket_count.argtypes = [cfgp]
+        L.orc_bucket_count.restype = ctypes.c_int64
+        L.orc_bucket_starts.argtypes = [cfgp, P(ctypes.c_int64)]
+        L.orc_bucket_starts.restype = None
         _lib = L
     return _lib
 
@@ -131,6 +146,15 @@ def layout(cfg: Config):
 
 def message_bytes(cfg: Config) -> int:
     return layout(cfg)[2]
+
+
+def bucket_starts(cfg: Config) -> np.ndarray:
+    """starts[0..nb]: bucket b covers [starts[b], starts[b+1])."""
+    c = cfg.c_struct()
+    nb = lib().orc_bucket_count(ctypes.byref(c))
+    out = np.zeros(nb + 1, dtype=np.int64)
+    lib().orc_bucket_starts(ctypes.byref(c), out.ctypes.data_as(ctypes.POINTER(ctypes.c_int64)))
+    return out
 
 
 def sign_l1(x: np.ndarray, bucket: int) -> float:

@@ -46,6 +46,9 @@ typedef struct orc_cfg {
   int32_t bits;     /* stochastic quantiser: bits per code */
   int32_t keep_lookahead; /* 1: also produce h = eta*F + e (Algorithm 2) */
   uint64_t seed;
+  int32_t nseg;     /* 0: buckets tile the flat vector; else the number of  */
+                    /* layer segments, each bucketed on its own             */
+  const int64_t* seg; /* nseg + 1 offsets: 0 = seg[0] < seg[1] < ... = d    */
 } orc_cfg;
 
 /* ------------------------------------------------------------------------ */
@@ -97,8 +100,35 @@ float orc_squant_uniform(uint64_t seed, int32_t worker, int64_t step, int64_t j)
 /* ------------------------------------------------------------------------ */
 static int64_t round256(int64_t x) { return (x + 255) / 256 * 256; }
 
+/* ------------------------------------------------------------------------ */
+/* Buckets.  Without segments, bucket b covers [b*n, min((b+1)*n, d)).  With */
+/* layer segments (the per-layer variant of Section 2.4's bucketing), each   */
+/* segment [seg[i], seg[i+1]) is cut into buckets of n from its own start,   */
+/* the last one partial; buckets are numbered in element order.             */
+/* ------------------------------------------------------------------------ */
+int64_t orc_bucket_count(const orc_cfg* c) {
+  if (c->nseg <= 0) return (c->d + c->bucket - 1) / c->bucket;
+  int64_t nb = 0;
+  for (int32_t i = 0; i < c->nseg; ++i) nb += (c->seg[i + 1] - c->seg[i] + c->bucket - 1) / c->bucket;
+  return nb;
+}
+
+/* starts[0..nb]: bucket b covers [starts[b], starts[b+1]). */
+void orc_bucket_starts(const orc_cfg* c, int64_t* starts) {
+  int64_t b = 0;
+  if (c->nseg <= 0) {
+    int64_t nb = orc_bucket_count(c);
+    for (b = 0; b < nb; ++b) starts[b] = b * c->bucket;
+    starts[nb] = c->d;
+    return;
+  }
+  for (int32_t i = 0; i < c->nseg; ++i)
+    for (int64_t j = c->seg[i]; j < c->seg[i + 1]; j += c->bucket) starts[b++] = j;
+  starts[b] = c->d;
+}
+
 int64_t orc_layout(const orc_cfg* c, int64_t* off_scales, int64_t* off_payload) {
-  int64_t nb = (c->d + c->bucket - 1) / c->bucket;
+  int64_t nb = (c->compressor == ORC_TOPK || c->compressor == ORC_IDENTITY) ? 0 : orc_bucket_count(c);
   *off_scales = 0;
   switch (c->compressor) {
     case ORC_SIGN: {
@@ -285,11 +315,17 @@ void orc_decode(const orc_cfg* c, const uint8_t* msg, float* q) {
     case ORC_SIGN: {
       const float* scales = (const float*)(msg + off_s);
       const uint32_t* words = (const uint32_t*)(msg + off_p);
-      for (int64_t j = 0; j < d; ++j) {
-        float s = scales[j / c->bucket];
-        int neg = (words[j >> 5] >> (j & 31)) & 1u;
-        q[j] = neg ? -s : s;
+      int64_t nb = orc_bucket_count(c);
+      int64_t* starts = (int64_t*)malloc((size_t)(nb + 1) * 8);
+      orc_bucket_starts(c, starts);
+      for (int64_t b = 0; b < nb; ++b) {
+        float s = scales[b];
+        for (int64_t j = starts[b]; j < starts[b + 1]; ++j) {
+          int neg = (words[j >> 5] >> (j & 31)) & 1u;
+          q[j] = neg ? -s : s;
+        }
       }
+      free(starts);
       break;
     }
     case ORC_SQUANT:
@@ -298,11 +334,17 @@ void orc_decode(const orc_cfg* c, const uint8_t* msg, float* q) {
       const uint32_t* words = (const uint32_t*)(msg + off_p);
       int32_t K = (1 << (c->bits - 1)) - 1;
       uint32_t mask = (1u << c->bits) - 1u;
-      for (int64_t j = 0; j < d; ++j) {
-        int64_t bitpos = j * c->bits;
-        int32_t code = (int32_t)((words[bitpos >> 5] >> (bitpos & 31)) & mask);
-        q[j] = orc_squant_decode(code, scales[j / c->bucket], K);
+      int64_t nb = orc_bucket_count(c);
+      int64_t* starts = (int64_t*)malloc((size_t)(nb + 1) * 8);
+      orc_bucket_starts(c, starts);
+      for (int64_t b = 0; b < nb; ++b) {
+        for (int64_t j = starts[b]; j < starts[b + 1]; ++j) {
+          int64_t bitpos = j * c->bits;
+          int32_t code = (int32_t)((words[bitpos >> 5] >> (bitpos & 31)) & mask);
+          q[j] = orc_squant_decode(code, scales[b], K);
+        }
       }
+      free(starts);
       break;
     }
     case ORC_TOPK: {
@@ -348,10 +390,12 @@ void orc_worker_step(const orc_cfg* c, int32_t worker, int64_t step, const float
     case ORC_SIGN: {
       float* scales = (float*)(msg + off_s);
       uint32_t* words = (uint32_t*)(msg + off_p);
-      int64_t nb = (d + c->bucket - 1) / c->bucket;
+      int64_t nb = orc_bucket_count(c);
+      int64_t* starts = (int64_t*)malloc((size_t)(nb + 1) * 8);
+      orc_bucket_starts(c, starts);
       for (int64_t b = 0; b < nb; ++b) {
-        int64_t start = b * c->bucket;
-        int64_t count = (d - start < c->bucket) ? d - start : c->bucket;
+        int64_t start = starts[b];
+        int64_t count = starts[b + 1] - start;
         float s = orc_sign_scale(p + start, count, c->bucket);
         scales[b] = s;
         for (int64_t j = start; j < start + count; ++j) {
@@ -360,6 +404,7 @@ void orc_worker_step(const orc_cfg* c, int32_t worker, int64_t step, const float
           q[j] = neg ? -s : s;
         }
       }
+      free(starts);
       break;
     }
     case ORC_SQUANT:
@@ -367,11 +412,13 @@ void orc_worker_step(const orc_cfg* c, int32_t worker, int64_t step, const float
       float* scales = (float*)(msg + off_s);
       uint32_t* words = (uint32_t*)(msg + off_p);
       int32_t K = (1 << (c->bits - 1)) - 1;
-      int64_t nb = (d + c->bucket - 1) / c->bucket;
+      int64_t nb = orc_bucket_count(c);
+      int64_t* starts = (int64_t*)malloc((size_t)(nb + 1) * 8);
+      orc_bucket_starts(c, starts);
       int32_t* codes = (int32_t*)malloc((size_t)c->bucket * 4);
       for (int64_t b = 0; b < nb; ++b) {
-        int64_t start = b * c->bucket;
-        int64_t count = (d - start < c->bucket) ? d - start : c->bucket;
+        int64_t start = starts[b];
+        int64_t count = starts[b + 1] - start;
         squant_bucket(c, worker, step, start, count, p + start, &scales[b], codes);
         for (int64_t j = 0; j < count; ++j) {
           int64_t bitpos = (start + j) * c->bits;
@@ -380,6 +427,7 @@ void orc_worker_step(const orc_cfg* c, int32_t worker, int64_t step, const float
         }
       }
       free(codes);
+      free(starts);
       break;
     }
     case ORC_TOPK: {

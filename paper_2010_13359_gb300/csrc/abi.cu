@@ -8,6 +8,7 @@
 #include <cstring>
 #include <new>
 #include <string>
+#include <vector>
 
 #include "internal.cuh"
 
@@ -23,6 +24,8 @@ struct dqgan_handle {
   void* scratch = nullptr;
   size_t scratch_bytes = 0;
   uint32_t* err_word = nullptr;  // device error word written by bounded waits
+  int64_t* seg_bstart = nullptr;     // layer segments: nb + 1 bucket starts (device)
+  uint32_t* seg_wbucket = nullptr;   // layer segments: bucket of every 32-element word (device)
   CUtensorMap words_map;         // TMA map of the last message buffer the server saw
   const void* words_map_msgs = nullptr;
   bool words_map_ok = false;
@@ -109,6 +112,7 @@ dq::CompressArgs compress_args(dqgan_handle* h, const float* g, int64_t g_stride
   a.msg_stride = msg_stride;
   a.d = h->cfg.d;
   a.nb = h->nb;
+  a.bstart = h->seg_bstart;
   a.off_payload = h->lay.off_payload;
   a.lr = h->cfg.lr;
   a.bucket = h->cfg.bucket;
@@ -283,6 +287,8 @@ int dqgan_destroy(dqgan_handle* h) {
   if (h->h) cudaFree(h->h);
   if (h->scratch) cudaFree(h->scratch);
   if (h->err_word) cudaFree(h->err_word);
+  if (h->seg_bstart) cudaFree(h->seg_bstart);
+  if (h->seg_wbucket) cudaFree(h->seg_wbucket);
   const cudaError_t st = cudaGetLastError();
   delete h;
   if (st != cudaSuccess) return set_error(nullptr, DQGAN_ERR_CUDA, "destroy: %s", cudaGetErrorString(st));
@@ -290,6 +296,70 @@ int dqgan_destroy(dqgan_handle* h) {
 }
 
 int64_t dqgan_message_bytes(const dqgan_handle* h) { return h ? h->lay.total : -1; }
+
+int dqgan_set_segments(dqgan_handle* h, const int64_t* offsets, int32_t nseg) {
+  if (!h) return set_error(nullptr, DQGAN_ERR_INVALID_ARG, "handle is NULL");
+  const dqgan_config& c = h->cfg;
+  if (c.compressor != DQGAN_SIGN && c.compressor != DQGAN_SQUANT && c.compressor != DQGAN_QSGD)
+    return set_error(h, DQGAN_ERR_UNSUPPORTED, "layer segments apply to the bucketed compressors only");
+  if (h->t != 1) return set_error(h, DQGAN_ERR_INVALID_ARG, "layer segments must be set before the first step");
+  if (nseg < 0 || (nseg > 0 && !offsets) || (nseg == 0 && offsets))
+    return set_error(h, DQGAN_ERR_INVALID_ARG, "nseg = %d with offsets %s", nseg, offsets ? "set" : "NULL");
+  std::vector<int64_t> starts;
+  if (nseg > 0) {
+    if (offsets[0] != 0 || offsets[nseg] != c.d)
+      return set_error(h, DQGAN_ERR_INVALID_ARG, "offsets must run from 0 to d = %lld", (long long)c.d);
+    for (int32_t i = 0; i < nseg; ++i) {
+      if (offsets[i + 1] <= offsets[i])
+        return set_error(h, DQGAN_ERR_INVALID_ARG, "offsets must increase (offset %d)", i + 1);
+      if (i > 0 && (offsets[i] & 31))
+        return set_error(h, DQGAN_ERR_INVALID_ARG, "offset %d = %lld is not a multiple of 32", i,
+                         (long long)offsets[i]);
+    }
+    for (int32_t i = 0; i < nseg; ++i)
+      for (int64_t j = offsets[i]; j < offsets[i + 1]; j += c.bucket) starts.push_back(j);
+    starts.push_back(c.d);
+  }
+  cudaError_t st = cudaStreamSynchronize(h->stream);  // no step is in flight; tables are replaced
+  if (st != cudaSuccess) return cuda_fail(h, st, "synchronize");
+  if (h->seg_bstart) cudaFree(h->seg_bstart);
+  if (h->seg_wbucket) cudaFree(h->seg_wbucket);
+  h->seg_bstart = nullptr;
+  h->seg_wbucket = nullptr;
+  h->words_map_msgs = nullptr;  // the payload moves with the scale section
+  dq::message_layout(c, &h->lay);
+  h->nb = (c.d + c.bucket - 1) / c.bucket;
+  if (nseg == 0) return DQGAN_OK;
+  const int64_t nb = (int64_t)starts.size() - 1;
+  const int64_t nwords = (c.d + 31) / 32;
+  std::vector<uint32_t> wb((size_t)nwords);
+  for (int64_t b = 0; b < nb; ++b)
+    for (int64_t w = starts[b] / 32; w < (starts[b + 1] + 31) / 32; ++w) wb[(size_t)w] = (uint32_t)b;
+  if ((st = cudaMalloc(&h->seg_bstart, starts.size() * sizeof(int64_t))) != cudaSuccess ||
+      (st = cudaMalloc(&h->seg_wbucket, wb.size() * sizeof(uint32_t))) != cudaSuccess) {
+    if (h->seg_bstart) cudaFree(h->seg_bstart);
+    h->seg_bstart = nullptr;
+    h->seg_wbucket = nullptr;
+    cudaGetLastError();
+    return set_error(h, st == cudaErrorMemoryAllocation ? DQGAN_ERR_OOM : DQGAN_ERR_CUDA, "segment tables: %s",
+                     cudaGetErrorString(st));
+  }
+  if ((st = cudaMemcpy(h->seg_bstart, starts.data(), starts.size() * sizeof(int64_t), cudaMemcpyHostToDevice)) !=
+          cudaSuccess ||
+      (st = cudaMemcpy(h->seg_wbucket, wb.data(), wb.size() * sizeof(uint32_t), cudaMemcpyHostToDevice)) !=
+          cudaSuccess) {
+    cudaFree(h->seg_bstart);
+    cudaFree(h->seg_wbucket);
+    h->seg_bstart = nullptr;
+    h->seg_wbucket = nullptr;
+    return cuda_fail(h, st, "copying the segment tables");
+  }
+  h->nb = nb;
+  h->lay.off_payload = round_up(4 * nb, 256);
+  const int64_t payload_words = c.compressor == DQGAN_SIGN ? nwords : (c.d * c.bits + 31) / 32;
+  h->lay.total = round_up(h->lay.off_payload + 4 * payload_words, 256);
+  return DQGAN_OK;
+}
 
 int dqgan_worker_compress(dqgan_handle* h, int32_t i, const float* g, void* out_msg) {
   if (!h) return set_error(nullptr, DQGAN_ERR_INVALID_ARG, "handle is NULL");
@@ -329,11 +399,13 @@ int dqgan_server_aggregate_update(dqgan_handle* h, const void* msgs_all, float* 
   s.M_pow2 = is_pow2(h->cfg.M) ? 1 : 0;
   s.inv_M = 1.0f / (float)h->cfg.M;
   s.err = h->err_word;
+  s.word_bucket = h->seg_wbucket;
   s.sign_words_map = nullptr;
   s.squant_words_map = nullptr;
-  const bool tma_sign = h->cfg.compressor == DQGAN_SIGN && h->cfg.bucket >= 1024 && h->cfg.M <= 32;
-  const bool tma_squant = (h->cfg.compressor == DQGAN_SQUANT || h->cfg.compressor == DQGAN_QSGD) && h->cfg.M <= 32 &&
-                          h->cfg.bucket >= 32 * (32 / h->cfg.bits);
+  const bool flat = h->seg_wbucket == nullptr;
+  const bool tma_sign = flat && h->cfg.compressor == DQGAN_SIGN && h->cfg.bucket >= 1024 && h->cfg.M <= 32;
+  const bool tma_squant = flat && (h->cfg.compressor == DQGAN_SQUANT || h->cfg.compressor == DQGAN_QSGD) &&
+                          h->cfg.M <= 32 && h->cfg.bucket >= 32 * (32 / h->cfg.bits);
   if (tma_sign || tma_squant) {
     if (h->words_map_msgs != msgs_all) {
       const int64_t payload_words = tma_sign ? (s.d + 31) / 32 : (s.d * s.bits + 31) / 32;

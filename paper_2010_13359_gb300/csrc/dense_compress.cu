@@ -18,12 +18,21 @@
 namespace dq {
 namespace {
 
-// Loads this thread's CPL chunks c = c0 + 32 i of the bucket starting at
-// element `base` and forms p.  Out-of-bucket or out-of-range elements read as
-// 0 and give p = 0.  sg (if HOLD) receives fl(eta * g) for the lookahead.
+// Bucket b covers [bucket_base, bucket_end): b*n up to n elements, or the
+// table of bucket starts when buckets restart at every layer segment.
+__device__ __forceinline__ int64_t bucket_base(const CompressArgs& a, int64_t b) {
+  return a.bstart ? a.bstart[b] : b * a.bucket;
+}
+__device__ __forceinline__ int64_t bucket_end(const CompressArgs& a, int64_t b) {
+  return a.bstart ? a.bstart[b + 1] : min64(b * a.bucket + a.bucket, a.d);
+}
+
+// Loads this thread's CPL chunks c = c0 + 32 i of the bucket [base, end) and
+// forms p.  Elements outside the bucket read as 0 and give p = 0.  sg (if
+// HOLD) receives fl(eta * g) for the lookahead.
 template <int CPL, bool HOLD>
 __device__ __forceinline__ void load_and_form(const CompressArgs& a, const float* g, const float* e,
-                                              int64_t base, int c0, bool full,
+                                              int64_t base, int64_t end, int c0, bool full,
                                               float (&p)[CPL][4], float (&sg)[HOLD ? CPL : 1][4]) {
   const int nchunk = a.bucket >> 2;
   if (full) {
@@ -51,7 +60,7 @@ __device__ __forceinline__ void load_and_form(const CompressArgs& a, const float
 #pragma unroll
       for (int q = 0; q < 4; ++q) {
         const int64_t j = base + 4 * c + q;
-        const bool ok = (c < nchunk) && (j < a.d);
+        const bool ok = (c < nchunk) && (j < end);
         const float gq = ok ? g[j] : 0.f;
         const float eq = ok ? e[j] : 0.f;
         const float s = __fmul_rn(a.lr, gq);
@@ -135,8 +144,9 @@ sign_compress_kernel(const CompressArgs a) {
   float* h = KEEP_H ? a.h + (int64_t)worker * a.ld : nullptr;
   uint8_t* msg = a.msg + (int64_t)row * a.msg_stride;
 
-  const int64_t base = b * a.bucket;
-  const int64_t count = valid ? min64((int64_t)a.bucket, a.d - base) : 0;
+  const int64_t base = valid ? bucket_base(a, b) : 0;
+  const int64_t end = valid ? bucket_end(a, b) : 0;
+  const int64_t count = end - base;
   const bool full = (count == a.bucket);
   const int nchunk = a.bucket >> 2;
   const int row0 = wib * CPT;  // first chunk row of this warp
@@ -144,7 +154,7 @@ sign_compress_kernel(const CompressArgs a) {
   float p[CPT][4];
   float sg[HOLD ? CPT : 1][4];
   if (valid) {
-    load_and_form<CPT, HOLD>(a, g, e, base, 32 * row0 + lane, full, p, sg);
+    load_and_form<CPT, HOLD>(a, g, e, base, end, 32 * row0 + lane, full, p, sg);
   } else {
 #pragma unroll
     for (int i = 0; i < CPT; ++i)
@@ -185,19 +195,18 @@ sign_compress_kernel(const CompressArgs a) {
 
   uint32_t* words = reinterpret_cast<uint32_t*>(msg + a.off_payload);
   const int64_t word0 = base >> 5;
-  const int64_t nwords = (a.d + 31) >> 5;
-  const int words_in_bucket = a.bucket >> 5;
+  const int64_t word_end = (end + 31) >> 5;  // buckets start on word boundaries
 #pragma unroll
   for (int i = 0; i < CPT; ++i) {
     const uint32_t wv = pack_sign_row(p[i][0], p[i][1], p[i][2], p[i][3], lane);
     if ((lane & 3) == 0 && lane < 16) {
       const int wib_word = 4 * (row0 + i) + (lane >> 2);
-      if (wib_word < words_in_bucket && word0 + wib_word < nwords) words[word0 + wib_word] = wv;
+      if (word0 + wib_word < word_end) words[word0 + wib_word] = wv;
     }
     const int c = 32 * (row0 + i) + lane;
     if (c < nchunk) {
       const int64_t j = base + 4 * c;
-      const int nvalid = (int)min64(4, a.d - j);
+      const int nvalid = (int)min64(4, end - j);
       if (nvalid > 0) {
         float en[4];
 #pragma unroll
@@ -244,8 +253,9 @@ squant_compress_kernel(const CompressArgs a) {
   float* h = KEEP_H ? a.h + (int64_t)worker * a.ld : nullptr;
   uint8_t* msg = a.msg + (int64_t)row * a.msg_stride;
 
-  const int64_t base = b * a.bucket;
-  const int64_t count = valid ? min64((int64_t)a.bucket, a.d - base) : 0;
+  const int64_t base = valid ? bucket_base(a, b) : 0;
+  const int64_t end = valid ? bucket_end(a, b) : 0;
+  const int64_t count = end - base;
   const bool full = (count == a.bucket);
   const int nchunk = a.bucket >> 2;
   const int row0 = wib * CPT;  // first chunk row of this warp
@@ -253,7 +263,7 @@ squant_compress_kernel(const CompressArgs a) {
   float p[CPT][4];
   float sg[HOLD ? CPT : 1][4];
   if (valid) {
-    load_and_form<CPT, HOLD>(a, g, e, base, 32 * row0 + lane, full, p, sg);
+    load_and_form<CPT, HOLD>(a, g, e, base, end, 32 * row0 + lane, full, p, sg);
   } else {
 #pragma unroll
     for (int i = 0; i < CPT; ++i)
@@ -320,7 +330,7 @@ squant_compress_kernel(const CompressArgs a) {
     const int c = 32 * (row0 + i) + lane;
     const int64_t j = base + 4 * c;
     const int64_t cg = j >> 2;  // global chunk index = Philox counter word 0
-    const int nvalid = (c < nchunk) ? (int)max64(0, min64(4, a.d - j)) : 0;
+    const int nvalid = (c < nchunk) ? (int)max64(0, min64(4, end - j)) : 0;
     const uint4 r4 = philox4x32_10(make_uint4((uint32_t)cg, (uint32_t)worker, a.step, kSquantTag),
                                    a.seed_lo, a.seed_hi);
     const uint32_t rq[4] = {r4.x, r4.y, r4.z, r4.w};
@@ -353,7 +363,9 @@ squant_compress_kernel(const CompressArgs a) {
       widx = cg >> 2;
       writer = (lane & 3) == 0;
     }
-    if (writer && c < nchunk && widx < nwords) words[widx] = wv;
+    // a code word holds 32 / BITS elements of one bucket (buckets start on
+    // multiples of 32): write the words that start inside this bucket
+    if (writer && c < nchunk && widx < nwords && widx * (32 / BITS) < end) words[widx] = wv;
     if (nvalid > 0) store_chunk<KEEP_H, HOLD, CPT>(a, g, e, h, j, full, nvalid, en, sg, i);
   }
 }

@@ -43,7 +43,8 @@ struct CompressArgs {
   uint8_t* msg;        // message of row y at msg + y * msg_stride
   int64_t msg_stride;  // bytes
   int64_t d;
-  int64_t nb;          // buckets: ceil(d / bucket)
+  int64_t nb;          // buckets: ceil(d / bucket), or the sum over layer segments
+  const int64_t* bstart;  // nb + 1 bucket starts (layer segments), or nullptr: b * bucket
   int64_t off_payload; // byte offset of the payload section in a message
   float lr;
   int32_t bucket;
@@ -69,6 +70,7 @@ struct ServerArgs {
   float inv_M;          // exact 1/M when M is a power of two
   int32_t M_pow2;       // 1 if M is a power of two (then x/M == x * inv_M exactly)
   uint32_t* err;        // device error word (bit 0: a bounded wait timed out)
+  const uint32_t* word_bucket;  // bucket of each 32-element word (layer segments), or nullptr: j / bucket
   const CUtensorMap* sign_words_map;    // TMA map of the M messages' sign words, or nullptr
   const CUtensorMap* squant_words_map;  // TMA map of the M messages' code words, or nullptr
 };

@@ -43,7 +43,7 @@ __global__ void __launch_bounds__(256) sign_server_kernel(const ServerArgs s) {
   const int64_t c = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   const int64_t j = 4 * c;
   if (j >= s.d) return;
-  const int64_t bkt = j / s.bucket;
+  const int64_t bkt = s.word_bucket ? (int64_t)s.word_bucket[j >> 5] : j / s.bucket;
   const int64_t word = j >> 5;
   const int shift = (int)(j & 31);
   float acc[4] = {0.f, 0.f, 0.f, 0.f};
@@ -428,7 +428,7 @@ __global__ void __launch_bounds__(256) squant_server_kernel(const ServerArgs s) 
   for (int64_t c = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; c < nchunks;
        c += (int64_t)gridDim.x * blockDim.x) {
     const int64_t j = 4 * c;
-    const int64_t bkt = j / s.bucket;
+    const int64_t bkt = s.word_bucket ? (int64_t)s.word_bucket[j >> 5] : j / s.bucket;
     const int64_t bitpos = j * BITS;  // a chunk's 4*BITS bits never straddle a word
     const int64_t word = bitpos >> 5;
     const int shift = (int)(bitpos & 31);
@@ -762,6 +762,11 @@ unsigned chunk_blocks(int64_t d, int threads) {
 }  // namespace
 
 cudaError_t launch_sign_server(const ServerArgs& s, cudaStream_t stream, uint64_t* launches) {
+  if (s.word_bucket) {  // buckets restart at layer segments: per-element scale lookup
+    sign_server_kernel<<<chunk_blocks(s.d, 256), 256, 0, stream>>>(s);
+    *launches += 1;
+    return cudaGetLastError();
+  }
   if (s.bucket >= 1024 && s.M <= 32 && s.sign_words_map != nullptr) {
     const bool p2 = s.M_pow2 != 0;
     cudaError_t st;
@@ -811,7 +816,7 @@ cudaError_t launch_sign_server(const ServerArgs& s, cudaStream_t stream, uint64_
 }
 
 cudaError_t launch_squant_server(const ServerArgs& s, cudaStream_t stream, uint64_t* launches) {
-  if (s.squant_words_map != nullptr && s.M <= 32 && s.bucket >= 32 * (32 / s.bits)) {
+  if (s.squant_words_map != nullptr && s.word_bucket == nullptr && s.M <= 32 && s.bucket >= 32 * (32 / s.bits)) {
     const bool p2 = s.M_pow2 != 0;
     cudaError_t st = cudaErrorInvalidValue;
     switch (s.bits) {

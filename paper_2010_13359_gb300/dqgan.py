@@ -90,6 +90,7 @@ def load_library(path: str = LIBRARY) -> ctypes.CDLL:
         "dqgan_last_error": (ctypes.c_char_p, [H]),
         "dqgan_topk_compress_noalloc": (ctypes.c_int, [P, P, P, i64, i64, ctypes.c_float, P]),
         "dqgan_selftest_wait_timeout": (ctypes.c_int, [H, ctypes.c_uint32]),
+        "dqgan_set_segments": (ctypes.c_int, [H, ctypes.POINTER(i64), i32]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(L, name)
@@ -168,6 +169,14 @@ class Handle:
         return self._h
 
     # -- hot path -------------------------------------------------------------
+    def set_segments(self, offsets) -> None:
+        """dqgan_set_segments: per-layer buckets; offsets from 0 to d (None: flat)."""
+        if offsets is None:
+            _check(load_library().dqgan_set_segments(self._h, None, 0), self._h)
+            return
+        arr = (ctypes.c_int64 * len(offsets))(*[int(x) for x in offsets])
+        _check(load_library().dqgan_set_segments(self._h, arr, len(offsets) - 1), self._h)
+
     def message_bytes(self) -> int:
         return int(load_library().dqgan_message_bytes(self._h))
 

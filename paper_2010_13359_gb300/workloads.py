@@ -47,6 +47,7 @@ class Workload:
     dist: str = "gauss"                    # "gauss" or "student_t3"
     dist_scale: float = 1.0
     w0_std: float = 0.02
+    layer_buckets: bool = False            # buckets restart at every segment (per-layer bucketing)
 
     # -- layer segments ------------------------------------------------------
     def segments(self) -> tuple[list[int], list[float]]:
@@ -68,6 +69,11 @@ class Workload:
             stds = [float(math.exp(v)) for v in rng.uniform(lo, hi, size=S)]
         assert sum(sizes) == self.d and len(sizes) == len(stds)
         return sizes, stds
+
+    def segment_offsets(self) -> tuple:
+        """0 = o_0 < o_1 < ... < o_S = d, the layer segment boundaries."""
+        sizes, _ = self.segments()
+        return tuple(int(x) for x in np.concatenate([[0], np.cumsum(sizes)]))
 
     def std_vector_np(self) -> np.ndarray:
         sizes, stds = self.segments()
@@ -168,6 +174,10 @@ WORKLOADS = {
     "resnet_squant_b8": _resnet("resnet_squant_b8", 8),
     # Same vector with QSGD's l2-scaled quantiser (Eq. (qsgd)), 8 bits.
     "resnet_qsgd_b8": _resnet("resnet_qsgd_b8", 8, QSGD),
+    # The same two vectors with buckets restarting at every layer segment.
+    "dcgan_sign_layers": _dcgan("dcgan_sign_layers", SIGN, bucket=1024, layer_buckets=True),
+    "resnet_squant_b8_layers": _resnet("resnet_squant_b8", 8).replace(name="resnet_squant_b8_layers",
+                                                                       layer_buckets=True),
     # Heavy-tailed stress case: d = 1e8, M = 32, sign per 4096, Student-t(3) * 1e-3.
     "stress_sign": Workload(name="stress_sign", d=100_000_000, M=32, compressor=SIGN, bucket=4096,
                             steps=20, n_segments=1, segment_sizes=(100_000_000,),

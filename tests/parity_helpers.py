@@ -37,7 +37,7 @@ def sections(ocfg: oracle.Config, msg: np.ndarray) -> dict:
     d = ocfg.d
     msg = np.asarray(msg, np.uint8)
     if ocfg.compressor in (oracle.SIGN, oracle.SQUANT, oracle.QSGD):
-        nb = -(-d // ocfg.bucket)
+        nb = len(oracle.bucket_starts(ocfg)) - 1
         nwords = -(-d // 32) if ocfg.compressor == oracle.SIGN else -(-d * ocfg.bits // 32)
         return {"scales": msg[off_s:off_s + 4 * nb].view(np.uint32),
                 "payload": msg[off_p:off_p + 4 * nwords].view(np.uint32)}
@@ -65,9 +65,9 @@ def assert_bits_equal(got: np.ndarray, want: np.ndarray, ctx: str = ""):
                              f"gpu {got[bad[:5]].tolist()} oracle {want[bad[:5]].tolist()}")
 
 
-def oracle_config(d, M, compressor, lr=1e-3, bucket=512, k=1, bits=8, seed=0, keep=False):
+def oracle_config(d, M, compressor, lr=1e-3, bucket=512, k=1, bits=8, seed=0, keep=False, segments=None):
     return oracle.Config(d=d, M=M, compressor=compressor, lr=lr, bucket=bucket, k=k, bits=bits,
-                         seed=seed, keep_lookahead=keep)
+                         seed=seed, keep_lookahead=keep, segments=segments)
 
 
 def slice_messages(ocfg: oracle.Config, msgs: np.ndarray, a: int, b: int):

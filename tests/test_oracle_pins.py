@@ -709,3 +709,112 @@ def test_qsgd_unbiased_and_variance_bound_over_philox_streams(bits):
     vv = np.sum(v.astype(np.float64) ** 2)
     assert resid <= min(n / K ** 2, math.sqrt(n) / K) * vv * 1.1
     assert resid < vv
+
+
+# --- per-layer-segment bucketing (buckets restart at every layer boundary) ---
+
+def _py_bucket_starts(segments, bucket):
+    starts = []
+    for a, b in zip(segments[:-1], segments[1:]):
+        starts.extend(range(a, b, bucket))
+    return starts + [segments[-1]]
+
+
+def _random_segments(rng, d, n):
+    cuts = np.sort(rng.choice(np.arange(1, d // 32), size=n - 1, replace=False)) * 32
+    return tuple([0, *cuts.tolist(), d])
+
+
+SEG_CASES = [(5_000, 512, (0, 32, 64, 4_000, 5_000)), (4_131, 256, (0, 4_131)),
+             (10_007, 1024, None), (3_000, 32, (0, 96, 2_048, 2_080, 3_000))]
+
+
+@pytest.mark.parametrize("d,bucket,segs", SEG_CASES)
+def test_segment_bucket_boundaries(d, bucket, segs):
+    segs = segs if segs is not None else _random_segments(np.random.default_rng(d), d, 7)
+    cfg = oracle.Config(d=d, M=1, compressor=oracle.SIGN, bucket=bucket, segments=segs)
+    got = oracle.bucket_starts(cfg)
+    assert got.tolist() == _py_bucket_starts(list(segs), bucket)
+    _, off_p, total = oracle.layout(cfg)
+    nb = len(got) - 1
+    assert off_p == -(-4 * nb // 256) * 256
+    assert total == -(-(off_p + 4 * (-(-d // 32))) // 256) * 256
+
+
+@pytest.mark.parametrize("d,bucket,segs", SEG_CASES)
+def test_segmented_sign_is_flat_sign_per_segment(d, bucket, segs):
+    """The sign compressor is deterministic and bucket-local: with segments,
+    each segment's scales and bits are those of the flat compressor run on
+    that segment alone."""
+    rng = np.random.default_rng(11)
+    segs = segs if segs is not None else _random_segments(np.random.default_rng(d), d, 7)
+    g = (rng.standard_normal(d) * np.exp(rng.uniform(-3, 2, d))).astype(np.float32)
+    cfg = oracle.Config(d=d, M=1, compressor=oracle.SIGN, bucket=bucket, lr=0.5, segments=segs)
+    e = np.zeros(d, np.float32)
+    msg = oracle.worker_step(cfg, 0, 1, g, e)
+    off_s, off_p, _ = oracle.layout(cfg)
+    scales = msg[off_s:].view(np.float32)
+    words = msg[off_p:].view(np.uint32)
+    b = 0
+    for a, z in zip(segs[:-1], segs[1:]):
+        sub = oracle.Config(d=z - a, M=1, compressor=oracle.SIGN, bucket=bucket, lr=0.5)
+        e_sub = np.zeros(z - a, np.float32)
+        m_sub = oracle.worker_step(sub, 0, 1, g[a:z].copy(), e_sub)
+        s_off, p_off, _ = oracle.layout(sub)
+        nb_sub = -(-(z - a) // bucket)
+        assert np.array_equal(scales[b:b + nb_sub].view(np.uint32),
+                              m_sub[s_off:s_off + 4 * nb_sub].view(np.uint32))
+        bits_seg = np.unpackbits(words.view(np.uint8), bitorder="little")[a:z]
+        bits_sub = np.unpackbits(m_sub[p_off:].view(np.uint8), bitorder="little")[:z - a]
+        assert np.array_equal(bits_seg, bits_sub)
+        assert_array_bits(e[a:z], e_sub)
+        b += nb_sub
+
+
+def assert_array_bits(x, y):
+    assert np.array_equal(np.asarray(x, np.float32).view(np.uint32), np.asarray(y, np.float32).view(np.uint32))
+
+
+@pytest.mark.parametrize("comp", [oracle.SQUANT, oracle.QSGD])
+@pytest.mark.parametrize("d,bucket,segs", SEG_CASES)
+def test_segmented_quantiser_scales_and_levels(comp, d, bucket, segs):
+    """Each bucket's scale is the max (or the l2 norm) over exactly its own
+    elements, and every decoded value is a level of that bucket's scale
+    bracketing |p_j| (Section 2.4, proof of Theorem 2)."""
+    rng = np.random.default_rng(5)
+    segs = segs if segs is not None else _random_segments(np.random.default_rng(d), d, 7)
+    bits = 4
+    K = 2 ** (bits - 1) - 1
+    g = (rng.standard_normal(d) * np.exp(rng.uniform(-3, 2, d))).astype(np.float32)
+    cfg = oracle.Config(d=d, M=1, compressor=comp, bucket=bucket, bits=bits, lr=1.0, seed=9, segments=segs)
+    e = np.zeros(d, np.float32)
+    msg = oracle.worker_step(cfg, 0, 3, g, e)
+    p = g.astype(np.float64)
+    q = oracle.decode(cfg, msg).astype(np.float64)
+    starts = _py_bucket_starts(list(segs), bucket)
+    scales = msg[oracle.layout(cfg)[0]:].view(np.float32)
+    for b in range(len(starts) - 1):
+        blk = p[starts[b]:starts[b + 1]]
+        want = np.max(np.abs(blk)) if comp == oracle.SQUANT else np.sqrt(np.sum(blk * blk))
+        assert abs(scales[b] - want) <= 1e-6 * want + 1e-30, (b, scales[b], want)
+        s = float(scales[b])
+        lv = np.abs(q[starts[b]:starts[b + 1]]) / s * K
+        t = np.abs(blk) / s * K
+        assert np.all(np.abs(lv - np.round(lv)) < 1e-4)
+        assert np.all(np.round(lv) >= np.floor(t * (1 - 1e-6)) - 1e-9)
+        assert np.all(np.round(lv) <= np.ceil(t * (1 + 1e-6)) + 1e-9)
+
+
+@pytest.mark.parametrize("comp", [oracle.SIGN, oracle.SQUANT, oracle.QSGD])
+def test_one_segment_is_the_flat_layout(comp):
+    rng = np.random.default_rng(2)
+    d = 9_001
+    g = rng.standard_normal((2, d)).astype(np.float32)
+    out = []
+    for segs in (None, (0, d)):
+        cfg = oracle.Config(d=d, M=2, compressor=comp, bucket=512, bits=8, lr=0.1, seed=4, segments=segs)
+        st = oracle.State(cfg)
+        w = np.zeros(d, np.float32)
+        out.append((st.step(g, w), w))
+    assert np.array_equal(out[0][0], out[1][0])
+    assert np.array_equal(out[0][1], out[1][1])
