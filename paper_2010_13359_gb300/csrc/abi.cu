@@ -404,7 +404,7 @@ int dqgan_server_aggregate_update(dqgan_handle* h, const void* msgs_all, float* 
   s.squant_words_map = nullptr;
   const bool flat = h->seg_wbucket == nullptr;
   const bool tma_sign = flat && h->cfg.compressor == DQGAN_SIGN && h->cfg.bucket >= 1024 && h->cfg.M <= 32;
-  const bool tma_squant = flat && (h->cfg.compressor == DQGAN_SQUANT || h->cfg.compressor == DQGAN_QSGD) &&
+  const bool tma_squant = (h->cfg.compressor == DQGAN_SQUANT || h->cfg.compressor == DQGAN_QSGD) &&
                           h->cfg.M <= 32 && h->cfg.bucket >= 32 * (32 / h->cfg.bits);
   if (tma_sign || tma_squant) {
     if (h->words_map_msgs != msgs_all) {

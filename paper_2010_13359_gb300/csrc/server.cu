@@ -487,7 +487,9 @@ __global__ void __launch_bounds__(256) squant_server_kernel(const ServerArgs s) 
 // b = 4: the worker's 15 products fl(s * V[c]), one per lane, looked up by
 // shuffle; b = 2: two bit tests, level-0 codes skipped).
 // Worker-order sums from +0, so the result equals the oracle's bit for bit.
-template <int BITS, bool POW2>
+// With layer segments (SEG) a slice may hold words of several buckets: each
+// lane then reads the workers' scales of its own word's bucket.
+template <int BITS, bool POW2, bool SEG>
 __global__ void __launch_bounds__(32 * kTmaWarps)
 squant_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap tmap) {
   constexpr int K = (1 << (BITS - 1)) - 1;
@@ -532,7 +534,7 @@ squant_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap
 
   const int spb = s.bucket / SLICE;  // slices per bucket
   const int64_t nb = (s.d + s.bucket - 1) / s.bucket;
-  const int64_t nslices = nb * spb;
+  const int64_t nslices = SEG ? (s.d + SLICE - 1) / SLICE : nb * spb;
   const int64_t stride = (int64_t)gridDim.x * kTmaWarps;
   const int32_t x0 = (int32_t)(s.off_payload >> 2);
   const bool active = lane < s.M;
@@ -566,8 +568,23 @@ squant_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap
         for (int r = 0; r < 4; ++r) wv[4 * q + r] = (j + r < s.d) ? s.w[j + r] : 0.f;
       }
     }
+    // The slice's bucket; with layer segments, each lane's word's bucket, and
+    // whether they differ within the slice (warp-uniform).
+    int64_t bkt = b, my_bkt = b;
+    bool mixed = false;
+    if constexpr (SEG) {
+      my_bkt = (j0 < s.d) ? (int64_t)__ldg(s.word_bucket + (j0 >> 5)) : -1;
+      bkt = __shfl_sync(kFullMask, my_bkt, 0);  // lane 0's elements always exist
+      if (my_bkt < 0) my_bkt = bkt;
+      mixed = !__all_sync(kFullMask, my_bkt == bkt);
+    }
     const float my_scale =
-        active ? __ldg(reinterpret_cast<const float*>(s.msgs + (int64_t)lane * s.msg_stride) + b) : 0.f;
+        active ? __ldg(reinterpret_cast<const float*>(s.msgs + (int64_t)lane * s.msg_stride) + bkt) : 0.f;
+    // worker m's scale for this lane's elements
+    auto scale_of = [&](int m) -> float {
+      if (SEG && mixed) return __ldg(reinterpret_cast<const float*>(s.msgs + (int64_t)m * s.msg_stride) + my_bkt);
+      return __shfl_sync(kFullMask, my_scale, m);
+    };
     ok = mbar_wait_bounded(&bar[cur], (it >> 1) & 1u, s.err);
     ok = __all_sync(kFullMask, ok);
     if (!ok) break;
@@ -592,8 +609,10 @@ squant_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap
         return;
       }
       // b = 4: lane c first forms this worker's decoded value of code c,
-      // fl(s * V[c]); each element then fetches its value with one shuffle
-      const float T4 = (BITS == 4) ? __fmul_rn(sc, V4) : 0.f;
+      // fl(s * V[c]); each element then fetches its value with one shuffle.
+      // (With layer segments the lanes' scales may differ: look up V[c] and
+      // multiply by the lane's own scale instead.)
+      const float T4 = (BITS == 4) ? __fmul_rn(mixed ? 1.0f : sc, V4) : 0.f;
 #pragma unroll
       for (int e = 0; e < EPL; ++e) {
         float v;
@@ -601,6 +620,7 @@ squant_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap
           v = 0.f;
         } else if constexpr (BITS == 4) {
           v = __shfl_sync(kFullMask, T4, (int)((word >> (4 * e)) & MASK));
+          if (mixed) v = __fmul_rn(sc, v);
         } else {
           v = __fmul_rn(sc, V8l[__byte_perm(word, 0u, 0x4440u | (uint32_t)e) * 32u]);
         }
@@ -611,8 +631,8 @@ squant_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap
     for (; m + 4 <= s.M; m += 4) {
       const uint32_t w0 = words[32 * m], w1 = words[32 * (m + 1)];
       const uint32_t w2 = words[32 * (m + 2)], w3 = words[32 * (m + 3)];
-      const float s0 = __shfl_sync(kFullMask, my_scale, m), s1 = __shfl_sync(kFullMask, my_scale, m + 1);
-      const float s2 = __shfl_sync(kFullMask, my_scale, m + 2), s3 = __shfl_sync(kFullMask, my_scale, m + 3);
+      const float s0 = scale_of(m), s1 = scale_of(m + 1);
+      const float s2 = scale_of(m + 2), s3 = scale_of(m + 3);
       add_worker(w0, s0);
       add_worker(w1, s1);
       add_worker(w2, s2);
@@ -628,13 +648,14 @@ squant_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap
         for (int u = 0; u < 4; ++u) {
           const bool ok = m + u < s.M;
           wq[u] = ok ? words[32 * (m + u)] : 0x55555555u;
-          sq[u] = __shfl_sync(kFullMask, my_scale, (m + u) & 31);
+          if constexpr (SEG) sq[u] = ok ? scale_of(m + u) : 0.f;
+          else sq[u] = __shfl_sync(kFullMask, my_scale, (m + u) & 31);
         }
 #pragma unroll
         for (int u = 0; u < 4; ++u) add_worker(wq[u], sq[u]);
       }
     } else {
-      for (; m < s.M; ++m) add_worker(words[32 * m], __shfl_sync(kFullMask, my_scale, m));
+      for (; m < s.M; ++m) add_worker(words[32 * m], scale_of(m));
     }
 #pragma unroll
     for (int q = 0; q < EPL / 4; ++q) {
@@ -735,9 +756,9 @@ cudaError_t launch_sign_tma(const ServerArgs& s, cudaStream_t stream) {
   return cudaGetLastError();
 }
 
-template <int BITS, bool POW2>
+template <int BITS, bool POW2, bool SEG>
 cudaError_t launch_squant_tma(const ServerArgs& s, cudaStream_t stream) {
-  auto kern = squant_server_tma_kernel<BITS, POW2>;
+  auto kern = squant_server_tma_kernel<BITS, POW2, SEG>;
   const int smem = kTmaWarps * 2 * s.M * 128 + 128;  // + alignment slack
   int dev = 0;
   cudaError_t st = cudaGetDevice(&dev);
@@ -747,7 +768,8 @@ cudaError_t launch_squant_tma(const ServerArgs& s, cudaStream_t stream) {
   if ((st = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return st;
   if ((st = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, 32 * kTmaWarps, smem)) != cudaSuccess)
     return st;
-  const int64_t nslices = ((s.d + s.bucket - 1) / s.bucket) * (s.bucket / (32 * (32 / BITS)));
+  const int64_t nslices = SEG ? (s.d + 32 * (32 / BITS) - 1) / (32 * (32 / BITS))
+                              : ((s.d + s.bucket - 1) / s.bucket) * (s.bucket / (32 * (32 / BITS)));
   const int64_t need = (nslices + kTmaWarps - 1) / kTmaWarps;
   const int64_t cap = (int64_t)sms * (per_sm > 0 ? per_sm : 1);
   kern<<<(unsigned)(need < cap ? need : cap), 32 * kTmaWarps, smem, stream>>>(s, *s.squant_words_map);
@@ -816,14 +838,20 @@ cudaError_t launch_sign_server(const ServerArgs& s, cudaStream_t stream, uint64_
 }
 
 cudaError_t launch_squant_server(const ServerArgs& s, cudaStream_t stream, uint64_t* launches) {
-  if (s.squant_words_map != nullptr && s.word_bucket == nullptr && s.M <= 32 && s.bucket >= 32 * (32 / s.bits)) {
+  if (s.squant_words_map != nullptr && s.M <= 32 && s.bucket >= 32 * (32 / s.bits)) {
     const bool p2 = s.M_pow2 != 0;
     cudaError_t st = cudaErrorInvalidValue;
+#define DQ_SQ_TMA(B)                                                                          \
+  st = s.word_bucket ? (p2 ? launch_squant_tma<B, true, true>(s, stream)                      \
+                           : launch_squant_tma<B, false, true>(s, stream))                    \
+                     : (p2 ? launch_squant_tma<B, true, false>(s, stream)                     \
+                           : launch_squant_tma<B, false, false>(s, stream))
     switch (s.bits) {
-      case 2: st = p2 ? launch_squant_tma<2, true>(s, stream) : launch_squant_tma<2, false>(s, stream); break;
-      case 4: st = p2 ? launch_squant_tma<4, true>(s, stream) : launch_squant_tma<4, false>(s, stream); break;
-      case 8: st = p2 ? launch_squant_tma<8, true>(s, stream) : launch_squant_tma<8, false>(s, stream); break;
+      case 2: DQ_SQ_TMA(2); break;
+      case 4: DQ_SQ_TMA(4); break;
+      case 8: DQ_SQ_TMA(8); break;
     }
+#undef DQ_SQ_TMA
     *launches += 1;
     return st;
   }
