@@ -18,15 +18,6 @@
 namespace dq {
 namespace {
 
-// Bucket b covers [bucket_base, bucket_end): b*n up to n elements, or the
-// table of bucket starts when buckets restart at every layer segment.
-__device__ __forceinline__ int64_t bucket_base(const CompressArgs& a, int64_t b) {
-  return a.bstart ? a.bstart[b] : b * a.bucket;
-}
-__device__ __forceinline__ int64_t bucket_end(const CompressArgs& a, int64_t b) {
-  return a.bstart ? a.bstart[b + 1] : min64(b * a.bucket + a.bucket, a.d);
-}
-
 // Loads this thread's CPL chunks c = c0 + 32 i of the bucket [base, end) and
 // forms p.  Elements outside the bucket read as 0 and give p = 0.  sg (if
 // HOLD) receives fl(eta * g) for the lookahead.
@@ -122,7 +113,7 @@ __device__ __forceinline__ void store_chunk(const CompressArgs& a, const float* 
 // and warp 0 runs the chains, so the sum is the same whatever WPB is.
 // ---------------------------------------------------------------------------
 
-template <int CPT, int WPB, bool KEEP_H>
+template <int CPT, int WPB, bool KEEP_H, bool SEG>
 __global__ void __launch_bounds__(32 * WPB * (WPB < 4 ? 4 / WPB : 1))
 sign_compress_kernel(const CompressArgs a) {
   constexpr bool HOLD = KEEP_H && CPT <= 8;
@@ -144,9 +135,10 @@ sign_compress_kernel(const CompressArgs a) {
   float* h = KEEP_H ? a.h + (int64_t)worker * a.ld : nullptr;
   uint8_t* msg = a.msg + (int64_t)row * a.msg_stride;
 
-  const int64_t base = valid ? bucket_base(a, b) : 0;
-  const int64_t end = valid ? bucket_end(a, b) : 0;
-  const int64_t count = end - base;
+  // flat buckets: [b n, b n + n) clipped to d; layer buckets (SEG): the table
+  const int64_t base = SEG ? (valid ? a.bstart[b] : 0) : b * a.bucket;
+  const int64_t end = SEG ? (valid ? a.bstart[b + 1] : 0) : a.d;  // elements at or past `end` are not this bucket's
+  const int64_t count = SEG ? end - base : (valid ? min64((int64_t)a.bucket, a.d - base) : 0);
   const bool full = (count == a.bucket);
   const int nchunk = a.bucket >> 2;
   const int row0 = wib * CPT;  // first chunk row of this warp
@@ -195,13 +187,14 @@ sign_compress_kernel(const CompressArgs a) {
 
   uint32_t* words = reinterpret_cast<uint32_t*>(msg + a.off_payload);
   const int64_t word0 = base >> 5;
-  const int64_t word_end = (end + 31) >> 5;  // buckets start on word boundaries
+  const int64_t word_end = SEG ? (end + 31) >> 5 : (a.d + 31) >> 5;  // buckets start on word boundaries
+  const int words_in_bucket = a.bucket >> 5;
 #pragma unroll
   for (int i = 0; i < CPT; ++i) {
     const uint32_t wv = pack_sign_row(p[i][0], p[i][1], p[i][2], p[i][3], lane);
     if ((lane & 3) == 0 && lane < 16) {
       const int wib_word = 4 * (row0 + i) + (lane >> 2);
-      if (word0 + wib_word < word_end) words[word0 + wib_word] = wv;
+      if (wib_word < words_in_bucket && word0 + wib_word < word_end) words[word0 + wib_word] = wv;
     }
     const int c = 32 * (row0 + i) + lane;
     if (c < nchunk) {
@@ -226,7 +219,7 @@ sign_compress_kernel(const CompressArgs a) {
 // ---------------------------------------------------------------------------
 // L2 = false: s_b = max |p_j| (Hou et al.); L2 = true: s_b = fl(sqrt(sum p_j^2))
 // (QSGD), the sum of squares in the fixed chain order of the scaled sign.
-template <int CPT, int WPB, int BITS, bool KEEP_H, bool L2>
+template <int CPT, int WPB, int BITS, bool KEEP_H, bool L2, bool SEG>
 __global__ void __launch_bounds__(32 * WPB * (WPB < 4 ? 4 / WPB : 1))
 squant_compress_kernel(const CompressArgs a) {
   constexpr int K = (1 << (BITS - 1)) - 1;
@@ -253,9 +246,10 @@ squant_compress_kernel(const CompressArgs a) {
   float* h = KEEP_H ? a.h + (int64_t)worker * a.ld : nullptr;
   uint8_t* msg = a.msg + (int64_t)row * a.msg_stride;
 
-  const int64_t base = valid ? bucket_base(a, b) : 0;
-  const int64_t end = valid ? bucket_end(a, b) : 0;
-  const int64_t count = end - base;
+  // flat buckets: [b n, b n + n) clipped to d; layer buckets (SEG): the table
+  const int64_t base = SEG ? (valid ? a.bstart[b] : 0) : b * a.bucket;
+  const int64_t end = SEG ? (valid ? a.bstart[b + 1] : 0) : a.d;  // elements at or past `end` are not this bucket's
+  const int64_t count = SEG ? end - base : (valid ? min64((int64_t)a.bucket, a.d - base) : 0);
   const bool full = (count == a.bucket);
   const int nchunk = a.bucket >> 2;
   const int row0 = wib * CPT;  // first chunk row of this warp
@@ -365,7 +359,7 @@ squant_compress_kernel(const CompressArgs a) {
     }
     // a code word holds 32 / BITS elements of one bucket (buckets start on
     // multiples of 32): write the words that start inside this bucket
-    if (writer && c < nchunk && widx < nwords && widx * (32 / BITS) < end) words[widx] = wv;
+    if (writer && c < nchunk && widx < nwords && (!SEG || widx * (32 / BITS) < end)) words[widx] = wv;
     if (nvalid > 0) store_chunk<KEEP_H, HOLD, CPT>(a, g, e, h, j, full, nvalid, en, sg, i);
   }
 }
@@ -420,8 +414,14 @@ cudaError_t sign_dispatch_keep(const CompressArgs& a, bool keep_h, cudaStream_t 
   constexpr int BPC = WPB < 4 ? 4 / WPB : 1;
   constexpr int THREADS = 32 * WPB * BPC;
   const dim3 grid((unsigned)((a.nb + BPC - 1) / BPC), (unsigned)a.nworkers);
-  if (keep_h) sign_compress_kernel<CPT, WPB, true><<<grid, THREADS, 0, stream>>>(a);
-  else sign_compress_kernel<CPT, WPB, false><<<grid, THREADS, 0, stream>>>(a);
+  const bool seg = a.bstart != nullptr;
+  if (keep_h) {
+    if (seg) sign_compress_kernel<CPT, WPB, true, true><<<grid, THREADS, 0, stream>>>(a);
+    else sign_compress_kernel<CPT, WPB, true, false><<<grid, THREADS, 0, stream>>>(a);
+  } else {
+    if (seg) sign_compress_kernel<CPT, WPB, false, true><<<grid, THREADS, 0, stream>>>(a);
+    else sign_compress_kernel<CPT, WPB, false, false><<<grid, THREADS, 0, stream>>>(a);
+  }
   return cudaGetLastError();
 }
 
@@ -430,8 +430,14 @@ cudaError_t squant_dispatch_keep(const CompressArgs& a, bool keep_h, cudaStream_
   constexpr int BPC = WPB < 4 ? 4 / WPB : 1;
   constexpr int THREADS = 32 * WPB * BPC;
   const dim3 grid((unsigned)((a.nb + BPC - 1) / BPC), (unsigned)a.nworkers);
-  if (keep_h) squant_compress_kernel<CPT, WPB, BITS, true, L2><<<grid, THREADS, 0, stream>>>(a);
-  else squant_compress_kernel<CPT, WPB, BITS, false, L2><<<grid, THREADS, 0, stream>>>(a);
+  const bool seg = a.bstart != nullptr;
+  if (keep_h) {
+    if (seg) squant_compress_kernel<CPT, WPB, BITS, true, L2, true><<<grid, THREADS, 0, stream>>>(a);
+    else squant_compress_kernel<CPT, WPB, BITS, true, L2, false><<<grid, THREADS, 0, stream>>>(a);
+  } else {
+    if (seg) squant_compress_kernel<CPT, WPB, BITS, false, L2, true><<<grid, THREADS, 0, stream>>>(a);
+    else squant_compress_kernel<CPT, WPB, BITS, false, L2, false><<<grid, THREADS, 0, stream>>>(a);
+  }
   return cudaGetLastError();
 }
 
