@@ -398,6 +398,12 @@ def run_gpu(args, rank, world, local):
         e2e_steps = max(1, min(args.steps, 10))
         copy_stream = torch.cuda.Stream(dev)
         copied = [torch.cuda.Event() for _ in range(wl.M)]
+        # the parameters go back on their own stream, overlapping the next
+        # step's gradient reads (the link is full duplex); the next server
+        # step waits for that copy before it updates w again
+        back_stream = torch.cuda.Stream(dev)
+        served, sent = torch.cuda.Event(), torch.cuda.Event()
+        sent.record(back_stream)
 
         def e2e_step():
             if args.e2e_mode == "copy":
@@ -414,8 +420,13 @@ def run_gpu(args, rank, world, local):
                     h.worker_compress(i, g[i], msgs[i])
             else:  # the kernels read the pinned host gradients in place
                 h.workers_compress_all(g_host, wl.d, msgs)
+            stream.wait_event(sent)
             h.server_aggregate_update(msgs, w)
-            w_host.copy_(w, non_blocking=True)
+            served.record(stream)
+            back_stream.wait_event(served)
+            with torch.cuda.stream(back_stream):
+                w_host.copy_(w, non_blocking=True)
+                sent.record(back_stream)
 
         e2e_step()
         torch.cuda.synchronize(dev)
@@ -424,12 +435,27 @@ def run_gpu(args, rank, world, local):
         a.record(stream)
         for _ in range(e2e_steps):
             e2e_step()
+        stream.wait_event(sent)  # the last step's parameters are on the host
         b.record(stream)
         torch.cuda.synchronize(dev)
         e2e_ms = max_over_ranks(a.elapsed_time(b), world, dev)
+        # the host link's own rate: a bulk copy of the same pinned gradients
+        lk = min(g_host.numel(), 1 << 28)
+        src, dst = g_host.view(-1)[:lk], g.view(-1)[:lk]
+        dst.copy_(src, non_blocking=True)
+        a.record(stream)
+        for _ in range(3):
+            dst.copy_(src, non_blocking=True)
+        b.record(stream)
+        torch.cuda.synchronize(dev)
+        link_gbs = 3 * lk * 4 / (a.elapsed_time(b) * 1e6)
+        h2d = int(g.numel() * 4)
         e2e = {"value": whole_job_rate(units, e2e_steps, world, e2e_ms), "unit": UNIT,
-               "h2d_bytes_per_step": int(g.numel() * 4), "d2h_bytes_per_step": int(w.numel() * 4),
-               "steps": e2e_steps, "ms_per_step": e2e_ms / e2e_steps, "mode": args.e2e_mode}
+               "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": int(w.numel() * 4),
+               "steps": e2e_steps, "ms_per_step": e2e_ms / e2e_steps, "mode": args.e2e_mode,
+               "host_link": {"bound": "host-to-device link", "measured_gbs": link_gbs,
+                             "achieved_gbs": h2d / (e2e_ms / e2e_steps * 1e6),
+                             "frac": h2d / (e2e_ms / e2e_steps * 1e6) / link_gbs}}
         del g_host, w_host
 
     h.synchronize()
