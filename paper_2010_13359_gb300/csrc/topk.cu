@@ -8,32 +8,34 @@
 // radix select (11 + 10 + 10 bits) without sorting.
 //
 // Two kernels per call, one pass over the dense vectors:
-//   1. form (tiles of 4096 elements): p -> e in place, h (optional), a
-//      histogram of the top key digit, and the tile's candidates -- the
-//      elements whose key is at least a threshold tau carried over from the
-//      worker's previous call (15/16 of its T) -- written in index order to
-//      the tile's slot, with the tile's count.
-//   2. select-and-compact, one cluster of 8 CTAs per worker.  Every CTA
-//      selects the top digit b0 of T from the histogram.  The candidates are
-//      split evenly over the 8 CTAs (by their index order, through a prefix
-//      of the tile counts), each CTA histograms the middle and then the low
-//      digit of its share, the cluster sums the histograms through
-//      distributed shared memory, and T and the number `need` of keys equal
-//      to T that are kept (the lowest indices) follow.  If T >= tau, every
-//      key >= T was a candidate and T is exact; otherwise (first call, or T
-//      fell below the carried threshold) each CTA re-extracts its tiles'
-//      elements with top digit >= b0 from p and the selection is repeated.
-//      Kept records are then written at position (number of keys > T before
-//      it) + min(number of keys == T before it, need).
+//   1. form (tiles of 4096 elements): p -> e in place, h (optional), and the
+//      tile's candidates -- the elements whose key is at least a threshold
+//      tau carried over from the worker's previous call (15/16 of its T) --
+//      written in index order to the tile's slot, with the tile's count.
+//   2. select-and-compact, one cluster of 8 CTAs per worker.  The candidates
+//      are split evenly over the 8 CTAs (by their index order, through a
+//      prefix of the tile counts); each CTA histograms the top, then the
+//      middle, then the low digit of its share, the cluster sums each
+//      histogram through distributed shared memory, and every CTA selects
+//      the same T and the number `need` of keys equal to T that are kept
+//      (the lowest indices).  If T >= tau, every key >= T was a candidate
+//      and T is exact; otherwise (first call, or T fell below the carried
+//      threshold) each CTA histograms the top digit over its tiles of p,
+//      re-extracts the elements whose top digit reaches the selected one,
+//      and the selection is repeated.  Kept records are then written at
+//      position (number of keys > T before it) + min(number of keys == T
+//      before it, need), the per-CTA counts taken from the CTA's own
+//      histograms.
 // The carried threshold only decides how much work the first pass saves the
 // second; the result is the same bit for bit either way.
 //
 // Server: w_j -= (sum over workers, in worker order, of the value recorded
 // for j) / M at the indices some worker sent; elsewhere w is unchanged (the
 // absent +0 terms leave the sum and w as they are).  A first kernel finds, for
-// each worker and each tile of 4096 indices, where the tile's records start;
-// a second kernel sums each tile's records in shared memory, worker by
-// worker, and updates the touched parameters.
+// each worker and each tile of 256 indices, where the tile's records start;
+// then one warp per tile sums the tile's records in shared memory, worker by
+// worker, and updates the touched parameters (one thread per record, with
+// searches narrowed to the tile, above 64 workers).
 #include <cooperative_groups.h>
 
 #include "device_common.cuh"
