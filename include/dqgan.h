@@ -178,6 +178,11 @@ DQGAN_API int dqgan_workers_compress_all(dqgan_handle* h, const float* g_all, in
  * parameters in place, w = fl(w - q_hat).  Then t <- t + 1.
  * msgs_all: device, M messages back to back (stride dqgan_message_bytes()).
  * params:   device, d fp32, caller-owned, read and written.
+ * SIGN with bucket >= 1024 and M <= 32 has two server kernels with the same
+ * results up to summation order; the library picks by size.  The environment
+ * variable DQGAN_SIGN_SERVER, read by dqgan_create, fixes the choice for the
+ * handle: "col" (per-lane bit transpose, parameters staged by TMA; needs
+ * d >= 32) or "tma" (warp bit transpose).  Any other value: by size.
  */
 DQGAN_API int dqgan_server_aggregate_update(dqgan_handle* h, const void* msgs_all, float* params);
 

@@ -5,6 +5,7 @@
 #include <cmath>
 #include <cstdarg>
 #include <cstdio>
+#include <cstdlib>
 #include <cstring>
 #include <new>
 #include <string>
@@ -29,6 +30,10 @@ struct dqgan_handle {
   CUtensorMap words_map;         // TMA map of the last message buffer the server saw
   const void* words_map_msgs = nullptr;
   bool words_map_ok = false;
+  CUtensorMap params_map;        // TMA map of the last parameter vector the sign server saw
+  const float* params_map_w = nullptr;
+  bool params_map_ok = false;
+  int32_t sign_path = 0;         // DQGAN_SIGN_SERVER at creation: 0 auto, 1 col, 2 tma
   int64_t t = 1;
   uint64_t launches = 0;
   std::string err;
@@ -240,6 +245,10 @@ int dqgan_create(const dqgan_config* cfg, dqgan_handle** out) {
   if (!h) return set_error(nullptr, DQGAN_ERR_OOM, "host allocation failed");
   h->cfg = *cfg;
   h->stream = reinterpret_cast<cudaStream_t>(cfg->cuda_stream);
+  if (const char* path = std::getenv("DQGAN_SIGN_SERVER")) {
+    if (std::strcmp(path, "col") == 0) h->sign_path = 1;
+    else if (std::strcmp(path, "tma") == 0) h->sign_path = 2;
+  }
   dq::message_layout(*cfg, &h->lay);
   h->nb = (cfg->d + cfg->bucket - 1) / (cfg->bucket > 0 ? cfg->bucket : 1);
   h->ld = round_up(cfg->d, 64);
@@ -414,6 +423,15 @@ int dqgan_server_aggregate_update(dqgan_handle* h, const void* msgs_all, float* 
       h->words_map_msgs = msgs_all;
     }
     if (h->words_map_ok) (tma_sign ? s.sign_words_map : s.squant_words_map) = &h->words_map;
+  }
+  s.params_map = nullptr;
+  s.sign_path = h->sign_path;
+  if (tma_sign && s.sign_words_map && s.d >= 32) {
+    if (h->params_map_w != params) {
+      h->params_map_ok = dq::encode_params_map(params, s.d, &h->params_map);
+      h->params_map_w = params;
+    }
+    if (h->params_map_ok) s.params_map = &h->params_map;
   }
   cudaError_t st = cudaSuccess;
   switch (h->cfg.compressor) {

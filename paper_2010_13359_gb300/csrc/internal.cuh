@@ -73,6 +73,8 @@ struct ServerArgs {
   const uint32_t* word_bucket;  // bucket of each 32-element word (layer segments), or nullptr: j / bucket
   const CUtensorMap* sign_words_map;    // TMA map of the M messages' sign words, or nullptr
   const CUtensorMap* squant_words_map;  // TMA map of the M messages' code words, or nullptr
+  const CUtensorMap* params_map;        // TMA map of w as rows of 32 floats, or nullptr
+  int32_t sign_path;  // sign, buckets >= 1024, M <= 32: 0 by size, 1 column kernel, 2 bit-transpose kernel
 };
 
 // TMA tensor map over the payload words of M messages: a 2-D array of u32,
@@ -81,6 +83,11 @@ struct ServerArgs {
 // outside.  Returns false if the driver entry point or the encoding fails.
 bool encode_words_map(const uint8_t* msgs, int64_t msg_stride, int64_t off_payload, int64_t payload_words,
                       int32_t M, bool swizzle128, CUtensorMap* out);
+
+// TMA tensor map over the parameters: floor(d / 32) rows of 32 fp32 (the
+// partial last row, if any, is outside it), boxes of 32 x 32, 128-byte
+// swizzle, zero fill.  Needs d >= 32 and w 16-byte aligned.
+bool encode_params_map(float* w, int64_t d, CUtensorMap* out);
 
 // Kernel launchers: each enqueues its kernels on `stream`, adds the number of
 // kernels it launched to *launches and returns the launch status.

@@ -357,6 +357,262 @@ sign_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap t
     mbar_wait_bounded(&bar[(it & 1u) ^ 1u], ((it + 1) >> 1) & 1u, s.err);
 }
 
+// Buckets of 1024..4096 with M <= 32 and d >= 32, column form.  Each warp
+// owns a contiguous range of 1024-element slices (32 message words).  TMA
+// brings the slice's words of every worker (box 32 words x M, 128-byte
+// swizzle) and the slice's 1024 parameters (box 32 rows x 32 floats of w
+// viewed as rows of 32, 128-byte swizzle) into shared memory.  Lane l reads
+// column l, word l of each worker, and transposes the 32 x 32 bit block in
+// its own registers, so that it holds the M sign bits of each of the 32
+// elements of that word; the worker sum comes from the five-worker group
+// tables looked up by shuffle (rebuilt only when the bucket changes).  The
+// lane updates its row of 32 parameters in shared memory and one TMA store
+// writes the box back.  Per warp kColWordBufs word buffers (with one, it is
+// refilled with the next slice's words as soon as the columns are in
+// registers; with two, the next slice's words load while this one is
+// decoded) and two parameter buffers (the next slice's parameters load while
+// this one is updated).
+// Against sign_server_tma_kernel: no warp transpose, 7 shuffles per element
+// at M = 32 instead of 12.
+constexpr int kColWarps = 12;
+constexpr int kColWordBufs = 2;
+constexpr int kColBox = 4096;                                  // bytes of one box
+constexpr int kColWarpBytes = (kColWordBufs + 2) * kColBox;    // word boxes + 2 parameter boxes
+constexpr int kColSmemBytes = kColWarps * kColWarpBytes + 1024;  // + alignment slack
+constexpr bool kColPairArith = false;  // workers 30, 31 by arithmetic instead of a seventh table
+
+// In-register transpose of a 32 x 32 bit block: on exit bit m of a[e] is
+// bit e of the entry a[m].  Block swaps of 16 and 8 bits by byte permutes,
+// then of 4, 2 and 1 bits by shifts and masks.
+template <int J>
+__device__ __forceinline__ void swap_stage(uint32_t (&a)[32], uint32_t m) {
+#pragma unroll
+  for (int k = 0; k < 32; ++k) {
+    if ((k & J) == 0) {
+      const uint32_t x = a[k], y = a[k + J];
+      a[k] = (x & m) | ((y << J) & ~m);
+      a[k + J] = ((x >> J) & m) | (y & ~m);
+    }
+  }
+}
+
+__device__ __forceinline__ void transpose32_regs(uint32_t (&a)[32]) {
+#pragma unroll
+  for (int k = 0; k < 16; ++k) {
+    const uint32_t x = a[k], y = a[k + 16];
+    a[k] = __byte_perm(x, y, 0x5410);
+    a[k + 16] = __byte_perm(x, y, 0x7632);
+  }
+#pragma unroll
+  for (int k = 0; k < 32; ++k) {
+    if ((k & 8) == 0) {
+      const uint32_t x = a[k], y = a[k + 8];
+      a[k] = __byte_perm(x, y, 0x6240);
+      a[k + 8] = __byte_perm(x, y, 0x7351);
+    }
+  }
+  swap_stage<4>(a, 0x0F0F0F0Fu);
+  swap_stage<2>(a, 0x33333333u);
+  swap_stage<1>(a, 0x55555555u);
+}
+
+// T_g[lane] for the first NGT five-worker groups (as build_group_tables).
+template <int NGT>
+__device__ __forceinline__ void build_tables(float my_scale, int M, int lane, float (&T)[7]) {
+#pragma unroll
+  for (int grp = 0; grp < 7; ++grp) {
+    float t = 0.f;
+    if (grp < NGT) {
+#pragma unroll
+      for (int r = 0; r < 5; ++r) {
+        const int wk = 5 * grp + r;
+        if (wk < 32) {
+          const float sc = __shfl_sync(kFullMask, my_scale, wk);
+          if (wk < M) t = __fadd_rn(t, ((lane >> r) & 1) ? -sc : sc);
+        }
+      }
+    }
+    T[grp] = t;
+  }
+}
+
+// Sum over the workers of one element's sign mask x: NG groups (with
+// kColPairArith the seventh, workers 30 and 31, by arithmetic from their
+// scales s30, s31), added pairwise, ((v0 + v1) + (v2 + v3)) + ((v4 + v5) + v6).
+template <int NG>
+__device__ __forceinline__ float column_sum(uint32_t x, const float (&T)[7], float s30, float s31) {
+  float v[NG];
+#pragma unroll
+  for (int grp = 0; grp < NG; ++grp) {
+    if (kColPairArith && grp == 6) {
+      const float q30 = __uint_as_float(__float_as_uint(s30) ^ ((x << 1) & 0x80000000u));
+      const float q31 = __uint_as_float(__float_as_uint(s31) ^ (x & 0x80000000u));
+      v[grp] = __fadd_rn(q30, q31);
+    } else {
+      v[grp] = __shfl_sync(kFullMask, T[grp], (int)(x >> (5 * grp)));
+    }
+  }
+#pragma unroll
+  for (int width = 1; width < NG; width *= 2)
+#pragma unroll
+    for (int i = 0; i + width < NG; i += 2 * width) v[i] = __fadd_rn(v[i], v[i + width]);
+  return v[0];
+}
+
+template <int NG, bool POW2>
+__global__ void __launch_bounds__(32 * kColWarps, 1)
+sign_server_col_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap wmap,
+                       const __grid_constant__ CUtensorMap pmap) {
+  constexpr int ROWS = 5 * NG < 32 ? 5 * NG : 32;  // message rows that can hold a worker
+  constexpr int NGT = (kColPairArith && NG == 7) ? 6 : NG;  // groups looked up in tables
+  extern __shared__ uint8_t smem_raw[];
+  __shared__ uint64_t bars[kColWarps][4];  // word boxes 0 and 1, parameter boxes 0 and 1
+  const int lane = threadIdx.x & 31;
+  const int warp = threadIdx.x >> 5;
+  const uint32_t raw = smem_addr(smem_raw);
+  uint8_t* const wbuf = smem_raw + ((1024u - (raw & 1023u)) & 1023u) + warp * kColWarpBytes;
+  uint8_t* const pbuf = wbuf + kColWordBufs * kColBox;  // word box i at wbuf + i * kColBox, parameter box i at pbuf + ...
+  uint64_t* wbar = &bars[warp][0];
+  uint64_t* pbar = &bars[warp][2];
+  if (lane == 0) {
+    for (int i = 0; i < 4; ++i) mbar_init(&bars[warp][i], 1);
+    mbar_fence_init();
+  }
+  __syncwarp();
+
+  const int words_per_bucket = s.bucket >> 5;  // 32..128
+  const int spb = words_per_bucket >> 5;       // slices per bucket
+  const int64_t nb = (s.d + s.bucket - 1) / s.bucket;
+  const int64_t nslices = nb * spb;
+  const int64_t nrows = s.d >> 5;              // rows of the parameter map
+  const int tail = (int)(s.d & 31);            // elements of the partial row nrows
+  const int32_t x0 = (int32_t)(s.off_payload >> 2);
+  const uint32_t wbytes = (uint32_t)(s.M < 32 ? s.M : 32) * 128u;
+  // this warp's slices [lo, hi): an even split of nslices over the grid's warps
+  const int64_t nwarps = (int64_t)gridDim.x * kColWarps;
+  const int64_t gw = (int64_t)blockIdx.x * kColWarps + warp;
+  const int64_t lo = nslices * gw / nwarps;
+  const int64_t hi = nslices * (gw + 1) / nwarps;
+  auto wbase_of = [&](int64_t slice) {
+    const int64_t b = slice / spb;
+    return b * words_per_bucket + (slice - b * spb) * 32;
+  };
+  // lane 0: copies of slice `slice` (the parameter box only if it starts inside the map)
+  // phases issued and waited for on each barrier (at most one outstanding)
+  uint32_t w_issued0 = 0, w_issued1 = 0, w_done0 = 0, w_done1 = 0;
+  uint32_t p_issued0 = 0, p_issued1 = 0, p_done0 = 0, p_done1 = 0;
+  auto issue_words = [&](int64_t slice, int i) {
+    if (i) ++w_issued1; else ++w_issued0;
+    mbar_arrive_expect_tx(&wbar[i], wbytes);
+    tma_load_2d(wbuf + i * kColBox, &wmap, x0 + (int32_t)wbase_of(slice), 0, &wbar[i]);
+  };
+  auto issue_params = [&](int64_t slice, int i) {
+    const int64_t wb = wbase_of(slice);
+    if (i) ++p_issued1; else ++p_issued0;
+    if (wb < nrows) {
+      mbar_arrive_expect_tx(&pbar[i], (uint32_t)kColBox);
+      tma_load_2d(pbuf + i * kColBox, &pmap, 0, (int32_t)wb, &pbar[i]);
+    } else {
+      mbar_arrive(&pbar[i]);  // nothing to copy: complete the phase
+    }
+  };
+  // byte offset of word `lane` in row m of a swizzled box: chunk (lane / 4) ^ (m mod 8)
+  const uint32_t lane_lo = (uint32_t)(lane & 3) << 2;
+  const uint32_t lane_chunk = (uint32_t)(lane >> 2);
+
+  if (lo < hi && lane == 0) {
+    issue_words(lo, 0);
+    issue_params(lo, 0);
+  }
+  float T[7];
+  float s30 = 0.f, s31 = 0.f;
+  int64_t table_b = -1;
+  uint32_t it = 0;
+  bool ok = true;
+  for (int64_t sl = lo; sl < hi; ++sl, ++it) {
+    const int cur = (int)(it & 1u);
+    const bool more = sl + 1 < hi;
+    const int wi = kColWordBufs == 2 ? cur : 0;  // this slice's word box
+    if (more && lane == 0) {
+      bulk_wait_read_all();        // the store of the previous slice has read its parameter box
+      fence_proxy_async_shared();  // this warp's reads of those boxes came before
+      issue_params(sl + 1, cur ^ 1);
+      if (kColWordBufs == 2) issue_words(sl + 1, cur ^ 1);
+    }
+    const int64_t b = sl / spb;
+    if (b != table_b) {  // warp-uniform
+      table_b = b;
+      const float my_scale =
+          lane < s.M ? __ldg(reinterpret_cast<const float*>(s.msgs + (int64_t)lane * s.msg_stride) + b) : 0.f;
+      build_tables<NGT>(my_scale, s.M, lane, T);
+      s30 = __shfl_sync(kFullMask, my_scale, 30);
+      s31 = __shfl_sync(kFullMask, my_scale, 31);
+    }
+    const int64_t wbase = wbase_of(sl);
+    ok = mbar_wait_bounded(&wbar[wi], (kColWordBufs == 2 ? it >> 1 : it) & 1u, s.err);
+    ok = __all_sync(kFullMask, ok);
+    if (!ok) break;
+    if (wi) ++w_done1; else ++w_done0;
+    const uint8_t* const wb = wbuf + wi * kColBox;
+    uint32_t x[32];
+#pragma unroll
+    for (int m = 0; m < 32; ++m) {
+      x[m] = 0u;
+      if (m < ROWS && m < s.M)
+        x[m] = *reinterpret_cast<const uint32_t*>(wb + m * 128 + (((lane_chunk ^ (uint32_t)(m & 7)) << 4) | lane_lo));
+    }
+    if (kColWordBufs == 1) {
+      __syncwarp();  // every lane has its columns: the word box may be refilled
+      if (more && lane == 0) {
+        fence_proxy_async_shared();
+        issue_words(sl + 1, 0);
+      }
+    }
+    transpose32_regs(x);  // x[e]: bit m = worker m's sign of element 32 (wbase + lane) + e
+    ok = mbar_wait_bounded(&pbar[cur], (it >> 1) & 1u, s.err);
+    ok = __all_sync(kFullMask, ok);
+    if (!ok) break;
+    if (cur) ++p_done1; else ++p_done0;
+    const int64_t row = wbase + lane;
+    const bool partial = row == nrows && tail != 0;  // the lane's row is the partial last one
+    float* const wg = s.w + 32 * row;
+    uint8_t* const prow = pbuf + cur * kColBox + lane * 128;
+#pragma unroll
+    for (int q = 0; q < 8; ++q) {
+      float4* slot = reinterpret_cast<float4*>(prow + ((q ^ (lane & 7)) << 4));
+      float4 wv = *slot;
+      float o[4] = {wv.x, wv.y, wv.z, wv.w};
+      if (partial) {
+#pragma unroll
+        for (int r = 0; r < 4; ++r) o[r] = (4 * q + r < tail) ? wg[4 * q + r] : 0.f;
+      }
+#pragma unroll
+      for (int r = 0; r < 4; ++r)
+        o[r] = __fsub_rn(o[r], average_t<POW2>(column_sum<NG>(x[4 * q + r], T, s30, s31), s));
+      if (partial) {
+#pragma unroll
+        for (int r = 0; r < 4; ++r)
+          if (4 * q + r < tail) wg[4 * q + r] = o[r];
+      }
+      *slot = make_float4(o[0], o[1], o[2], o[3]);
+    }
+    fence_proxy_async_shared();  // the box writes above, before the store reads them
+    __syncwarp();
+    if (lane == 0 && wbase < nrows) tma_store_2d(&pmap, 0, (int32_t)wbase, pbuf + cur * kColBox);
+    __syncwarp();
+  }
+  if (lane == 0) {
+    bulk_wait_all();  // stores complete before the block's shared memory is released
+    // after a time-out, copies already issued may still be in flight
+    if (!ok) {
+      if (w_issued0 > w_done0) mbar_wait_bounded(&wbar[0], w_done0 & 1u, s.err);
+      if (w_issued1 > w_done1) mbar_wait_bounded(&wbar[1], w_done1 & 1u, s.err);
+      if (p_issued0 > p_done0) mbar_wait_bounded(&pbar[0], p_done0 & 1u, s.err);
+      if (p_issued1 > p_done1) mbar_wait_bounded(&pbar[1], p_done1 & 1u, s.err);
+    }
+  }
+}
+
 // Any M: workers taken 32 at a time, groups added in order, w updated at the end.
 __global__ void __launch_bounds__(256) sign_server_slabs_kernel(const ServerArgs s) {
   const int lane = threadIdx.x & 31;
@@ -756,6 +1012,46 @@ cudaError_t launch_sign_tma(const ServerArgs& s, cudaStream_t stream) {
   return cudaGetLastError();
 }
 
+template <int NG, bool POW2>
+cudaError_t launch_sign_col(const ServerArgs& s, cudaStream_t stream) {
+  auto kern = sign_server_col_kernel<NG, POW2>;
+  int dev = 0;
+  cudaError_t st = cudaGetDevice(&dev);
+  if (st != cudaSuccess) return st;
+  static int blocks_for[64] = {0};
+  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+  if (blocks_for[dev] == 0) {
+    if ((st = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kColSmemBytes)) !=
+        cudaSuccess)
+      return st;
+    int sms = 0, per_sm = 0;
+    if ((st = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return st;
+    if ((st = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, 32 * kColWarps, kColSmemBytes)) !=
+        cudaSuccess)
+      return st;
+    blocks_for[dev] = sms * (per_sm > 0 ? per_sm : 1);
+  }
+  const int64_t nb = (s.d + s.bucket - 1) / s.bucket;
+  const int64_t warps = nb * (s.bucket / 1024);
+  const int64_t need = (warps + kColWarps - 1) / kColWarps;
+  const unsigned blocks = (unsigned)(need < blocks_for[dev] ? need : blocks_for[dev]);
+  kern<<<blocks, 32 * kColWarps, kColSmemBytes, stream>>>(s, *s.sign_words_map, *s.params_map);
+  return cudaGetLastError();
+}
+
+// The column kernel pays once every resident warp has several slices: with
+// one or two the latency of a slice's chain (copies in, transpose, store)
+// shows and the bit-transpose kernel is as fast or faster.
+bool sign_col_pays(const ServerArgs& s) {
+  static int sms[64] = {0};
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return false;
+  if (sms[dev] == 0 && cudaDeviceGetAttribute(&sms[dev], cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+    return false;
+  const int64_t nslices = ((s.d + s.bucket - 1) / s.bucket) * (s.bucket / 1024);
+  return nslices >= 4ll * sms[dev] * kColWarps;
+}
+
 template <int BITS, bool POW2, bool SEG>
 cudaError_t launch_squant_tma(const ServerArgs& s, cudaStream_t stream) {
   auto kern = squant_server_tma_kernel<BITS, POW2, SEG>;
@@ -791,8 +1087,11 @@ cudaError_t launch_sign_server(const ServerArgs& s, cudaStream_t stream, uint64_
   }
   if (s.bucket >= 1024 && s.M <= 32 && s.sign_words_map != nullptr) {
     const bool p2 = s.M_pow2 != 0;
+    const bool col = s.params_map != nullptr && (s.sign_path == 1 || (s.sign_path == 0 && sign_col_pays(s)));
     cudaError_t st;
-#define DQ_SIGN_TMA(NG) st = (p2 ? launch_sign_tma<NG, true>(s, stream) : launch_sign_tma<NG, false>(s, stream))
+#define DQ_SIGN_TMA(NG)                                                                           \
+  st = col ? (p2 ? launch_sign_col<NG, true>(s, stream) : launch_sign_col<NG, false>(s, stream)) \
+           : (p2 ? launch_sign_tma<NG, true>(s, stream) : launch_sign_tma<NG, false>(s, stream))
     switch ((s.M + 4) / 5) {
       case 1: DQ_SIGN_TMA(1); break;
       case 2: DQ_SIGN_TMA(2); break;
@@ -889,11 +1188,15 @@ cudaError_t launch_lookahead(const float* w, const float* h, float* out, int64_t
 
 namespace dq {
 
-bool encode_words_map(const uint8_t* msgs, int64_t msg_stride, int64_t off_payload, int64_t payload_words,
-                      int32_t M, bool swizzle128, CUtensorMap* out) {
-  using EncodeFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
-                                const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
-                                CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+namespace {
+
+using EncodeFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                              const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                              CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+// cuTensorMapEncodeTiled through the runtime's driver entry point (no link
+// against libcuda); nullptr if it is unavailable.
+EncodeFn tensor_map_encoder() {
   static EncodeFn encode = nullptr;
   static bool looked_up = false;
   if (!looked_up) {
@@ -905,6 +1208,14 @@ bool encode_words_map(const uint8_t* msgs, int64_t msg_stride, int64_t off_paylo
         q == cudaDriverEntryPointSuccess)
       encode = reinterpret_cast<EncodeFn>(fn);
   }
+  return encode;
+}
+
+}  // namespace
+
+bool encode_words_map(const uint8_t* msgs, int64_t msg_stride, int64_t off_payload, int64_t payload_words,
+                      int32_t M, bool swizzle128, CUtensorMap* out) {
+  const EncodeFn encode = tensor_map_encoder();
   if (!encode || M < 1) return false;
   const cuuint64_t dims[2] = {(cuuint64_t)(off_payload / 4 + payload_words), (cuuint64_t)M};
   const cuuint64_t strides[1] = {(cuuint64_t)msg_stride};
@@ -913,6 +1224,18 @@ bool encode_words_map(const uint8_t* msgs, int64_t msg_stride, int64_t off_paylo
   return encode(out, CU_TENSOR_MAP_DATA_TYPE_UINT32, 2, const_cast<uint8_t*>(msgs), dims, strides, box, elem,
                 CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle128 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE,
                 CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
+                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+bool encode_params_map(float* w, int64_t d, CUtensorMap* out) {
+  const EncodeFn encode = tensor_map_encoder();
+  if (!encode || d < 32 || ((uintptr_t)w & 15u) != 0) return false;
+  const cuuint64_t dims[2] = {32u, (cuuint64_t)(d / 32)};
+  const cuuint64_t strides[1] = {128u};
+  const cuuint32_t box[2] = {32u, 32u};
+  const cuuint32_t elem[2] = {1u, 1u};
+  return encode(out, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, w, dims, strides, box, elem, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
                 CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
