@@ -27,6 +27,8 @@ struct dqgan_handle {
   uint32_t* err_word = nullptr;  // device error word written by bounded waits
   int64_t* seg_bstart = nullptr;     // layer segments: nb + 1 bucket starts (device)
   uint32_t* seg_wbucket = nullptr;   // layer segments: bucket of every 32-element word (device)
+  uint32_t* seg_slices = nullptr;    // layer segments, sign: {first word, bucket | (rows - 1) << 27} per slice
+  int64_t seg_nslices = 0;
   CUtensorMap words_map;         // TMA map of the last message buffer the server saw
   const void* words_map_msgs = nullptr;
   bool words_map_ok = false;
@@ -298,6 +300,7 @@ int dqgan_destroy(dqgan_handle* h) {
   if (h->err_word) cudaFree(h->err_word);
   if (h->seg_bstart) cudaFree(h->seg_bstart);
   if (h->seg_wbucket) cudaFree(h->seg_wbucket);
+  if (h->seg_slices) cudaFree(h->seg_slices);
   const cudaError_t st = cudaGetLastError();
   delete h;
   if (st != cudaSuccess) return set_error(nullptr, DQGAN_ERR_CUDA, "destroy: %s", cudaGetErrorString(st));
@@ -333,8 +336,11 @@ int dqgan_set_segments(dqgan_handle* h, const int64_t* offsets, int32_t nseg) {
   if (st != cudaSuccess) return cuda_fail(h, st, "synchronize");
   if (h->seg_bstart) cudaFree(h->seg_bstart);
   if (h->seg_wbucket) cudaFree(h->seg_wbucket);
+  if (h->seg_slices) cudaFree(h->seg_slices);
   h->seg_bstart = nullptr;
   h->seg_wbucket = nullptr;
+  h->seg_slices = nullptr;
+  h->seg_nslices = 0;
   h->words_map_msgs = nullptr;  // the payload moves with the scale section
   dq::message_layout(c, &h->lay);
   h->nb = (c.d + c.bucket - 1) / c.bucket;
@@ -344,11 +350,26 @@ int dqgan_set_segments(dqgan_handle* h, const int64_t* offsets, int32_t nseg) {
   std::vector<uint32_t> wb((size_t)nwords);
   for (int64_t b = 0; b < nb; ++b)
     for (int64_t w = starts[b] / 32; w < (starts[b + 1] + 31) / 32; ++w) wb[(size_t)w] = (uint32_t)b;
+  // sign server slices: each bucket's words in runs of up to 32 (every bucket
+  // starts on a word: inner segment offsets are multiples of 32)
+  std::vector<uint32_t> slices;
+  if (c.compressor == DQGAN_SIGN)
+    for (int64_t b = 0; b < nb; ++b) {
+      const int64_t we = (starts[b + 1] + 31) / 32;
+      for (int64_t w = starts[b] / 32; w < we; w += 32) {
+        const int64_t rows = we - w < 32 ? we - w : 32;
+        slices.push_back((uint32_t)w);
+        slices.push_back((uint32_t)b | (uint32_t)(rows - 1) << 27);
+      }
+    }
   if ((st = cudaMalloc(&h->seg_bstart, starts.size() * sizeof(int64_t))) != cudaSuccess ||
-      (st = cudaMalloc(&h->seg_wbucket, wb.size() * sizeof(uint32_t))) != cudaSuccess) {
+      (st = cudaMalloc(&h->seg_wbucket, wb.size() * sizeof(uint32_t))) != cudaSuccess ||
+      (!slices.empty() && (st = cudaMalloc(&h->seg_slices, slices.size() * sizeof(uint32_t))) != cudaSuccess)) {
     if (h->seg_bstart) cudaFree(h->seg_bstart);
+    if (h->seg_wbucket) cudaFree(h->seg_wbucket);
     h->seg_bstart = nullptr;
     h->seg_wbucket = nullptr;
+    h->seg_slices = nullptr;
     cudaGetLastError();
     return set_error(h, st == cudaErrorMemoryAllocation ? DQGAN_ERR_OOM : DQGAN_ERR_CUDA, "segment tables: %s",
                      cudaGetErrorString(st));
@@ -356,13 +377,18 @@ int dqgan_set_segments(dqgan_handle* h, const int64_t* offsets, int32_t nseg) {
   if ((st = cudaMemcpy(h->seg_bstart, starts.data(), starts.size() * sizeof(int64_t), cudaMemcpyHostToDevice)) !=
           cudaSuccess ||
       (st = cudaMemcpy(h->seg_wbucket, wb.data(), wb.size() * sizeof(uint32_t), cudaMemcpyHostToDevice)) !=
-          cudaSuccess) {
+          cudaSuccess ||
+      (h->seg_slices && (st = cudaMemcpy(h->seg_slices, slices.data(), slices.size() * sizeof(uint32_t),
+                                         cudaMemcpyHostToDevice)) != cudaSuccess)) {
     cudaFree(h->seg_bstart);
     cudaFree(h->seg_wbucket);
+    if (h->seg_slices) cudaFree(h->seg_slices);
     h->seg_bstart = nullptr;
     h->seg_wbucket = nullptr;
+    h->seg_slices = nullptr;
     return cuda_fail(h, st, "copying the segment tables");
   }
+  h->seg_nslices = (int64_t)slices.size() / 2;
   h->nb = nb;
   h->lay.off_payload = round_up(4 * nb, 256);
   const int64_t payload_words = c.compressor == DQGAN_SIGN ? nwords : (c.d * c.bits + 31) / 32;
@@ -411,15 +437,20 @@ int dqgan_server_aggregate_update(dqgan_handle* h, const void* msgs_all, float* 
   s.word_bucket = h->seg_wbucket;
   s.sign_words_map = nullptr;
   s.squant_words_map = nullptr;
+  s.seg_slices = h->seg_slices;
+  s.seg_nslices = h->seg_nslices;
   const bool flat = h->seg_wbucket == nullptr;
-  const bool tma_sign = flat && h->cfg.compressor == DQGAN_SIGN && h->cfg.bucket >= 1024 && h->cfg.M <= 32;
+  // sign, buckets >= 1024, M <= 32: the TMA kernels (flat: 32-word boxes,
+  // 128-byte swizzle; layer segments: 36-word boxes without swizzle)
+  const bool tma_sign = h->cfg.compressor == DQGAN_SIGN && h->cfg.bucket >= 1024 && h->cfg.M <= 32 &&
+                        (flat || h->seg_slices != nullptr);
   const bool tma_squant = (h->cfg.compressor == DQGAN_SQUANT || h->cfg.compressor == DQGAN_QSGD) &&
                           h->cfg.M <= 32 && h->cfg.bucket >= 32 * (32 / h->cfg.bits);
   if (tma_sign || tma_squant) {
     if (h->words_map_msgs != msgs_all) {
       const int64_t payload_words = tma_sign ? (s.d + 31) / 32 : (s.d * s.bits + 31) / 32;
-      h->words_map_ok = dq::encode_words_map(s.msgs, s.msg_stride, s.off_payload, payload_words, s.M, tma_sign,
-                                             &h->words_map);
+      h->words_map_ok = dq::encode_words_map(s.msgs, s.msg_stride, s.off_payload, payload_words, s.M,
+                                             tma_sign && flat, tma_sign && !flat ? dq::kSignSegBoxWords : 32, &h->words_map);
       h->words_map_msgs = msgs_all;
     }
     if (h->words_map_ok) (tma_sign ? s.sign_words_map : s.squant_words_map) = &h->words_map;

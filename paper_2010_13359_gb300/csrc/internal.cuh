@@ -75,14 +75,21 @@ struct ServerArgs {
   const CUtensorMap* squant_words_map;  // TMA map of the M messages' code words, or nullptr
   const CUtensorMap* params_map;        // TMA map of w as rows of 32 floats, or nullptr
   int32_t sign_path;  // sign, buckets >= 1024, M <= 32: 0 by size, 1 column kernel, 2 bit-transpose kernel
+  // sign with layer segments: per slice {first word, bucket | (rows - 1) << 27}, or nullptr
+  const uint32_t* seg_slices;
+  int64_t seg_nslices;
 };
 
 // TMA tensor map over the payload words of M messages: a 2-D array of u32,
 // rows = workers (M), columns = message words up to the end of the payload;
-// boxes of 32 words x min(M, 32) workers, 128-byte swizzle or none, zero fill
-// outside.  Returns false if the driver entry point or the encoding fails.
+// boxes of box_words words (a multiple of 4; 32 with the 128-byte swizzle)
+// x min(M, 32) workers, zero fill outside.  Returns false if the driver entry
+// point or the encoding fails.
 bool encode_words_map(const uint8_t* msgs, int64_t msg_stride, int64_t off_payload, int64_t payload_words,
-                      int32_t M, bool swizzle128, CUtensorMap* out);
+                      int32_t M, bool swizzle128, int32_t box_words, CUtensorMap* out);
+// Width in words of the sign server's word boxes with layer segments: a box
+// starts at the 16-byte boundary at or before its 32-word slice.
+constexpr int kSignSegBoxWords = 36;
 
 // TMA tensor map over the parameters: floor(d / 32) rows of 32 fp32 (the
 // partial last row, if any, is outside it), boxes of 32 x 32, 128-byte

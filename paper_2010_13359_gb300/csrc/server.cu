@@ -367,19 +367,30 @@ sign_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap t
 // elements of that word; the worker sum comes from the five-worker group
 // tables looked up by shuffle (rebuilt only when the bucket changes).  The
 // lane updates its row of 32 parameters in shared memory and one TMA store
-// writes the box back.  Per warp kColWordBufs word buffers (with one, it is
-// refilled with the next slice's words as soon as the columns are in
-// registers; with two, the next slice's words load while this one is
-// decoded) and two parameter buffers (the next slice's parameters load while
-// this one is updated).
+// writes the box back.  Per warp two word and two parameter buffers: the
+// next slice's boxes load while this one is decoded and updated.
+// With layer segments (SEG) every slice lies inside one bucket: a host-built
+// table lists each bucket's runs of up to 32 words; the word box starts at
+// the 16-byte boundary at or before the slice (36 words wide, no swizzle),
+// and a slice shorter than 32 rows, or one that reaches the partial last
+// row, updates its parameters with plain loads and stores (a box store would
+// overlap the next slice).
 // Against sign_server_tma_kernel: no warp transpose, 7 shuffles per element
 // at M = 32 instead of 12.
 constexpr int kColWarps = 12;
-constexpr int kColWordBufs = 2;
-constexpr int kColBox = 4096;                                  // bytes of one box
-constexpr int kColWarpBytes = (kColWordBufs + 2) * kColBox;    // word boxes + 2 parameter boxes
-constexpr int kColSmemBytes = kColWarps * kColWarpBytes + 1024;  // + alignment slack
+constexpr int kColBox = 4096;        // bytes of a parameter box, and of a word box of the flat form
+constexpr int kSegBoxWords = kSignSegBoxWords;
 constexpr bool kColPairArith = false;  // workers 30, 31 by arithmetic instead of a seventh table
+
+// Per-warp shared memory of the column kernel: two parameter boxes, then two
+// word boxes (every swizzled box 1024-byte aligned).
+template <bool SEG>
+struct ColLayout {
+  static constexpr int kWBox = SEG ? 32 * kSegBoxWords * 4 : kColBox;
+  static constexpr int kWarpBytes = 2 * kColBox + 2 * kWBox;
+  static constexpr int kSmem = kColWarps * kWarpBytes + 1024;  // + alignment slack
+  static_assert(kWarpBytes % 1024 == 0, "boxes stay 1024-byte aligned");
+};
 
 // In-register transpose of a 32 x 32 bit block: on exit bit m of a[e] is
 // bit e of the entry a[m].  Block swaps of 16 and 8 bits by byte permutes,
@@ -459,10 +470,11 @@ __device__ __forceinline__ float column_sum(uint32_t x, const float (&T)[7], flo
   return v[0];
 }
 
-template <int NG, bool POW2>
+template <int NG, bool POW2, bool SEG>
 __global__ void __launch_bounds__(32 * kColWarps, 1)
 sign_server_col_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap wmap,
                        const __grid_constant__ CUtensorMap pmap) {
+  using L = ColLayout<SEG>;
   constexpr int ROWS = 5 * NG < 32 ? 5 * NG : 32;  // message rows that can hold a worker
   constexpr int NGT = (kColPairArith && NG == 7) ? 6 : NG;  // groups looked up in tables
   extern __shared__ uint8_t smem_raw[];
@@ -470,8 +482,8 @@ sign_server_col_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap w
   const int lane = threadIdx.x & 31;
   const int warp = threadIdx.x >> 5;
   const uint32_t raw = smem_addr(smem_raw);
-  uint8_t* const wbuf = smem_raw + ((1024u - (raw & 1023u)) & 1023u) + warp * kColWarpBytes;
-  uint8_t* const pbuf = wbuf + kColWordBufs * kColBox;  // word box i at wbuf + i * kColBox, parameter box i at pbuf + ...
+  uint8_t* const pbuf = smem_raw + ((1024u - (raw & 1023u)) & 1023u) + warp * L::kWarpBytes;  // + i * kColBox
+  uint8_t* const wbuf = pbuf + 2 * kColBox;                                                     // + i * L::kWBox
   uint64_t* wbar = &bars[warp][0];
   uint64_t* pbar = &bars[warp][2];
   if (lane == 0) {
@@ -481,37 +493,48 @@ sign_server_col_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap w
   __syncwarp();
 
   const int words_per_bucket = s.bucket >> 5;  // 32..128
-  const int spb = words_per_bucket >> 5;       // slices per bucket
-  const int64_t nb = (s.d + s.bucket - 1) / s.bucket;
-  const int64_t nslices = nb * spb;
+  const int spb = words_per_bucket >> 5;       // slices per bucket (flat form)
+  const int64_t nslices = SEG ? s.seg_nslices : ((s.d + s.bucket - 1) / s.bucket) * spb;
   const int64_t nrows = s.d >> 5;              // rows of the parameter map
   const int tail = (int)(s.d & 31);            // elements of the partial row nrows
   const int32_t x0 = (int32_t)(s.off_payload >> 2);
-  const uint32_t wbytes = (uint32_t)(s.M < 32 ? s.M : 32) * 128u;
+  const uint32_t wbytes = (uint32_t)(s.M < 32 ? s.M : 32) * (SEG ? 4u * kSegBoxWords : 128u);
   // this warp's slices [lo, hi): an even split of nslices over the grid's warps
   const int64_t nwarps = (int64_t)gridDim.x * kColWarps;
   const int64_t gw = (int64_t)blockIdx.x * kColWarps + warp;
   const int64_t lo = nslices * gw / nwarps;
   const int64_t hi = nslices * (gw + 1) / nwarps;
-  auto wbase_of = [&](int64_t slice) {
-    const int64_t b = slice / spb;
-    return b * words_per_bucket + (slice - b * spb) * 32;
+  struct Slice {
+    int64_t word;    // first message word = first parameter row
+    int64_t bucket;
+    int rows;        // words (rows) in the slice, 1..32
   };
-  // lane 0: copies of slice `slice` (the parameter box only if it starts inside the map)
-  // phases issued and waited for on each barrier (at most one outstanding)
+  auto slice_of = [&](int64_t sl) -> Slice {
+    if constexpr (SEG) {
+      const uint2 e = __ldg(reinterpret_cast<const uint2*>(s.seg_slices) + sl);
+      return Slice{(int64_t)e.x, (int64_t)(e.y & 0x7FFFFFFu), (int)(e.y >> 27) + 1};
+    } else {
+      const int64_t b = sl / spb;
+      return Slice{b * words_per_bucket + (sl - b * spb) * 32, b, 32};
+    }
+  };
+  // whether the slice's parameters move as one TMA box: flat, the box starts
+  // inside the map (its rows past the map read as zero and are not stored);
+  // layer segments, all 32 rows lie inside the map
+  auto boxed = [&](const Slice& c) { return SEG ? (c.rows == 32 && c.word + 32 <= nrows) : (c.word < nrows); };
+  // lane 0: copies of slice c into buffers i (phases issued and waited for
+  // on each barrier are counted; at most one is outstanding)
   uint32_t w_issued0 = 0, w_issued1 = 0, w_done0 = 0, w_done1 = 0;
   uint32_t p_issued0 = 0, p_issued1 = 0, p_done0 = 0, p_done1 = 0;
-  auto issue_words = [&](int64_t slice, int i) {
+  auto issue = [&](const Slice& c, int i) {
     if (i) ++w_issued1; else ++w_issued0;
     mbar_arrive_expect_tx(&wbar[i], wbytes);
-    tma_load_2d(wbuf + i * kColBox, &wmap, x0 + (int32_t)wbase_of(slice), 0, &wbar[i]);
-  };
-  auto issue_params = [&](int64_t slice, int i) {
-    const int64_t wb = wbase_of(slice);
+    const int32_t x = x0 + (int32_t)c.word;
+    tma_load_2d(wbuf + i * L::kWBox, &wmap, SEG ? (x & ~3) : x, 0, &wbar[i]);
     if (i) ++p_issued1; else ++p_issued0;
-    if (wb < nrows) {
+    if (boxed(c)) {
       mbar_arrive_expect_tx(&pbar[i], (uint32_t)kColBox);
-      tma_load_2d(pbuf + i * kColBox, &pmap, 0, (int32_t)wb, &pbar[i]);
+      tma_load_2d(pbuf + i * kColBox, &pmap, 0, (int32_t)c.word, &pbar[i]);
     } else {
       mbar_arrive(&pbar[i]);  // nothing to copy: complete the phase
     }
@@ -520,10 +543,8 @@ sign_server_col_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap w
   const uint32_t lane_lo = (uint32_t)(lane & 3) << 2;
   const uint32_t lane_chunk = (uint32_t)(lane >> 2);
 
-  if (lo < hi && lane == 0) {
-    issue_words(lo, 0);
-    issue_params(lo, 0);
-  }
+  Slice c = lo < hi ? slice_of(lo) : Slice{0, 0, 0};
+  if (lo < hi && lane == 0) issue(c, 0);
   float T[7];
   float s30 = 0.f, s31 = 0.f;
   int64_t table_b = -1;
@@ -532,74 +553,78 @@ sign_server_col_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap w
   for (int64_t sl = lo; sl < hi; ++sl, ++it) {
     const int cur = (int)(it & 1u);
     const bool more = sl + 1 < hi;
-    const int wi = kColWordBufs == 2 ? cur : 0;  // this slice's word box
+    const Slice cn = more ? slice_of(sl + 1) : c;
     if (more && lane == 0) {
       bulk_wait_read_all();        // the store of the previous slice has read its parameter box
       fence_proxy_async_shared();  // this warp's reads of those boxes came before
-      issue_params(sl + 1, cur ^ 1);
-      if (kColWordBufs == 2) issue_words(sl + 1, cur ^ 1);
+      issue(cn, cur ^ 1);
     }
-    const int64_t b = sl / spb;
-    if (b != table_b) {  // warp-uniform
-      table_b = b;
+    if (c.bucket != table_b) {  // warp-uniform
+      table_b = c.bucket;
       const float my_scale =
-          lane < s.M ? __ldg(reinterpret_cast<const float*>(s.msgs + (int64_t)lane * s.msg_stride) + b) : 0.f;
+          lane < s.M ? __ldg(reinterpret_cast<const float*>(s.msgs + (int64_t)lane * s.msg_stride) + c.bucket)
+                     : 0.f;
       build_tables<NGT>(my_scale, s.M, lane, T);
       s30 = __shfl_sync(kFullMask, my_scale, 30);
       s31 = __shfl_sync(kFullMask, my_scale, 31);
     }
-    const int64_t wbase = wbase_of(sl);
-    ok = mbar_wait_bounded(&wbar[wi], (kColWordBufs == 2 ? it >> 1 : it) & 1u, s.err);
+    ok = mbar_wait_bounded(&wbar[cur], (it >> 1) & 1u, s.err);
     ok = __all_sync(kFullMask, ok);
     if (!ok) break;
-    if (wi) ++w_done1; else ++w_done0;
-    const uint8_t* const wb = wbuf + wi * kColBox;
+    if (cur) ++w_done1; else ++w_done0;
+    const uint8_t* const wb = wbuf + cur * L::kWBox;
+    const uint32_t seg_off = SEG ? (((uint32_t)(x0 + c.word) & 3u) + (uint32_t)lane) * 4u : 0u;
     uint32_t x[32];
 #pragma unroll
     for (int m = 0; m < 32; ++m) {
       x[m] = 0u;
-      if (m < ROWS && m < s.M)
-        x[m] = *reinterpret_cast<const uint32_t*>(wb + m * 128 + (((lane_chunk ^ (uint32_t)(m & 7)) << 4) | lane_lo));
-    }
-    if (kColWordBufs == 1) {
-      __syncwarp();  // every lane has its columns: the word box may be refilled
-      if (more && lane == 0) {
-        fence_proxy_async_shared();
-        issue_words(sl + 1, 0);
+      if (m < ROWS && m < s.M) {
+        const uint32_t off = SEG ? (uint32_t)(m * 4 * kSegBoxWords) + seg_off
+                                 : (uint32_t)(m * 128) + (((lane_chunk ^ (uint32_t)(m & 7)) << 4) | lane_lo);
+        x[m] = *reinterpret_cast<const uint32_t*>(wb + off);
       }
     }
-    transpose32_regs(x);  // x[e]: bit m = worker m's sign of element 32 (wbase + lane) + e
+    transpose32_regs(x);  // x[e]: bit m = worker m's sign of element 32 (c.word + lane) + e
     ok = mbar_wait_bounded(&pbar[cur], (it >> 1) & 1u, s.err);
     ok = __all_sync(kFullMask, ok);
     if (!ok) break;
     if (cur) ++p_done1; else ++p_done0;
-    const int64_t row = wbase + lane;
-    const bool partial = row == nrows && tail != 0;  // the lane's row is the partial last one
+    const bool in_box = boxed(c);
+    const int64_t row = c.word + lane;
+    // rows updated with plain loads and stores: flat, the partial last row
+    // (rows past it hold no parameters); layer segments, the partial last row
+    // of a boxed slice, or every row of a slice without a box
+    const bool direct = (SEG && !in_box) ? (lane < c.rows) : (row == nrows && tail != 0);
+    const int cnt = row == nrows ? tail : 32;  // parameters in the row
     float* const wg = s.w + 32 * row;
     uint8_t* const prow = pbuf + cur * kColBox + lane * 128;
 #pragma unroll
     for (int q = 0; q < 8; ++q) {
       float4* slot = reinterpret_cast<float4*>(prow + ((q ^ (lane & 7)) << 4));
-      float4 wv = *slot;
-      float o[4] = {wv.x, wv.y, wv.z, wv.w};
-      if (partial) {
+      float o[4] = {0.f, 0.f, 0.f, 0.f};
+      if (in_box) {
+        const float4 wv = *slot;
+        o[0] = wv.x; o[1] = wv.y; o[2] = wv.z; o[3] = wv.w;
+      }
+      if (direct) {
 #pragma unroll
-        for (int r = 0; r < 4; ++r) o[r] = (4 * q + r < tail) ? wg[4 * q + r] : 0.f;
+        for (int r = 0; r < 4; ++r) o[r] = (4 * q + r < cnt) ? wg[4 * q + r] : 0.f;
       }
 #pragma unroll
       for (int r = 0; r < 4; ++r)
         o[r] = __fsub_rn(o[r], average_t<POW2>(column_sum<NG>(x[4 * q + r], T, s30, s31), s));
-      if (partial) {
+      if (direct) {
 #pragma unroll
         for (int r = 0; r < 4; ++r)
-          if (4 * q + r < tail) wg[4 * q + r] = o[r];
+          if (4 * q + r < cnt) wg[4 * q + r] = o[r];
       }
-      *slot = make_float4(o[0], o[1], o[2], o[3]);
+      if (in_box) *slot = make_float4(o[0], o[1], o[2], o[3]);
     }
     fence_proxy_async_shared();  // the box writes above, before the store reads them
     __syncwarp();
-    if (lane == 0 && wbase < nrows) tma_store_2d(&pmap, 0, (int32_t)wbase, pbuf + cur * kColBox);
+    if (lane == 0 && in_box) tma_store_2d(&pmap, 0, (int32_t)c.word, pbuf + cur * kColBox);
     __syncwarp();
+    c = cn;
   }
   if (lane == 0) {
     bulk_wait_all();  // stores complete before the block's shared memory is released
@@ -1012,30 +1037,29 @@ cudaError_t launch_sign_tma(const ServerArgs& s, cudaStream_t stream) {
   return cudaGetLastError();
 }
 
-template <int NG, bool POW2>
+template <int NG, bool POW2, bool SEG>
 cudaError_t launch_sign_col(const ServerArgs& s, cudaStream_t stream) {
-  auto kern = sign_server_col_kernel<NG, POW2>;
+  auto kern = sign_server_col_kernel<NG, POW2, SEG>;
+  constexpr int smem = ColLayout<SEG>::kSmem;
   int dev = 0;
   cudaError_t st = cudaGetDevice(&dev);
   if (st != cudaSuccess) return st;
   static int blocks_for[64] = {0};
   if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
   if (blocks_for[dev] == 0) {
-    if ((st = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kColSmemBytes)) !=
-        cudaSuccess)
+    if ((st = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem)) != cudaSuccess)
       return st;
     int sms = 0, per_sm = 0;
     if ((st = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return st;
-    if ((st = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, 32 * kColWarps, kColSmemBytes)) !=
-        cudaSuccess)
+    if ((st = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, 32 * kColWarps, smem)) != cudaSuccess)
       return st;
     blocks_for[dev] = sms * (per_sm > 0 ? per_sm : 1);
   }
-  const int64_t nb = (s.d + s.bucket - 1) / s.bucket;
-  const int64_t warps = nb * (s.bucket / 1024);
-  const int64_t need = (warps + kColWarps - 1) / kColWarps;
+  const int64_t nslices = SEG ? s.seg_nslices : ((s.d + s.bucket - 1) / s.bucket) * (s.bucket / 1024);
+  const int64_t need = (nslices + kColWarps - 1) / kColWarps;
   const unsigned blocks = (unsigned)(need < blocks_for[dev] ? need : blocks_for[dev]);
-  kern<<<blocks, 32 * kColWarps, kColSmemBytes, stream>>>(s, *s.sign_words_map, *s.params_map);
+  if (blocks == 0) return cudaSuccess;
+  kern<<<blocks, 32 * kColWarps, smem, stream>>>(s, *s.sign_words_map, *s.params_map);
   return cudaGetLastError();
 }
 
@@ -1080,8 +1104,25 @@ unsigned chunk_blocks(int64_t d, int threads) {
 }  // namespace
 
 cudaError_t launch_sign_server(const ServerArgs& s, cudaStream_t stream, uint64_t* launches) {
-  if (s.word_bucket) {  // buckets restart at layer segments: per-element scale lookup
-    sign_server_kernel<<<chunk_blocks(s.d, 256), 256, 0, stream>>>(s);
+  if (s.word_bucket) {  // buckets restart at layer segments
+    if (s.seg_slices && s.sign_words_map && s.params_map && s.bucket >= 1024 && s.M <= 32) {
+      const bool p2 = s.M_pow2 != 0;
+      cudaError_t st;
+#define DQ_SIGN_SEG(NG) st = (p2 ? launch_sign_col<NG, true, true>(s, stream) : launch_sign_col<NG, false, true>(s, stream))
+      switch ((s.M + 4) / 5) {
+        case 1: DQ_SIGN_SEG(1); break;
+        case 2: DQ_SIGN_SEG(2); break;
+        case 3: DQ_SIGN_SEG(3); break;
+        case 4: DQ_SIGN_SEG(4); break;
+        case 5: DQ_SIGN_SEG(5); break;
+        case 6: DQ_SIGN_SEG(6); break;
+        default: DQ_SIGN_SEG(7); break;
+      }
+#undef DQ_SIGN_SEG
+      *launches += 1;
+      return st;
+    }
+    sign_server_kernel<<<chunk_blocks(s.d, 256), 256, 0, stream>>>(s);  // per-element scale lookup
     *launches += 1;
     return cudaGetLastError();
   }
@@ -1090,7 +1131,7 @@ cudaError_t launch_sign_server(const ServerArgs& s, cudaStream_t stream, uint64_
     const bool col = s.params_map != nullptr && (s.sign_path == 1 || (s.sign_path == 0 && sign_col_pays(s)));
     cudaError_t st;
 #define DQ_SIGN_TMA(NG)                                                                           \
-  st = col ? (p2 ? launch_sign_col<NG, true>(s, stream) : launch_sign_col<NG, false>(s, stream)) \
+  st = col ? (p2 ? launch_sign_col<NG, true, false>(s, stream) : launch_sign_col<NG, false, false>(s, stream)) \
            : (p2 ? launch_sign_tma<NG, true>(s, stream) : launch_sign_tma<NG, false>(s, stream))
     switch ((s.M + 4) / 5) {
       case 1: DQ_SIGN_TMA(1); break;
@@ -1214,12 +1255,12 @@ EncodeFn tensor_map_encoder() {
 }  // namespace
 
 bool encode_words_map(const uint8_t* msgs, int64_t msg_stride, int64_t off_payload, int64_t payload_words,
-                      int32_t M, bool swizzle128, CUtensorMap* out) {
+                      int32_t M, bool swizzle128, int32_t box_words, CUtensorMap* out) {
   const EncodeFn encode = tensor_map_encoder();
-  if (!encode || M < 1) return false;
+  if (!encode || M < 1 || (swizzle128 && box_words != 32)) return false;
   const cuuint64_t dims[2] = {(cuuint64_t)(off_payload / 4 + payload_words), (cuuint64_t)M};
   const cuuint64_t strides[1] = {(cuuint64_t)msg_stride};
-  const cuuint32_t box[2] = {32u, (cuuint32_t)(M < 32 ? M : 32)};
+  const cuuint32_t box[2] = {(cuuint32_t)box_words, (cuuint32_t)(M < 32 ? M : 32)};
   const cuuint32_t elem[2] = {1u, 1u};
   return encode(out, CU_TENSOR_MAP_DATA_TYPE_UINT32, 2, const_cast<uint8_t*>(msgs), dims, strides, box, elem,
                 CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle128 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE,

@@ -103,3 +103,63 @@ def test_sign_server_paths(P, d, M, bucket, path, monkeypatch):
     assert np.all(tail == 12345.0), "parameters past d were written"
     assert torch.all(alt[d:] == 0.0)
     h.destroy()
+
+
+def layer_offsets(kind, d, rng):
+    if kind == "tiny":  # many one-word layers, then a long one
+        return tuple([0, *range(32, 32 * 40, 32), d])
+    if kind == "odd":  # layer sizes that leave every bucket off the 16-byte grid of the payload
+        offs, at = [0], 0
+        while True:
+            at += 32 * int(rng.integers(1, 90))
+            if at >= d:
+                break
+            offs.append(at)
+        return tuple(offs + [d])
+    cuts = np.sort(rng.choice(np.arange(1, d // 32), size=15, replace=False)) * 32
+    return tuple([0, *cuts.tolist(), d])
+
+
+SEG_CASES = [
+    (20_011, 3, 1024, "tiny"), (65_536, 8, 1024, "odd"), (65_536 + 7, 32, 4096, "odd"),
+    (200_003, 13, 2048, "random16"), (2_000_000, 8, 1024, "random16"), (1_000_003, 31, 4096, "random16"),
+]
+
+
+@pytest.mark.parametrize("d,M,bucket,kind", SEG_CASES, ids=[f"d{d}-M{M}-b{b}-{k}" for d, M, b, k in SEG_CASES])
+def test_sign_server_segments(P, d, M, bucket, kind):
+    """Layer segments: every slice of the column kernel lies inside one
+    bucket; short slices update their rows with plain stores."""
+    dev = torch.device("cuda:0")
+    stream = torch.cuda.current_stream(dev)
+    rng = np.random.default_rng(d + bucket)
+    segs = layer_offsets(kind, d, rng)
+    ocfg = oracle_config(d, M, oracle.SIGN, lr=0.03, bucket=bucket, seed=M, segments=segs)
+    h = P.create(P.make_config(d=d, M=M, compressor=P.SIGN, lr=0.03, bucket=bucket, seed=M,
+                               cuda_stream=stream.cuda_stream))
+    h.set_segments(segs)
+    st = oracle.State(ocfg)
+    ld = (d + 3) // 4 * 4
+    guard = 64
+    w0 = (rng.standard_normal(d) * 0.02).astype(np.float32)
+    buf = torch.full((d + guard,), -777.0, dtype=torch.float32, device=dev)
+    buf[:d] = torch.from_numpy(w0).to(dev)
+    w_gpu = buf[:d]
+    w_orc = w0.copy()
+    msgs = torch.zeros((M, h.message_bytes()), dtype=torch.uint8, device=dev)
+    for t in range(2):
+        g = (rng.standard_normal((M, d)) * np.exp(rng.uniform(-3, 1, (M, d)))).astype(np.float32)
+        g_dev = torch.zeros((M, ld), dtype=torch.float32, device=dev)
+        g_dev[:, :d] = torch.from_numpy(g).to(dev)
+        h.workers_compress_all(g_dev, ld, msgs)
+        want = st.compress_all(g)
+        got = msgs.cpu().numpy()
+        for i in range(M):
+            assert_messages_equal(ocfg, got[i], want[i], f"worker {i} step {t}")
+        h.server_aggregate_update(msgs, w_gpu)
+        st.server(want, w_orc)
+        h.synchronize()
+        err = rel_err(w_gpu.cpu().numpy(), w_orc)
+        assert err <= STEP_RTOL, f"step {t}: rel err {err}"
+    assert np.all(buf[d:].cpu().numpy() == -777.0), "parameters past d were written"
+    h.destroy()
