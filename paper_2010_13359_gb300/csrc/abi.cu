@@ -437,8 +437,6 @@ int dqgan_server_aggregate_update(dqgan_handle* h, const void* msgs_all, float* 
   s.word_bucket = h->seg_wbucket;
   s.sign_words_map = nullptr;
   s.squant_words_map = nullptr;
-  s.seg_slices = h->seg_slices;
-  s.seg_nslices = h->seg_nslices;
   const bool flat = h->seg_wbucket == nullptr;
   // sign, buckets >= 1024, M <= 32: the TMA kernels (flat: 32-word boxes,
   // 128-byte swizzle; layer segments: 36-word boxes without swizzle)
@@ -455,18 +453,20 @@ int dqgan_server_aggregate_update(dqgan_handle* h, const void* msgs_all, float* 
     }
     if (h->words_map_ok) (tma_sign ? s.sign_words_map : s.squant_words_map) = &h->words_map;
   }
-  s.params_map = nullptr;
-  s.sign_path = h->sign_path;
+  dq::SignServerExtras x{};
+  x.path = h->sign_path;
+  x.seg_slices = h->seg_slices;
+  x.seg_nslices = h->seg_nslices;
   if (tma_sign && s.sign_words_map && s.d >= 32) {
     if (h->params_map_w != params) {
       h->params_map_ok = dq::encode_params_map(params, s.d, &h->params_map);
       h->params_map_w = params;
     }
-    if (h->params_map_ok) s.params_map = &h->params_map;
+    if (h->params_map_ok) x.params_map = &h->params_map;
   }
   cudaError_t st = cudaSuccess;
   switch (h->cfg.compressor) {
-    case DQGAN_SIGN: st = dq::launch_sign_server(s, h->stream, &h->launches); break;
+    case DQGAN_SIGN: st = dq::launch_sign_server(s, x, h->stream, &h->launches); break;
     case DQGAN_SQUANT:
     case DQGAN_QSGD: st = dq::launch_squant_server(s, h->stream, &h->launches); break;
     case DQGAN_IDENTITY: st = dq::launch_identity_server(s, h->stream, &h->launches); break;

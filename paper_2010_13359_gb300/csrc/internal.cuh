@@ -73,10 +73,14 @@ struct ServerArgs {
   const uint32_t* word_bucket;  // bucket of each 32-element word (layer segments), or nullptr: j / bucket
   const CUtensorMap* sign_words_map;    // TMA map of the M messages' sign words, or nullptr
   const CUtensorMap* squant_words_map;  // TMA map of the M messages' code words, or nullptr
-  const CUtensorMap* params_map;        // TMA map of w as rows of 32 floats, or nullptr
-  int32_t sign_path;  // sign, buckets >= 1024, M <= 32: 0 by size, 1 column kernel, 2 bit-transpose kernel
-  // sign with layer segments: per slice {first word, bucket | (rows - 1) << 27}, or nullptr
-  const uint32_t* seg_slices;
+};
+
+// The sign server's further inputs (kept out of ServerArgs, which every
+// server kernel takes as its parameter block).
+struct SignServerExtras {
+  const CUtensorMap* params_map;  // TMA map of w as rows of 32 floats, or nullptr
+  int32_t path;                   // buckets >= 1024, M <= 32: 0 by size, 1 column kernel, 2 bit-transpose kernel
+  const uint32_t* seg_slices;     // layer segments: per slice {first word, bucket | (rows - 1) << 27}, or nullptr
   int64_t seg_nslices;
 };
 
@@ -116,7 +120,8 @@ size_t topk_scratch_clear_bytes(int64_t d);
 cudaError_t launch_topk_compress(const CompressArgs& a, int64_t k, bool keep_h, void* scratch,
                                  cudaStream_t stream, uint64_t* launches);
 
-cudaError_t launch_sign_server(const ServerArgs& s, cudaStream_t stream, uint64_t* launches);
+cudaError_t launch_sign_server(const ServerArgs& s, const SignServerExtras& x, cudaStream_t stream,
+                               uint64_t* launches);
 cudaError_t launch_squant_server(const ServerArgs& s, cudaStream_t stream, uint64_t* launches);
 cudaError_t launch_identity_server(const ServerArgs& s, cudaStream_t stream, uint64_t* launches);
 cudaError_t launch_topk_server(const ServerArgs& s, void* scratch, cudaStream_t stream, uint64_t* launches);

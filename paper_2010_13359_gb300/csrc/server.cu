@@ -470,9 +470,15 @@ __device__ __forceinline__ float column_sum(uint32_t x, const float (&T)[7], flo
   return v[0];
 }
 
+// The slice table of the layer-segmented form.
+struct SegSlices {
+  const uint32_t* slices;  // per slice {first word, bucket | (rows - 1) << 27}
+  int64_t n;
+};
+
 template <int NG, bool POW2, bool SEG>
 __global__ void __launch_bounds__(32 * kColWarps, 1)
-sign_server_col_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap wmap,
+sign_server_col_kernel(const ServerArgs s, const SegSlices seg, const __grid_constant__ CUtensorMap wmap,
                        const __grid_constant__ CUtensorMap pmap) {
   using L = ColLayout<SEG>;
   constexpr int ROWS = 5 * NG < 32 ? 5 * NG : 32;  // message rows that can hold a worker
@@ -494,7 +500,7 @@ sign_server_col_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap w
 
   const int words_per_bucket = s.bucket >> 5;  // 32..128
   const int spb = words_per_bucket >> 5;       // slices per bucket (flat form)
-  const int64_t nslices = SEG ? s.seg_nslices : ((s.d + s.bucket - 1) / s.bucket) * spb;
+  const int64_t nslices = SEG ? seg.n : ((s.d + s.bucket - 1) / s.bucket) * spb;
   const int64_t nrows = s.d >> 5;              // rows of the parameter map
   const int tail = (int)(s.d & 31);            // elements of the partial row nrows
   const int32_t x0 = (int32_t)(s.off_payload >> 2);
@@ -511,7 +517,7 @@ sign_server_col_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap w
   };
   auto slice_of = [&](int64_t sl) -> Slice {
     if constexpr (SEG) {
-      const uint2 e = __ldg(reinterpret_cast<const uint2*>(s.seg_slices) + sl);
+      const uint2 e = __ldg(reinterpret_cast<const uint2*>(seg.slices) + sl);
       return Slice{(int64_t)e.x, (int64_t)(e.y & 0x7FFFFFFu), (int)(e.y >> 27) + 1};
     } else {
       const int64_t b = sl / spb;
@@ -1038,7 +1044,7 @@ cudaError_t launch_sign_tma(const ServerArgs& s, cudaStream_t stream) {
 }
 
 template <int NG, bool POW2, bool SEG>
-cudaError_t launch_sign_col(const ServerArgs& s, cudaStream_t stream) {
+cudaError_t launch_sign_col(const ServerArgs& s, const SignServerExtras& x, cudaStream_t stream) {
   auto kern = sign_server_col_kernel<NG, POW2, SEG>;
   constexpr int smem = ColLayout<SEG>::kSmem;
   int dev = 0;
@@ -1055,11 +1061,12 @@ cudaError_t launch_sign_col(const ServerArgs& s, cudaStream_t stream) {
       return st;
     blocks_for[dev] = sms * (per_sm > 0 ? per_sm : 1);
   }
-  const int64_t nslices = SEG ? s.seg_nslices : ((s.d + s.bucket - 1) / s.bucket) * (s.bucket / 1024);
+  const int64_t nslices = SEG ? x.seg_nslices : ((s.d + s.bucket - 1) / s.bucket) * (s.bucket / 1024);
   const int64_t need = (nslices + kColWarps - 1) / kColWarps;
   const unsigned blocks = (unsigned)(need < blocks_for[dev] ? need : blocks_for[dev]);
   if (blocks == 0) return cudaSuccess;
-  kern<<<blocks, 32 * kColWarps, smem, stream>>>(s, *s.sign_words_map, *s.params_map);
+  kern<<<blocks, 32 * kColWarps, smem, stream>>>(s, SegSlices{x.seg_slices, x.seg_nslices}, *s.sign_words_map,
+                                                  *x.params_map);
   return cudaGetLastError();
 }
 
@@ -1103,12 +1110,14 @@ unsigned chunk_blocks(int64_t d, int threads) {
 
 }  // namespace
 
-cudaError_t launch_sign_server(const ServerArgs& s, cudaStream_t stream, uint64_t* launches) {
+cudaError_t launch_sign_server(const ServerArgs& s, const SignServerExtras& x, cudaStream_t stream,
+                               uint64_t* launches) {
   if (s.word_bucket) {  // buckets restart at layer segments
-    if (s.seg_slices && s.sign_words_map && s.params_map && s.bucket >= 1024 && s.M <= 32) {
+    if (x.seg_slices && s.sign_words_map && x.params_map && s.bucket >= 1024 && s.M <= 32) {
       const bool p2 = s.M_pow2 != 0;
       cudaError_t st;
-#define DQ_SIGN_SEG(NG) st = (p2 ? launch_sign_col<NG, true, true>(s, stream) : launch_sign_col<NG, false, true>(s, stream))
+#define DQ_SIGN_SEG(NG) \
+  st = (p2 ? launch_sign_col<NG, true, true>(s, x, stream) : launch_sign_col<NG, false, true>(s, x, stream))
       switch ((s.M + 4) / 5) {
         case 1: DQ_SIGN_SEG(1); break;
         case 2: DQ_SIGN_SEG(2); break;
@@ -1128,10 +1137,10 @@ cudaError_t launch_sign_server(const ServerArgs& s, cudaStream_t stream, uint64_
   }
   if (s.bucket >= 1024 && s.M <= 32 && s.sign_words_map != nullptr) {
     const bool p2 = s.M_pow2 != 0;
-    const bool col = s.params_map != nullptr && (s.sign_path == 1 || (s.sign_path == 0 && sign_col_pays(s)));
+    const bool col = x.params_map != nullptr && (x.path == 1 || (x.path == 0 && sign_col_pays(s)));
     cudaError_t st;
 #define DQ_SIGN_TMA(NG)                                                                           \
-  st = col ? (p2 ? launch_sign_col<NG, true, false>(s, stream) : launch_sign_col<NG, false, false>(s, stream)) \
+  st = col ? (p2 ? launch_sign_col<NG, true, false>(s, x, stream) : launch_sign_col<NG, false, false>(s, x, stream)) \
            : (p2 ? launch_sign_tma<NG, true>(s, stream) : launch_sign_tma<NG, false>(s, stream))
     switch ((s.M + 4) / 5) {
       case 1: DQ_SIGN_TMA(1); break;
