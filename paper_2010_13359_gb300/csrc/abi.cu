@@ -32,7 +32,7 @@ struct dqgan_handle {
   CUtensorMap words_map;         // TMA map of the last message buffer the server saw
   const void* words_map_msgs = nullptr;
   bool words_map_ok = false;
-  CUtensorMap params_map;        // TMA map of the last parameter vector the sign server saw
+  CUtensorMap params_map;        // TMA map of the last parameter vector the sign / squant server saw
   const float* params_map_w = nullptr;
   bool params_map_ok = false;
   int32_t sign_path = 0;         // DQGAN_SIGN_SERVER at creation: 0 auto, 1 col, 2 tma
@@ -457,9 +457,13 @@ int dqgan_server_aggregate_update(dqgan_handle* h, const void* msgs_all, float* 
   x.path = h->sign_path;
   x.seg_slices = h->seg_slices;
   x.seg_nslices = h->seg_nslices;
-  if (tma_sign && s.sign_words_map && s.d >= 32) {
+  // parameter boxes: 32 rows for the sign column kernel, one slice of
+  // 32 * (32 / b) elements for the b = 2, 4 quantiser server
+  const bool boxed_squant = tma_squant && s.squant_words_map && h->cfg.bits != 8;
+  if (((tma_sign && s.sign_words_map) || boxed_squant) && s.d >= 32) {
     if (h->params_map_w != params) {
-      h->params_map_ok = dq::encode_params_map(params, s.d, &h->params_map);
+      const int32_t rows = boxed_squant ? 32 / h->cfg.bits : 32;
+      h->params_map_ok = dq::encode_params_map(params, s.d, rows, &h->params_map);
       h->params_map_w = params;
     }
     if (h->params_map_ok) x.params_map = &h->params_map;
@@ -468,7 +472,7 @@ int dqgan_server_aggregate_update(dqgan_handle* h, const void* msgs_all, float* 
   switch (h->cfg.compressor) {
     case DQGAN_SIGN: st = dq::launch_sign_server(s, x, h->stream, &h->launches); break;
     case DQGAN_SQUANT:
-    case DQGAN_QSGD: st = dq::launch_squant_server(s, h->stream, &h->launches); break;
+    case DQGAN_QSGD: st = dq::launch_squant_server(s, x.params_map, h->stream, &h->launches); break;
     case DQGAN_IDENTITY: st = dq::launch_identity_server(s, h->stream, &h->launches); break;
     case DQGAN_TOPK: st = dq::launch_topk_server(s, h->scratch, h->stream, &h->launches); break;
   }

@@ -96,9 +96,11 @@ bool encode_words_map(const uint8_t* msgs, int64_t msg_stride, int64_t off_paylo
 constexpr int kSignSegBoxWords = 36;
 
 // TMA tensor map over the parameters: floor(d / 32) rows of 32 fp32 (the
-// partial last row, if any, is outside it), boxes of 32 x 32, 128-byte
-// swizzle, zero fill.  Needs d >= 32 and w 16-byte aligned.
-bool encode_params_map(float* w, int64_t d, CUtensorMap* out);
+// partial last row, if any, is outside it), boxes of 32 floats x box_rows
+// rows (32 for the sign server's column kernel; 32 * (32 / b) / 32 for the
+// b-bit quantiser's server at b = 2, 4), 128-byte swizzle, zero fill.  Needs
+// d >= 32 and w 16-byte aligned.
+bool encode_params_map(float* w, int64_t d, int32_t box_rows, CUtensorMap* out);
 
 // Kernel launchers: each enqueues its kernels on `stream`, adds the number of
 // kernels it launched to *launches and returns the launch status.
@@ -122,7 +124,10 @@ cudaError_t launch_topk_compress(const CompressArgs& a, int64_t k, bool keep_h, 
 
 cudaError_t launch_sign_server(const ServerArgs& s, const SignServerExtras& x, cudaStream_t stream,
                                uint64_t* launches);
-cudaError_t launch_squant_server(const ServerArgs& s, cudaStream_t stream, uint64_t* launches);
+// params_map: encode_params_map(w, d, 32 * (32 / bits) / 32) for bits 2 and 4,
+// or nullptr (then those widths take the kernel without TMA).
+cudaError_t launch_squant_server(const ServerArgs& s, const CUtensorMap* params_map, cudaStream_t stream,
+                                 uint64_t* launches);
 cudaError_t launch_identity_server(const ServerArgs& s, cudaStream_t stream, uint64_t* launches);
 cudaError_t launch_topk_server(const ServerArgs& s, void* scratch, cudaStream_t stream, uint64_t* launches);
 

@@ -764,6 +764,97 @@ __global__ void __launch_bounds__(256) squant_server_kernel(const ServerArgs s) 
   }
 }
 
+// Transpose of a 16 x 16 block of 2-bit entries held one row per register:
+// on entry entry e of a[m] is at bits 2e; on exit entry m of a[e] is the old
+// entry e of a[m].  Block swaps of 8 and 4 entries by byte permutes, then of
+// 2 and 1 entries by shifts and masks (rows k and k + B, S = 2B bits).
+template <int B, int S>
+__device__ __forceinline__ void swap_stage16(uint32_t (&a)[16], uint32_t m) {
+#pragma unroll
+  for (int k = 0; k < 16; ++k) {
+    if ((k & B) == 0) {
+      const uint32_t x = a[k], y = a[k + B];
+      a[k] = (x & m) | ((y << S) & ~m);
+      a[k + B] = ((x >> S) & m) | (y & ~m);
+    }
+  }
+}
+
+__device__ __forceinline__ void transpose16x2_regs(uint32_t (&a)[16]) {
+#pragma unroll
+  for (int k = 0; k < 8; ++k) {
+    const uint32_t x = a[k], y = a[k + 8];
+    a[k] = __byte_perm(x, y, 0x5410);
+    a[k + 8] = __byte_perm(x, y, 0x7632);
+  }
+#pragma unroll
+  for (int k = 0; k < 16; ++k) {
+    if ((k & 4) == 0) {
+      const uint32_t x = a[k], y = a[k + 4];
+      a[k] = __byte_perm(x, y, 0x6240);
+      a[k + 4] = __byte_perm(x, y, 0x7351);
+    }
+  }
+  swap_stage16<2, 4>(a, 0x0F0F0F0Fu);
+  swap_stage16<1, 2>(a, 0x33333333u);
+}
+
+// b = 2 sums over workers by pair tables.  The decoded value of a 2-bit code
+// is v(0, s) = -s, v(1, s) = +0, v(2, s) = +s (code 3 never occurs; 0 here).
+// Pair p = workers (2p, 2p + 1): lane l holds
+//   T_p[l mod 16] = fl(v(l mod 4, s_2p) + v((l / 4) mod 4, s_2p+1)),
+// the pair's contribution for the 4-bit field code_2p | code_2p+1 << 2.  A
+// worker at or beyond M has scale 0 and adds only zeros.
+template <int NP>
+__device__ __forceinline__ void build_pair_tables(float my_scale, int lane, float (&T)[NP]) {
+  const int ca = lane & 3, cb = (lane >> 2) & 3;
+  const float fa = ca == 0 ? -1.f : (ca == 2 ? 1.f : 0.f);  // v(c, s) = f(c) * s exactly
+  const float fb = cb == 0 ? -1.f : (cb == 2 ? 1.f : 0.f);
+#pragma unroll
+  for (int p = 0; p < NP; ++p) {
+    const float sa = __shfl_sync(kFullMask, my_scale, 2 * p);
+    const float sb = __shfl_sync(kFullMask, my_scale, 2 * p + 1);
+    T[p] = __fadd_rn(__fmul_rn(fa, sa), __fmul_rn(fb, sb));
+  }
+}
+
+// The b = 2 server update of this lane's 16 elements, w_j = fl(w_j - sum_j / M)
+// in wv, with the worker sums by pair tables: the lane's code word of
+// each worker (16 per set of workers) is transposed so that one register
+// holds one element's codes of 16 workers, whose 4-bit pair fields index the
+// pair tables by shuffle (the lane index is taken mod 32: the tables repeat
+// in lanes 16..31, so the bits above a field do not matter).  The eight pair
+// values of a set are added pairwise, the two sets' sums last.
+template <int NSET, bool POW2>
+__device__ __forceinline__ void b2_pair_table_update(const uint32_t* words, const ServerArgs& s,
+                                                     const float (&T)[8 * NSET], float (&wv)[16]) {
+  float acc[16];
+#pragma unroll
+  for (int set = 0; set < NSET; ++set) {
+    uint32_t z[16];
+#pragma unroll
+    for (int r = 0; r < 16; ++r) {
+      const int m = 16 * set + r;
+      z[r] = m < s.M ? words[32 * m] : 0x55555555u;  // rows past M: level-0 codes (never read past the box)
+    }
+    transpose16x2_regs(z);
+#pragma unroll
+    for (int e = 0; e < 16; ++e) {
+      float v[8];
+#pragma unroll
+      for (int p = 0; p < 8; ++p) v[p] = __shfl_sync(kFullMask, T[8 * set + p], (int)(z[e] >> (4 * p)));
+      const float sum = __fadd_rn(__fadd_rn(__fadd_rn(v[0], v[1]), __fadd_rn(v[2], v[3])),
+                                  __fadd_rn(__fadd_rn(v[4], v[5]), __fadd_rn(v[6], v[7])));
+      acc[e] = set == 0 ? sum : __fadd_rn(acc[e], sum);
+      if (set + 1 == NSET) wv[e] = __fsub_rn(wv[e], average_t<POW2>(acc[e], s));
+    }
+  }
+}
+
+// Whether the squant server stages the parameters by TMA (b = 2 and 4; for
+// b = 8 a lane's 16 bytes of w are contiguous across the warp already).
+constexpr bool sq_params_boxed(int bits) { return bits != 8; }
+
 // b-bit stochastic quantiser with M <= 32 and buckets of at least 32*32/b
 // elements: the code words are staged by TMA like the sign words above (a
 // box is 32 words of every worker, M rows of 128 bytes, no swizzle: lane l
@@ -772,25 +863,45 @@ __global__ void __launch_bounds__(256) squant_server_kernel(const ServerArgs s) 
 // order, it decodes them with the worker's scale (broadcast by shuffle from
 // the lane that loaded it) and V[code] (b = 8: the bank-replicated table;
 // b = 4: the worker's 15 products fl(s * V[c]), one per lane, looked up by
-// shuffle; b = 2: two bit tests, level-0 codes skipped).
-// Worker-order sums from +0, so the result equals the oracle's bit for bit.
+// shuffle).  Worker-order sums from +0, so the result equals the oracle's
+// bit for bit.  b = 2 sums by pair tables instead (b2_pair_table_update, NSET
+// sets of 16 workers; tables rebuilt only when the bucket changes): not
+// worker order, so w agrees with the oracle up to the summation order.
 // With layer segments (SEG) a slice may hold words of several buckets: each
-// lane then reads the workers' scales of its own word's bucket.
-template <int BITS, bool POW2, bool SEG>
+// lane then reads the workers' scales of its own word's bucket (b = 2: two
+// bit tests per worker and element, level-0 codes skipped, worker order).
+// For b = 2 and 4 (a lane owns 64 or 32 contiguous bytes of w, which plain
+// loads would fetch at a 64- or 32-byte lane stride) the slice's parameters
+// come by TMA as well: w viewed as rows of 32 floats (pmap), a box of
+// R = 32 (32 / b) / 32 rows with 128-byte swizzle (16-byte chunk c of row r
+// at chunk c ^ (r mod 8), so the lanes' 16-byte accesses never conflict),
+// loaded with the code words on the same mbarrier and stored back by TMA.
+// Rows past the map read as zero and are not stored; the partial last row
+// (d mod 32 elements, outside the map) is read and written directly.
+// Per warp two buffers of each kind: slice i + 1 loads while slice i is
+// decoded.
+template <int BITS, bool POW2, bool SEG, int NSET>
 __global__ void __launch_bounds__(32 * kTmaWarps)
-squant_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap tmap) {
+squant_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap tmap,
+                         const __grid_constant__ CUtensorMap pmap) {
   constexpr int K = (1 << (BITS - 1)) - 1;
-  constexpr uint32_t MASK = (1u << BITS) - 1u;
   constexpr int EPL = 32 / BITS;  // elements per lane (one code word)
   constexpr int SLICE = 32 * EPL; // elements per slice
+  constexpr bool WB = sq_params_boxed(BITS);
+  constexpr int R = SLICE / 32;                 // parameter rows per slice
+  constexpr uint32_t PBOX = WB ? R * 128u : 0u;  // bytes of a parameter box (1024-byte multiple)
+  constexpr int LPR = 32 / EPL;                 // lanes per parameter row
   extern __shared__ uint8_t smem_raw[];
   __shared__ uint64_t bars[kTmaWarps][2];
   __shared__ float V8[BITS == 8 ? 256 * 32 : 1];
   const int lane = threadIdx.x & 31;
   const int warp = threadIdx.x >> 5;
   const uint32_t box_bytes = (uint32_t)s.M * 128u;
-  const uint32_t raw = smem_addr(smem_raw);  // 128-byte aligned boxes
-  uint8_t* const buf0 = smem_raw + ((128u - (raw & 127u)) & 127u) + warp * 2 * box_bytes;  // buffer i at + i*box
+  const uint32_t raw = smem_addr(smem_raw);
+  // parameter boxes of every warp first (1024-byte aligned), then the word boxes
+  uint8_t* const pbuf0 = smem_raw + ((1024u - (raw & 1023u)) & 1023u) + warp * 2 * PBOX;  // + i * PBOX
+  uint8_t* const buf0 = smem_raw + ((1024u - (raw & 1023u)) & 1023u) + kTmaWarps * 2 * PBOX +
+                        warp * 2 * box_bytes;  // + i * box_bytes
   uint64_t* bar = bars[warp];
   if constexpr (BITS == 8) {
     for (int t = threadIdx.x; t < 256 * 32; t += blockDim.x) {
@@ -804,10 +915,10 @@ squant_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap
       V8[t] = v;
     }
   }
-  float V4 = 0.f;  // b = 4: lane c holds V[c]
+  float V4 = 0.f;  // b = 4: lane l holds V[l mod 16]
   if constexpr (BITS == 4) {
-    const int level = lane - K;
-    if (lane <= 2 * K && level != 0) {
+    const int level = (lane & 15) - K;
+    if ((lane & 15) <= 2 * K && level != 0) {
       const float mag = __fdiv_rn((float)(level < 0 ? -level : level), (float)K);
       V4 = level < 0 ? -mag : mag;
     }
@@ -824,35 +935,51 @@ squant_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap
   const int64_t nslices = SEG ? (s.d + SLICE - 1) / SLICE : nb * spb;
   const int64_t stride = (int64_t)gridDim.x * kTmaWarps;
   const int32_t x0 = (int32_t)(s.off_payload >> 2);
+  const int64_t nrows = s.d >> 5;     // rows of the parameter map
+  const int tail = (int)(s.d & 31);   // elements of the partial row nrows
   const bool active = lane < s.M;
+  // slice sl covers code words [32 sl, 32 sl + 32) and parameter rows
+  // [R sl, R sl + R): buckets hold whole slices
+  auto issue = [&](int64_t sl_, int i) {
+    const bool boxed = WB && R * sl_ < nrows;
+    mbar_arrive_expect_tx(&bar[i], box_bytes + (boxed ? PBOX : 0u));
+    tma_load_2d(buf0 + i * box_bytes, &tmap, x0 + (int32_t)(32 * sl_), 0, &bar[i]);
+    if (boxed) tma_load_2d(pbuf0 + i * PBOX, &pmap, 0, (int32_t)(R * sl_), &bar[i]);
+  };
   int64_t sl = (int64_t)blockIdx.x * kTmaWarps + warp;
-  // slice sl covers code words [32 sl, 32 sl + 32): buckets hold whole slices
-  if (sl < nslices && lane == 0) {
-    mbar_arrive_expect_tx(&bar[0], box_bytes);
-    tma_load_2d(buf0, &tmap, x0 + (int32_t)(32 * sl), 0, &bar[0]);
-  }
+  if (sl < nslices && lane == 0) issue(sl, 0);
   uint32_t it = 0;
   bool ok = true;
+  float T2[8 * NSET];  // b = 2 pair tables of bucket t2_bkt
+  int64_t t2_bkt = -1;
   for (; sl < nslices; sl += stride, ++it) {
     const int cur = (int)(it & 1u);
     const int64_t nxt = sl + stride;
     if (nxt < nslices && lane == 0) {
-      fence_proxy_async_shared();
-      mbar_arrive_expect_tx(&bar[cur ^ 1], box_bytes);
-      tma_load_2d(buf0 + (cur ^ 1) * box_bytes, &tmap, x0 + (int32_t)(32 * nxt), 0, &bar[cur ^ 1]);
+      if constexpr (WB) bulk_wait_read_all();  // the previous slice's store has read its box
+      fence_proxy_async_shared();  // this warp's accesses of those buffers came before
+      issue(nxt, cur ^ 1);
     }
     const int64_t b = sl / spb;
     const int64_t j0 = SLICE * sl + EPL * lane;  // this lane's first element
+    // the lane's parameters: row pr of the box, 16-byte chunks pc0 ..
+    const int pr = lane / LPR;
+    const int pc0 = (lane % LPR) * (EPL / 4);
+    const bool boxed = WB && R * sl < nrows;
+    const bool direct = WB && R * sl + pr == nrows && tail != 0;  // the partial last row
+    uint8_t* const prow = pbuf0 + cur * PBOX + pr * 128;
     float wv[EPL];
+    if constexpr (!WB) {
 #pragma unroll
-    for (int q = 0; q < EPL / 4; ++q) {
-      const int64_t j = j0 + 4 * q;
-      if (j + 3 < s.d) {
-        const float4 x = __ldcs(reinterpret_cast<const float4*>(s.w + j));
-        wv[4 * q] = x.x; wv[4 * q + 1] = x.y; wv[4 * q + 2] = x.z; wv[4 * q + 3] = x.w;
-      } else {
+      for (int q = 0; q < EPL / 4; ++q) {
+        const int64_t j = j0 + 4 * q;
+        if (j + 3 < s.d) {
+          const float4 x = __ldcs(reinterpret_cast<const float4*>(s.w + j));
+          wv[4 * q] = x.x; wv[4 * q + 1] = x.y; wv[4 * q + 2] = x.z; wv[4 * q + 3] = x.w;
+        } else {
 #pragma unroll
-        for (int r = 0; r < 4; ++r) wv[4 * q + r] = (j + r < s.d) ? s.w[j + r] : 0.f;
+          for (int r = 0; r < 4; ++r) wv[4 * q + r] = (j + r < s.d) ? s.w[j + r] : 0.f;
+        }
       }
     }
     // The slice's bucket; with layer segments, each lane's word's bucket, and
@@ -875,6 +1002,21 @@ squant_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap
     ok = mbar_wait_bounded(&bar[cur], (it >> 1) & 1u, s.err);
     ok = __all_sync(kFullMask, ok);
     if (!ok) break;
+    if constexpr (WB) {
+#pragma unroll
+      for (int q = 0; q < EPL / 4; ++q) {
+        float4 x = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (boxed) x = *reinterpret_cast<const float4*>(prow + (((pc0 + q) ^ (pr & 7)) << 4));
+        if (direct) {
+          const int64_t j = j0 + 4 * q;
+          x.x = j < s.d ? s.w[j] : 0.f;
+          x.y = j + 1 < s.d ? s.w[j + 1] : 0.f;
+          x.z = j + 2 < s.d ? s.w[j + 2] : 0.f;
+          x.w = j + 3 < s.d ? s.w[j + 3] : 0.f;
+        }
+        wv[4 * q] = x.x; wv[4 * q + 1] = x.y; wv[4 * q + 2] = x.z; wv[4 * q + 3] = x.w;
+      }
+    }
     const uint32_t* words = reinterpret_cast<const uint32_t*>(buf0 + cur * box_bytes) + lane;
     const float* V8l = V8 + lane;
     float acc[EPL];
@@ -895,10 +1037,12 @@ squant_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap
         }
         return;
       }
-      // b = 4: lane c first forms this worker's decoded value of code c,
-      // fl(s * V[c]); each element then fetches its value with one shuffle.
-      // (With layer segments the lanes' scales may differ: look up V[c] and
-      // multiply by the lane's own scale instead.)
+      // b = 4: lane c first forms this worker's decoded value of code c mod 16,
+      // fl(s * V[c mod 16]); each element then fetches its value with one
+      // shuffle (the lane index is taken mod 32 and the values repeat in lanes
+      // 16..31, so the bits above the element's code need no mask).  (With
+      // layer segments the lanes' scales may differ: look up V[c] and multiply
+      // by the lane's own scale instead.)
       const float T4 = (BITS == 4) ? __fmul_rn(mixed ? 1.0f : sc, V4) : 0.f;
 #pragma unroll
       for (int e = 0; e < EPL; ++e) {
@@ -906,7 +1050,7 @@ squant_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap
         if constexpr (BITS == 2) {
           v = 0.f;
         } else if constexpr (BITS == 4) {
-          v = __shfl_sync(kFullMask, T4, (int)((word >> (4 * e)) & MASK));
+          v = __shfl_sync(kFullMask, T4, (int)(word >> (4 * e)));
           if (mixed) v = __fmul_rn(sc, v);
         } else {
           v = __fmul_rn(sc, V8l[__byte_perm(word, 0u, 0x4440u | (uint32_t)e) * 32u]);
@@ -915,42 +1059,64 @@ squant_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap
       }
     };
     int m = 0;
-    for (; m + 4 <= s.M; m += 4) {
-      const uint32_t w0 = words[32 * m], w1 = words[32 * (m + 1)];
-      const uint32_t w2 = words[32 * (m + 2)], w3 = words[32 * (m + 3)];
-      const float s0 = scale_of(m), s1 = scale_of(m + 1);
-      const float s2 = scale_of(m + 2), s3 = scale_of(m + 3);
-      add_worker(w0, s0);
-      add_worker(w1, s1);
-      add_worker(w2, s2);
-      add_worker(w3, s3);
-    }
     if constexpr (BITS == 2) {
-      // the last M mod 4 workers as one more group of four: the missing
-      // workers read as all-level-0 words, which add nothing
-      if (m < s.M) {
-        uint32_t wq[4];
-        float sq[4];
-#pragma unroll
-        for (int u = 0; u < 4; ++u) {
-          const bool ok = m + u < s.M;
-          wq[u] = ok ? words[32 * (m + u)] : 0x55555555u;
-          if constexpr (SEG) sq[u] = ok ? scale_of(m + u) : 0.f;
-          else sq[u] = __shfl_sync(kFullMask, my_scale, (m + u) & 31);
+      if (!(SEG && mixed)) {
+        if (bkt != t2_bkt) {
+          build_pair_tables<8 * NSET>(my_scale, lane, T2);
+          t2_bkt = bkt;
         }
-#pragma unroll
-        for (int u = 0; u < 4; ++u) add_worker(wq[u], sq[u]);
+        b2_pair_table_update<NSET, POW2>(words, s, T2, wv);
+        m = s.M;
       }
-    } else {
-      for (; m < s.M; ++m) add_worker(words[32 * m], scale_of(m));
+    }
+    // per-worker decode: b = 4, 8, and b = 2 on slices that span layer segments
+    const bool per_worker = BITS != 2 || (SEG && mixed);
+    if (BITS != 2 || SEG) {
+      for (; m + 4 <= s.M; m += 4) {
+        const uint32_t w0 = words[32 * m], w1 = words[32 * (m + 1)];
+        const uint32_t w2 = words[32 * (m + 2)], w3 = words[32 * (m + 3)];
+        const float s0 = scale_of(m), s1 = scale_of(m + 1);
+        const float s2 = scale_of(m + 2), s3 = scale_of(m + 3);
+        add_worker(w0, s0);
+        add_worker(w1, s1);
+        add_worker(w2, s2);
+        add_worker(w3, s3);
+      }
+      if constexpr (BITS == 2) {
+        // the last M mod 4 workers as one more group of four: the missing
+        // workers read as all-level-0 words, which add nothing
+        if (m < s.M) {
+          uint32_t wq[4];
+          float sq[4];
+#pragma unroll
+          for (int u = 0; u < 4; ++u) {
+            const bool ok = m + u < s.M;
+            wq[u] = ok ? words[32 * (m + u)] : 0x55555555u;
+            sq[u] = ok ? scale_of(m + u) : 0.f;
+          }
+#pragma unroll
+          for (int u = 0; u < 4; ++u) add_worker(wq[u], sq[u]);
+        }
+      } else {
+        for (; m < s.M; ++m) add_worker(words[32 * m], scale_of(m));
+      }
     }
 #pragma unroll
     for (int q = 0; q < EPL / 4; ++q) {
       const int64_t j = j0 + 4 * q;
       float o[4];
 #pragma unroll
-      for (int r = 0; r < 4; ++r) o[r] = __fsub_rn(wv[4 * q + r], average_t<POW2>(acc[4 * q + r], s));
-      if (j + 3 < s.d) {
+      for (int r = 0; r < 4; ++r)
+        o[r] = per_worker ? __fsub_rn(wv[4 * q + r], average_t<POW2>(acc[4 * q + r], s)) : wv[4 * q + r];
+      if constexpr (WB) {
+        if (boxed)
+          *reinterpret_cast<float4*>(prow + (((pc0 + q) ^ (pr & 7)) << 4)) = make_float4(o[0], o[1], o[2], o[3]);
+        if (direct) {
+#pragma unroll
+          for (int r = 0; r < 4; ++r)
+            if (j + r < s.d) s.w[j + r] = o[r];
+        }
+      } else if (j + 3 < s.d) {
         __stcs(reinterpret_cast<float4*>(s.w + j), make_float4(o[0], o[1], o[2], o[3]));
       } else {
 #pragma unroll
@@ -958,10 +1124,16 @@ squant_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap
           if (j + r < s.d) s.w[j + r] = o[r];
       }
     }
+    if constexpr (WB) fence_proxy_async_shared();  // the box writes above, before the store reads them
+    __syncwarp();
+    if (WB && lane == 0 && boxed) tma_store_2d(&pmap, 0, (int32_t)(R * sl), pbuf0 + cur * PBOX);
     __syncwarp();
   }
-  if (!ok && lane == 0 && sl + stride < nslices)
-    mbar_wait_bounded(&bar[(it & 1u) ^ 1u], ((it + 1) >> 1) & 1u, s.err);
+  if (lane == 0) {
+    if constexpr (WB) bulk_wait_all();  // stores complete before the block's shared memory is released
+    // after a time-out, the copy of the next slice may still be in flight
+    if (!ok && sl + stride < nslices) mbar_wait_bounded(&bar[(it & 1u) ^ 1u], ((it + 1) >> 1) & 1u, s.err);
+  }
 }
 
 // Identity: the messages are the p vectors themselves (worker order).
@@ -1083,10 +1255,11 @@ bool sign_col_pays(const ServerArgs& s) {
   return nslices >= 4ll * sms[dev] * kColWarps;
 }
 
-template <int BITS, bool POW2, bool SEG>
-cudaError_t launch_squant_tma(const ServerArgs& s, cudaStream_t stream) {
-  auto kern = squant_server_tma_kernel<BITS, POW2, SEG>;
-  const int smem = kTmaWarps * 2 * s.M * 128 + 128;  // + alignment slack
+template <int BITS, bool POW2, bool SEG, int NSET>
+cudaError_t launch_squant_tma(const ServerArgs& s, const CUtensorMap* params_map, cudaStream_t stream) {
+  auto kern = squant_server_tma_kernel<BITS, POW2, SEG, NSET>;
+  constexpr int pbox = sq_params_boxed(BITS) ? 32 * (32 / BITS) * 4 : 0;  // bytes of a parameter box
+  const int smem = kTmaWarps * 2 * (pbox + s.M * 128) + 1024;  // + alignment slack
   int dev = 0;
   cudaError_t st = cudaGetDevice(&dev);
   if (st != cudaSuccess) return st;
@@ -1099,7 +1272,9 @@ cudaError_t launch_squant_tma(const ServerArgs& s, cudaStream_t stream) {
                               : ((s.d + s.bucket - 1) / s.bucket) * (s.bucket / (32 * (32 / BITS)));
   const int64_t need = (nslices + kTmaWarps - 1) / kTmaWarps;
   const int64_t cap = (int64_t)sms * (per_sm > 0 ? per_sm : 1);
-  kern<<<(unsigned)(need < cap ? need : cap), 32 * kTmaWarps, smem, stream>>>(s, *s.squant_words_map);
+  // (b = 8 takes no parameter map: the word map stands in for the unused argument)
+  kern<<<(unsigned)(need < cap ? need : cap), 32 * kTmaWarps, smem, stream>>>(
+      s, *s.squant_words_map, sq_params_boxed(BITS) ? *params_map : *s.squant_words_map);
   return cudaGetLastError();
 }
 
@@ -1186,19 +1361,24 @@ cudaError_t launch_sign_server(const ServerArgs& s, const SignServerExtras& x, c
   return cudaGetLastError();
 }
 
-cudaError_t launch_squant_server(const ServerArgs& s, cudaStream_t stream, uint64_t* launches) {
-  if (s.squant_words_map != nullptr && s.M <= 32 && s.bucket >= 32 * (32 / s.bits)) {
+cudaError_t launch_squant_server(const ServerArgs& s, const CUtensorMap* params_map, cudaStream_t stream,
+                                 uint64_t* launches) {
+  if (s.squant_words_map != nullptr && s.M <= 32 && s.bucket >= 32 * (32 / s.bits) &&
+      (params_map != nullptr || !sq_params_boxed(s.bits))) {
     const bool p2 = s.M_pow2 != 0;
     cudaError_t st = cudaErrorInvalidValue;
-#define DQ_SQ_TMA(B)                                                                          \
-  st = s.word_bucket ? (p2 ? launch_squant_tma<B, true, true>(s, stream)                      \
-                           : launch_squant_tma<B, false, true>(s, stream))                    \
-                     : (p2 ? launch_squant_tma<B, true, false>(s, stream)                     \
-                           : launch_squant_tma<B, false, false>(s, stream))
+#define DQ_SQ_TMA(B, NSET)                                                                              \
+  st = s.word_bucket ? (p2 ? launch_squant_tma<B, true, true, NSET>(s, params_map, stream)              \
+                           : launch_squant_tma<B, false, true, NSET>(s, params_map, stream))            \
+                     : (p2 ? launch_squant_tma<B, true, false, NSET>(s, params_map, stream)             \
+                           : launch_squant_tma<B, false, false, NSET>(s, params_map, stream))
     switch (s.bits) {
-      case 2: DQ_SQ_TMA(2); break;
-      case 4: DQ_SQ_TMA(4); break;
-      case 8: DQ_SQ_TMA(8); break;
+      case 2:
+        if (s.M <= 16) DQ_SQ_TMA(2, 1);
+        else DQ_SQ_TMA(2, 2);
+        break;
+      case 4: DQ_SQ_TMA(4, 1); break;
+      case 8: DQ_SQ_TMA(8, 1); break;
     }
 #undef DQ_SQ_TMA
     *launches += 1;
@@ -1277,12 +1457,12 @@ bool encode_words_map(const uint8_t* msgs, int64_t msg_stride, int64_t off_paylo
                 CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-bool encode_params_map(float* w, int64_t d, CUtensorMap* out) {
+bool encode_params_map(float* w, int64_t d, int32_t box_rows, CUtensorMap* out) {
   const EncodeFn encode = tensor_map_encoder();
-  if (!encode || d < 32 || ((uintptr_t)w & 15u) != 0) return false;
+  if (!encode || d < 32 || ((uintptr_t)w & 15u) != 0 || box_rows < 1 || box_rows > 256) return false;
   const cuuint64_t dims[2] = {32u, (cuuint64_t)(d / 32)};
   const cuuint64_t strides[1] = {128u};
-  const cuuint32_t box[2] = {32u, 32u};
+  const cuuint32_t box[2] = {32u, (cuuint32_t)box_rows};
   const cuuint32_t elem[2] = {1u, 1u};
   return encode(out, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2, w, dims, strides, box, elem, CU_TENSOR_MAP_INTERLEAVE_NONE,
                 CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,

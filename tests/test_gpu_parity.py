@@ -167,6 +167,17 @@ def test_worker_counts(P, M, comp, bucket):
     run_parity(P, ocfg, T=3, seed=M)
 
 
+@pytest.mark.parametrize("M", [1, 7, 16, 17, 32])
+@pytest.mark.parametrize("comp,bits,bucket", [(oracle.SQUANT, 2, 512), (oracle.SQUANT, 2, 1024),
+                                              (oracle.QSGD, 2, 2048), (oracle.SQUANT, 4, 512)])
+def test_squant_server_worker_counts(P, M, comp, bits, bucket):
+    """The TMA quantiser servers at every worker count they take: b = 2 in
+    one or two sets of 16 workers (pair tables, several slices per bucket),
+    b = 4 by per-worker lookups; ragged last bucket."""
+    ocfg = oracle_config(3 * 4096 + 2 * 512 + 100, M, comp, lr=1e-2, bucket=bucket, bits=bits, seed=M + bits)
+    run_parity(P, ocfg, T=3, seed=M)
+
+
 def test_multi_tile_topk_many_steps(P):
     """Top-k over many 4096-element tiles with a ragged last tile, 6 steps."""
     ocfg = oracle_config(3 * 4096 * 7 + 123, 3, oracle.TOPK, lr=0.1, k=1500, keep=True)
