@@ -332,10 +332,8 @@ squant_compress_kernel(const CompressArgs a) {
     float en[4];
 #pragma unroll
     for (int q = 0; q < 4; ++q) {
-      int code = K;
-      float qv = 0.f;
-      if (s > 0.f) squant_element<K>(p[i][q], s, inv, rq[q], level_value, &code, &qv);
-      en[q] = __fsub_rn(p[i][q], qv);
+      int code;
+      squant_element<K>(p[i][q], s, inv, rq[q], level_value, &code, &en[q]);
       if (q < nvalid) chunk_bits |= (uint32_t)code << (q * BITS);
     }
     // pack: a chunk is 4*BITS bits; 32 / (4*BITS) neighbouring lanes share a word

@@ -72,26 +72,27 @@ __device__ __forceinline__ uint4 philox4x32_10(uint4 x, uint32_t k0, uint32_t k1
   return x;
 }
 
-// One element of the b-bit stochastic quantiser (s > 0): code and Q(p).
+// One element of the b-bit stochastic quantiser: code and the residual p - Q(p).
 // t = min(fl(|p| * inv), K); r = floor(t); rounds up iff u < t - r, u the top
-// 24 bits of the Philox word; code = K -+ level; Q = sign * fl(s * fl(level/K)).
+// 24 bits of the Philox word; code = K -+ level; Q = sign * fl(s * fl(level/K)),
+// +0 at level 0.  With s = 0 the caller passes inv = 0, so every element
+// takes level 0 (code K) and keeps e = p.
+// No clamp of the level is needed: r <= K, and r = K only when t = K, where
+// the fraction is 0 and never rounds up.  The residual is formed as p + mag
+// for p < 0 and p - mag otherwise, which equals fl(p - Q) for every level:
+// at level 0, mag = fl(s * 0) = +0 and p -+ (+0) = p - (+0).
 template <int K>
 __device__ __forceinline__ void squant_element(float p, float s, float inv, uint32_t rnd,
-                                               const float* level_value, int* code, float* q) {
+                                               const float* level_value, int* code, float* resid) {
   const float t = fminf(__fmul_rn(fabsf(p), inv), (float)K);
   const float r = floorf(t);
   const float f = __fsub_rn(t, r);
   const float u = __fmul_rn(__uint2float_rn(rnd >> 8), 0x1p-24f);
-  int level = (int)r + (u < f ? 1 : 0);
-  level = level < K ? level : K;
+  const int level = (int)r + (u < f ? 1 : 0);
   const bool neg = p < 0.f;
   *code = neg ? K - level : K + level;
-  float qv = 0.f;
-  if (level != 0) {
-    const float mag = __fmul_rn(s, level_value[level]);
-    qv = neg ? -mag : mag;
-  }
-  *q = qv;
+  const float mag = __fmul_rn(s, level_value[level]);
+  *resid = neg ? __fadd_rn(p, mag) : __fsub_rn(p, mag);
 }
 
 // ---------------------------------------------------------------------------
