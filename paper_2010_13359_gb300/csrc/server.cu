@@ -551,6 +551,12 @@ sign_server_col_kernel(const ServerArgs s, const SegSlices seg, const __grid_con
 
   Slice c = lo < hi ? slice_of(lo) : Slice{0, 0, 0};
   if (lo < hi && lane == 0) issue(c, 0);
+  // worker `lane`'s scale of a bucket; loaded one slice ahead, so that a new
+  // bucket's tables do not wait for it
+  auto scale_of_bucket = [&](int64_t bkt) -> float {
+    return lane < s.M ? __ldg(reinterpret_cast<const float*>(s.msgs + (int64_t)lane * s.msg_stride) + bkt) : 0.f;
+  };
+  float scale_next = lo < hi ? scale_of_bucket(c.bucket) : 0.f;
   float T[7];
   float s30 = 0.f, s31 = 0.f;
   int64_t table_b = -1;
@@ -565,11 +571,11 @@ sign_server_col_kernel(const ServerArgs s, const SegSlices seg, const __grid_con
       fence_proxy_async_shared();  // this warp's reads of those boxes came before
       issue(cn, cur ^ 1);
     }
+    const float scale_cur = scale_next;  // of bucket c.bucket
+    if (more && cn.bucket != c.bucket) scale_next = scale_of_bucket(cn.bucket);
     if (c.bucket != table_b) {  // warp-uniform
       table_b = c.bucket;
-      const float my_scale =
-          lane < s.M ? __ldg(reinterpret_cast<const float*>(s.msgs + (int64_t)lane * s.msg_stride) + c.bucket)
-                     : 0.f;
+      const float my_scale = scale_cur;
       build_tables<NGT>(my_scale, s.M, lane, T);
       s30 = __shfl_sync(kFullMask, my_scale, 30);
       s31 = __shfl_sync(kFullMask, my_scale, 31);
@@ -948,6 +954,13 @@ squant_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap
   };
   int64_t sl = (int64_t)blockIdx.x * kTmaWarps + warp;
   if (sl < nslices && lane == 0) issue(sl, 0);
+  // with layer segments: the bucket of this lane's word, loaded one slice
+  // ahead so that the scale load does not wait for it (-1 past d)
+  auto word_bucket_of = [&](int64_t sl_) -> int64_t {
+    const int64_t j = SLICE * sl_ + EPL * lane;
+    return (sl_ < nslices && j < s.d) ? (int64_t)__ldg(s.word_bucket + (j >> 5)) : -1;
+  };
+  int64_t wb_next = SEG ? word_bucket_of(sl) : 0;
   uint32_t it = 0;
   bool ok = true;
   float T2[8 * NSET];  // b = 2 pair tables of bucket t2_bkt
@@ -960,6 +973,8 @@ squant_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap
       fence_proxy_async_shared();  // this warp's accesses of those buffers came before
       issue(nxt, cur ^ 1);
     }
+    const int64_t wb_cur = wb_next;
+    if constexpr (SEG) wb_next = word_bucket_of(nxt);
     const int64_t b = sl / spb;
     const int64_t j0 = SLICE * sl + EPL * lane;  // this lane's first element
     // the lane's parameters: row pr of the box, 16-byte chunks pc0 ..
@@ -987,7 +1002,7 @@ squant_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap
     int64_t bkt = b, my_bkt = b;
     bool mixed = false;
     if constexpr (SEG) {
-      my_bkt = (j0 < s.d) ? (int64_t)__ldg(s.word_bucket + (j0 >> 5)) : -1;
+      my_bkt = wb_cur;
       bkt = __shfl_sync(kFullMask, my_bkt, 0);  // lane 0's elements always exist
       if (my_bkt < 0) my_bkt = bkt;
       mixed = !__all_sync(kFullMask, my_bkt == bkt);
