@@ -18,10 +18,10 @@
 namespace dq {
 namespace {
 
-// Loads this thread's CPL chunks c = c0 + 32 i of the bucket [base, end) and
-// forms p.  Elements outside the bucket read as 0 and give p = 0.  sg (if
+// Loads this thread's CPL chunks c = c0 + CSTRIDE i of the bucket [base, end)
+// and forms p.  Elements outside the bucket read as 0 and give p = 0.  sg (if
 // HOLD) receives fl(eta * g) for the lookahead.
-template <int CPL, bool HOLD>
+template <int CPL, bool HOLD, int CSTRIDE = 32>
 __device__ __forceinline__ void load_and_form(const CompressArgs& a, const float* g, const float* e,
                                               int64_t base, int64_t end, int c0, bool full,
                                               float (&p)[CPL][4], float (&sg)[HOLD ? CPL : 1][4]) {
@@ -29,7 +29,7 @@ __device__ __forceinline__ void load_and_form(const CompressArgs& a, const float
   if (full) {
 #pragma unroll
     for (int i = 0; i < CPL; ++i) {
-      const int c = c0 + 32 * i;
+      const int c = c0 + CSTRIDE * i;
       float4 gv = make_float4(0.f, 0.f, 0.f, 0.f), ev = gv;
       if (c < nchunk) {
         gv = ld_stream4(g + base + 4 * c);
@@ -47,7 +47,7 @@ __device__ __forceinline__ void load_and_form(const CompressArgs& a, const float
   } else {
 #pragma unroll
     for (int i = 0; i < CPL; ++i) {
-      const int c = c0 + 32 * i;
+      const int c = c0 + CSTRIDE * i;
 #pragma unroll
       for (int q = 0; q < 4; ++q) {
         const int64_t j = base + 4 * c + q;
@@ -226,6 +226,12 @@ squant_compress_kernel(const CompressArgs a) {
   constexpr bool HOLD = KEEP_H && CPT <= 8;
   constexpr int BPC = WPB < 4 ? 4 / WPB : 1;  // buckets per CTA (CTA = max(4, WPB) warps)
   constexpr int CHAIN = 32 * CPT * WPB;
+  // b = 2, 4 with the max-abs scale and one warp per bucket: lane l takes the
+  // CPT consecutive chunks CPT l .. CPT l + CPT - 1, which hold whole code
+  // words, so its codes are packed without shuffles (the max is the same in
+  // any order; the l2 chain order of QSGD needs the interleaved mapping).
+  constexpr bool LC = WPB == 1 && !L2 && BITS < 8 && (CPT * 4 * BITS) % 32 == 0;
+  constexpr int CPW = 8 / BITS;  // chunks per code word
   __shared__ float level_value[K + 1];        // fl(r / K)
   __shared__ float warp_max[BPC * WPB];
   __shared__ float chain[(L2 && WPB > 1) ? BPC * CHAIN : 1];
@@ -257,7 +263,7 @@ squant_compress_kernel(const CompressArgs a) {
   float p[CPT][4];
   float sg[HOLD ? CPT : 1][4];
   if (valid) {
-    load_and_form<CPT, HOLD>(a, g, e, base, end, 32 * row0 + lane, full, p, sg);
+    load_and_form<CPT, HOLD, LC ? 1 : 32>(a, g, e, base, end, LC ? CPT * lane : 32 * row0 + lane, full, p, sg);
   } else {
 #pragma unroll
     for (int i = 0; i < CPT; ++i)
@@ -319,9 +325,10 @@ squant_compress_kernel(const CompressArgs a) {
 
   uint32_t* words = reinterpret_cast<uint32_t*>(msg + a.off_payload);
   const int64_t nwords = (a.d * BITS + 31) >> 5;
+  uint32_t lc_word = 0;  // LC: the code word being filled
 #pragma unroll
   for (int i = 0; i < CPT; ++i) {
-    const int c = 32 * (row0 + i) + lane;
+    const int c = LC ? CPT * lane + i : 32 * (row0 + i) + lane;
     const int64_t j = base + 4 * c;
     const int64_t cg = j >> 2;  // global chunk index = Philox counter word 0
     const int nvalid = (c < nchunk) ? (int)max64(0, min64(4, end - j)) : 0;
@@ -336,11 +343,18 @@ squant_compress_kernel(const CompressArgs a) {
       squant_element<K>(p[i][q], s, inv, rq[q], level_value, &code, &en[q]);
       if (q < nvalid) chunk_bits |= (uint32_t)code << (q * BITS);
     }
-    // pack: a chunk is 4*BITS bits; 32 / (4*BITS) neighbouring lanes share a word
+    // pack: a chunk is 4*BITS bits; 32 / (4*BITS) neighbouring chunks share a word
     uint32_t wv = chunk_bits;
     int64_t widx;
     bool writer;
-    if constexpr (BITS == 8) {
+    if constexpr (LC) {
+      // this lane's chunks c - CPW + 1 .. c complete a word
+      lc_word |= chunk_bits << (4 * BITS * (i % CPW));
+      wv = lc_word;
+      widx = (cg - (CPW - 1)) / CPW;
+      writer = (i + 1) % CPW == 0;
+      if (writer) lc_word = 0;
+    } else if constexpr (BITS == 8) {
       widx = cg;
       writer = true;
     } else if constexpr (BITS == 4) {
@@ -357,7 +371,8 @@ squant_compress_kernel(const CompressArgs a) {
     }
     // a code word holds 32 / BITS elements of one bucket (buckets start on
     // multiples of 32): write the words that start inside this bucket
-    if (writer && c < nchunk && widx < nwords && (!SEG || widx * (32 / BITS) < end)) words[widx] = wv;
+    const int c_first = LC ? c - (CPW - 1) : c;  // the word's first chunk
+    if (writer && c_first < nchunk && widx < nwords && (!SEG || widx * (32 / BITS) < end)) words[widx] = wv;
     if (nvalid > 0) store_chunk<KEEP_H, HOLD, CPT>(a, g, e, h, j, full, nvalid, en, sg, i);
   }
 }
