@@ -242,9 +242,6 @@ squant_compress_kernel(const CompressArgs a) {
   const int warp = threadIdx.x >> 5;
   const int slot = warp / WPB;  // bucket within the CTA
   const int wib = warp % WPB;   // warp within the bucket
-  const int64_t b = (int64_t)blockIdx.x * BPC + slot;
-  const bool valid = b < a.nb;
-  if (WPB == 1 && !valid) return;
   const int row = blockIdx.y;
   const int worker = a.worker0 + row;
   const float* g = a.g + (int64_t)row * a.g_stride;
@@ -252,9 +249,36 @@ squant_compress_kernel(const CompressArgs a) {
   float* h = KEEP_H ? a.h + (int64_t)worker * a.ld : nullptr;
   uint8_t* msg = a.msg + (int64_t)row * a.msg_stride;
 
+  // With one warp per bucket the grid is persistent: a warp takes buckets b,
+  // b + stride, ... (the level table above is built once per CTA, not once
+  // per four buckets) and, with layer segments, loads the next bucket's
+  // bounds from the table while it quantises this one, so the data loads of
+  // a bucket never wait for the table.  Otherwise one bucket per warp.
+  constexpr bool PERSIST = WPB == 1;
+  const int64_t bstride = (int64_t)gridDim.x * BPC;
+  int64_t b = (int64_t)blockIdx.x * BPC + slot;
+  int64_t next_base = 0, next_end = 0;
+  if (PERSIST && SEG && b < a.nb) {
+    next_base = a.bstart[b];
+    next_end = a.bstart[b + 1];
+  }
+  for (;; b += bstride) {
+  const bool valid = b < a.nb;
+  if (WPB == 1 && !valid) return;
+
   // flat buckets: [b n, b n + n) clipped to d; layer buckets (SEG): the table
-  const int64_t base = SEG ? (valid ? a.bstart[b] : 0) : b * a.bucket;
-  const int64_t end = SEG ? (valid ? a.bstart[b + 1] : 0) : a.d;  // elements at or past `end` are not this bucket's
+  int64_t base, end;  // elements at or past `end` are not this bucket's
+  if constexpr (PERSIST && SEG) {
+    base = next_base;
+    end = next_end;
+    if (b + bstride < a.nb) {
+      next_base = a.bstart[b + bstride];
+      next_end = a.bstart[b + bstride + 1];
+    }
+  } else {
+    base = SEG ? (valid ? a.bstart[b] : 0) : b * a.bucket;
+    end = SEG ? (valid ? a.bstart[b + 1] : 0) : a.d;
+  }
   const int64_t count = SEG ? end - base : (valid ? min64((int64_t)a.bucket, a.d - base) : 0);
   const bool full = (count == a.bucket);
   const int nchunk = a.bucket >> 2;
@@ -375,6 +399,8 @@ squant_compress_kernel(const CompressArgs a) {
     if (writer && c_first < nchunk && widx < nwords && (!SEG || widx * (32 / BITS) < end)) words[widx] = wv;
     if (nvalid > 0) store_chunk<KEEP_H, HOLD, CPT>(a, g, e, h, j, full, nvalid, en, sg, i);
   }
+  if constexpr (!PERSIST) break;
+  }
 }
 
 // ---------------------------------------------------------------------------
@@ -442,8 +468,22 @@ template <int CPT, int WPB, int BITS, bool L2>
 cudaError_t squant_dispatch_keep(const CompressArgs& a, bool keep_h, cudaStream_t stream) {
   constexpr int BPC = WPB < 4 ? 4 / WPB : 1;
   constexpr int THREADS = 32 * WPB * BPC;
-  const dim3 grid((unsigned)((a.nb + BPC - 1) / BPC), (unsigned)a.nworkers);
   const bool seg = a.bstart != nullptr;
+  int64_t gx = (a.nb + BPC - 1) / BPC;
+  if (WPB == 1) {
+    // persistent over buckets: about four waves of resident CTAs in all rows
+    static int sms[64] = {0};
+    int dev = 0;
+    if (cudaGetDevice(&dev) == cudaSuccess && dev >= 0 && dev < 64) {
+      if (sms[dev] == 0 && cudaDeviceGetAttribute(&sms[dev], cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+        sms[dev] = 0;
+      if (sms[dev] > 0) {
+        const int64_t cap = ((int64_t)sms[dev] * 4 * (2048 / THREADS) + a.nworkers - 1) / a.nworkers;
+        gx = gx < cap ? gx : (cap > 0 ? cap : 1);
+      }
+    }
+  }
+  const dim3 grid((unsigned)gx, (unsigned)a.nworkers);
   if (keep_h) {
     if (seg) squant_compress_kernel<CPT, WPB, BITS, true, L2, true><<<grid, THREADS, 0, stream>>>(a);
     else squant_compress_kernel<CPT, WPB, BITS, true, L2, false><<<grid, THREADS, 0, stream>>>(a);
