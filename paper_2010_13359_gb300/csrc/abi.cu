@@ -11,6 +11,8 @@
 #include <string>
 #include <vector>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include "internal.cuh"
 
 struct dqgan_handle {
@@ -42,6 +44,16 @@ struct dqgan_handle {
 };
 
 namespace {
+
+// A named NVTX range over one host call (worker compress, server update,
+// lookahead), so that profilers show the hot-path stages by name; without
+// a profiler attached the push and pop do nothing.
+struct NvtxRange {
+  explicit NvtxRange(const char* name) { nvtxRangePushA(name); }
+  ~NvtxRange() { nvtxRangePop(); }
+  NvtxRange(const NvtxRange&) = delete;
+  NvtxRange& operator=(const NvtxRange&) = delete;
+};
 
 thread_local std::string tl_err;
 
@@ -134,6 +146,7 @@ dq::CompressArgs compress_args(dqgan_handle* h, const float* g, int64_t g_stride
 }
 
 int run_compress(dqgan_handle* h, const dq::CompressArgs& a) {
+  NvtxRange range("dqgan worker compress");
   const bool keep = (h->cfg.flags & DQGAN_KEEP_LOOKAHEAD) != 0;
   cudaError_t st = cudaSuccess;
   switch (h->cfg.compressor) {
@@ -421,6 +434,7 @@ int dqgan_server_aggregate_update(dqgan_handle* h, const void* msgs_all, float* 
   if (!msgs_all || !params) return set_error(h, DQGAN_ERR_INVALID_ARG, "NULL message or parameter pointer");
   if (!aligned16(msgs_all) || !aligned16(params))
     return set_error(h, DQGAN_ERR_INVALID_ARG, "messages and parameters must be 16-byte aligned");
+  NvtxRange range("dqgan server aggregate update");
   dq::ServerArgs s{};
   s.msgs = reinterpret_cast<const uint8_t*>(msgs_all);
   s.msg_stride = h->lay.total;
@@ -489,6 +503,7 @@ int dqgan_worker_lookahead(dqgan_handle* h, int32_t i, const float* params, floa
   if (!params || !out_w_half) return set_error(h, DQGAN_ERR_INVALID_ARG, "NULL pointer");
   if (!aligned16(params) || !aligned16(out_w_half))
     return set_error(h, DQGAN_ERR_INVALID_ARG, "pointers must be 16-byte aligned");
+  NvtxRange range("dqgan worker lookahead");
   const cudaError_t st = dq::launch_lookahead(params, h->h + (int64_t)i * h->ld, out_w_half, h->cfg.d,
                                               h->stream, &h->launches);
   if (st != cudaSuccess) return cuda_fail(h, st, "lookahead launch");
