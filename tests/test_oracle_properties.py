@@ -15,6 +15,8 @@ input they check what the definitions fix, by an independent route:
 * b-bit stochastic quantiser (Hou et al., proof of Theorem 2): s_b = max
   |p_j| of the bucket. Q_j is 0 or has the sign of p_j, |Q_j| <= s_b, and
   |Q_j - p_j| <= s_b / K (one level step), up to rounding. e = fl(p - Q);
+* QSGD's variant (Eq. (qsgd)): s_b = ||p_b||_2 within the fp32 bound, the
+  same sign and one-step properties;
 * server (Algorithm 2): w_new = w - (1/M) sum_m Q_m, within the rounding of
   an M-term fp32 sum (float64 reference).
 
@@ -148,3 +150,33 @@ def test_server_subtracts_the_average(M, x, comp, seed):
     avg = qs.sum(axis=0) / M
     bound = (M + 1) * U * np.sum(np.abs(qs), axis=0) / M + U * np.abs(w0.astype(np.float64) - avg)
     assert np.all(np.abs(w.astype(np.float64) - (w0.astype(np.float64) - avg)) <= bound + 1e-45)
+
+
+@SETTINGS
+@given(x=vectors(), bits=st.sampled_from([2, 4, 8]), bucket=st.sampled_from([32, 64]),
+       seed=st.integers(min_value=0, max_value=2**32 - 1))
+def test_qsgd_scale_is_the_l2_norm_and_levels_step_by_s_over_K(x, bits, bucket, seed):
+    """QSGD's variant (Section 2.4, Eq. (qsgd)): s_b = ||p_b||_2 within the
+    fp32 bound of an n-term sum of squares and one square root; Q_j is 0 or
+    has the sign of p_j, and |Q_j - p_j| <= s_b / K up to rounding."""
+    d = x.size
+    K = (1 << (bits - 1)) - 1
+    cfg = oracle.Config(d=d, M=1, compressor=oracle.QSGD, lr=1.0, bucket=bucket, bits=bits, seed=seed)
+    p, msg, e = run_worker(cfg, x)
+    q = oracle.decode(cfg, msg)
+    off_s = oracle.layout(cfg)[0]
+    nb = -(-d // bucket)
+    scales = msg[off_s:off_s + 4 * nb].view(np.float32)
+    for b in range(nb):
+        pb = p[b * bucket:(b + 1) * bucket].astype(np.float64)
+        qb = q[b * bucket:(b + 1) * bucket].astype(np.float64)
+        n = pb.size
+        l2 = float(np.sqrt(np.sum(pb * pb)))
+        s = float(scales[b])
+        if l2 < 1e-18:  # squares below the fp32 range flush the sum
+            continue
+        assert abs(s - l2) <= (n * U + 2 * U) * l2
+        assert np.all((qb == 0) | (np.sign(qb) == np.sign(pb)))
+        assert np.all(np.abs(qb) <= s * (1 + 2 * U))
+        assert np.all(np.abs(qb - pb) <= s / K * (1 + 4 * U) + 2 * U * s)
+    assert np.array_equal(e.view(np.uint32), (p - q).astype(np.float32).view(np.uint32))
