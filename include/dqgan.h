@@ -275,19 +275,26 @@ DQGAN_API uint64_t dqgan_launch_count(const dqgan_handle* h);
  * g:       device, d fp32, read only.
  * e:       device, d fp32, caller-owned residual, read and written.
  * out_msg: device, at least 8*k bytes, written.
- * All three 16-byte aligned.  1 <= d <= 1,048,576 (2^20); 1 <= k <= d.
+ * All three 16-byte aligned.  1 <= d <= DQGAN_NOALLOC_MAX_D (2^20); 1 <= k <= d.
  * cuda_stream: the cudaStream_t to enqueue on (NULL: legacy stream).
- * Scratch: a fixed 4.25 MiB array in this library's device memory, reserved
- * on every GPU that loads the library until the process exits.  Nothing is
- * allocated or freed.  The first call on a device looks up the array's
- * device address (cudaGetSymbolAddress); make that first call before any
- * stream capture.  Every call clears the part of the array it uses, and all
- * calls share the array: calls whose work overlaps on the GPU (other
+ * Scratch: a fixed array of DQGAN_NOALLOC_SCRATCH_BYTES (8.75 MiB) in this
+ * library's device memory, reserved on every GPU that loads the library
+ * until the process exits.  Nothing is allocated or freed.  The first call
+ * on a device looks up the array's device address (cudaGetSymbolAddress) and
+ * keeps it for the life of the process: make that first call before any
+ * stream capture, and do not reset the device while the library is loaded.
+ * The kernels rewrite the array's counts, prefixes and candidates in full on
+ * every call, so nothing needs clearing; the one word that carries over from
+ * call to call is the previous call's candidate threshold, which only
+ * decides how much work the first pass saves and never changes a result.
+ * All calls share the array: calls whose work overlaps on the GPU (other
  * streams, other host threads) race and give wrong results.
  * Returns DQGAN_OK, DQGAN_ERR_INVALID_ARG (sizes beyond the limit, NULL or
  * misaligned pointers) or DQGAN_ERR_CUDA; the reason is in
  * dqgan_last_error(NULL).
  */
+#define DQGAN_NOALLOC_MAX_D (1 << 20)
+#define DQGAN_NOALLOC_SCRATCH_BYTES (35 << 18)
 DQGAN_API int dqgan_topk_compress_noalloc(const float* g, float* e, void* out_msg, int64_t d, int64_t k,
                                           float lr, void* cuda_stream);
 

@@ -112,13 +112,13 @@ cudaError_t launch_squant_compress(const CompressArgs& a, bool keep_h, bool l2_s
 cudaError_t launch_identity_compress(const CompressArgs& a, bool keep_h, cudaStream_t stream,
                                      uint64_t* launches);
 
-// Scratch of the top-k path: one row per worker (kept across calls: the
-// candidate threshold carried from call to call lives there) and the
-// server's record-range table for `nworkers` messages.
+// Scratch of the top-k path: one row per worker and the server's
+// record-range table for `nworkers` messages.  A row needs no clearing
+// between calls: every call rewrites its tile counts, tile prefixes and
+// candidates in full.  Only the row's last state word carries over -- the
+// candidate threshold of the worker's previous call (0 before the first),
+// which decides how much work the first pass saves and never a result.
 size_t topk_scratch_bytes(int64_t d, int32_t nworkers);
-// Leading bytes of a row that must be zero before a first call; the rest of
-// the row needs no clearing.
-size_t topk_scratch_clear_bytes(int64_t d);
 cudaError_t launch_topk_compress(const CompressArgs& a, int64_t k, bool keep_h, void* scratch,
                                  cudaStream_t stream, uint64_t* launches);
 

@@ -11,7 +11,9 @@
 // The array below is reserved on every GPU that loads the library and stays
 // reserved until the process exits.  In host code its name is only a
 // host-side stand-in, not a device address: the device address is looked up
-// with cudaGetSymbolAddress once per device, with that device current.
+// with cudaGetSymbolAddress once per device, with that device current, and
+// kept for the life of the process (so a device reset, which reloads the
+// module, is not supported while this library is loaded).
 #include <cmath>
 #include <cstdio>
 #include <mutex>
@@ -22,9 +24,10 @@ namespace dq {
 namespace {
 
 // Largest d the fixed scratch supports, and the scratch itself (8.75 MiB;
-// one worker's top-k scratch at that d needs just under 8.02 MiB).
-constexpr int64_t kNoAllocMaxD = 1 << 20;
-constexpr size_t kNoAllocScratchBytes = (size_t)35 << 18;
+// one worker's top-k scratch at that d needs just under 8.02 MiB).  Both
+// numbers are the ones dqgan.h states.
+constexpr int64_t kNoAllocMaxD = DQGAN_NOALLOC_MAX_D;
+constexpr size_t kNoAllocScratchBytes = (size_t)DQGAN_NOALLOC_SCRATCH_BYTES;
 constexpr int kMaxDevices = 64;
 
 static __device__ __align__(256) unsigned char noalloc_scratch[kNoAllocScratchBytes];
@@ -82,15 +85,11 @@ extern "C" int dqgan_topk_compress_noalloc(const float* g, float* e, void* out_m
   }
 
   cudaStream_t stream = reinterpret_cast<cudaStream_t>(cuda_stream);
-  // the histogram and counters of the top-k stages must start at zero (the
-  // kernels return them to zero; clearing makes each call independent of how
-  // an earlier one ended).  The candidate threshold carried from the previous
-  // call stays: it only decides how much work the first pass does.
-  st = cudaMemsetAsync(scratch, 0, dq::topk_scratch_clear_bytes(d), stream);
-  if (st != cudaSuccess) {
-    snprintf(why, sizeof why, "clearing the scratch: %s", cudaGetErrorString(st));
-    return dq::set_thread_error(DQGAN_ERR_CUDA, why);
-  }
+  // No clearing: the top-k kernels rewrite the tile counts, tile prefixes and
+  // candidates of the row in full on every call.  The one word that carries
+  // over is the candidate threshold of the previous call (zero in the array
+  // as loaded, i.e. none); it decides how much work the first pass saves and
+  // never changes a result, whatever d and k the previous call had.
   dq::CompressArgs a{};
   a.g = g;
   a.g_stride = 0;

@@ -36,6 +36,8 @@
 // then one warp per tile sums the tile's records in shared memory, worker by
 // worker, and updates the touched parameters (one thread per record, with
 // searches narrowed to the tile, above 64 workers).
+#include <atomic>
+
 #include <cooperative_groups.h>
 
 #include "device_common.cuh"
@@ -1064,36 +1066,44 @@ size_t topk_scratch_bytes(int64_t d, int32_t nworkers) {
   return (size_t)(row_words(d) * nworkers + server_words) * 4u;
 }
 
-size_t topk_scratch_clear_bytes(int64_t d) {
-  (void)d;
-  return (size_t)ST_TAU * 4u;
-}
-
 // Raises a kernel's dynamic shared memory limit when its static plus dynamic
-// shared memory exceeds the default 48 KB (the value only grows; the
-// attribute is per function, for every device).
+// shared memory exceeds the default 48 KB.  The attribute belongs to the
+// function on the current device, so what has been set is remembered per
+// device ordinal (`done` has kSmemDevices slots; the value only grows).
+// Several host threads may race to set it; setting it twice is harmless.
+constexpr int kSmemDevices = 64;
+
 template <typename K>
-cudaError_t ensure_smem(K kernel, size_t bytes, size_t static_bytes, size_t* done) {
-  if (bytes + static_bytes <= 48u * 1024u || bytes <= *done) return cudaSuccess;
-  const cudaError_t st = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
-  if (st == cudaSuccess) *done = bytes;
+cudaError_t ensure_smem(K kernel, size_t bytes, size_t static_bytes, std::atomic<size_t> (&done)[kSmemDevices]) {
+  if (bytes + static_bytes <= 48u * 1024u) return cudaSuccess;
+  int dev = 0;
+  cudaError_t st = cudaGetDevice(&dev);
+  if (st != cudaSuccess) return st;
+  const bool cached = dev >= 0 && dev < kSmemDevices;
+  if (cached && done[dev].load(std::memory_order_acquire) >= bytes) return cudaSuccess;
+  st = cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)bytes);
+  if (st == cudaSuccess && cached) {
+    size_t cur = done[dev].load(std::memory_order_relaxed);
+    while (cur < bytes && !done[dev].compare_exchange_weak(cur, bytes, std::memory_order_release)) {
+    }
+  }
   return st;
 }
 
 cudaError_t launch_topk_compress(const CompressArgs& a, int64_t k, bool keep_h, void* scratch,
                                  cudaStream_t stream, uint64_t* launches) {
-  static size_t smem_done[2] = {0, 0};
+  static std::atomic<size_t> smem_done[2][kSmemDevices];
   const unsigned rows = (unsigned)a.nworkers;
   const dim3 tiles((unsigned)tiles_of(a.d), rows);
   const dim3 clusters(kCluster, rows);
   const size_t smem = sizeof(SelectSmem);
   cudaError_t st;
   if (keep_h) {
-    if ((st = ensure_smem(topk_select_kernel<true>, smem, 0, &smem_done[1])) != cudaSuccess) return st;
+    if ((st = ensure_smem(topk_select_kernel<true>, smem, 0, smem_done[1])) != cudaSuccess) return st;
     topk_form_kernel<true><<<tiles, kFormThreads, 0, stream>>>(a, scratch);
     topk_select_kernel<true><<<clusters, kSelThreads, smem, stream>>>(a, k, scratch);
   } else {
-    if ((st = ensure_smem(topk_select_kernel<false>, smem, 0, &smem_done[0])) != cudaSuccess) return st;
+    if ((st = ensure_smem(topk_select_kernel<false>, smem, 0, smem_done[0])) != cudaSuccess) return st;
     topk_form_kernel<false><<<tiles, kFormThreads, 0, stream>>>(a, scratch);
     topk_select_kernel<false><<<clusters, kSelThreads, smem, stream>>>(a, k, scratch);
   }
@@ -1106,12 +1116,12 @@ cudaError_t launch_topk_server(const ServerArgs& s, void* scratch, cudaStream_t 
   const int64_t n = (int64_t)s.M * s.k;
   topk_server_starts_kernel<<<dim3((unsigned)((s.k + 255) / 256), (unsigned)s.M), 256, 0, stream>>>(s, starts);
   if (s.M <= kSrvWarpMaxM) {
-    static size_t smem_done[2] = {0, 0};
+    static std::atomic<size_t> smem_done[2][kSmemDevices];
     const size_t smem = sizeof(SrvWarpSmem) * kSrvWarps;
     const unsigned blocks = (unsigned)((srv_tiles(s.d) + kSrvWarps - 1) / kSrvWarps);
     cudaError_t st;
-    if (s.M_pow2) st = ensure_smem(topk_server_warp_kernel<true>, smem, 0, &smem_done[1]);
-    else st = ensure_smem(topk_server_warp_kernel<false>, smem, 0, &smem_done[0]);
+    if (s.M_pow2) st = ensure_smem(topk_server_warp_kernel<true>, smem, 0, smem_done[1]);
+    else st = ensure_smem(topk_server_warp_kernel<false>, smem, 0, smem_done[0]);
     if (st != cudaSuccess) return st;
     if (s.M_pow2) topk_server_warp_kernel<true><<<blocks, kSrvThreads, smem, stream>>>(s, starts);
     else topk_server_warp_kernel<false><<<blocks, kSrvThreads, smem, stream>>>(s, starts);

@@ -56,6 +56,38 @@ def test_noalloc_topk_matches_handle_path(P, d, k):
     h.destroy()
 
 
+def test_noalloc_exact_size_views_odd_d(P):
+    """g and e are views of exactly d floats at an odd d, with guard words
+    on both sides inside the same allocation: the scalar tail path must
+    neither read past d (NaN guards would reach the selection and change the
+    records against the oracle) nor write outside [0, d) of e."""
+    import oracle
+    dev = torch.device("cuda:0")
+    stream = torch.cuda.current_stream(dev)
+    d, k, lr, lead, tail = 300_007, 2_999, 0.01, 16, 61
+    guard = np.float32(np.nan)
+    g_buf = torch.full((lead + d + tail,), float(guard), dtype=torch.float32, device=dev)
+    e_buf = torch.full((lead + d + tail,), float(guard), dtype=torch.float32, device=dev)
+    g, e = g_buf[lead:lead + d], e_buf[lead:lead + d]
+    assert g.data_ptr() % 16 == 0 and e.data_ptr() % 16 == 0
+    e.zero_()
+    e_orc = np.zeros(d, np.float32)
+    cfg = oracle.Config(d=d, M=1, compressor=oracle.TOPK, lr=lr, k=k)
+    rng = np.random.default_rng(7)
+    msg = torch.zeros(8 * k, dtype=torch.uint8, device=dev)
+    for call in range(2):
+        g_host = (rng.standard_normal(d) * np.exp(rng.uniform(-3, 1, d))).astype(np.float32)
+        g.copy_(torch.from_numpy(g_host))
+        P.dqgan.topk_compress_noalloc(g, e, msg, d, k, lr, stream.cuda_stream)
+        torch.cuda.synchronize(dev)
+        want = oracle.worker_step(cfg, 0, call + 1, g_host, e_orc)
+        assert np.array_equal(msg.cpu().numpy(), want[:8 * k]), f"call {call}: records differ from the oracle"
+        assert np.array_equal(e.cpu().numpy().view(np.uint32), e_orc.view(np.uint32)), f"call {call}: residual"
+        for name, buf in (("g", g_buf), ("e", e_buf)):
+            host = buf.cpu().numpy()
+            assert np.isnan(host[:lead]).all() and np.isnan(host[lead + d:]).all(), f"{name} guard words changed"
+
+
 def test_noalloc_rejects_sizes_beyond_the_limit(P):
     dev = torch.device("cuda:0")
     buf = torch.zeros(16, dtype=torch.float32, device=dev)
