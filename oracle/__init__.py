@@ -103,6 +103,8 @@ def lib() -> ctypes.CDLL:
         L.orc_decode.restype = None
         L.orc_worker_step.argtypes = [cfgp, ctypes.c_int32, ctypes.c_int64, f32p, f32p, f32p, u8p]
         L.orc_worker_step.restype = None
+        L.orc_pairwise_sum.argtypes = [f32p, ctypes.c_int32]
+        L.orc_pairwise_sum.restype = ctypes.c_float
         L.orc_server_step.argtypes = [cfgp, u8p, ctypes.c_int64, f32p]
         L.orc_server_step.restype = None
         L.orc_lookahead.argtypes = [ctypes.c_int64, f32p, f32p, f32p]
@@ -202,6 +204,18 @@ def worker_step(cfg: Config, worker: int, step: int, g: np.ndarray, e: np.ndarra
     hp = _f32(h) if h is not None else ctypes.POINTER(ctypes.c_float)()
     lib().orc_worker_step(ctypes.byref(cfg.c_struct()), worker, step, _f32(g), _f32(e), hp, _u8(msg))
     return msg
+
+
+def pairwise_sum(values) -> float:
+    """The server's fixed-order sum of M values (padded with +0 to a power of two, summed pairwise)."""
+    v = np.ascontiguousarray(values, dtype=np.float32)
+    M = v.size
+    P = 1
+    while P < M:
+        P *= 2
+    buf = np.zeros(P, dtype=np.float32)
+    buf[:M] = v
+    return float(lib().orc_pairwise_sum(_f32(buf), M))
 
 
 def server_step(cfg: Config, msgs: np.ndarray, w: np.ndarray) -> None:

@@ -305,63 +305,100 @@ void orc_topk_select(const float* p, int64_t d, int64_t k, uint8_t* selected) {
 }
 
 /* ------------------------------------------------------------------------ */
-/* Dense decode of one message: q = Q(p) as the server sees it.             */
+/* Decode of elements [j0, j1) of one message: q[j - j0] = Q(p)_j as the    */
+/* server sees it.  starts: the nb + 1 bucket starts (sign, quantisers).    */
 /* ------------------------------------------------------------------------ */
-void orc_decode(const orc_cfg* c, const uint8_t* msg, float* q) {
+static void decode_range(const orc_cfg* c, const uint8_t* msg, const int64_t* starts, int64_t nb,
+                         int64_t j0, int64_t j1, float* q) {
   int64_t off_s, off_p;
   orc_layout(c, &off_s, &off_p);
-  int64_t d = c->d;
   switch (c->compressor) {
-    case ORC_SIGN: {
-      const float* scales = (const float*)(msg + off_s);
-      const uint32_t* words = (const uint32_t*)(msg + off_p);
-      int64_t nb = orc_bucket_count(c);
-      int64_t* starts = (int64_t*)malloc((size_t)(nb + 1) * 8);
-      orc_bucket_starts(c, starts);
-      for (int64_t b = 0; b < nb; ++b) {
-        float s = scales[b];
-        for (int64_t j = starts[b]; j < starts[b + 1]; ++j) {
-          int neg = (words[j >> 5] >> (j & 31)) & 1u;
-          q[j] = neg ? -s : s;
-        }
-      }
-      free(starts);
-      break;
-    }
+    case ORC_SIGN:
     case ORC_SQUANT:
     case ORC_QSGD: {
       const float* scales = (const float*)(msg + off_s);
       const uint32_t* words = (const uint32_t*)(msg + off_p);
       int32_t K = (1 << (c->bits - 1)) - 1;
       uint32_t mask = (1u << c->bits) - 1u;
-      int64_t nb = orc_bucket_count(c);
-      int64_t* starts = (int64_t*)malloc((size_t)(nb + 1) * 8);
-      orc_bucket_starts(c, starts);
-      for (int64_t b = 0; b < nb; ++b) {
-        for (int64_t j = starts[b]; j < starts[b + 1]; ++j) {
+      /* the bucket holding j0: the last b with starts[b] <= j0 */
+      int64_t lo = 0, hi = nb;
+      while (hi - lo > 1) {
+        int64_t mid = (lo + hi) / 2;
+        if (starts[mid] <= j0) lo = mid;
+        else hi = mid;
+      }
+      int64_t b = lo;
+      for (int64_t j = j0; j < j1; ++j) {
+        while (starts[b + 1] <= j) ++b;
+        if (c->compressor == ORC_SIGN) {
+          int neg = (words[j >> 5] >> (j & 31)) & 1u;
+          q[j - j0] = neg ? -scales[b] : scales[b];
+        } else {
           int64_t bitpos = j * c->bits;
           int32_t code = (int32_t)((words[bitpos >> 5] >> (bitpos & 31)) & mask);
-          q[j] = orc_squant_decode(code, scales[b], K);
+          q[j - j0] = orc_squant_decode(code, scales[b], K);
         }
       }
-      free(starts);
       break;
     }
     case ORC_TOPK: {
-      for (int64_t j = 0; j < d; ++j) q[j] = 0.0f;
-      for (int64_t r = 0; r < c->k; ++r) {
+      for (int64_t j = j0; j < j1; ++j) q[j - j0] = 0.0f;
+      /* records ascend by index: the first one at or after j0 */
+      int64_t lo = 0, hi = c->k;
+      while (lo < hi) {
+        int64_t mid = (lo + hi) / 2;
+        uint32_t idx;
+        memcpy(&idx, msg + 8 * mid, 4);
+        if ((int64_t)idx < j0) lo = mid + 1;
+        else hi = mid;
+      }
+      for (int64_t r = lo; r < c->k; ++r) {
         uint32_t idx;
         float val;
         memcpy(&idx, msg + 8 * r, 4);
+        if ((int64_t)idx >= j1) break;
         memcpy(&val, msg + 8 * r + 4, 4);
-        q[idx] = val;
+        q[idx - j0] = val;
       }
       break;
     }
     case ORC_IDENTITY:
-      memcpy(q, msg, (size_t)d * 4);
+      memcpy(q, msg + 4 * j0, (size_t)(j1 - j0) * 4);
       break;
   }
+}
+
+static int64_t* bucket_starts_alloc(const orc_cfg* c, int64_t* nb_out) {
+  int64_t nb = (c->compressor == ORC_TOPK || c->compressor == ORC_IDENTITY) ? 0 : orc_bucket_count(c);
+  int64_t* starts = (int64_t*)malloc((size_t)(nb + 1) * 8);
+  if (nb > 0) orc_bucket_starts(c, starts);
+  else starts[0] = c->d;
+  *nb_out = nb;
+  return starts;
+}
+
+/* Dense decode of one message: q = Q(p) as the server sees it. */
+void orc_decode(const orc_cfg* c, const uint8_t* msg, float* q) {
+  int64_t nb;
+  int64_t* starts = bucket_starts_alloc(c, &nb);
+  decode_range(c, msg, starts, nb, 0, c->d, q);
+  free(starts);
+}
+
+/* ------------------------------------------------------------------------ */
+/* The sum over the M workers of Algorithm 2's server, in one fixed order   */
+/* (the paper leaves the order open; fixing it makes the parameters        */
+/* reproducible bit for bit): the M values, padded with +0 to the next     */
+/* power of two P >= M, are summed pairwise -- at every level x_i becomes  */
+/* x_2i + x_2i+1 -- until one value is left.  x: P floats, overwritten.    */
+/* ------------------------------------------------------------------------ */
+float orc_pairwise_sum(float* x, int32_t M) {
+  int32_t P = 1;
+  while (P < M) P *= 2;
+  for (int32_t i = M; i < P; ++i) x[i] = 0.0f;
+  for (int32_t width = 1; width < P; width *= 2)
+    for (int32_t i = 0; i < P; i += 2 * width) x[i] = x[i] + x[i + width];
+  return x[0];
 }
 
 /* ------------------------------------------------------------------------ */
@@ -466,25 +503,37 @@ void orc_worker_step(const orc_cfg* c, int32_t worker, int64_t step, const float
 }
 
 /* ------------------------------------------------------------------------ */
-/* Server step of Algorithm 2: q_hat = (1/M) sum_m p_hat^(m), summed in      */
-/* worker order starting from +0, then w = w - q_hat.                       */
+/* Server step of Algorithm 2: q_hat = (1/M) sum_m p_hat^(m), the sum taken */
+/* by orc_pairwise_sum, then w = w - q_hat.  Elements are handled a chunk   */
+/* at a time (every message's values of the chunk decoded first) only to   */
+/* bound the memory; each element's arithmetic is the one stated.          */
 /* msgs: M messages, message m at msgs + m * msg_stride.  w: d floats.      */
 /* ------------------------------------------------------------------------ */
+#define ORC_SERVER_CHUNK 4096
+
 void orc_server_step(const orc_cfg* c, const uint8_t* msgs, int64_t msg_stride, float* w) {
   int64_t d = c->d;
-  float* acc = (float*)malloc((size_t)(d > 0 ? d : 1) * 4);
-  float* q = (float*)malloc((size_t)(d > 0 ? d : 1) * 4);
-  for (int64_t j = 0; j < d; ++j) acc[j] = 0.0f;
-  for (int32_t m = 0; m < c->M; ++m) {
-    orc_decode(c, msgs + (int64_t)m * msg_stride, q);
-    for (int64_t j = 0; j < d; ++j) acc[j] = acc[j] + q[j];
+  int32_t M = c->M;
+  int32_t P = 1;
+  while (P < M) P *= 2;
+  int64_t nb;
+  int64_t* starts = bucket_starts_alloc(c, &nb);
+  float* q = (float*)malloc((size_t)M * ORC_SERVER_CHUNK * 4);
+  float* x = (float*)malloc((size_t)P * 4);
+  for (int64_t j0 = 0; j0 < d; j0 += ORC_SERVER_CHUNK) {
+    int64_t j1 = j0 + ORC_SERVER_CHUNK < d ? j0 + ORC_SERVER_CHUNK : d;
+    for (int32_t m = 0; m < M; ++m)
+      decode_range(c, msgs + (int64_t)m * msg_stride, starts, nb, j0, j1, q + (int64_t)m * ORC_SERVER_CHUNK);
+    for (int64_t j = j0; j < j1; ++j) {
+      for (int32_t m = 0; m < M; ++m) x[m] = q[(int64_t)m * ORC_SERVER_CHUNK + (j - j0)];
+      float sum = orc_pairwise_sum(x, M);
+      float q_hat = sum / (float)M;
+      w[j] = w[j] - q_hat;
+    }
   }
-  for (int64_t j = 0; j < d; ++j) {
-    float q_hat = acc[j] / (float)c->M;
-    w[j] = w[j] - q_hat;
-  }
-  free(acc);
+  free(x);
   free(q);
+  free(starts);
 }
 
 /* Lookahead of Algorithm 2: w_{t-1/2} = w_{t-1} - h, h = eta*F_prev + e_prev. */

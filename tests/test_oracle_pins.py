@@ -512,6 +512,77 @@ def test_identity_reduces_to_uncompressed_distributed_omd():
         assert err <= (t + 1) * 8 * Fraction(U32) * (scale + 1)
 
 
+# ---------------------------------------------------------------------------
+# The server's sum over workers.  Algorithm 2 averages the M decoded messages;
+# the paper leaves the order of the sum open, and the reading taken fixes it
+# to pairwise summation over the M values padded with +0 to a power of two.
+# Two facts of the mathematics pin that order: (1) pairwise summation's
+# forward error is at most ceil(log2 M) u sum|x| (Higham, Accuracy and
+# Stability of Numerical Algorithms, section 4.2), a bound that recursive
+# (worker-order) summation breaks on adversarial inputs; (2) where every
+# pairwise partial sum is exact, the average is the exact average.
+# ---------------------------------------------------------------------------
+U_HALF = 2.0 ** -24  # unit roundoff of binary32
+
+
+@pytest.mark.parametrize("M", [2, 3, 5, 8, 13, 16, 33, 64, 100])
+def test_server_sum_is_within_the_pairwise_error_bound(M):
+    r = rng(90 + M)
+    cases = [r.standard_normal(M), np.abs(r.standard_normal(M)) * 2.0 ** r.integers(-20, 20, M),
+             np.concatenate([[1.0], np.full(M - 1, U_HALF)])]
+    levels = int(np.ceil(np.log2(M)))
+    for x in cases:
+        x = np.asarray(x, np.float32)
+        exact_sum = sum((Fraction(float(v)) for v in x), Fraction(0))
+        got = Fraction(oracle.pairwise_sum(x))
+        bound = Fraction(levels) * Fraction(U_HALF) * sum(abs(Fraction(float(v))) for v in x)
+        assert abs(got - exact_sum) <= bound * (1 + Fraction(1, 10 ** 6)), (M, float(got), float(exact_sum))
+
+
+def test_worker_order_summation_would_break_the_bound():
+    """The adversarial input of the test above separates the orders: adding
+    63 halves of an ulp to 1 one at a time loses every one of them."""
+    x = np.concatenate([[1.0], np.full(63, U_HALF)]).astype(np.float32)
+    seq = np.float32(0.0)
+    for v in x:
+        seq = np.float32(seq + v)
+    exact_sum = Fraction(1) + 63 * Fraction(U_HALF)
+    bound = 6 * Fraction(U_HALF) * exact_sum
+    assert abs(Fraction(float(seq)) - exact_sum) > bound
+    assert abs(Fraction(oracle.pairwise_sum(x)) - exact_sum) <= bound
+
+
+@pytest.mark.parametrize("vals", [(1.0, 0.0, U_HALF, U_HALF), (1.0, 0.0, 0.0, 0.0) + (U_HALF,) * 4,
+                                  (0.0, 0.0, 1.0, 0.0, 2 * U_HALF, 0.0, 2 * U_HALF, 0.0)])
+def test_server_average_is_exact_when_pairwise_partial_sums_are(vals):
+    """Identity messages carrying these values per element: the exact
+    average sum/M is representable and every pairwise partial sum is exact,
+    so the server must subtract exactly sum/M (a worker-order sum would drop
+    the small terms against the 1)."""
+    M, d = len(vals), 8
+    cfg = oracle.Config(d=d, M=M, compressor=oracle.IDENTITY)
+    msgs = np.zeros((M, oracle.message_bytes(cfg)), np.uint8)
+    for m, v in enumerate(vals):
+        msgs[m, :4 * d] = np.full(d, v, np.float32).view(np.uint8)
+    w = np.zeros(d, np.float32)
+    oracle.server_step(cfg, msgs, w)
+    want = -(sum((Fraction(float(np.float32(v))) for v in vals), Fraction(0)) / M)
+    assert all(Fraction(float(x)) == want for x in w), (w[0], float(want))
+
+
+def test_pairwise_sum_pads_with_positive_zero():
+    """A power-of-two count is not padded (one -0 stays -0); any other count
+    adds +0 leaves, which turn a -0 partial sum into +0."""
+    assert math.copysign(1.0, oracle.pairwise_sum([-0.0])) < 0
+    assert math.copysign(1.0, oracle.pairwise_sum([-0.0, -0.0])) < 0
+    three = oracle.pairwise_sum([-0.0, -0.0, -0.0])
+    assert three == 0.0 and math.copysign(1.0, three) > 0
+    # the padding is exactly zero: the smallest subnormal survives it
+    tiny = 2.0 ** -149
+    assert oracle.pairwise_sum([tiny, 0.0, 0.0]) == tiny
+    assert oracle.pairwise_sum([-tiny] * 5) == -5 * tiny
+
+
 def bilinear_F(w):
     """F(x, y) = (y, -x): the operator of the bilinear game min_x max_y x.y."""
     half = len(w) // 2
