@@ -16,9 +16,10 @@ Default workload: the d = 1e8, M = 32, sign-per-4096 stress configuration
 independent replicas -- the simulated workers share nothing across GPUs --
 and reports the whole-job rate over the max-over-ranks time.
 
---impl reference times the CPU oracle (single thread, the code as the tests
-use it) on a bounded sample of the same workload and prints the same line
-with "impl": "reference".
+--impl reference times the CPU oracle (the code as the tests use it) over
+whole steps of the same workload on all host cores (worker steps and server
+element ranges in parallel threads) and prints the same line with
+"impl": "reference".
 """
 from __future__ import annotations
 
@@ -241,12 +242,92 @@ class ClockSampler:
 # CPU oracle timing (cpu_baseline leg and the reference arm)
 # ---------------------------------------------------------------------------
 
-def oracle_step_time(wl, worker_fraction: float = 1.0, server_fraction: float = 1 / 64):
+def host_threads() -> int:
+    try:
+        return len(os.sched_getaffinity(0))
+    except Exception:
+        return os.cpu_count() or 1
+
+
+def cpu_model() -> str:
+    """The host CPU's model name (lscpu, else /proc/cpuinfo, else the platform)."""
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.startswith("Model name:"):
+                return line.split(":", 1)[1].strip()
+    except Exception:
+        pass
+    try:
+        with open("/proc/cpuinfo") as f:
+            for line in f:
+                if line.lower().startswith("model name"):
+                    return line.split(":", 1)[1].strip()
+    except Exception:
+        pass
+    import platform
+    return platform.processor() or platform.machine()
+
+
+class OracleSteps:
+    """Whole steps of Algorithm 2 on the oracle, as the tests run it, spread
+    over `threads` host threads: the M worker steps in parallel, then the
+    server step in parallel element ranges (the oracle is a C library called
+    through ctypes, which releases the GIL).  The gradients are one seeded
+    batch generated up front (outside any timing) and used at every step."""
+
+    def __init__(self, wl, threads: int):
+        from concurrent.futures import ThreadPoolExecutor
+
+        import numpy as np
+
+        import oracle
+
+        self.np, self.oracle = np, oracle
+        self.wl, self.threads = wl, threads
+        segs = wl.segment_offsets() if wl.layer_buckets else None
+        self.cfg = oracle.Config(d=wl.d, M=wl.M, compressor=wl.compressor, lr=wl.lr, bucket=wl.bucket,
+                                 k=wl.k, bits=wl.bits, seed=wl.seed, segments=segs)
+        self.pool = ThreadPoolExecutor(threads)
+        self.E = np.zeros((wl.M, wl.d), np.float32)
+        self.G = np.empty((wl.M, wl.d), np.float32)
+
+        def gen(i):
+            self.G[i] = wl.gradient_np(1, i)
+
+        list(self.pool.map(gen, range(wl.M)))
+        self.w = wl.w0_np()
+        self.msgs = np.zeros((wl.M, oracle.message_bytes(self.cfg)), np.uint8)
+        parts = 4 * threads
+        cuts = sorted({wl.d * i // parts for i in range(parts + 1)})
+        self.ranges = [(x, y) for x, y in zip(cuts[:-1], cuts[1:]) if y > x]
+        self.t = 1
+
+    def step(self) -> float:
+        """One whole step; returns its wall time in seconds."""
+        cfg, oracle, t = self.cfg, self.oracle, self.t
+
+        def worker(i):
+            self.msgs[i] = oracle.worker_step(cfg, i, t, self.G[i], self.E[i])
+
+        t0 = time.perf_counter()
+        list(self.pool.map(worker, range(self.wl.M)))
+        list(self.pool.map(lambda r: oracle.server_step_range(cfg, self.msgs, self.w, r[0], r[1]), self.ranges))
+        dt = time.perf_counter() - t0
+        self.t += 1
+        return dt
+
+    def close(self):
+        self.pool.shutdown()
+        self.E = self.G = self.msgs = None
+
+
+def oracle_single_thread_estimate(wl, worker_fraction: float = 1 / 8, server_fraction: float = 1 / 64):
     """Single-thread oracle time for one full step of `wl`, estimated from a
     bounded sample: one worker step on a bucket-aligned prefix of the vector
     (`worker_fraction` of d; every worker's step costs the same per
-    parameter) and the server step on a bucket-aligned prefix
-    (`server_fraction` of d), both scaled to all M workers and all of d."""
+    parameter) and the server step on a prefix (`server_fraction` of d),
+    both scaled to all M workers and all of d."""
     import numpy as np
 
     import oracle
@@ -278,30 +359,53 @@ def oracle_step_time(wl, worker_fraction: float = 1.0, server_fraction: float = 
     oracle.server_step(sub, msgs, w)
     t_server = (time.perf_counter() - t0) * (wl.d / sd)
     step = wl.M * t_worker + t_server
-    sample = (f"one worker step on {wd} of d = {wl.d} parameters ({t_worker:.2f} s scaled to d, "
-              f"x M = {wl.M}) + the server step on {sd} parameters ({t_server:.2f} s scaled to d); "
-              f"one host thread")
+    sample = (f"projection, not a whole step: one worker step on {wd} of d = {wl.d} parameters "
+              f"({t_worker:.2f} s scaled to d, x M = {wl.M}) + the server step on {sd} parameters "
+              f"({t_server:.2f} s scaled to d); one host thread")
     return step, sample
 
 
+def cpu_baseline_leg(wl):
+    """The GPU arm's cpu_baseline: one whole step of the workload on all host
+    cores (timed after one untimed step), and the one-thread projection."""
+    threads = host_threads()
+    run = OracleSteps(wl, threads)
+    run.step()
+    dt = run.step()
+    run.close()
+    st1, sample1 = oracle_single_thread_estimate(wl)
+    units = wl.d * wl.M
+    return {"value": units / dt, "unit": UNIT, "cores": threads, "cpu_model": cpu_model(), "kind": "oracle",
+            "sample": (f"one whole step of this workload (all M = {wl.M} worker steps and the server "
+                       f"over all d = {wl.d}), timed after one untimed step, on {threads} host threads "
+                       f"(worker steps and server element ranges in parallel): {dt:.2f} s"),
+            "single_thread": {"value": units / st1, "unit": UNIT, "cores": 1, "sample": sample1}}
+
+
 def run_reference(args, rank, world):
+    """The oracle on the host cores, whole steps: W untimed, then K timed."""
     if rank != 0:
         return 0
     wl = selected_workload(args)
-    step_times = []
-    sample = ""
-    for i in range(args.warmup + args.steps):
-        st, sample = oracle_step_time(wl, worker_fraction=1 / 8, server_fraction=1 / 64)
-        if i >= args.warmup:
-            step_times.append(st)
-    total = sum(step_times)
-    value = wl.d * wl.M * len(step_times) / total
+    threads = host_threads()
+    run = OracleSteps(wl, threads)
+    for _ in range(args.warmup):
+        run.step()
+    step_s = [run.step() for _ in range(args.steps)]
+    run.close()
+    total = sum(step_s)
+    value = wl.d * wl.M * len(step_s) / total
+    sample = (f"whole steps of this workload: {args.warmup} untimed, then {args.steps} timed, each all "
+              f"M = {wl.M} worker steps and the server over all d = {wl.d}, on {threads} host threads "
+              f"(worker steps and server element ranges in parallel); gradients: one seeded batch "
+              f"generated before timing, used at every step")
     line = {
         "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": args.gpus,
-        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * total / len(step_times),
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * total / len(step_s),
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
         "data": "synthetic", "config": workload_config(wl, args),
-        "cpu_baseline": {"value": value, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample},
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": threads, "cpu_model": cpu_model(),
+                         "kind": "oracle", "sample": sample},
         "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
     }
     print(json.dumps(line), flush=True)
@@ -533,8 +637,7 @@ def run_gpu(args, rank, world, local):
                        "algorithmic_bytes": sb, "ms": serv_avg, "timing": timing}
     cpu = None
     if world == 1 and not args.no_cpu_baseline:
-        st, sample = oracle_step_time(wl)
-        cpu = {"value": units / st, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": sample}
+        cpu = cpu_baseline_leg(wl)
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": total_ms / args.steps, "higher_is_better": True,

@@ -107,6 +107,8 @@ def lib() -> ctypes.CDLL:
         L.orc_pairwise_sum.restype = ctypes.c_float
         L.orc_server_step.argtypes = [cfgp, u8p, ctypes.c_int64, f32p]
         L.orc_server_step.restype = None
+        L.orc_server_step_range.argtypes = [cfgp, u8p, ctypes.c_int64, f32p, ctypes.c_int64, ctypes.c_int64]
+        L.orc_server_step_range.restype = None
         L.orc_lookahead.argtypes = [ctypes.c_int64, f32p, f32p, f32p]
         L.orc_lookahead.restype = None
         L.orc_bucket_count.argtypes = [cfgp]
@@ -223,6 +225,13 @@ def server_step(cfg: Config, msgs: np.ndarray, w: np.ndarray) -> None:
     msgs = np.ascontiguousarray(msgs, dtype=np.uint8)
     assert msgs.ndim == 2 and msgs.shape[0] == cfg.M
     lib().orc_server_step(ctypes.byref(cfg.c_struct()), _u8(msgs), msgs.shape[1], _f32(w))
+
+
+def server_step_range(cfg: Config, msgs: np.ndarray, w: np.ndarray, j0: int, j1: int) -> None:
+    """The server step on elements [j0, j1) of w only (disjoint ranges may run in parallel threads)."""
+    assert msgs.dtype == np.uint8 and msgs.flags.c_contiguous and msgs.ndim == 2 and msgs.shape[0] == cfg.M
+    assert 0 <= j0 <= j1 <= cfg.d and w.size == cfg.d
+    lib().orc_server_step_range(ctypes.byref(cfg.c_struct()), _u8(msgs), msgs.shape[1], _f32(w), j0, j1)
 
 
 def lookahead(w: np.ndarray, h: np.ndarray) -> np.ndarray:

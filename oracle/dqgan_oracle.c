@@ -511,8 +511,11 @@ void orc_worker_step(const orc_cfg* c, int32_t worker, int64_t step, const float
 /* ------------------------------------------------------------------------ */
 #define ORC_SERVER_CHUNK 4096
 
-void orc_server_step(const orc_cfg* c, const uint8_t* msgs, int64_t msg_stride, float* w) {
-  int64_t d = c->d;
+/* The server step restricted to elements [j0, j1): each element's update
+ * depends on that element alone, so disjoint ranges may run concurrently
+ * (the full step is the range [0, d)). */
+void orc_server_step_range(const orc_cfg* c, const uint8_t* msgs, int64_t msg_stride, float* w, int64_t j0,
+                           int64_t j1) {
   int32_t M = c->M;
   int32_t P = 1;
   while (P < M) P *= 2;
@@ -520,12 +523,12 @@ void orc_server_step(const orc_cfg* c, const uint8_t* msgs, int64_t msg_stride, 
   int64_t* starts = bucket_starts_alloc(c, &nb);
   float* q = (float*)malloc((size_t)M * ORC_SERVER_CHUNK * 4);
   float* x = (float*)malloc((size_t)P * 4);
-  for (int64_t j0 = 0; j0 < d; j0 += ORC_SERVER_CHUNK) {
-    int64_t j1 = j0 + ORC_SERVER_CHUNK < d ? j0 + ORC_SERVER_CHUNK : d;
+  for (int64_t c0 = j0; c0 < j1; c0 += ORC_SERVER_CHUNK) {
+    int64_t c1 = c0 + ORC_SERVER_CHUNK < j1 ? c0 + ORC_SERVER_CHUNK : j1;
     for (int32_t m = 0; m < M; ++m)
-      decode_range(c, msgs + (int64_t)m * msg_stride, starts, nb, j0, j1, q + (int64_t)m * ORC_SERVER_CHUNK);
-    for (int64_t j = j0; j < j1; ++j) {
-      for (int32_t m = 0; m < M; ++m) x[m] = q[(int64_t)m * ORC_SERVER_CHUNK + (j - j0)];
+      decode_range(c, msgs + (int64_t)m * msg_stride, starts, nb, c0, c1, q + (int64_t)m * ORC_SERVER_CHUNK);
+    for (int64_t j = c0; j < c1; ++j) {
+      for (int32_t m = 0; m < M; ++m) x[m] = q[(int64_t)m * ORC_SERVER_CHUNK + (j - c0)];
       float sum = orc_pairwise_sum(x, M);
       float q_hat = sum / (float)M;
       w[j] = w[j] - q_hat;
@@ -534,6 +537,10 @@ void orc_server_step(const orc_cfg* c, const uint8_t* msgs, int64_t msg_stride, 
   free(x);
   free(q);
   free(starts);
+}
+
+void orc_server_step(const orc_cfg* c, const uint8_t* msgs, int64_t msg_stride, float* w) {
+  orc_server_step_range(c, msgs, msg_stride, w, 0, c->d);
 }
 
 /* Lookahead of Algorithm 2: w_{t-1/2} = w_{t-1} - h, h = eta*F_prev + e_prev. */

@@ -96,6 +96,97 @@ __device__ __forceinline__ void squant_element(float p, float s, float inv, uint
 }
 
 // ---------------------------------------------------------------------------
+// The server's sum over workers (Algorithm 2, server part).  The order is
+// fixed so that the parameters are reproducible bit for bit: the M decoded
+// values of an element, padded with +0 to the next power of two P >= M, are
+// summed pairwise (x_i <- x_2i + x_2i+1 at every level).  Kernels reach that
+// tree from groups of consecutive workers whose size is a power of two: a
+// full group is a subtree, a partial last group is padded with +0 inside,
+// and the group values are combined by the same rule (padding whole groups
+// with +0).  Adding a +0 leaf is done as an addition, so that a -0 partial
+// sum becomes +0 exactly where the padded tree says.
+// ---------------------------------------------------------------------------
+__host__ __device__ constexpr int next_pow2(int n) {
+  int p = 1;
+  while (p < n) p *= 2;
+  return p;
+}
+
+// A full group of four consecutive workers: (a + b) + (c + d).
+__device__ __forceinline__ float tree4(float a, float b, float c, float d) {
+  return __fadd_rn(__fadd_rn(a, b), __fadd_rn(c, d));
+}
+
+// The value of a group of four (leaves past M given as +0): a subtree of
+// the padded tree when M > 4; for M <= 4 the group is the whole tree, over
+// P = next_pow2(M) leaves only.
+__device__ __forceinline__ float group4(float a, float b, float c, float d, int M) {
+  if (M > 2) return tree4(a, b, c, d);
+  return M == 2 ? __fadd_rn(a, b) : a;
+}
+
+// Pairwise sum of N values (N fixed at compile time), padded with +0 to
+// next_pow2(N).
+template <int N>
+__device__ __forceinline__ float pairwise_n(const float (&v)[N]) {
+  constexpr int P = next_pow2(N);
+  float x[P];
+#pragma unroll
+  for (int i = 0; i < P; ++i) x[i] = i < N ? v[i] : 0.f;
+#pragma unroll
+  for (int w = 1; w < P; w *= 2)
+#pragma unroll
+    for (int i = 0; i + w < P; i += 2 * w) x[i] = __fadd_rn(x[i], x[i + w]);
+  return x[0];
+}
+
+// The same sum for a count known only at run time, fed one value (or one
+// group value) at a time in order: a binary counter of complete blocks,
+// block L holding the sum of 2^L consecutive values.  LEVELS must exceed
+// log2 of the largest count.  result() pads with +0 to the next power of
+// two: a block whose right sibling is all padding is added to +0.
+template <int LEVELS>
+struct PairwiseAcc {
+  float lvl[LEVELS];
+  uint32_t n = 0;
+
+  __device__ __forceinline__ void push(float x) {
+    float c = x;
+    bool placed = false;
+#pragma unroll
+    for (int L = 0; L < LEVELS; ++L) {
+      if (!placed) {
+        if ((n >> L) & 1u) {
+          c = __fadd_rn(lvl[L], c);
+        } else {
+          lvl[L] = c;
+          placed = true;
+        }
+      }
+    }
+    ++n;
+  }
+
+  __device__ __forceinline__ float result() const {
+    float c = 0.f, whole = 0.f;
+    bool have = false;
+#pragma unroll
+    for (int L = 0; L < LEVELS; ++L) {
+      if (n == (1u << L)) whole = lvl[L];
+      if ((1u << L) < n) {  // the levels below the root of the padded tree
+        if ((n >> L) & 1u) {
+          c = __fadd_rn(lvl[L], have ? c : 0.f);
+          have = true;
+        } else if (have) {
+          c = __fadd_rn(c, 0.f);
+        }
+      }
+    }
+    return (n & (n - 1u)) == 0u ? whole : c;
+  }
+};
+
+// ---------------------------------------------------------------------------
 // mbarrier + 1-D TMA bulk copy (cp.async.bulk) primitives.  Every wait is
 // bounded: after kSpinLimit polls (each may sleep up to kSuspendNs) it sets
 // kErrTimeout in the launch's error word and returns false.

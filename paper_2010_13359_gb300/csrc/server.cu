@@ -2,11 +2,18 @@
 //   decode the M messages, q_hat = fl(sum_m Q_m / M), w = fl(w - q_hat).
 // and the worker lookahead w_{t-1/2} = fl(w - h).
 //
+// Every kernel takes the sum over workers in the one order the library fixes
+// (device_common.cuh): the M values padded with +0 to a power of two and
+// summed pairwise, reached through groups of consecutive workers (four for
+// the sign tables and the generic kernels, two for the b = 2 pair tables).
+// The parameters therefore come out the same bit for bit whichever kernel
+// runs.
+//
 // Stochastic quantiser, identity, and sign with buckets < 512: one thread per
-// 4-element chunk of w walks the M messages in worker order with 4 fp32
-// accumulators, fetching the message words of 8 (4) workers before using
-// them.  Sign with buckets >= 512: bit-transposed table decode (below).
-// w is read and written once.
+// 4-element chunk of w walks the M messages in groups of four workers,
+// fetching the message words of 8 workers before using them.  Sign with
+// buckets >= 512: bit-transposed table decode (below).  w is read and
+// written once.
 #include "device_common.cuh"
 
 namespace dq {
@@ -37,8 +44,10 @@ __device__ __forceinline__ void apply_chunk(const ServerArgs& s, int64_t j, cons
   }
 }
 
-// Scaled sign, any bucket: Q_m(p)_j = bit ? -s_m : s_m summed in worker
-// order, message words and scales fetched 8 workers at a time.
+// Scaled sign, any bucket: Q_m(p)_j = bit ? -s_m : s_m, message words and
+// scales fetched 8 workers at a time, summed as two groups of four.
+constexpr int kSumLevels = 11;  // group counts up to 1024 (M <= 4096)
+
 __global__ void __launch_bounds__(256) sign_server_kernel(const ServerArgs s) {
   const int64_t c = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   const int64_t j = 4 * c;
@@ -46,7 +55,7 @@ __global__ void __launch_bounds__(256) sign_server_kernel(const ServerArgs s) {
   const int64_t bkt = s.word_bucket ? (int64_t)s.word_bucket[j >> 5] : j / s.bucket;
   const int64_t word = j >> 5;
   const int shift = (int)(j & 31);
-  float acc[4] = {0.f, 0.f, 0.f, 0.f};
+  PairwiseAcc<kSumLevels> acc[4];
   for (int m0 = 0; m0 < s.M; m0 += 8) {
     float sc[8];
     uint32_t bits[8];
@@ -61,12 +70,25 @@ __global__ void __launch_bounds__(256) sign_server_kernel(const ServerArgs s) {
       }
     }
 #pragma unroll
-    for (int u = 0; u < 8; ++u)
-      if (m0 + u < s.M)
+    for (int h = 0; h < 2; ++h) {
+      if (m0 + 4 * h < s.M) {
 #pragma unroll
-        for (int q = 0; q < 4; ++q) acc[q] = __fadd_rn(acc[q], ((bits[u] >> q) & 1u) ? -sc[u] : sc[u]);
+        for (int q = 0; q < 4; ++q) {
+          float v[4];
+#pragma unroll
+          for (int u = 0; u < 4; ++u) {
+            const int x = 4 * h + u;
+            v[u] = (m0 + x < s.M) ? (((bits[x] >> q) & 1u) ? -sc[x] : sc[x]) : 0.f;  // +0 past M
+          }
+          acc[q].push(group4(v[0], v[1], v[2], v[3], s.M));
+        }
+      }
+    }
   }
-  apply_chunk(s, j, acc);
+  float sum[4];
+#pragma unroll
+  for (int q = 0; q < 4; ++q) sum[q] = acc[q].result();
+  apply_chunk(s, j, sum);
 }
 
 // 32x32 bit transpose across a warp: on entry lane m holds row m; on exit
@@ -102,30 +124,46 @@ __device__ __forceinline__ uint32_t warp_transpose32(uint32_t x, const Transpose
 // message words = 1024 elements), no shared memory and no block barriers.
 // Lane m loads worker m's words of the slice (32 contiguous bytes at a time)
 // and a warp transpose gives lane l the M sign bits of one element.  The sum
-// over workers comes from per-bucket tables of partial sums over groups of
-// five workers, T_g[v] = sum_{r<5} (bit r of v ? -s_{5g+r} : s_{5g+r}) (in
-// r order), held in registers: lane l keeps T_g[l], and a lookup is one
-// shuffle whose source lane is the 5-bit field (shuffles use the lane index
-// mod 32).  Up to 32 workers the group values are added pairwise,
-// ((T_0 + T_1) + (T_2 + T_3)) + ((T_4 + T_5) + T_6); beyond 32, slab after
-// slab and group after group.  Neither is worker order.
+// over workers comes from per-bucket tables of four-worker group values:
+// T_g[v] = the group's subtree (a + b) + (c + d) over the leaves
+// bit r of v ? -s_{4g+r} : s_{4g+r} (+0 past M), held in registers two
+// groups per register -- lane l of register a keeps T_{2a + l/16}[l mod 16]
+// -- so that a lookup is one shuffle whose source lane is the group's 4-bit
+// field, plus 16 for an odd group (shuffles take the lane index mod 32).
+// The NG = ceil(M/4) group values are then summed pairwise, padded with +0
+// groups to a power of two: the library's fixed order of the sum.
 constexpr int kSliceWords = 32;
 
-// T_g[lane] for the 7 groups of five workers of one 32-worker slab.
-__device__ __forceinline__ void build_group_tables(float my_scale, int in_slab, int lane, float (&T)[7]) {
+// T[a] of groups 2a (lanes 0..15) and 2a + 1 (lanes 16..31) for the
+// workers of one 32-worker slab: in_slab of them present, M in all.
+template <int NR>
+__device__ __forceinline__ void build_group_tables(float my_scale, int in_slab, int M, int lane, float (&T)[NR]) {
+  const int pat = lane & 15;
+  const int hi = lane >> 4;
 #pragma unroll
-  for (int grp = 0; grp < 7; ++grp) {
-    float t = 0.f;
+  for (int a = 0; a < NR; ++a) {
+    float leaf[4];
 #pragma unroll
-    for (int r = 0; r < 5; ++r) {
-      const int wk = 5 * grp + r;
-      if (wk < 32) {
-        const float sc = __shfl_sync(kFullMask, my_scale, wk);
-        if (wk < in_slab) t = __fadd_rn(t, ((lane >> r) & 1) ? -sc : sc);
-      }
+    for (int r = 0; r < 4; ++r) {
+      const int wk = 4 * (2 * a + hi) + r;  // <= 31
+      const float sc = __shfl_sync(kFullMask, my_scale, wk);
+      leaf[r] = wk < in_slab ? (((pat >> r) & 1) ? -sc : sc) : 0.f;
     }
-    T[grp] = t;
+    T[a] = group4(leaf[0], leaf[1], leaf[2], leaf[3], M);
   }
+}
+
+// The sum over the NG groups of one element's transposed sign mask x (bit
+// m: worker m negative): one lookup per group, then pairwise.
+template <int NG, int NR>
+__device__ __forceinline__ float group_sum(uint32_t x, const float (&T)[NR]) {
+  static_assert(NR == (NG + 1) / 2, "two groups per table register");
+  const uint32_t xe = x & 0x0F0F0F0Fu;                          // fields of groups 0, 2, 4, 6
+  const uint32_t xo = ((x >> 4) & 0x0F0F0F0Fu) | 0x10101010u;  // groups 1, 3, 5, 7, in lanes 16..31
+  float v[NG];
+#pragma unroll
+  for (int g = 0; g < NG; ++g) v[g] = __shfl_sync(kFullMask, T[g >> 1], (int)(((g & 1) ? xo : xe) >> (8 * (g >> 1))));
+  return pairwise_n<NG>(v);
 }
 
 // This lane's 8 message words starting at word w0 (zero past the message).
@@ -146,43 +184,15 @@ __device__ __forceinline__ void load_words8(const uint32_t* wp, int64_t w0, int6
   }
 }
 
-// Sum over the NG five-worker groups of one element's transposed sign mask x:
-// the lookups are added pairwise, ((v0 + v1) + (v2 + v3)) + ((v4 + v5) + v6).
-template <int NG>
-__device__ __forceinline__ float group_sum(uint32_t x, const float (&T)[7]) {
-  float v[NG];
-#pragma unroll
-  for (int grp = 0; grp < NG; ++grp) v[grp] = __shfl_sync(kFullMask, T[grp], (int)(x >> (5 * grp)));
-#pragma unroll
-  for (int width = 1; width < NG; width *= 2)
-#pragma unroll
-    for (int i = 0; i + width < NG; i += 2 * width) v[i] = __fadd_rn(v[i], v[i + width]);
-  return v[0];
-}
-
 // The table sums of 8 transposed words.
-template <int NG>
-__device__ __forceinline__ void sums8(const uint32_t (&wd)[8], const float (&T)[7], const TransposeLane& tl,
+template <int NG, int NR>
+__device__ __forceinline__ void sums8(const uint32_t (&wd)[8], const float (&T)[NR], const TransposeLane& tl,
                                       float (&out)[8]) {
 #pragma unroll
   for (int k = 0; k < 8; ++k) out[k] = group_sum<NG>(warp_transpose32(wd[k], tl), T);
 }
 
-template <int NG>
-__device__ __forceinline__ void accumulate8_dyn(const uint32_t (&wd)[8], const float (&T)[7], int ngroups,
-                                                const TransposeLane& tl, float* acc) {
-#pragma unroll
-  for (int k = 0; k < 8; ++k) {
-    const uint32_t x = warp_transpose32(wd[k], tl);
-    float a = acc[k];
-#pragma unroll
-    for (int grp = 0; grp < 7; ++grp)
-      if (grp < ngroups) a = __fadd_rn(a, __shfl_sync(kFullMask, T[grp], (int)(x >> (5 * grp))));
-    acc[k] = a;
-  }
-}
-
-// M <= 32 workers in NG = ceil(M / 5) groups; w updated after every 8 words.
+// M <= 32 workers in NG = ceil(M / 4) groups; w updated after every 8 words.
 // The next 8 words and parameters are fetched before the current ones are
 // decoded.
 template <int NG, bool POW2>
@@ -201,8 +211,8 @@ __global__ void __launch_bounds__(256) sign_server_shfl_kernel(const ServerArgs 
   const uint8_t* my_msg = s.msgs + (int64_t)lane * s.msg_stride;
   const bool active = lane < s.M;
   const float my_scale = active ? __ldg(reinterpret_cast<const float*>(my_msg) + b) : 0.f;
-  float T[7];
-  build_group_tables(my_scale, s.M, lane, T);
+  float T[(NG + 1) / 2];
+  build_group_tables(my_scale, s.M, s.M, lane, T);
   const uint32_t* wp = reinterpret_cast<const uint32_t*>(my_msg + s.off_payload) + wbase;
   float* wl = s.w + 32 * wbase + lane;
   const int64_t jmax = s.d - 32 * wbase - lane;  // wl[32 i] is a parameter iff 32 i < jmax
@@ -311,8 +321,8 @@ sign_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap t
     for (int k = 0; k < 8; ++k) wv[k] = (32 * k < jmax) ? __ldcs(wl + 32 * k) : 0.f;
     const float my_scale =
         active ? __ldg(reinterpret_cast<const float*>(s.msgs + (int64_t)lane * s.msg_stride) + b) : 0.f;
-    float T[7];
-    build_group_tables(my_scale, s.M, lane, T);
+    float T[(NG + 1) / 2];
+    build_group_tables(my_scale, s.M, s.M, lane, T);
     ok = mbar_wait_bounded(&bar[cur], (it >> 1) & 1u, s.err);
     ok = __all_sync(kFullMask, ok);
     if (!ok) break;
@@ -364,7 +374,7 @@ sign_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap t
 // viewed as rows of 32, 128-byte swizzle) into shared memory.  Lane l reads
 // column l, word l of each worker, and transposes the 32 x 32 bit block in
 // its own registers, so that it holds the M sign bits of each of the 32
-// elements of that word; the worker sum comes from the five-worker group
+// elements of that word; the worker sum comes from the four-worker group
 // tables looked up by shuffle (rebuilt only when the bucket changes).  The
 // lane updates its row of 32 parameters in shared memory and one TMA store
 // writes the box back.  Per warp two word and two parameter buffers: the
@@ -375,12 +385,11 @@ sign_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap t
 // and a slice shorter than 32 rows, or one that reaches the partial last
 // row, updates its parameters with plain loads and stores (a box store would
 // overlap the next slice).
-// Against sign_server_tma_kernel: no warp transpose, 7 shuffles per element
-// at M = 32 instead of 12.
+// Against sign_server_tma_kernel: no warp transpose, 8 shuffles per element
+// at M = 32 instead of 13.
 constexpr int kColWarps = 12;
 constexpr int kColBox = 4096;        // bytes of a parameter box, and of a word box of the flat form
 constexpr int kSegBoxWords = kSignSegBoxWords;
-constexpr bool kColPairArith = false;  // workers 30, 31 by arithmetic instead of a seventh table
 
 // Per-warp shared memory of the column kernel: two parameter boxes, then two
 // word boxes (every swizzled box 1024-byte aligned).
@@ -427,49 +436,6 @@ __device__ __forceinline__ void transpose32_regs(uint32_t (&a)[32]) {
   swap_stage<1>(a, 0x55555555u);
 }
 
-// T_g[lane] for the first NGT five-worker groups (as build_group_tables).
-template <int NGT>
-__device__ __forceinline__ void build_tables(float my_scale, int M, int lane, float (&T)[7]) {
-#pragma unroll
-  for (int grp = 0; grp < 7; ++grp) {
-    float t = 0.f;
-    if (grp < NGT) {
-#pragma unroll
-      for (int r = 0; r < 5; ++r) {
-        const int wk = 5 * grp + r;
-        if (wk < 32) {
-          const float sc = __shfl_sync(kFullMask, my_scale, wk);
-          if (wk < M) t = __fadd_rn(t, ((lane >> r) & 1) ? -sc : sc);
-        }
-      }
-    }
-    T[grp] = t;
-  }
-}
-
-// Sum over the workers of one element's sign mask x: NG groups (with
-// kColPairArith the seventh, workers 30 and 31, by arithmetic from their
-// scales s30, s31), added pairwise, ((v0 + v1) + (v2 + v3)) + ((v4 + v5) + v6).
-template <int NG>
-__device__ __forceinline__ float column_sum(uint32_t x, const float (&T)[7], float s30, float s31) {
-  float v[NG];
-#pragma unroll
-  for (int grp = 0; grp < NG; ++grp) {
-    if (kColPairArith && grp == 6) {
-      const float q30 = __uint_as_float(__float_as_uint(s30) ^ ((x << 1) & 0x80000000u));
-      const float q31 = __uint_as_float(__float_as_uint(s31) ^ (x & 0x80000000u));
-      v[grp] = __fadd_rn(q30, q31);
-    } else {
-      v[grp] = __shfl_sync(kFullMask, T[grp], (int)(x >> (5 * grp)));
-    }
-  }
-#pragma unroll
-  for (int width = 1; width < NG; width *= 2)
-#pragma unroll
-    for (int i = 0; i + width < NG; i += 2 * width) v[i] = __fadd_rn(v[i], v[i + width]);
-  return v[0];
-}
-
 // The slice table of the layer-segmented form.
 struct SegSlices {
   const uint32_t* slices;  // per slice {first word, bucket | (rows - 1) << 27}
@@ -481,8 +447,7 @@ __global__ void __launch_bounds__(32 * kColWarps, 1)
 sign_server_col_kernel(const ServerArgs s, const SegSlices seg, const __grid_constant__ CUtensorMap wmap,
                        const __grid_constant__ CUtensorMap pmap) {
   using L = ColLayout<SEG>;
-  constexpr int ROWS = 5 * NG < 32 ? 5 * NG : 32;  // message rows that can hold a worker
-  constexpr int NGT = (kColPairArith && NG == 7) ? 6 : NG;  // groups looked up in tables
+  constexpr int ROWS = 4 * NG < 32 ? 4 * NG : 32;  // message rows that can hold a worker
   extern __shared__ uint8_t smem_raw[];
   __shared__ uint64_t bars[kColWarps][4];  // word boxes 0 and 1, parameter boxes 0 and 1
   const int lane = threadIdx.x & 31;
@@ -557,8 +522,7 @@ sign_server_col_kernel(const ServerArgs s, const SegSlices seg, const __grid_con
     return lane < s.M ? __ldg(reinterpret_cast<const float*>(s.msgs + (int64_t)lane * s.msg_stride) + bkt) : 0.f;
   };
   float scale_next = lo < hi ? scale_of_bucket(c.bucket) : 0.f;
-  float T[7];
-  float s30 = 0.f, s31 = 0.f;
+  float T[(NG + 1) / 2];
   int64_t table_b = -1;
   uint32_t it = 0;
   bool ok = true;
@@ -576,9 +540,7 @@ sign_server_col_kernel(const ServerArgs s, const SegSlices seg, const __grid_con
     if (c.bucket != table_b) {  // warp-uniform
       table_b = c.bucket;
       const float my_scale = scale_cur;
-      build_tables<NGT>(my_scale, s.M, lane, T);
-      s30 = __shfl_sync(kFullMask, my_scale, 30);
-      s31 = __shfl_sync(kFullMask, my_scale, 31);
+      build_group_tables(my_scale, s.M, s.M, lane, T);
     }
     ok = mbar_wait_bounded(&wbar[cur], (it >> 1) & 1u, s.err);
     ok = __all_sync(kFullMask, ok);
@@ -624,7 +586,7 @@ sign_server_col_kernel(const ServerArgs s, const SegSlices seg, const __grid_con
       }
 #pragma unroll
       for (int r = 0; r < 4; ++r)
-        o[r] = __fsub_rn(o[r], average_t<POW2>(column_sum<NG>(x[4 * q + r], T, s30, s31), s));
+        o[r] = __fsub_rn(o[r], average_t<POW2>(group_sum<NG>(x[4 * q + r], T), s));
       if (direct) {
 #pragma unroll
         for (int r = 0; r < 4; ++r)
@@ -650,7 +612,13 @@ sign_server_col_kernel(const ServerArgs s, const SegSlices seg, const __grid_con
   }
 }
 
-// Any M: workers taken 32 at a time, groups added in order, w updated at the end.
+// M above 32: workers taken 32 at a time.  With M > 32 the padded tree has
+// at least 64 leaves, so each 32-worker slab (the last one padded with +0
+// groups) is a subtree: per 8-word chunk of the slice, every slab's sum of
+// the chunk's elements goes into a per-element pairwise accumulator over
+// slabs, and w is updated once all slabs are in.
+constexpr int kSlabLevels = 8;  // up to 128 slabs (M <= 4096)
+
 __global__ void __launch_bounds__(256) sign_server_slabs_kernel(const ServerArgs s) {
   const int lane = threadIdx.x & 31;
   const int64_t gw = (int64_t)blockIdx.x * 8 + (threadIdx.x >> 5);
@@ -663,37 +631,36 @@ __global__ void __launch_bounds__(256) sign_server_slabs_kernel(const ServerArgs
   const int64_t wbase = b * words_per_bucket + (gw % spb) * sw;
   const int64_t nwords = (s.d + 31) >> 5;
   const TransposeLane tl(lane);
-  float acc[kSliceWords];
+  const int nslabs = (s.M + 31) / 32;
+  for (int it = 0; it * 8 < sw; ++it) {
+    PairwiseAcc<kSlabLevels> acc[8];
+    for (int slab = 0; slab < nslabs; ++slab) {
+      const int in_slab = min(32, s.M - slab * 32);
+      const uint8_t* my_msg = s.msgs + (int64_t)(slab * 32 + lane) * s.msg_stride;
+      const float my_scale = (lane < in_slab) ? __ldg(reinterpret_cast<const float*>(my_msg) + b) : 0.f;
+      float T[4];
+      build_group_tables(my_scale, in_slab, s.M, lane, T);
+      const int64_t w0 = wbase + 8 * it;
+      uint32_t wd[8];
+      load_words8(reinterpret_cast<const uint32_t*>(my_msg + s.off_payload) + w0, w0, nwords, lane < in_slab, wd);
+      float v[8];
+      sums8<8>(wd, T, tl, v);
 #pragma unroll
-  for (int i = 0; i < kSliceWords; ++i) acc[i] = 0.f;
-  for (int slab = 0; slab * 32 < s.M; ++slab) {
-    const int in_slab = min(32, s.M - slab * 32);
-    const uint8_t* my_msg = s.msgs + (int64_t)(slab * 32 + lane) * s.msg_stride;
-    const float my_scale = (lane < in_slab) ? __ldg(reinterpret_cast<const float*>(my_msg) + b) : 0.f;
-    float T[7];
-    build_group_tables(my_scale, in_slab, lane, T);
-    const int ngroups = (in_slab + 4) / 5;
-    const uint32_t* wp = reinterpret_cast<const uint32_t*>(my_msg + s.off_payload) + wbase;
-#pragma unroll
-    for (int it = 0; it < kSliceWords / 8; ++it) {
-      if (it * 8 < sw) {
-        uint32_t wd[8];
-        load_words8(wp + 8 * it, wbase + 8 * it, nwords, lane < in_slab, wd);
-        accumulate8_dyn<7>(wd, T, ngroups, tl, acc + 8 * it);
-      }
+      for (int k = 0; k < 8; ++k) acc[k].push(v[k]);
     }
-  }
 #pragma unroll
-  for (int i = 0; i < kSliceWords; ++i) {
-    const int64_t j = 32 * (wbase + i) + lane;
-    if (i < sw && j < s.d) __stcs(s.w + j, __fsub_rn(__ldcs(s.w + j), average(acc[i], s)));
+    for (int k = 0; k < 8; ++k) {
+      const int64_t j = 32 * (wbase + 8 * it + k) + lane;
+      if (j < s.d) __stcs(s.w + j, __fsub_rn(__ldcs(s.w + j), average(acc[k].result(), s)));
+    }
   }
 }
 
 // b-bit stochastic quantiser: Q_m(p)_j = fl(s_m * V[code]) with
-// V[code] = sign(code - K) * fl(|code - K| / K) (so V[K] = +0), summed in
-// worker order.  One thread per 4-element chunk (a fixed grid strides over
-// the chunks), code words of 8 workers fetched before they are decoded.  For
+// V[code] = sign(code - K) * fl(|code - K| / K) (so V[K] = +0), summed as
+// groups of four workers in the library's pairwise order.  One thread per
+// 4-element chunk (a fixed grid strides over the chunks), code words of 8
+// workers fetched before they are decoded.  For
 // b = 4, 8 V lives in shared memory replicated once per bank (entry c of lane
 // l at [c][l]), so the random code lookups of a warp never conflict; for
 // b = 2 (V in {-1, 0, +1}) the value is a select.
@@ -727,7 +694,7 @@ __global__ void __launch_bounds__(256) squant_server_kernel(const ServerArgs s) 
     const int shift = (int)(bitpos & 31);
     const uint8_t* m_scale = s.msgs + 4 * bkt;
     const uint8_t* m_word = s.msgs + s.off_payload + 4 * word;
-    float acc[4] = {0.f, 0.f, 0.f, 0.f};
+    PairwiseAcc<kSumLevels> sum[4];
     for (int m0 = 0; m0 < s.M; m0 += 8) {
       uint32_t bits[8];
       float sc[8];
@@ -739,24 +706,32 @@ __global__ void __launch_bounds__(256) squant_server_kernel(const ServerArgs s) 
         sc[u] = ok ? __ldg(reinterpret_cast<const float*>(m_scale + off)) : 0.f;
       }
 #pragma unroll
-      for (int u = 0; u < 8; ++u) {
-        if (m0 + u < s.M) {
+      for (int h = 0; h < 2; ++h) {
+        if (m0 + 4 * h < s.M) {
 #pragma unroll
           for (int q = 0; q < 4; ++q) {
-            float v;
-            if constexpr (BITS == 2) {
-              const uint32_t code = (bits[u] >> (2 * q)) & 3u;
-              v = (code == 0) ? -sc[u] : (code == 2 ? sc[u] : 0.f);  // fl(s * 1) = s
-            } else if constexpr (BITS == 8) {
-              v = __fmul_rn(sc[u], Vl[__byte_perm(bits[u], 0, 0x4440 | q) << 5]);
-            } else {
-              v = __fmul_rn(sc[u], Vl[((bits[u] >> (q * BITS)) & MASK) << 5]);
+            float v[4];
+#pragma unroll
+            for (int x = 0; x < 4; ++x) {
+              const int u = 4 * h + x;
+              if constexpr (BITS == 2) {
+                const uint32_t code = (bits[u] >> (2 * q)) & 3u;
+                v[x] = (code == 0) ? -sc[u] : (code == 2 ? sc[u] : 0.f);  // fl(s * 1) = s
+              } else if constexpr (BITS == 8) {
+                v[x] = __fmul_rn(sc[u], Vl[__byte_perm(bits[u], 0, 0x4440 | q) << 5]);
+              } else {
+                v[x] = __fmul_rn(sc[u], Vl[((bits[u] >> (q * BITS)) & MASK) << 5]);
+              }
+              if (m0 + u >= s.M) v[x] = 0.f;  // padding leaves
             }
-            acc[q] = __fadd_rn(acc[q], v);
+            sum[q].push(group4(v[0], v[1], v[2], v[3], s.M));
           }
         }
       }
     }
+    float acc[4];
+#pragma unroll
+    for (int q = 0; q < 4; ++q) acc[q] = sum[q].result();
     if (j + 3 < s.d) {
       float4 wv = __ldcs(reinterpret_cast<const float4*>(s.w + j));
       wv.x = __fsub_rn(wv.x, average_t<POW2>(acc[0], s));
@@ -807,12 +782,14 @@ __device__ __forceinline__ void transpose16x2_regs(uint32_t (&a)[16]) {
 
 // b = 2 sums over workers by pair tables.  The decoded value of a 2-bit code
 // is v(0, s) = -s, v(1, s) = +0, v(2, s) = +s (code 3 never occurs; 0 here).
-// Pair p = workers (2p, 2p + 1): lane l holds
+// Pair p = workers (2p, 2p + 1), the lowest subtrees of the padded tree once
+// M >= 2: lane l holds
 //   T_p[l mod 16] = fl(v(l mod 4, s_2p) + v((l / 4) mod 4, s_2p+1)),
-// the pair's contribution for the 4-bit field code_2p | code_2p+1 << 2.  A
-// worker at or beyond M has scale 0 and adds only zeros.
+// the pair's value for the 4-bit field code_2p | code_2p+1 << 2.  A worker at
+// or beyond M has scale 0 and reads as code 1, so it adds a +0 leaf; with
+// M = 1 the tree is the single leaf and T_0 holds v(c, s_0) alone.
 template <int NP>
-__device__ __forceinline__ void build_pair_tables(float my_scale, int lane, float (&T)[NP]) {
+__device__ __forceinline__ void build_pair_tables(float my_scale, int lane, int M, float (&T)[NP]) {
   const int ca = lane & 3, cb = (lane >> 2) & 3;
   const float fa = ca == 0 ? -1.f : (ca == 2 ? 1.f : 0.f);  // v(c, s) = f(c) * s exactly
   const float fb = cb == 0 ? -1.f : (cb == 2 ? 1.f : 0.f);
@@ -820,7 +797,8 @@ __device__ __forceinline__ void build_pair_tables(float my_scale, int lane, floa
   for (int p = 0; p < NP; ++p) {
     const float sa = __shfl_sync(kFullMask, my_scale, 2 * p);
     const float sb = __shfl_sync(kFullMask, my_scale, 2 * p + 1);
-    T[p] = __fadd_rn(__fmul_rn(fa, sa), __fmul_rn(fb, sb));
+    const float va = __fmul_rn(fa, sa);
+    T[p] = M == 1 ? va : __fadd_rn(va, __fmul_rn(fb, sb));
   }
 }
 
@@ -829,11 +807,14 @@ __device__ __forceinline__ void build_pair_tables(float my_scale, int lane, floa
 // each worker (16 per set of workers) is transposed so that one register
 // holds one element's codes of 16 workers, whose 4-bit pair fields index the
 // pair tables by shuffle (the lane index is taken mod 32: the tables repeat
-// in lanes 16..31, so the bits above a field do not matter).  The eight pair
-// values of a set are added pairwise, the two sets' sums last.
+// in lanes 16..31, so the bits above a field do not matter).  The pair
+// values are summed pairwise over the padded tree's next_pow2(ceil(M/2))
+// pairs (one set: 1, 2, 4 or 8 of them, the level picked by M; two sets:
+// the two 8-pair sums added last).
 template <int NSET, bool POW2>
 __device__ __forceinline__ void b2_pair_table_update(const uint32_t* words, const ServerArgs& s,
                                                      const float (&T)[8 * NSET], float (&wv)[16]) {
+  const int np = next_pow2((s.M + 1) / 2);  // pairs in the padded tree (NSET = 2: 16)
   float acc[16];
 #pragma unroll
   for (int set = 0; set < NSET; ++set) {
@@ -849,8 +830,10 @@ __device__ __forceinline__ void b2_pair_table_update(const uint32_t* words, cons
       float v[8];
 #pragma unroll
       for (int p = 0; p < 8; ++p) v[p] = __shfl_sync(kFullMask, T[8 * set + p], (int)(z[e] >> (4 * p)));
-      const float sum = __fadd_rn(__fadd_rn(__fadd_rn(v[0], v[1]), __fadd_rn(v[2], v[3])),
-                                  __fadd_rn(__fadd_rn(v[4], v[5]), __fadd_rn(v[6], v[7])));
+      const float a01 = __fadd_rn(v[0], v[1]), a23 = __fadd_rn(v[2], v[3]);
+      const float a03 = __fadd_rn(a01, a23);
+      const float sum = np >= 8 ? __fadd_rn(a03, __fadd_rn(__fadd_rn(v[4], v[5]), __fadd_rn(v[6], v[7])))
+                                : (np == 4 ? a03 : (np == 2 ? a01 : v[0]));
       acc[e] = set == 0 ? sum : __fadd_rn(acc[e], sum);
       if (set + 1 == NSET) wv[e] = __fsub_rn(wv[e], average_t<POW2>(acc[e], s));
     }
@@ -865,17 +848,17 @@ constexpr bool sq_params_boxed(int bits) { return bits != 8; }
 // elements: the code words are staged by TMA like the sign words above (a
 // box is 32 words of every worker, M rows of 128 bytes, no swizzle: lane l
 // reads word l of row m, one conflict-free 128-byte row per worker).  Lane l
-// owns the 32/b consecutive elements of its word; per worker, in worker
-// order, it decodes them with the worker's scale (broadcast by shuffle from
-// the lane that loaded it) and V[code] (b = 8: the bank-replicated table;
-// b = 4: the worker's 15 products fl(s * V[c]), one per lane, looked up by
-// shuffle).  Worker-order sums from +0, so the result equals the oracle's
-// bit for bit.  b = 2 sums by pair tables instead (b2_pair_table_update, NSET
-// sets of 16 workers; tables rebuilt only when the bucket changes): not
-// worker order, so w agrees with the oracle up to the summation order.
+// owns the 32/b consecutive elements of its word; per worker it decodes them
+// with the worker's scale (broadcast by shuffle from the lane that loaded it)
+// and V[code] (b = 8: the bank-replicated table; b = 4: the worker's 15
+// products fl(s * V[c]), one per lane, looked up by shuffle), four workers
+// at a time into the group value (a + b) + (c + d), and the groups are
+// summed pairwise: the library's fixed order.  b = 2 sums by pair tables
+// instead (b2_pair_table_update, NSET sets of 16 workers; tables rebuilt only
+// when the bucket changes), which reach the same tree from pairs of workers.
 // With layer segments (SEG) a slice may hold words of several buckets: each
 // lane then reads the workers' scales of its own word's bucket (b = 2: two
-// bit tests per worker and element, level-0 codes skipped, worker order).
+// bit tests per worker and element, then the groups of four).
 // For b = 2 and 4 (a lane owns 64 or 32 contiguous bytes of w, which plain
 // loads would fetch at a 64- or 32-byte lane stride) the slice's parameters
 // come by TMA as well: w viewed as rows of 32 floats (pmap), a box of
@@ -1034,21 +1017,16 @@ squant_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap
     }
     const uint32_t* words = reinterpret_cast<const uint32_t*>(buf0 + cur * box_bytes) + lane;
     const float* V8l = V8 + lane;
-    float acc[EPL];
-#pragma unroll
-    for (int e = 0; e < EPL; ++e) acc[e] = 0.f;
-    // one worker's contribution, added in worker order
-    auto add_worker = [&](uint32_t word, float sc) {
+    // one worker's decoded values of this lane's EPL elements
+    auto decode_worker = [&](uint32_t word, float sc, float (&v)[EPL]) {
       if constexpr (BITS == 2) {
-        // code 0: -s, 1: +0, 2: +s (fl(s * 1) = s).  Adding +0 never changes
-        // the sum (it starts at +0 and so is never -0), so level-0 codes are
-        // skipped: per element one bit test picks the sign, one the add.
+        // code 0: -s, 1: +0, 2: +s (fl(s * 1) = s): one bit test picks +0,
+        // one the sign
         const float nsc = -sc;
 #pragma unroll
         for (int e = 0; e < EPL; ++e) {
           const bool zero = (word >> (2 * e)) & 1u;
-          const float v = ((word >> (2 * e + 1)) & 1u) ? sc : nsc;
-          acc[e] = zero ? acc[e] : __fadd_rn(acc[e], v);
+          v[e] = zero ? 0.f : (((word >> (2 * e + 1)) & 1u) ? sc : nsc);
         }
         return;
       }
@@ -1061,59 +1039,101 @@ squant_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap
       const float T4 = (BITS == 4) ? __fmul_rn(mixed ? 1.0f : sc, V4) : 0.f;
 #pragma unroll
       for (int e = 0; e < EPL; ++e) {
-        float v;
-        if constexpr (BITS == 2) {
-          v = 0.f;
-        } else if constexpr (BITS == 4) {
-          v = __shfl_sync(kFullMask, T4, (int)(word >> (4 * e)));
-          if (mixed) v = __fmul_rn(sc, v);
+        if constexpr (BITS == 4) {
+          v[e] = __shfl_sync(kFullMask, T4, (int)(word >> (4 * e)));
+          if (mixed) v[e] = __fmul_rn(sc, v[e]);
         } else {
-          v = __fmul_rn(sc, V8l[__byte_perm(word, 0u, 0x4440u | (uint32_t)e) * 32u]);
+          v[e] = __fmul_rn(sc, V8l[__byte_perm(word, 0u, 0x4440u | (uint32_t)e) * 32u]);
         }
-        acc[e] = __fadd_rn(acc[e], v);
       }
     };
-    int m = 0;
+    float acc[EPL] = {};
     if constexpr (BITS == 2) {
       if (!(SEG && mixed)) {
         if (bkt != t2_bkt) {
-          build_pair_tables<8 * NSET>(my_scale, lane, T2);
+          build_pair_tables<8 * NSET>(my_scale, lane, s.M, T2);
           t2_bkt = bkt;
         }
         b2_pair_table_update<NSET, POW2>(words, s, T2, wv);
-        m = s.M;
       }
     }
-    // per-worker decode: b = 4, 8, and b = 2 on slices that span layer segments
+    // per-worker decode (b = 4, 8, and b = 2 on slices that span layer
+    // segments): groups of four workers, G = (a + b) + (c + d) with +0 past
+    // M, combined as the padded tree over the next_pow2(ceil(M / 4)) <= 8
+    // groups: G0; G0 + G1; (G0 + G1) + (G2 + G3); then + ((G4 + G5) + (G6 + G7)),
+    // groups past M being +0 (M is warp-uniform, so are the branches)
     const bool per_worker = BITS != 2 || (SEG && mixed);
-    if (BITS != 2 || SEG) {
-      for (; m + 4 <= s.M; m += 4) {
-        const uint32_t w0 = words[32 * m], w1 = words[32 * (m + 1)];
-        const uint32_t w2 = words[32 * (m + 2)], w3 = words[32 * (m + 3)];
-        const float s0 = scale_of(m), s1 = scale_of(m + 1);
-        const float s2 = scale_of(m + 2), s3 = scale_of(m + 3);
-        add_worker(w0, s0);
-        add_worker(w1, s1);
-        add_worker(w2, s2);
-        add_worker(w3, s3);
-      }
-      if constexpr (BITS == 2) {
-        // the last M mod 4 workers as one more group of four: the missing
-        // workers read as all-level-0 words, which add nothing
-        if (m < s.M) {
-          uint32_t wq[4];
-          float sq[4];
+    if (per_worker) {
+      // group value of workers m .. m + 3 into g
+      auto group = [&](int m, float (&g)[EPL]) {
+        float va[EPL], vb[EPL];
+        decode_worker(words[32 * m], scale_of(m), va);
+        if (m + 1 < s.M) {
+          decode_worker(words[32 * (m + 1)], scale_of(m + 1), vb);
+        } else {
 #pragma unroll
-          for (int u = 0; u < 4; ++u) {
-            const bool ok = m + u < s.M;
-            wq[u] = ok ? words[32 * (m + u)] : 0x55555555u;
-            sq[u] = ok ? scale_of(m + u) : 0.f;
-          }
-#pragma unroll
-          for (int u = 0; u < 4; ++u) add_worker(wq[u], sq[u]);
+          for (int e = 0; e < EPL; ++e) vb[e] = 0.f;
         }
-      } else {
-        for (; m < s.M; ++m) add_worker(words[32 * m], scale_of(m));
+#pragma unroll
+        for (int e = 0; e < EPL; ++e) g[e] = s.M == 1 ? va[e] : __fadd_rn(va[e], vb[e]);
+        if (s.M <= 2) return;
+        if (m + 2 < s.M) {
+          decode_worker(words[32 * (m + 2)], scale_of(m + 2), va);
+        } else {
+#pragma unroll
+          for (int e = 0; e < EPL; ++e) va[e] = 0.f;
+        }
+        if (m + 3 < s.M) {
+          decode_worker(words[32 * (m + 3)], scale_of(m + 3), vb);
+        } else {
+#pragma unroll
+          for (int e = 0; e < EPL; ++e) vb[e] = 0.f;
+        }
+#pragma unroll
+        for (int e = 0; e < EPL; ++e) g[e] = __fadd_rn(g[e], __fadd_rn(va[e], vb[e]));
+      };
+      // x <- x + (value of groups i, i + 1), the second +0 past M
+      auto add_pair = [&](int i, float (&x)[EPL]) {
+        float t[EPL], g[EPL];
+        group(4 * i, t);
+        if (4 * (i + 1) < s.M) {
+          group(4 * (i + 1), g);
+        } else {
+#pragma unroll
+          for (int e = 0; e < EPL; ++e) g[e] = 0.f;
+        }
+#pragma unroll
+        for (int e = 0; e < EPL; ++e) x[e] = __fadd_rn(x[e], __fadd_rn(t[e], g[e]));
+      };
+      group(0, acc);
+      if (s.M > 4) {
+        float g[EPL];
+        group(4, g);
+#pragma unroll
+        for (int e = 0; e < EPL; ++e) acc[e] = __fadd_rn(acc[e], g[e]);
+        if (s.M > 8) {
+          add_pair(2, acc);
+          if (s.M > 16) {
+            float h[EPL];
+            group(16, h);
+            if (s.M > 20) {
+              group(20, g);
+            } else {
+#pragma unroll
+              for (int e = 0; e < EPL; ++e) g[e] = 0.f;
+            }
+#pragma unroll
+            for (int e = 0; e < EPL; ++e) h[e] = __fadd_rn(h[e], g[e]);
+            if (s.M > 24) {
+              add_pair(6, h);
+            } else {
+#pragma unroll
+              for (int e = 0; e < EPL; ++e) h[e] = __fadd_rn(h[e], 0.f);
+            }
+#pragma unroll
+            for (int e = 0; e < EPL; ++e) acc[e] = __fadd_rn(acc[e], h[e]);
+          }
+        }
       }
     }
 #pragma unroll
@@ -1151,18 +1171,19 @@ squant_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap
   }
 }
 
-// Identity: the messages are the p vectors themselves (worker order).
+// Identity: the messages are the p vectors themselves, summed in groups of
+// four workers in the library's pairwise order.
 __global__ void __launch_bounds__(256) identity_server_kernel(const ServerArgs s) {
   const int64_t c = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   const int64_t j = 4 * c;
   if (j >= s.d) return;
-  float acc[4] = {0.f, 0.f, 0.f, 0.f};
+  PairwiseAcc<kSumLevels> sum[4];
   const bool vec = j + 3 < s.d;
   for (int m0 = 0; m0 < s.M; m0 += 4) {
     float4 v[4];
 #pragma unroll
     for (int u = 0; u < 4; ++u) {
-      v[u] = make_float4(0.f, 0.f, 0.f, 0.f);
+      v[u] = make_float4(0.f, 0.f, 0.f, 0.f);  // +0 leaves past M and past d
       if (m0 + u < s.M) {
         const float* vals = reinterpret_cast<const float*>(s.msgs + (int64_t)(m0 + u) * s.msg_stride);
         if (vec) {
@@ -1174,16 +1195,14 @@ __global__ void __launch_bounds__(256) identity_server_kernel(const ServerArgs s
         }
       }
     }
-#pragma unroll
-    for (int u = 0; u < 4; ++u) {
-      if (m0 + u < s.M) {
-        acc[0] = __fadd_rn(acc[0], v[u].x);
-        acc[1] = __fadd_rn(acc[1], v[u].y);
-        acc[2] = __fadd_rn(acc[2], v[u].z);
-        acc[3] = __fadd_rn(acc[3], v[u].w);
-      }
-    }
+    sum[0].push(group4(v[0].x, v[1].x, v[2].x, v[3].x, s.M));
+    sum[1].push(group4(v[0].y, v[1].y, v[2].y, v[3].y, s.M));
+    sum[2].push(group4(v[0].z, v[1].z, v[2].z, v[3].z, s.M));
+    sum[3].push(group4(v[0].w, v[1].w, v[2].w, v[3].w, s.M));
   }
+  float acc[4];
+#pragma unroll
+  for (int q = 0; q < 4; ++q) acc[q] = sum[q].result();
   apply_chunk(s, j, acc);
 }
 
@@ -1308,14 +1327,15 @@ cudaError_t launch_sign_server(const ServerArgs& s, const SignServerExtras& x, c
       cudaError_t st;
 #define DQ_SIGN_SEG(NG) \
   st = (p2 ? launch_sign_col<NG, true, true>(s, x, stream) : launch_sign_col<NG, false, true>(s, x, stream))
-      switch ((s.M + 4) / 5) {
+      switch ((s.M + 3) / 4) {
         case 1: DQ_SIGN_SEG(1); break;
         case 2: DQ_SIGN_SEG(2); break;
         case 3: DQ_SIGN_SEG(3); break;
         case 4: DQ_SIGN_SEG(4); break;
         case 5: DQ_SIGN_SEG(5); break;
         case 6: DQ_SIGN_SEG(6); break;
-        default: DQ_SIGN_SEG(7); break;
+        case 7: DQ_SIGN_SEG(7); break;
+        default: DQ_SIGN_SEG(8); break;
       }
 #undef DQ_SIGN_SEG
       *launches += 1;
@@ -1332,14 +1352,15 @@ cudaError_t launch_sign_server(const ServerArgs& s, const SignServerExtras& x, c
 #define DQ_SIGN_TMA(NG)                                                                           \
   st = col ? (p2 ? launch_sign_col<NG, true, false>(s, x, stream) : launch_sign_col<NG, false, false>(s, x, stream)) \
            : (p2 ? launch_sign_tma<NG, true>(s, stream) : launch_sign_tma<NG, false>(s, stream))
-    switch ((s.M + 4) / 5) {
+    switch ((s.M + 3) / 4) {
       case 1: DQ_SIGN_TMA(1); break;
       case 2: DQ_SIGN_TMA(2); break;
       case 3: DQ_SIGN_TMA(3); break;
       case 4: DQ_SIGN_TMA(4); break;
       case 5: DQ_SIGN_TMA(5); break;
       case 6: DQ_SIGN_TMA(6); break;
-      default: DQ_SIGN_TMA(7); break;
+      case 7: DQ_SIGN_TMA(7); break;
+      default: DQ_SIGN_TMA(8); break;
     }
 #undef DQ_SIGN_TMA
     *launches += 1;
@@ -1353,7 +1374,7 @@ cudaError_t launch_sign_server(const ServerArgs& s, const SignServerExtras& x, c
     if (s.M > 32) {
       sign_server_slabs_kernel<<<blocks, 256, 0, stream>>>(s);
     } else {
-      const int ng = (s.M + 4) / 5;
+      const int ng = (s.M + 3) / 4;
       const bool p2 = s.M_pow2 != 0;
 #define DQ_SIGN_SERVER(NG) \
       (p2 ? sign_server_shfl_kernel<NG, true><<<blocks, 256, 0, stream>>>(s) \
@@ -1365,7 +1386,8 @@ cudaError_t launch_sign_server(const ServerArgs& s, const SignServerExtras& x, c
         case 4: DQ_SIGN_SERVER(4); break;
         case 5: DQ_SIGN_SERVER(5); break;
         case 6: DQ_SIGN_SERVER(6); break;
-        default: DQ_SIGN_SERVER(7); break;
+        case 7: DQ_SIGN_SERVER(7); break;
+        default: DQ_SIGN_SERVER(8); break;
       }
 #undef DQ_SIGN_SERVER
     }

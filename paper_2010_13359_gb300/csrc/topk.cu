@@ -29,13 +29,13 @@
 // The carried threshold only decides how much work the first pass saves the
 // second; the result is the same bit for bit either way.
 //
-// Server: w_j -= (sum over workers, in worker order, of the value recorded
-// for j) / M at the indices some worker sent; elsewhere w is unchanged (the
-// absent +0 terms leave the sum and w as they are).  A first kernel finds, for
-// each worker and each tile of 256 indices, where the tile's records start;
-// then one warp per tile sums the tile's records in shared memory, worker by
-// worker, and updates the touched parameters (one thread per record, with
-// searches narrowed to the tile, above 64 workers).
+// Server: w_j -= (sum over workers of the value recorded for j, absent
+// workers as +0, in the library's pairwise order) / M at the indices some
+// worker sent; elsewhere the sum is +0 and w is unchanged.  A first kernel
+// finds, for each worker and each tile of 256 indices, where the tile's
+// records start; then one warp per tile builds the tile's per-index sums in
+// shared memory, worker by worker, and updates the touched parameters (one
+// thread per record, with searches narrowed to the tile, above 64 workers).
 #include <atomic>
 
 #include <cooperative_groups.h>
@@ -856,32 +856,75 @@ __device__ __forceinline__ float srv_average(float acc, const ServerArgs& s) {
   else return __fdiv_rn(acc, (float)s.M);
 }
 
+// Per index, the server's sum over workers in the library's order (the
+// M values padded with +0 to P = next_pow2(M), summed pairwise), built
+// worker by worker with absent workers as +0 leaves: stk holds the index's
+// complete blocks (level L: the sum of 2^L consecutive workers, column
+// `off` of row L, rows kSrvTile floats apart), n the workers accounted for.
+// Pushes the block of 2^L workers starting at n (n a multiple of 2^L).
+__device__ __forceinline__ void srv_push_block(float* stk, int off, uint32_t n, int L, float v) {
+  float c = v;
+  uint32_t k = n >> L;
+  int l = L;
+  while (k & 1u) {
+    c = __fadd_rn(stk[l * kSrvTile + off], c);
+    k >>= 1;
+    ++l;
+  }
+  stk[l * kSrvTile + off] = c;
+}
+
+// Accounts for workers n .. t - 1 as +0 leaves, in the largest aligned
+// blocks (a block of +0 leaves sums to +0); returns t.
+__device__ __forceinline__ uint32_t srv_push_zeros(float* stk, int off, uint32_t n, uint32_t t) {
+  while (n < t) {
+    int L = 31 - __clz((int)(t - n));  // the largest block that fits
+    if (n) L = min(L, __ffs((int)n) - 1);  // and that starts on a multiple of its size
+    srv_push_block(stk, off, n, L, 0.f);
+    n += 1u << L;
+  }
+  return n;
+}
+
 // One warp per tile of kSrvTile indices (M <= kSrvWarpMaxM).  The warp
 // stages the tile's records of all workers in shared memory (one flat,
-// worker-ordered batch of loads), adds them into the tile's sums worker by
-// worker -- program order within the warp keeps worker order, so no block
-// barrier is needed -- and updates the touched w_j (all loads of w issued
-// before the stores).
-struct SrvWarpSmem {
-  float acc[kSrvTile];
-  uint32_t touched[kSrvTile / 32];
-  uint2 buf[kSrvWarpBuf];
-  uint32_t first[kSrvWarpMaxM];
-  uint32_t pre[kSrvWarpMaxM + 1];
-};
+// worker-ordered batch of loads) and pushes them into the per-index
+// pairwise sums worker by worker -- program order within the warp keeps
+// worker order, so no block barrier is needed -- then completes every
+// touched index's sum to P leaves and updates the touched w_j (all loads of
+// w issued before the stores).  Untouched indices sum to +0 and keep w_j.
+// Per-warp shared memory (srv_warp_bytes): the record buffer, then
+// srv_levels(M) rows of per-index blocks, the per-worker record ranges, and
+// one count byte per index.
+__host__ __device__ constexpr int srv_levels(int M) {
+  int l = 1;
+  while ((1 << (l - 1)) < M) ++l;
+  return l;  // log2(next_pow2(M)) + 1
+}
+__host__ __device__ constexpr size_t srv_warp_bytes(int M) {
+  return (size_t)kSrvWarpBuf * 8 + (size_t)srv_levels(M) * kSrvTile * 4 + (kSrvWarpMaxM + kSrvWarpMaxM + 4) * 4 +
+         kSrvTile;
+}
 constexpr int kSrvWarps = kSrvThreads / 32;
 
 template <bool POW2>
 __global__ void __launch_bounds__(kSrvThreads) topk_server_warp_kernel(const ServerArgs s, const uint32_t* starts) {
   extern __shared__ __align__(16) unsigned char smem_raw[];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  SrvWarpSmem& sm = reinterpret_cast<SrvWarpSmem*>(smem_raw)[warp];
+  const int M = s.M;
+  const int nlev = srv_levels(M);
+  unsigned char* region = smem_raw + (size_t)warp * srv_warp_bytes(M);
+  uint2* buf = reinterpret_cast<uint2*>(region);
+  float* stk = reinterpret_cast<float*>(region + (size_t)kSrvWarpBuf * 8);
+  uint32_t* first = reinterpret_cast<uint32_t*>(stk + nlev * kSrvTile);
+  uint32_t* pre = first + kSrvWarpMaxM;
+  uint8_t* cnt = reinterpret_cast<uint8_t*>(pre + kSrvWarpMaxM + 4);
   const int64_t nts = srv_tiles(s.d);
   const int64_t t = (int64_t)blockIdx.x * kSrvWarps + warp;
   if (t >= nts) return;  // the whole warp
   const int64_t tile0 = t * kSrvTile;
-  const int M = s.M;
-  if (lane < kSrvTile / 32) sm.touched[lane] = 0;
+#pragma unroll
+  for (int q = 0; q < kSrvTile / 32; ++q) cnt[q * 32 + lane] = 0;
   // this tile's record range of every worker, and the flat prefix
   uint32_t run = 0;
   for (int base = 0; base < M; base += 32) {
@@ -891,7 +934,7 @@ __global__ void __launch_bounds__(kSrvThreads) topk_server_warp_kernel(const Ser
       const uint32_t* st = starts + (int64_t)m * (nts + 1);
       const uint32_t a0 = (uint32_t)min64(st[t], s.k), a1 = (uint32_t)min64(st[t + 1], s.k);
       n = a1 > a0 ? a1 - a0 : 0u;
-      sm.first[m] = a0;
+      first[m] = a0;
     }
     uint32_t x = n;
 #pragma unroll
@@ -899,10 +942,10 @@ __global__ void __launch_bounds__(kSrvThreads) topk_server_warp_kernel(const Ser
       const uint32_t y = __shfl_up_sync(kFullMask, x, off);
       if (lane >= off) x += y;
     }
-    if (m < M) sm.pre[m] = run + x - n;
+    if (m < M) pre[m] = run + x - n;
     run += __shfl_sync(kFullMask, x, 31);
   }
-  if (lane == 0) sm.pre[M] = run;
+  if (lane == 0) pre[M] = run;
   __syncwarp();
   const uint32_t N = run;
   for (uint32_t b = 0; b < N; b += kSrvWarpBuf) {
@@ -920,69 +963,67 @@ __global__ void __launch_bounds__(kSrvThreads) topk_server_warp_kernel(const Ser
           int lo = 0, hi = M;  // pre[lo] <= f < pre[hi]
           while (hi - lo > 1) {
             const int mid = (lo + hi) >> 1;
-            if (sm.pre[mid] <= f) lo = mid;
+            if (pre[mid] <= f) lo = mid;
             else hi = mid;
           }
           const uint2* msg = reinterpret_cast<const uint2*>(s.msgs + (int64_t)lo * s.msg_stride);
-          v[u] = msg[sm.first[lo] + (f - sm.pre[lo])];
+          v[u] = msg[first[lo] + (f - pre[lo])];
         }
       }
 #pragma unroll
       for (int u = 0; u < kStage; ++u) {
         const uint32_t i = i0 + u * 32 + lane;
-        if (i < nb) sm.buf[i] = v[u];
+        if (i < nb) buf[i] = v[u];
       }
     }
     __syncwarp();
     for (int m = 0; m < M; ++m) {
-      const uint32_t f0 = max64(sm.pre[m], b), f1 = min64(sm.pre[m + 1], b + nb);
-      // a worker's indices are distinct: its records update distinct sums,
-      // four per lane at a time
-      for (uint32_t fb = f0; fb < f1; fb += 4 * 32) {
-        uint2 r[4];
-#pragma unroll
-        for (int u = 0; u < 4; ++u) {
-          const uint32_t f = fb + u * 32 + lane;
-          r[u] = f < f1 ? sm.buf[f - b] : make_uint2(0xFFFFFFFFu, 0u);
-        }
-#pragma unroll
-        for (int u = 0; u < 4; ++u) {
-          const int64_t off = (int64_t)r[u].x - tile0;
-          if (fb + u * 32 + lane < f1 && off >= 0 && off < kSrvTile && (int64_t)r[u].x < s.d) {
-            const uint32_t bit = 1u << (off & 31);
-            const bool seen = (sm.touched[off >> 5] & bit) != 0;
-            // the sum starts at +0 (as a dense sum over all workers would)
-            sm.acc[off] = __fadd_rn(seen ? sm.acc[off] : 0.f, __uint_as_float(r[u].y));
-            if (!seen) atomicOr(&sm.touched[off >> 5], bit);
-          }
+      const uint32_t f0 = max64(pre[m], b), f1 = min64(pre[m + 1], b + nb);
+      // a worker's indices are distinct: its records go to distinct sums,
+      // one per lane at a time
+      for (uint32_t f = f0 + lane; f < f1; f += 32) {
+        const uint2 r = buf[f - b];
+        const int64_t off = (int64_t)r.x - tile0;
+        if (off >= 0 && off < kSrvTile && (int64_t)r.x < s.d) {
+          const uint32_t n = srv_push_zeros(stk, (int)off, cnt[off], (uint32_t)m);
+          srv_push_block(stk, (int)off, n, 0, __uint_as_float(r.y));
+          cnt[off] = (uint8_t)(m + 1);
         }
       }
       __syncwarp();
     }
   }
+  const uint32_t P = 1u << (nlev - 1);
   constexpr int kPer = kSrvTile / 32;
   constexpr int kHalf = kPer / 2;
 #pragma unroll
   for (int half = 0; half < 2; ++half) {
-    float wv[kHalf];
+    float wv[kHalf], sum[kHalf];
 #pragma unroll
     for (int q = 0; q < kHalf; ++q) {
       const int i = (half * kHalf + q) * 32 + lane;
-      wv[q] = ((sm.touched[i >> 5] >> (i & 31)) & 1u) ? s.w[tile0 + i] : 0.f;
+      const uint32_t n = cnt[i];
+      wv[q] = 0.f;
+      sum[q] = 0.f;
+      if (n) {
+        wv[q] = s.w[tile0 + i];
+        srv_push_zeros(stk, i, n, P);
+        sum[q] = stk[(nlev - 1) * kSrvTile + i];
+      }
     }
 #pragma unroll
     for (int q = 0; q < kHalf; ++q) {
       const int i = (half * kHalf + q) * 32 + lane;
-      if ((sm.touched[i >> 5] >> (i & 31)) & 1u) s.w[tile0 + i] = __fsub_rn(wv[q], srv_average<POW2>(sm.acc[i], s));
+      if (cnt[i]) s.w[tile0 + i] = __fsub_rn(wv[q], srv_average<POW2>(sum[q], s));
     }
   }
 }
 
 // One thread per record of every worker.  The record of the lowest worker
-// holding index j owns j: it sums the values recorded for j over the
-// workers in worker order (the sum starts at +0, as a dense sum over all
-// workers would) and applies w_j -= sum / M; the others find an earlier
-// worker holding j and stop.  Each search looks only at the other worker's
+// holding index j owns j: it sums the values recorded for j over all M
+// workers (absent ones as +0 leaves) in the library's pairwise order and
+// applies w_j -= sum / M; the others find an earlier worker holding j and
+// stop.  Each search looks only at the other worker's
 // records in j's tile of kSrvTile indices (the starts table), and the
 // searches in kSrvGroup workers' lists advance in lockstep so that their
 // loads are in flight together.
@@ -999,7 +1040,9 @@ __global__ void __launch_bounds__(kSrvThreads) topk_server_owner_kernel(const Se
   if ((int64_t)j >= s.d) return;  // records come from the compressor and are < d
   const int64_t nts = srv_tiles(s.d);
   const int64_t t = j / kSrvTile;
-  float acc = __fadd_rn(0.f, __uint_as_float(mine.y));
+  PairwiseAcc<13> sum;  // M <= 4096
+  for (int m2 = 0; m2 < m; ++m2) sum.push(0.f);  // no earlier worker holds j (else it owns j)
+  sum.push(__uint_as_float(mine.y));
   for (int m0 = 0; m0 < s.M; m0 += kSrvGroup) {
     uint32_t lo[kSrvGroup], hi[kSrvGroup], end[kSrvGroup];
 #pragma unroll
@@ -1051,12 +1094,11 @@ __global__ void __launch_bounds__(kSrvThreads) topk_server_owner_kernel(const Se
     }
 #pragma unroll
     for (int u = 0; u < kSrvGroup; ++u) {
-      if (!has[u]) continue;
-      if (m0 + u < m) return;  // an earlier worker owns j
-      acc = __fadd_rn(acc, val[u]);
+      if (has[u] && m0 + u < m) return;  // an earlier worker owns j
+      if (m0 + u > m && m0 + u < s.M) sum.push(has[u] ? val[u] : 0.f);
     }
   }
-  s.w[j] = __fsub_rn(s.w[j], srv_average<POW2>(acc, s));
+  s.w[j] = __fsub_rn(s.w[j], srv_average<POW2>(sum.result(), s));
 }
 
 }  // namespace
@@ -1117,7 +1159,7 @@ cudaError_t launch_topk_server(const ServerArgs& s, void* scratch, cudaStream_t 
   topk_server_starts_kernel<<<dim3((unsigned)((s.k + 255) / 256), (unsigned)s.M), 256, 0, stream>>>(s, starts);
   if (s.M <= kSrvWarpMaxM) {
     static std::atomic<size_t> smem_done[2][kSmemDevices];
-    const size_t smem = sizeof(SrvWarpSmem) * kSrvWarps;
+    const size_t smem = srv_warp_bytes(s.M) * kSrvWarps;
     const unsigned blocks = (unsigned)((srv_tiles(s.d) + kSrvWarps - 1) / kSrvWarps);
     cudaError_t st;
     if (s.M_pow2) st = ensure_smem(topk_server_warp_kernel<true>, smem, 0, smem_done[1]);

@@ -17,7 +17,7 @@ import numpy as np
 import pytest
 
 import oracle
-from parity_helpers import STEP_RTOL, assert_bits_equal, assert_messages_equal, oracle_config, rel_err
+from parity_helpers import STEP_RTOL, assert_bits_equal, assert_messages_equal, oracle_config, assert_params_equal
 from paper_2010_13359_gb300.workloads import game_diag_np, game_noise_np
 
 pytestmark = pytest.mark.gpu
@@ -87,8 +87,7 @@ def test_closed_loop_matches_oracle(P, comp, kw, locked):
     for t in range(1, T + 1):
         closed_loop(h, game, w_gpu, steps=1, step0=t, on_step=on_step)
         h.synchronize()
-        err = rel_err(w_gpu.cpu().numpy(), w_orc)
-        assert err <= STEP_RTOL, f"params step {t}: {err}"
+        assert_params_equal(w_gpu.cpu().numpy(), w_orc, f"params step {t}")
         for i in range(M):
             e_i, h_i = np.empty(d, np.float32), np.empty(d, np.float32)
             h.get_residual(i, e_i)

@@ -10,7 +10,7 @@ import numpy as np
 import pytest
 
 import oracle
-from parity_helpers import STEP_RTOL, assert_bits_equal, assert_messages_equal, oracle_config, rel_err
+from parity_helpers import STEP_RTOL, assert_bits_equal, assert_messages_equal, oracle_config, assert_params_equal
 
 pytestmark = pytest.mark.gpu
 
@@ -66,7 +66,7 @@ def test_bounded_wait_times_out_and_the_handle_survives(P, polls):
     h.server_aggregate_update(msgs, w_gpu)
     st.server(want, w_orc)
     h.synchronize()
-    assert rel_err(w_gpu.cpu().numpy(), w_orc) <= STEP_RTOL
+    assert_params_equal(w_gpu.cpu().numpy(), w_orc, "params")
     e0 = np.empty(d, np.float32)
     h.get_residual(0, e0)
     assert_bits_equal(e0, st.e[0], "residual after the time-out")

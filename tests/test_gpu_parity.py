@@ -13,7 +13,7 @@ import pytest
 
 import oracle
 from parity_helpers import (STEP_RTOL, assert_bits_equal, assert_messages_equal, oracle_config,
-                            rel_err)
+                            assert_params_equal)
 
 pytestmark = pytest.mark.gpu
 
@@ -49,7 +49,7 @@ def grads(kind, M, d, rng):
 
 def run_parity(P, ocfg, T, kind="gauss", batched=True, seed=0):
     """T free-running steps on both sides; every step compares messages,
-    e and h bit for bit and w within STEP_RTOL."""
+    e, h and w bit for bit (w also within STEP_RTOL per element)."""
     dev = torch.device("cuda:0")
     stream = torch.cuda.current_stream(dev)
     rng = np.random.default_rng(seed)
@@ -92,8 +92,7 @@ def run_parity(P, ocfg, T, kind="gauss", batched=True, seed=0):
         h.server_aggregate_update(msgs, w_gpu)
         st.server(msgs_orc, w_orc)
         h.synchronize()
-        err = rel_err(w_gpu.cpu().numpy(), w_orc)
-        assert err <= STEP_RTOL, f"params step {t}: rel err {err}"
+        assert_params_equal(w_gpu.cpu().numpy(), w_orc, f"params step {t}")
         assert h.get_step() == st.t == t + 1
     h.destroy()
 

@@ -9,7 +9,7 @@ import numpy as np
 import pytest
 
 import oracle
-from parity_helpers import STEP_RTOL, assert_bits_equal, assert_messages_equal, oracle_config, rel_err
+from parity_helpers import STEP_RTOL, assert_bits_equal, assert_messages_equal, oracle_config, assert_params_equal
 from paper_2010_13359_gb300.workloads import WORKLOADS
 
 pytestmark = pytest.mark.gpu
@@ -65,7 +65,7 @@ def run_segmented(P, ocfg, T, seed):
         h.server_aggregate_update(msgs, w_gpu)
         st.server(want, w_orc)
         h.synchronize()
-        assert rel_err(w_gpu.cpu().numpy(), w_orc) <= STEP_RTOL
+        assert_params_equal(w_gpu.cpu().numpy(), w_orc, "params")
     h.destroy()
 
 

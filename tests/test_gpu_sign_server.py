@@ -21,7 +21,7 @@ import numpy as np
 import pytest
 
 import oracle
-from parity_helpers import STEP_RTOL, assert_messages_equal, oracle_config, rel_err
+from parity_helpers import STEP_RTOL, assert_messages_equal, oracle_config, assert_params_equal
 
 pytestmark = pytest.mark.gpu
 
@@ -97,8 +97,7 @@ def test_sign_server_paths(P, d, M, bucket, path, monkeypatch):
             h.server_aggregate_update(msgs, w_gpu)
         st.server(msgs_orc, w_orc)
         h.synchronize()
-        err = rel_err(w_gpu.cpu().numpy(), w_orc)
-        assert err <= STEP_RTOL, f"step {t}: rel err {err}"
+        assert_params_equal(w_gpu.cpu().numpy(), w_orc, f"step {t}")
     tail = buf[d:].cpu().numpy()
     assert np.all(tail == 12345.0), "parameters past d were written"
     assert torch.all(alt[d:] == 0.0)
@@ -159,7 +158,6 @@ def test_sign_server_segments(P, d, M, bucket, kind):
         h.server_aggregate_update(msgs, w_gpu)
         st.server(want, w_orc)
         h.synchronize()
-        err = rel_err(w_gpu.cpu().numpy(), w_orc)
-        assert err <= STEP_RTOL, f"step {t}: rel err {err}"
+        assert_params_equal(w_gpu.cpu().numpy(), w_orc, f"step {t}")
     assert np.all(buf[d:].cpu().numpy() == -777.0), "parameters past d were written"
     h.destroy()
