@@ -43,6 +43,32 @@ class _OrcCfg(ctypes.Structure):
     ]
 
 
+class _OrcOAdam(ctypes.Structure):
+    _fields_ = [
+        ("alpha", ctypes.c_float),
+        ("beta1", ctypes.c_float),
+        ("beta2", ctypes.c_float),
+        ("eps", ctypes.c_float),
+        ("adaptive", ctypes.c_int32),
+        ("bias_correction", ctypes.c_int32),
+    ]
+
+
+@dataclasses.dataclass
+class OAdam:
+    """Optimistic Adam server update (see orc_oadam_update)."""
+    alpha: float = 1e-3
+    beta1: float = 0.5
+    beta2: float = 0.999
+    eps: float = 1e-8
+    adaptive: bool = True
+    bias_correction: bool = True
+
+    def c_struct(self) -> _OrcOAdam:
+        return _OrcOAdam(alpha=self.alpha, beta1=self.beta1, beta2=self.beta2, eps=self.eps,
+                         adaptive=1 if self.adaptive else 0, bias_correction=1 if self.bias_correction else 0)
+
+
 @dataclasses.dataclass
 class Config:
     d: int
@@ -109,6 +135,16 @@ def lib() -> ctypes.CDLL:
         L.orc_server_step.restype = None
         L.orc_server_step_range.argtypes = [cfgp, u8p, ctypes.c_int64, f32p, ctypes.c_int64, ctypes.c_int64]
         L.orc_server_step_range.restype = None
+        L.orc_server_average_range.argtypes = [cfgp, u8p, ctypes.c_int64, f32p, ctypes.c_int64, ctypes.c_int64]
+        L.orc_server_average_range.restype = None
+        L.orc_pow_steps.argtypes = [ctypes.c_float, ctypes.c_int64]
+        L.orc_pow_steps.restype = ctypes.c_float
+        oap = P(_OrcOAdam)
+        L.orc_oadam_update.argtypes = [oap, ctypes.c_int64, ctypes.c_int64, f32p, f32p, f32p, f32p, f32p]
+        L.orc_oadam_update.restype = None
+        L.orc_server_step_oadam_range.argtypes = [cfgp, u8p, ctypes.c_int64, oap, ctypes.c_int64, f32p, f32p,
+                                                  f32p, f32p, ctypes.c_int64, ctypes.c_int64]
+        L.orc_server_step_oadam_range.restype = None
         L.orc_lookahead.argtypes = [ctypes.c_int64, f32p, f32p, f32p]
         L.orc_lookahead.restype = None
         L.orc_bucket_count.argtypes = [cfgp]
@@ -232,6 +268,43 @@ def server_step_range(cfg: Config, msgs: np.ndarray, w: np.ndarray, j0: int, j1:
     assert msgs.dtype == np.uint8 and msgs.flags.c_contiguous and msgs.ndim == 2 and msgs.shape[0] == cfg.M
     assert 0 <= j0 <= j1 <= cfg.d and w.size == cfg.d
     lib().orc_server_step_range(ctypes.byref(cfg.c_struct()), _u8(msgs), msgs.shape[1], _f32(w), j0, j1)
+
+
+def server_average(cfg: Config, msgs: np.ndarray, j0: int = 0, j1: int | None = None) -> np.ndarray:
+    """q_hat = (1/M) sum_m Q_m for elements [j0, j1) (the server's fixed-order average)."""
+    j1 = cfg.d if j1 is None else j1
+    msgs = np.ascontiguousarray(msgs, dtype=np.uint8)
+    out = np.zeros(max(j1 - j0, 1), np.float32)
+    lib().orc_server_average_range(ctypes.byref(cfg.c_struct()), _u8(msgs), msgs.shape[1], _f32(out), j0, j1)
+    return out[:j1 - j0]
+
+
+def pow_steps(b: float, t: int) -> float:
+    return float(lib().orc_pow_steps(b, t))
+
+
+class OAdamState:
+    """The server's Optimistic Adam state for d parameters: m, v, u_prev (zero at the start)."""
+
+    def __init__(self, d: int, opt: OAdam):
+        self.opt = opt
+        self.m = np.zeros(d, np.float32)
+        self.v = np.zeros(d, np.float32)
+        self.u = np.zeros(d, np.float32)
+
+    def update(self, t: int, q_hat: np.ndarray, w: np.ndarray) -> None:
+        """One Optimistic Adam step at iteration t on w (in place) from the averaged update q_hat."""
+        q_hat = np.ascontiguousarray(q_hat, dtype=np.float32)
+        c = self.opt.c_struct()
+        lib().orc_oadam_update(ctypes.byref(c), t, w.size, _f32(q_hat), _f32(self.m), _f32(self.v), _f32(self.u),
+                               _f32(w))
+
+    def server_step_range(self, cfg: Config, t: int, msgs: np.ndarray, w: np.ndarray, j0: int, j1: int) -> None:
+        """Server step of Algorithm 2 with the Optimistic Adam update, on elements [j0, j1)."""
+        msgs = np.ascontiguousarray(msgs, dtype=np.uint8)
+        c = self.opt.c_struct()
+        lib().orc_server_step_oadam_range(ctypes.byref(cfg.c_struct()), _u8(msgs), msgs.shape[1], ctypes.byref(c), t,
+                                          _f32(self.m), _f32(self.v), _f32(self.u), _f32(w), j0, j1)
 
 
 def lookahead(w: np.ndarray, h: np.ndarray) -> np.ndarray:

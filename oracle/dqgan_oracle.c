@@ -511,11 +511,12 @@ void orc_worker_step(const orc_cfg* c, int32_t worker, int64_t step, const float
 /* ------------------------------------------------------------------------ */
 #define ORC_SERVER_CHUNK 4096
 
-/* The server step restricted to elements [j0, j1): each element's update
- * depends on that element alone, so disjoint ranges may run concurrently
- * (the full step is the range [0, d)). */
-void orc_server_step_range(const orc_cfg* c, const uint8_t* msgs, int64_t msg_stride, float* w, int64_t j0,
-                           int64_t j1) {
+/* The averaged update q_hat of Algorithm 2's server for elements [j0, j1),
+ * element j written to q_hat[j - j0]: the sum over workers taken by
+ * orc_pairwise_sum, then divided by M.  Each element depends on that element alone, so disjoint
+ * ranges may run concurrently. */
+void orc_server_average_range(const orc_cfg* c, const uint8_t* msgs, int64_t msg_stride, float* q_hat,
+                              int64_t j0, int64_t j1) {
   int32_t M = c->M;
   int32_t P = 1;
   while (P < M) P *= 2;
@@ -530,8 +531,7 @@ void orc_server_step_range(const orc_cfg* c, const uint8_t* msgs, int64_t msg_st
     for (int64_t j = c0; j < c1; ++j) {
       for (int32_t m = 0; m < M; ++m) x[m] = q[(int64_t)m * ORC_SERVER_CHUNK + (j - c0)];
       float sum = orc_pairwise_sum(x, M);
-      float q_hat = sum / (float)M;
-      w[j] = w[j] - q_hat;
+      q_hat[j - j0] = sum / (float)M;
     }
   }
   free(x);
@@ -539,8 +539,83 @@ void orc_server_step_range(const orc_cfg* c, const uint8_t* msgs, int64_t msg_st
   free(starts);
 }
 
+/* The server step (w = w - q_hat) restricted to elements [j0, j1). */
+void orc_server_step_range(const orc_cfg* c, const uint8_t* msgs, int64_t msg_stride, float* w, int64_t j0,
+                           int64_t j1) {
+  float* q_hat = (float*)malloc((size_t)(j1 > j0 ? j1 - j0 : 1) * 4);
+  orc_server_average_range(c, msgs, msg_stride, q_hat, j0, j1);
+  for (int64_t j = j0; j < j1; ++j) w[j] = w[j] - q_hat[j - j0];
+  free(q_hat);
+}
+
 void orc_server_step(const orc_cfg* c, const uint8_t* msgs, int64_t msg_stride, float* w) {
   orc_server_step_range(c, msgs, msg_stride, w, 0, c->d);
+}
+
+/* ------------------------------------------------------------------------ */
+/* Optimistic Adam on the server (the CPOAdam family that Section 4 compares */
+/* against).  The paper prints no rule for it; the reading taken is the     */
+/* Optimistic Adam of Daskalakis, Ilyas, Syrgkanis and Zeng ("Training GANs  */
+/* with Optimism", ICLR 2018), fed the averaged update q_hat of Algorithm 2  */
+/* in place of the plain step w = w - q_hat:                                 */
+/*   m = b1 m + (1 - b1) q_hat,   v = b2 v + ((1 - b2) q_hat) q_hat          */
+/*   with bias correction m_hat = m / (1 - b1^t), v_hat = v / (1 - b2^t),   */
+/*   else m_hat = m, v_hat = v                                               */
+/*   adaptive: u = m_hat / (sqrt(v_hat) + eps), and u = 0 where m_hat = 0;  */
+/*   else u = m_hat (the identity preconditioner)                           */
+/*   w = w - alpha (2 u - u_prev),   u_prev = u                              */
+/* in fp32, one rounding per operation in the order written; b^t is the     */
+/* product of t factors b taken left to right.  m, v, u_prev start at 0.    */
+/* With b1 = 0, the identity preconditioner and alpha = 1 the update is     */
+/* w_t = w_{t-1} - 2 q_hat_t + q_hat_{t-1}, the one-line OMD recurrence of  */
+/* Section 2.2.                                                              */
+/* ------------------------------------------------------------------------ */
+typedef struct orc_oadam {
+  float alpha;
+  float beta1;
+  float beta2;
+  float eps;
+  int32_t adaptive;         /* 1: divide by sqrt(v_hat) + eps */
+  int32_t bias_correction;  /* 1: divide m, v by 1 - b^t */
+} orc_oadam;
+
+float orc_pow_steps(float b, int64_t t) {
+  float r = 1.0f;
+  for (int64_t i = 0; i < t; ++i) r = r * b;
+  return r;
+}
+
+/* One Optimistic Adam step at iteration t (1-based) on n elements. */
+void orc_oadam_update(const orc_oadam* p, int64_t t, int64_t n, const float* q_hat, float* m, float* v, float* u,
+                      float* w) {
+  float one_m_b1 = 1.0f - p->beta1;
+  float one_m_b2 = 1.0f - p->beta2;
+  float c1 = p->bias_correction ? 1.0f - orc_pow_steps(p->beta1, t) : 1.0f;
+  float c2 = p->bias_correction ? 1.0f - orc_pow_steps(p->beta2, t) : 1.0f;
+  for (int64_t j = 0; j < n; ++j) {
+    float g = q_hat[j];
+    float mj = p->beta1 * m[j] + one_m_b1 * g;
+    float vj = p->beta2 * v[j] + (one_m_b2 * g) * g;
+    float mh = p->bias_correction ? mj / c1 : mj;
+    float vh = p->bias_correction ? vj / c2 : vj;
+    float uj = mh;
+    if (p->adaptive) uj = (mh == 0.0f) ? 0.0f : mh / (sqrtf(vh) + p->eps);
+    float step = 2.0f * uj - u[j];
+    w[j] = w[j] - p->alpha * step;
+    m[j] = mj;
+    v[j] = vj;
+    u[j] = uj;
+  }
+}
+
+/* The server step with Optimistic Adam on elements [j0, j1): q_hat as in   */
+/* orc_server_average_range, then orc_oadam_update (m, v, u: d floats).      */
+void orc_server_step_oadam_range(const orc_cfg* c, const uint8_t* msgs, int64_t msg_stride, const orc_oadam* p,
+                                 int64_t t, float* m, float* v, float* u, float* w, int64_t j0, int64_t j1) {
+  float* q_hat = (float*)malloc((size_t)(j1 > j0 ? j1 - j0 : 1) * 4);
+  orc_server_average_range(c, msgs, msg_stride, q_hat, j0, j1);
+  orc_oadam_update(p, t, j1 - j0, q_hat, m + j0, v + j0, u + j0, w + j0);
+  free(q_hat);
 }
 
 /* Lookahead of Algorithm 2: w_{t-1/2} = w_{t-1} - h, h = eta*F_prev + e_prev. */

@@ -131,3 +131,50 @@ class ExactDQGAN:
         rec["w"] = list(self.w)
         self.history.append(rec)
         return rec
+
+
+# --- Optimistic Adam server update (the CPOAdam family of Section 4) --------
+
+def exact_sqrt(x: Fraction) -> Fraction:
+    """The square root of x when it is rational (x a square of a rational); else ValueError."""
+    from math import isqrt
+    if x < 0:
+        raise ValueError("negative")
+    n, d = x.numerator, x.denominator
+    rn, rd = isqrt(n), isqrt(d)
+    if rn * rn != n or rd * rd != d:
+        raise ValueError("not a rational square")
+    return Fraction(rn, rd)
+
+
+class ExactOAdam:
+    """Optimistic Adam (Daskalakis et al., ICLR 2018) on the server's
+    averaged update, in exact arithmetic:
+    m = b1 m + (1 - b1) q; v = b2 v + (1 - b2) q^2; with bias correction
+    m_hat = m / (1 - b1^t), v_hat = v / (1 - b2^t); adaptive:
+    u = m_hat / (sqrt(v_hat) + eps) (u = 0 where m_hat = 0), else u = m_hat;
+    w = w - alpha (2 u - u_prev).  The square root must be rational (for
+    example b2 = 0, where sqrt(v_hat) = |q|)."""
+
+    def __init__(self, d: int, alpha, beta1, beta2, eps, adaptive: bool = True, bias_correction: bool = True):
+        self.alpha, self.b1, self.b2, self.eps = (Fraction(x) for x in (alpha, beta1, beta2, eps))
+        self.adaptive, self.bc = adaptive, bias_correction
+        self.m = [Fraction(0)] * d
+        self.v = [Fraction(0)] * d
+        self.u = [Fraction(0)] * d
+
+    def update(self, t: int, q_hat: Vec, w: Vec) -> Vec:
+        c1 = 1 - self.b1 ** t if self.bc else Fraction(1)
+        c2 = 1 - self.b2 ** t if self.bc else Fraction(1)
+        out = []
+        for j, (g, x) in enumerate(zip(q_hat, w)):
+            self.m[j] = self.b1 * self.m[j] + (1 - self.b1) * g
+            self.v[j] = self.b2 * self.v[j] + (1 - self.b2) * g * g
+            mh, vh = self.m[j] / c1, self.v[j] / c2
+            if self.adaptive:
+                u = Fraction(0) if mh == 0 else mh / (exact_sqrt(vh) + self.eps)
+            else:
+                u = mh
+            out.append(x - self.alpha * (2 * u - self.u[j]))
+            self.u[j] = u
+        return out

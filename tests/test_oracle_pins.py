@@ -889,3 +889,157 @@ def test_one_segment_is_the_flat_layout(comp):
         out.append((st.step(g, w), w))
     assert np.array_equal(out[0][0], out[1][0])
     assert np.array_equal(out[0][1], out[1][1])
+
+
+# ---------------------------------------------------------------------------
+# Optimistic Adam server update (the CPOAdam family of Section 4; the rule of
+# Daskalakis et al., ICLR 2018, fed the averaged update q_hat).
+# ---------------------------------------------------------------------------
+
+def dyadic(r, shape, bits=8, scale=1.0):
+    """Random values with at most `bits` significant bits (products and squares stay exact in fp32)."""
+    ints = r.integers(-(2 ** bits) + 1, 2 ** bits, size=shape)
+    ints[ints == 0] = 1
+    return (ints.astype(np.float64) * scale / 2 ** bits).astype(np.float32)
+
+
+def test_oadam_reduces_to_the_one_line_omd_recurrence():
+    """b1 = 0, identity preconditioner, alpha = 1, one worker, identity Q, the
+    gradient taken at the current iterate: Algorithm 2's server with this
+    update obeys w_{t+1} = w_t - 2 eta F(w_t) + eta F(w_{t-1}) (Section 2.2)
+    exactly (dyadic data: no operation rounds)."""
+    d, T = 8, 6
+    lr = 0.125
+    cfg = oracle.Config(d=d, M=1, compressor=oracle.IDENTITY, lr=lr)
+    st = oracle.State(cfg)
+    opt = oracle.OAdamState(d, oracle.OAdam(alpha=1.0, beta1=0.0, beta2=0.0, eps=0.0, adaptive=False,
+                                            bias_correction=False))
+    w = dyadic(rng(100), d, bits=6)
+    w_exact = exact.frac_vec(w)
+    F_prev = [Fraction(0)] * d
+    for t in range(1, T + 1):
+        F = bilinear_F(w_exact)
+        g = np.array([float(x) for x in F], np.float32)
+        msgs = st.compress_all(g[None, :])
+        q_hat = oracle.server_average(cfg, msgs)
+        opt.update(t, q_hat, w)
+        st.t += 1
+        w_exact = [x - 2 * Fraction(lr) * f + Fraction(lr) * fp for x, f, fp in zip(w_exact, F, F_prev)]
+        F_prev = F
+        assert [Fraction(float(x)) for x in w] == w_exact, t
+
+
+def test_oadam_first_step_is_a_signed_step():
+    """t = 1 with bias correction and eps = 0: m_hat = q, v_hat = q^2, so
+    u = sign(q) and w_1 = w_0 - 2 alpha sign(q) exactly (dyadic b1, b2)."""
+    d = 500
+    r = rng(101)
+    q = dyadic(r, d, bits=10, scale=2.0 ** -7)
+    w0 = dyadic(r, d, bits=12)
+    w = w0.copy()
+    st = oracle.OAdamState(d, oracle.OAdam(alpha=0.0625, beta1=0.5, beta2=0.75, eps=0.0))
+    st.update(1, q, w)
+    assert np.array_equal(st.u, np.sign(q).astype(np.float32))
+    assert np.array_equal(w, (w0 - np.float32(0.125) * np.sign(q)).astype(np.float32))
+
+
+def test_oadam_matches_the_exact_replay():
+    """b2 = 0 makes sqrt(v_hat) = |q| rational, so the rule can be replayed in
+    exact arithmetic; the fp32 oracle stays within a few roundings of it over
+    8 steps (adaptive and identity preconditioner, with and without bias
+    correction)."""
+    d, T = 16, 8
+    for adaptive in (True, False):
+        for bc in (True, False):
+            r = rng(102)
+            opt = oracle.OAdam(alpha=0.0625, beta1=0.75, beta2=0.0, eps=2.0 ** -6, adaptive=adaptive,
+                               bias_correction=bc)
+            st = oracle.OAdamState(d, opt)
+            ex = exact.ExactOAdam(d, opt.alpha, opt.beta1, opt.beta2, opt.eps, adaptive, bc)
+            w = dyadic(r, d, bits=10)
+            w_ex = exact.frac_vec(w)
+            for t in range(1, T + 1):
+                q = dyadic(r, d, bits=6, scale=2.0 ** -3)
+                st.update(t, q, w)
+                w_ex = ex.update(t, exact.frac_vec(q), w_ex)
+                scale = max(abs(x) for x in w_ex) + 1
+                err = max(abs(Fraction(float(a)) - b) for a, b in zip(w, w_ex))
+                assert err <= 64 * t * Fraction(U32) * scale, (adaptive, bc, t, float(err))
+
+
+def test_oadam_is_invariant_to_power_of_two_gradient_scaling():
+    """With eps = 0 the update u depends on q only through q / sqrt(E q^2):
+    scaling every q by 2^k scales m by 2^k, v by 4^k and leaves u and w bit
+    for bit unchanged (no operation rounds differently)."""
+    d, T = 1000, 6
+    qs = [(rng(103 + t).standard_normal(d) * 1e-3).astype(np.float32) for t in range(T)]
+    w0 = rng(110).standard_normal(d).astype(np.float32)
+    runs = []
+    for k in (0, 7, -9):
+        st = oracle.OAdamState(d, oracle.OAdam(alpha=1e-3, beta1=0.5, beta2=0.999, eps=0.0))
+        w = w0.copy()
+        for t, q in enumerate(qs, 1):
+            st.update(t, (q * np.float32(2.0 ** k)).astype(np.float32), w)
+        runs.append((w, st.u.copy()))
+    for w, u in runs[1:]:
+        assert np.array_equal(w.view(np.uint32), runs[0][0].view(np.uint32))
+        assert np.array_equal(u.view(np.uint32), runs[0][1].view(np.uint32))
+
+
+def test_oadam_is_odd_in_the_gradients():
+    """Negating every q and w_0 negates m, u and w exactly and leaves v."""
+    d, T = 777, 5
+    qs = [(rng(120 + t).standard_normal(d)).astype(np.float32) for t in range(T)]
+    w0 = rng(130).standard_normal(d).astype(np.float32)
+    opt = oracle.OAdam(alpha=1e-2, beta1=0.9, beta2=0.99, eps=1e-6)
+    a, b = oracle.OAdamState(d, opt), oracle.OAdamState(d, opt)
+    wa, wb = w0.copy(), (-w0).astype(np.float32)
+    for t, q in enumerate(qs, 1):
+        a.update(t, q, wa)
+        b.update(t, (-q).astype(np.float32), wb)
+    assert np.array_equal(wb, -wa) and np.array_equal(b.u, -a.u) and np.array_equal(b.m, -a.m)
+    assert np.array_equal(b.v, a.v)
+
+
+@pytest.mark.parametrize("beta1,beta2", [(0.5, 0.999), (0.9, 0.999), (0.0, 0.9), (0.9, 0.99)])
+def test_oadam_step_is_bounded(beta1, beta2):
+    """Cauchy-Schwarz on m_t = (1-b1) sum b1^(t-s) q_s against
+    v_t = (1-b2) sum b2^(t-s) q_s^2 bounds every update (eps = 0):
+    |u_t| <= (1-b1) sqrt(S_t) sqrt(1-b2^t) / ((1-b1^t) sqrt(1-b2)),
+    S_t = sum_{k<t} (b1^2/b2)^k -- for any gradients, heavy-tailed included."""
+    d, T = 4000, 12
+    r = rng(140)
+    st = oracle.OAdamState(d, oracle.OAdam(alpha=1e-3, beta1=beta1, beta2=beta2, eps=0.0))
+    w = np.zeros(d, np.float32)
+    for t in range(1, T + 1):
+        q = (r.standard_t(2, d) * 10.0 ** r.uniform(-4, 1, d)).astype(np.float32)
+        st.update(t, q, w)
+        S = sum((beta1 ** 2 / beta2) ** k for k in range(t))
+        bound = (1 - beta1) * math.sqrt(S) * math.sqrt(1 - beta2 ** t) / ((1 - beta1 ** t) * math.sqrt(1 - beta2))
+        assert np.max(np.abs(st.u)) <= bound * (1 + 1e-5), (t, float(np.max(np.abs(st.u))), bound)
+
+
+def test_oadam_bias_correction_power_is_a_running_product():
+    """b^t is the product of t factors: b^0 = 1, b^1 = b, and b^(t+1) = fl(b^t * b)."""
+    for b in (0.9, 0.999, 0.5):
+        assert oracle.pow_steps(b, 0) == 1.0 and oracle.pow_steps(b, 1) == np.float32(b)
+        for t in (2, 7, 100):
+            assert oracle.pow_steps(b, t) == np.float32(np.float32(oracle.pow_steps(b, t - 1)) * np.float32(b))
+
+
+def test_oadam_constant_gradient_gives_unit_steps():
+    """A constant gradient q: with bias correction m_hat_t = q and
+    v_hat_t = q^2 exactly at every t (the corrections undo the zero start),
+    so u_t = sign(q) and w_t = w_{t-1} - alpha sign(q) after the first step.
+    Powers of two for q and dyadic b1, b2 keep every operation exact."""
+    d, T = 64, 9
+    r = rng(150)
+    q = (np.where(r.random(d) < 0.5, -1.0, 1.0) * 2.0 ** r.integers(-12, 4, d)).astype(np.float32)
+    st = oracle.OAdamState(d, oracle.OAdam(alpha=0.125, beta1=0.5, beta2=0.75, eps=0.0))
+    w = np.zeros(d, np.float32)
+    for t in range(1, T + 1):
+        before = w.copy()
+        st.update(t, q, w)
+        assert np.array_equal(st.u, np.sign(q).astype(np.float32)), t
+        step = np.float32(0.125) * (np.float32(2.0 if t == 1 else 1.0) * np.sign(q)).astype(np.float32)
+        assert np.array_equal(w, (before - step).astype(np.float32)), t
