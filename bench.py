@@ -65,6 +65,9 @@ def parse_args():
     ap.add_argument("--sweep", action="store_true",
                     help="instead of the one-line result, print one line per d = 2^16 .. 2^27 "
                          "(M = 8, sign per 1024, DCGAN gradient law): the roofline curve")
+    ap.add_argument("--server", default="omd", choices=["omd", "oadam"],
+                    help="server update: Algorithm 2's w = w - q_hat, or Optimistic Adam on q_hat "
+                         "(alpha 1e-3, b1 0.5, b2 0.999, eps 1e-8, bias-corrected)")
     ap.add_argument("--override", action="append", default=[], metavar="FIELD=VALUE",
                     help="change a workload field (e.g. M=4 for a smaller profiling case)")
     return ap.parse_args()
@@ -115,8 +118,15 @@ def compress_bytes(wl, lookahead: bool) -> int:
     return wl.M * per_worker
 
 
-def server_bytes(wl) -> int:
-    """Read and write w, read all M messages (top-k: read and write only the touched w)."""
+OADAM = dict(alpha=1e-3, beta1=0.5, beta2=0.999, eps=1e-8)
+
+
+def server_bytes(wl, oadam: bool = False) -> int:
+    """Read and write w, read all M messages (top-k: read and write only the
+    touched w); Optimistic Adam also reads and writes m, v, u_prev of every
+    parameter (and so every w)."""
+    if oadam:
+        return 32 * wl.d + wl.M * message_payload_bytes(wl)
     if wl.compressor == TOPK:
         return wl.M * 8 * wl.k + 8 * min(wl.d, wl.M * wl.k)
     return 8 * wl.d + wl.M * message_payload_bytes(wl)
@@ -276,7 +286,7 @@ class OracleSteps:
     through ctypes, which releases the GIL).  The gradients are one seeded
     batch generated up front (outside any timing) and used at every step."""
 
-    def __init__(self, wl, threads: int):
+    def __init__(self, wl, threads: int, server: str = "omd"):
         from concurrent.futures import ThreadPoolExecutor
 
         import numpy as np
@@ -301,6 +311,7 @@ class OracleSteps:
         parts = 4 * threads
         cuts = sorted({wl.d * i // parts for i in range(parts + 1)})
         self.ranges = [(x, y) for x, y in zip(cuts[:-1], cuts[1:]) if y > x]
+        self.opt = oracle.OAdamState(wl.d, oracle.OAdam(**OADAM)) if server == "oadam" else None
         self.t = 1
 
     def step(self) -> float:
@@ -312,7 +323,11 @@ class OracleSteps:
 
         t0 = time.perf_counter()
         list(self.pool.map(worker, range(self.wl.M)))
-        list(self.pool.map(lambda r: oracle.server_step_range(cfg, self.msgs, self.w, r[0], r[1]), self.ranges))
+        if self.opt is None:
+            list(self.pool.map(lambda r: oracle.server_step_range(cfg, self.msgs, self.w, r[0], r[1]), self.ranges))
+        else:
+            list(self.pool.map(lambda r: self.opt.server_step_range(cfg, t, self.msgs, self.w, r[0], r[1]),
+                               self.ranges))
         dt = time.perf_counter() - t0
         self.t += 1
         return dt
@@ -365,11 +380,11 @@ def oracle_single_thread_estimate(wl, worker_fraction: float = 1 / 8, server_fra
     return step, sample
 
 
-def cpu_baseline_leg(wl):
+def cpu_baseline_leg(wl, server: str = "omd"):
     """The GPU arm's cpu_baseline: one whole step of the workload on all host
     cores (timed after one untimed step), and the one-thread projection."""
     threads = host_threads()
-    run = OracleSteps(wl, threads)
+    run = OracleSteps(wl, threads, server)
     run.step()
     dt = run.step()
     run.close()
@@ -388,7 +403,7 @@ def run_reference(args, rank, world):
         return 0
     wl = selected_workload(args)
     threads = host_threads()
-    run = OracleSteps(wl, threads)
+    run = OracleSteps(wl, threads, args.server)
     for _ in range(args.warmup):
         run.step()
     step_s = [run.step() for _ in range(args.steps)]
@@ -420,7 +435,9 @@ def workload_config(wl, args):
          "lookahead": bool(args.lookahead),
          "l2": ("not flushed: every step reads and writes more than twice the 129 MB L2" if big else
                 "flushed before every timed step (256 MB write, outside the timed region)"),
-         "parallelism": f"replicas{args.gpus}" if args.gpus > 1 else "single"}
+         "parallelism": f"replicas{args.gpus}" if args.gpus > 1 else "single",
+         "server": ("optimistic_adam " + ", ".join(f"{k} {v:g}" for k, v in OADAM.items()) + ", bias-corrected"
+                    if getattr(args, "server", "omd") == "oadam" else "omd: w = w - q_hat")}
     if wl.compressor in (SIGN, SQUANT, QSGD):
         c["bucket"] = wl.bucket
         c["buckets"] = "per layer segment" if wl.layer_buckets else "flat"
@@ -458,6 +475,8 @@ def run_gpu(args, rank, world, local):
                                cuda_stream=stream.cuda_stream))
     if wl.layer_buckets:
         h.set_segments(wl.segment_offsets())
+    if args.server == "oadam":
+        h.set_server_optimizer(P.dqgan.oadam(**OADAM))
     mb = h.message_bytes()
     msgs = torch.empty((wl.M, mb), dtype=torch.uint8, device=dev)
     w = wl.w0_torch(dev)
@@ -622,7 +641,7 @@ def run_gpu(args, rank, world, local):
     comp_avg = statistics.mean(comp_ms)
     serv_avg = statistics.mean(serv_ms)
     cb = compress_bytes(wl, args.lookahead)
-    sb = server_bytes(wl)
+    sb = server_bytes(wl, args.server == "oadam")
     timing = ("CUDA events around each launch, each step after an L2 flush" if need_flush else
               f"CUDA events around {args.steps} launches of the kernel back to back, averaged")
     comp_gbs = cb / (comp_avg / 1e3) / 1e9
@@ -632,12 +651,13 @@ def run_gpu(args, rank, world, local):
                 "achieved": comp_gbs, "peak": peak, "unit": "GB/s", "frac": comp_gbs / peak,
                 "traffic": traffic, "algorithmic_bytes": cb, "ms": comp_avg,
                 "peak_source": f"{peak_kind} hbm_gbs", "timing": timing}
-    roofline_server = {"bound": "hbm", "kernel": f"{COMPRESSOR_NAME[wl.compressor]}_server",
+    roofline_server = {"bound": "hbm", "kernel": f"{COMPRESSOR_NAME[wl.compressor]}_server"
+                                                  + ("_oadam" if args.server == "oadam" else ""),
                        "achieved": serv_gbs, "peak": peak, "unit": "GB/s", "frac": serv_gbs / peak,
                        "algorithmic_bytes": sb, "ms": serv_avg, "timing": timing}
     cpu = None
     if world == 1 and not args.no_cpu_baseline:
-        cpu = cpu_baseline_leg(wl)
+        cpu = cpu_baseline_leg(wl, args.server)
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
         "warmup": args.warmup, "ms_per_step": total_ms / args.steps, "higher_is_better": True,

@@ -138,7 +138,10 @@ DQGAN_API int dqgan_validate_config(const dqgan_config* cfg);
  * e_0 = 0), h (M x d fp32, zero, only with DQGAN_KEEP_LOOKAHEAD: F(w_{-1/2})
  * is taken as 0 so that w_{1/2} = w_0), and top-k scratch.  Sets t = 1.
  * *out receives the handle; on error *out is NULL and
- * dqgan_last_error(NULL) holds the reason.
+ * dqgan_last_error(NULL) holds the reason, and nothing stays allocated.
+ * Test hook: with the environment variable DQGAN_TEST_FAIL_ALLOC=N set, the
+ * N-th device allocation this thread makes from this call on (through later
+ * calls as well) fails as out of memory, once.
  */
 DQGAN_API int dqgan_create(const dqgan_config* cfg, dqgan_handle** out);
 
@@ -170,6 +173,34 @@ DQGAN_API int dqgan_worker_compress(dqgan_handle* h, int32_t i, const float* g, 
  */
 DQGAN_API int dqgan_workers_compress_all(dqgan_handle* h, const float* g_all, int64_t g_stride,
                                void* msgs_all);
+
+/*
+ * The worker step for workers first .. first + count - 1 in one launch per
+ * kernel stage (the part of Algorithm 2 one rank runs when the M workers are
+ * sharded over several GPUs: each rank compresses its workers into its rows
+ * of the message buffer, the ranks all-gather the messages -- the push and
+ * pull of Section 2.3 -- and every rank runs the same server step).
+ * g:    worker first + r's gradient at g + r * g_stride (floats), device or
+ *       pinned host memory; g_stride >= d and a multiple of 4.
+ * msgs: device, worker first + r's message at msgs + r * dqgan_message_bytes().
+ * The workers must lie in the handle's local range (all M unless
+ * dqgan_set_local_workers chose fewer).
+ */
+DQGAN_API int dqgan_workers_compress_range(dqgan_handle* h, int32_t first, int32_t count, const float* g,
+                                           int64_t g_stride, void* msgs);
+
+/*
+ * Keep the worker state (residuals e, lookahead offsets h, top-k scratch) of
+ * workers first .. first + count - 1 only, instead of all M: the handle of
+ * one rank when the M workers are sharded over several GPUs.  The server
+ * step still averages all M messages.  Only before the first step (step
+ * counter 1, else DQGAN_ERR_INVALID_ARG); replaces the state with zeroed
+ * rows for the range (DQGAN_ERR_OOM if that fails; the handle then keeps its
+ * old state).  Afterwards the per-worker calls accept only workers in the
+ * range, dqgan_workers_compress_all is refused unless the range is all M,
+ * and the checkpoint state holds the range's rows.  Synchronous.
+ */
+DQGAN_API int dqgan_set_local_workers(dqgan_handle* h, int32_t first, int32_t count);
 
 /*
  * Server step of Algorithm 2, fused: decode the M messages, average them
@@ -231,8 +262,11 @@ DQGAN_API int dqgan_set_step(dqgan_handle* h, int64_t t);
 
 /*
  * Checkpoint / resume.  The state is a 64-byte header (magic, d, M,
- * compressor, flags, t) followed by e (M x d fp32) and, with
- * DQGAN_KEEP_LOOKAHEAD, h (M x d fp32).  host buffers of at least
+ * compressor, flags, t, server rule, local worker range) followed by e
+ * (one d fp32 row per local worker), with DQGAN_KEEP_LOOKAHEAD h (the same
+ * rows), and under DQGAN_SERVER_OADAM m, v and
+ * u_prev (d fp32 each; the rule's parameters are not stored: set the same
+ * rule on the handle before loading).  host buffers of at least
  * dqgan_state_bytes() bytes.  Synchronous.  Loading checks that the header
  * matches the handle's config (else DQGAN_ERR_INVALID_ARG).
  */
@@ -258,6 +292,56 @@ DQGAN_API int dqgan_load_state(dqgan_handle* h, const void* host_src, int64_t by
  * With segments the servers take their per-element scale-lookup paths.
  */
 DQGAN_API int dqgan_set_segments(dqgan_handle* h, const int64_t* offsets, int32_t nseg);
+
+/*
+ * Server update rule.  Algorithm 2's server steps w = fl(w - q_hat)
+ * (DQGAN_SERVER_OMD, the default).  DQGAN_SERVER_OADAM replaces that step by
+ * Optimistic Adam on the averaged update q_hat -- the optimizer family of the
+ * CPOAdam systems Section 4 compares against, for which the paper prints no
+ * rule; this is the rule of Daskalakis, Ilyas, Syrgkanis and Zeng, "Training
+ * GANs with Optimism" (ICLR 2018).  Per parameter j, in fp32 with one
+ * rounding per operation in this order (one dense pass after the server
+ * kernel, which then writes q_hat to a library-owned buffer):
+ *   m = b1 m + (1 - b1) q_hat;   v = b2 v + ((1 - b2) q_hat) q_hat;
+ *   m_hat = m / (1 - b1^t), v_hat = v / (1 - b2^t)   (DQGAN_OADAM_BIAS_CORRECTION,
+ *                                    b^t the fp32 product of t factors, t the step);
+ *   u = m_hat / (sqrt(v_hat) + eps), u = 0 where m_hat = 0   (DQGAN_OADAM_ADAPTIVE),
+ *   else u = m_hat;
+ *   w = w - alpha (2 u - u_prev);   u_prev = u.
+ * m, v and u_prev start at 0 and are library-owned (with the q_hat buffer,
+ * 4 x d fp32).  With
+ * b1 = 0, no DQGAN_OADAM_ADAPTIVE and alpha = 1 the update is
+ * w_t = w_{t-1} - 2 q_hat_t + q_hat_{t-1}, the one-line OMD recurrence of
+ * Section 2.2.  With top-k messages every parameter moves, not only the
+ * indices sent.  28 bytes, no implicit padding.
+ */
+#define DQGAN_SERVER_OMD 0
+#define DQGAN_SERVER_OADAM 1
+#define DQGAN_OADAM_ADAPTIVE 1u
+#define DQGAN_OADAM_BIAS_CORRECTION 2u
+
+typedef struct dqgan_server_optimizer {
+  int32_t kind;    /* DQGAN_SERVER_OMD or DQGAN_SERVER_OADAM */
+  uint32_t flags;  /* DQGAN_OADAM_ADAPTIVE | DQGAN_OADAM_BIAS_CORRECTION */
+  float alpha;     /* step size, finite */
+  float beta1;     /* in [0, 1) */
+  float beta2;     /* in [0, 1) */
+  float eps;       /* >= 0, finite */
+  uint32_t reserved; /* 0 */
+} dqgan_server_optimizer;
+
+/* Choose the server update rule; only before the first step (step counter
+ * 1, else DQGAN_ERR_INVALID_ARG).  DQGAN_SERVER_OADAM allocates m, v, u_prev
+ * and the q_hat buffer (4 x d fp32, zero; DQGAN_ERR_OOM if that fails) and
+ * adds m, v, u_prev to the
+ * checkpoint state; DQGAN_SERVER_OMD frees them.  DQGAN_ERR_UNSUPPORTED for
+ * DQGAN_TOPK with more than 64 workers.  Synchronous. */
+DQGAN_API int dqgan_set_server_optimizer(dqgan_handle* h, const dqgan_server_optimizer* opt);
+
+/* Copy the Optimistic Adam state to dst (host or device, d fp32):
+ * which = 0: m, 1: v, 2: u_prev.  DQGAN_ERR_UNSUPPORTED under DQGAN_SERVER_OMD.
+ * Synchronous. */
+DQGAN_API int dqgan_get_server_state(dqgan_handle* h, int32_t which, float* dst);
 
 /* Kernels this handle has launched so far. */
 DQGAN_API uint64_t dqgan_launch_count(const dqgan_handle* h);

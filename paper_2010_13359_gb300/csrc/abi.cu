@@ -38,6 +38,15 @@ struct dqgan_handle {
   const float* params_map_w = nullptr;
   bool params_map_ok = false;
   int32_t sign_path = 0;         // DQGAN_SIGN_SERVER at creation: 0 auto, 1 col, 2 tma
+  dqgan_server_optimizer opt{};  // server update rule (kind DQGAN_SERVER_OMD: w = w - q_hat)
+  float* opt_m = nullptr;        // Optimistic Adam: m, v, u_prev and the server's q_hat
+  float* opt_v = nullptr;        // (d fp32 each, rows of one allocation)
+  float* opt_u = nullptr;
+  float* opt_q = nullptr;
+  float pow1 = 1.f, pow2 = 1.f;  // b1^pow_t, b2^pow_t as fp32 running products
+  int64_t pow_t = 0;
+  int32_t row0 = 0;              // the handle holds the state of workers [row0, row0 + nlocal)
+  int32_t nlocal = 0;            // (all M unless dqgan_set_local_workers chose a range)
   int64_t t = 1;
   uint64_t launches = 0;
   std::string err;
@@ -66,6 +75,38 @@ int set_error(dqgan_handle* h, int code, const char* fmt, ...) {
   if (h) h->err = buf;
   else tl_err = buf;
   return code;
+}
+
+// Every device allocation of the library goes through dq_malloc.  For the
+// tests of the out-of-memory paths, the environment variable
+// DQGAN_TEST_FAIL_ALLOC=N, read by dqgan_create, makes the N-th allocation
+// made by this thread from then on fail with cudaErrorMemoryAllocation
+// (nothing is allocated); N counts on through later calls such as
+// dqgan_set_segments, and the hook is spent once it fires.
+thread_local int64_t tl_fail_countdown = 0;
+
+void arm_allocation_failure() {
+  tl_fail_countdown = 0;
+  if (const char* v = std::getenv("DQGAN_TEST_FAIL_ALLOC")) {
+    const long long n = std::atoll(v);
+    if (n > 0) tl_fail_countdown = n;
+  }
+}
+
+cudaError_t dq_malloc(void** p, size_t bytes) {
+  if (tl_fail_countdown > 0 && --tl_fail_countdown == 0) {
+    *p = nullptr;
+    return cudaErrorMemoryAllocation;
+  }
+  return cudaMalloc(p, bytes);
+}
+
+template <typename T>
+cudaError_t dq_malloc(T** p, size_t bytes) {
+  void* q = nullptr;
+  const cudaError_t st = dq_malloc(&q, bytes);
+  *p = static_cast<T*>(q);
+  return st;
 }
 
 bool is_pow2(int64_t x) { return x > 0 && (x & (x - 1)) == 0; }
@@ -138,6 +179,7 @@ dq::CompressArgs compress_args(dqgan_handle* h, const float* g, int64_t g_stride
   a.bits = h->cfg.bits;
   a.worker0 = worker0;
   a.nworkers = nworkers;
+  a.row0 = h->row0;
   a.seed_lo = (uint32_t)(h->cfg.seed & 0xFFFFFFFFu);
   a.seed_hi = (uint32_t)(h->cfg.seed >> 32);
   a.step = (uint32_t)h->t;
@@ -165,13 +207,14 @@ int run_compress(dqgan_handle* h, const dq::CompressArgs& a) {
 }
 
 int check_worker(dqgan_handle* h, int32_t i) {
-  if (i < 0 || i >= h->cfg.M)
-    return set_error(h, DQGAN_ERR_INVALID_ARG, "worker %d outside [0, %d)", i, h->cfg.M);
+  if (i < h->row0 || i >= h->row0 + h->nlocal)
+    return set_error(h, DQGAN_ERR_INVALID_ARG, "worker %d outside the handle's workers [%d, %d)", i, h->row0,
+                     h->row0 + h->nlocal);
   return DQGAN_OK;
 }
 
 int copy_rows(dqgan_handle* h, float* base, int32_t i, void* dst, const void* src) {
-  float* row = base + (int64_t)i * h->ld;
+  float* row = base + (int64_t)(i - h->row0) * h->ld;
   cudaError_t st;
   if (dst) st = cudaMemcpyAsync(dst, row, (size_t)h->cfg.d * 4, cudaMemcpyDefault, h->stream);
   else st = cudaMemcpyAsync(row, src, (size_t)h->cfg.d * 4, cudaMemcpyDefault, h->stream);
@@ -179,6 +222,52 @@ int copy_rows(dqgan_handle* h, float* base, int32_t i, void* dst, const void* sr
   st = cudaStreamSynchronize(h->stream);
   if (st != cudaSuccess) return cuda_fail(h, st, "copy sync");
   return DQGAN_OK;
+}
+
+// b^t as the fp32 product of t factors, t the handle's step (the bias
+// corrections of Optimistic Adam); advanced one factor per step, recomputed
+// after the step counter is set.
+void advance_powers(dqgan_handle* h) {
+  if (h->pow_t > h->t) {
+    h->pow1 = h->pow2 = 1.f;
+    h->pow_t = 0;
+  }
+  while (h->pow_t < h->t) {
+    const float n1 = h->pow1 * h->opt.beta1, n2 = h->pow2 * h->opt.beta2;
+    if (n1 == h->pow1 && n2 == h->pow2) {  // a fixed point (0, or a subnormal that rounds to itself)
+      h->pow_t = h->t;
+      break;
+    }
+    h->pow1 = n1;
+    h->pow2 = n2;
+    ++h->pow_t;
+  }
+}
+
+dq::OAdamArgs oadam_args(dqgan_handle* h, float* params) {
+  advance_powers(h);
+  dq::OAdamArgs a{};
+  a.q = h->opt_q;
+  a.w = params;
+  a.m = h->opt_m;
+  a.v = h->opt_v;
+  a.u = h->opt_u;
+  a.d = h->cfg.d;
+  a.alpha = h->opt.alpha;
+  a.beta1 = h->opt.beta1;
+  a.one_m_beta1 = 1.f - h->opt.beta1;
+  a.beta2 = h->opt.beta2;
+  a.one_m_beta2 = 1.f - h->opt.beta2;
+  a.eps = h->opt.eps;
+  a.bias_correction = (h->opt.flags & DQGAN_OADAM_BIAS_CORRECTION) ? 1 : 0;
+  a.adaptive = (h->opt.flags & DQGAN_OADAM_ADAPTIVE) ? 1 : 0;
+  a.c1 = a.bias_correction ? 1.f - h->pow1 : 1.f;
+  a.c2 = a.bias_correction ? 1.f - h->pow2 : 1.f;
+  return a;
+}
+
+int64_t opt_state_floats(const dqgan_handle* h) {
+  return h->opt_m ? 3 * h->cfg.d : 0;
 }
 
 struct StateHeader {
@@ -191,9 +280,11 @@ struct StateHeader {
   int32_t bucket;
   int32_t bits;
   uint32_t flags;
-  uint32_t reserved;
+  uint32_t server_kind;  // DQGAN_SERVER_OMD, or DQGAN_SERVER_OADAM (then m, v, u_prev follow e and h)
+  int32_t row0;          // the local workers [row0, row0 + nlocal) whose rows follow
+  int32_t nlocal;
 };
-static_assert(sizeof(StateHeader) == 56, "state header layout");
+static_assert(sizeof(StateHeader) == 64, "state header layout");
 constexpr int64_t kHeaderBytes = 64;
 
 }  // namespace
@@ -256,6 +347,7 @@ int dqgan_create(const dqgan_config* cfg, dqgan_handle** out) {
   *out = nullptr;
   const std::string why = check_config(cfg);
   if (!why.empty()) return set_error(nullptr, DQGAN_ERR_INVALID_ARG, "%s", why.c_str());
+  arm_allocation_failure();
   dqgan_handle* h = new (std::nothrow) dqgan_handle();
   if (!h) return set_error(nullptr, DQGAN_ERR_OOM, "host allocation failed");
   h->cfg = *cfg;
@@ -283,14 +375,14 @@ int dqgan_create(const dqgan_config* cfg, dqgan_handle** out) {
     return set_error(nullptr, e == cudaErrorMemoryAllocation ? DQGAN_ERR_OOM : DQGAN_ERR_CUDA,
                      "%s: %s", what, cudaGetErrorString(e));
   };
-  if ((st = cudaMalloc(&h->err_word, 256)) != cudaSuccess) return fail_oom("allocating the error word", st);
+  if ((st = dq_malloc(&h->err_word, 256)) != cudaSuccess) return fail_oom("allocating the error word", st);
   if ((st = cudaMemsetAsync(h->err_word, 0, 256, h->stream)) != cudaSuccess) return fail_oom("zeroing the error word", st);
-  if ((st = cudaMalloc(&h->e, rows_bytes)) != cudaSuccess) return fail_oom("allocating e", st);
+  if ((st = dq_malloc(&h->e, rows_bytes)) != cudaSuccess) return fail_oom("allocating e", st);
   if (cfg->flags & DQGAN_KEEP_LOOKAHEAD)
-    if ((st = cudaMalloc(&h->h, rows_bytes)) != cudaSuccess) return fail_oom("allocating h", st);
+    if ((st = dq_malloc(&h->h, rows_bytes)) != cudaSuccess) return fail_oom("allocating h", st);
   if (cfg->compressor == DQGAN_TOPK) {
-    h->scratch_bytes = dq::topk_scratch_bytes(cfg->d, cfg->M);
-    if ((st = cudaMalloc(&h->scratch, h->scratch_bytes)) != cudaSuccess)
+    h->scratch_bytes = dq::topk_scratch_bytes(cfg->d, cfg->M, cfg->M);
+    if ((st = dq_malloc(&h->scratch, h->scratch_bytes)) != cudaSuccess)
       return fail_oom("allocating top-k scratch", st);
   }
   if ((st = cudaMemsetAsync(h->e, 0, rows_bytes, h->stream)) != cudaSuccess) return fail_oom("zeroing e", st);
@@ -300,6 +392,8 @@ int dqgan_create(const dqgan_config* cfg, dqgan_handle** out) {
     return fail_oom("zeroing scratch", st);
   if ((st = cudaStreamSynchronize(h->stream)) != cudaSuccess) return fail_oom("create sync", st);
   h->t = 1;
+  h->row0 = 0;
+  h->nlocal = cfg->M;
   *out = h;
   return DQGAN_OK;
 }
@@ -314,6 +408,7 @@ int dqgan_destroy(dqgan_handle* h) {
   if (h->seg_bstart) cudaFree(h->seg_bstart);
   if (h->seg_wbucket) cudaFree(h->seg_wbucket);
   if (h->seg_slices) cudaFree(h->seg_slices);
+  if (h->opt_m) cudaFree(h->opt_m);
   const cudaError_t st = cudaGetLastError();
   delete h;
   if (st != cudaSuccess) return set_error(nullptr, DQGAN_ERR_CUDA, "destroy: %s", cudaGetErrorString(st));
@@ -375,9 +470,9 @@ int dqgan_set_segments(dqgan_handle* h, const int64_t* offsets, int32_t nseg) {
         slices.push_back((uint32_t)b | (uint32_t)(rows - 1) << 27);
       }
     }
-  if ((st = cudaMalloc(&h->seg_bstart, starts.size() * sizeof(int64_t))) != cudaSuccess ||
-      (st = cudaMalloc(&h->seg_wbucket, wb.size() * sizeof(uint32_t))) != cudaSuccess ||
-      (!slices.empty() && (st = cudaMalloc(&h->seg_slices, slices.size() * sizeof(uint32_t))) != cudaSuccess)) {
+  if ((st = dq_malloc(&h->seg_bstart, starts.size() * sizeof(int64_t))) != cudaSuccess ||
+      (st = dq_malloc(&h->seg_wbucket, wb.size() * sizeof(uint32_t))) != cudaSuccess ||
+      (!slices.empty() && (st = dq_malloc(&h->seg_slices, slices.size() * sizeof(uint32_t))) != cudaSuccess)) {
     if (h->seg_bstart) cudaFree(h->seg_bstart);
     if (h->seg_wbucket) cudaFree(h->seg_wbucket);
     h->seg_bstart = nullptr;
@@ -426,7 +521,64 @@ int dqgan_workers_compress_all(dqgan_handle* h, const float* g_all, int64_t g_st
   if (g_stride < h->cfg.d || (g_stride & 3))
     return set_error(h, DQGAN_ERR_INVALID_ARG, "g_stride = %lld must be >= d and a multiple of 4",
                      (long long)g_stride);
+  if (h->nlocal != h->cfg.M)
+    return set_error(h, DQGAN_ERR_INVALID_ARG, "the handle holds workers [%d, %d) only: use dqgan_workers_compress_range",
+                     h->row0, h->row0 + h->nlocal);
   return run_compress(h, compress_args(h, g_all, g_stride, msgs_all, h->lay.total, 0, h->cfg.M));
+}
+
+int dqgan_workers_compress_range(dqgan_handle* h, int32_t first, int32_t count, const float* g, int64_t g_stride,
+                                 void* msgs) {
+  if (!h) return set_error(nullptr, DQGAN_ERR_INVALID_ARG, "handle is NULL");
+  if (count < 1 || first < h->row0 || (int64_t)first + count > (int64_t)h->row0 + h->nlocal)
+    return set_error(h, DQGAN_ERR_INVALID_ARG, "workers [%d, %d) outside the handle's workers [%d, %d)", first,
+                     first + count, h->row0, h->row0 + h->nlocal);
+  if (!g || !msgs) return set_error(h, DQGAN_ERR_INVALID_ARG, "NULL gradient or message pointer");
+  if (!aligned16(g) || !aligned16(msgs))
+    return set_error(h, DQGAN_ERR_INVALID_ARG, "gradients and messages must be 16-byte aligned");
+  if (g_stride < h->cfg.d || (g_stride & 3))
+    return set_error(h, DQGAN_ERR_INVALID_ARG, "g_stride = %lld must be >= d and a multiple of 4",
+                     (long long)g_stride);
+  return run_compress(h, compress_args(h, g, g_stride, msgs, h->lay.total, first, count));
+}
+
+int dqgan_set_local_workers(dqgan_handle* h, int32_t first, int32_t count) {
+  if (!h) return set_error(nullptr, DQGAN_ERR_INVALID_ARG, "handle is NULL");
+  if (h->t != 1) return set_error(h, DQGAN_ERR_INVALID_ARG, "local workers must be set before the first step");
+  if (count < 1 || first < 0 || (int64_t)first + count > h->cfg.M)
+    return set_error(h, DQGAN_ERR_INVALID_ARG, "workers [%d, %d) outside [0, %d)", first, first + count, h->cfg.M);
+  cudaError_t st = cudaStreamSynchronize(h->stream);  // no step in flight
+  if (st != cudaSuccess) return cuda_fail(h, st, "synchronize");
+  const size_t rows_bytes = (size_t)count * (size_t)h->ld * sizeof(float);
+  const size_t scratch_bytes =
+      h->cfg.compressor == DQGAN_TOPK ? dq::topk_scratch_bytes(h->cfg.d, count, h->cfg.M) : 0;
+  float *e = nullptr, *hh = nullptr;
+  void* scratch = nullptr;
+  auto fail = [&](const char* what, cudaError_t err) {
+    cudaGetLastError();
+    if (e) cudaFree(e);
+    if (hh) cudaFree(hh);
+    if (scratch) cudaFree(scratch);
+    return set_error(h, err == cudaErrorMemoryAllocation ? DQGAN_ERR_OOM : DQGAN_ERR_CUDA, "%s: %s", what,
+                     cudaGetErrorString(err));
+  };
+  if ((st = dq_malloc(&e, rows_bytes)) != cudaSuccess) return fail("allocating e", st);
+  if (h->h && (st = dq_malloc(&hh, rows_bytes)) != cudaSuccess) return fail("allocating h", st);
+  if (scratch_bytes && (st = dq_malloc(&scratch, scratch_bytes)) != cudaSuccess)
+    return fail("allocating top-k scratch", st);
+  if ((st = cudaMemset(e, 0, rows_bytes)) != cudaSuccess || (hh && (st = cudaMemset(hh, 0, rows_bytes)) != cudaSuccess) ||
+      (scratch && (st = cudaMemset(scratch, 0, scratch_bytes)) != cudaSuccess))
+    return fail("zeroing the worker state", st);
+  cudaFree(h->e);
+  if (h->h) cudaFree(h->h);
+  if (h->scratch) cudaFree(h->scratch);
+  h->e = e;
+  h->h = hh;
+  h->scratch = scratch;
+  h->scratch_bytes = scratch_bytes;
+  h->row0 = first;
+  h->nlocal = count;
+  return DQGAN_OK;
 }
 
 int dqgan_server_aggregate_update(dqgan_handle* h, const void* msgs_all, float* params) {
@@ -451,6 +603,14 @@ int dqgan_server_aggregate_update(dqgan_handle* h, const void* msgs_all, float* 
   s.word_bucket = h->seg_wbucket;
   s.sign_words_map = nullptr;
   s.squant_words_map = nullptr;
+  // Optimistic Adam: the server kernel writes q_hat to the handle's buffer,
+  // then one dense pass updates m, v, u_prev and the parameters
+  const bool oadam = h->opt_m != nullptr;
+  if (oadam) {
+    s.w = h->opt_q;
+    s.store_q = 1;
+  }
+  float* const target = s.w;
   const bool flat = h->seg_wbucket == nullptr;
   // sign, buckets >= 1024, M <= 32: the TMA kernels (flat: 32-word boxes,
   // 128-byte swizzle; layer segments: 36-word boxes without swizzle)
@@ -475,10 +635,10 @@ int dqgan_server_aggregate_update(dqgan_handle* h, const void* msgs_all, float* 
   // 32 * (32 / b) elements for the b = 2, 4 quantiser server
   const bool boxed_squant = tma_squant && s.squant_words_map && h->cfg.bits != 8;
   if (((tma_sign && s.sign_words_map) || boxed_squant) && s.d >= 32) {
-    if (h->params_map_w != params) {
+    if (h->params_map_w != target) {
       const int32_t rows = boxed_squant ? 32 / h->cfg.bits : 32;
-      h->params_map_ok = dq::encode_params_map(params, s.d, rows, &h->params_map);
-      h->params_map_w = params;
+      h->params_map_ok = dq::encode_params_map(target, s.d, rows, &h->params_map);
+      h->params_map_w = target;
     }
     if (h->params_map_ok) x.params_map = &h->params_map;
   }
@@ -488,9 +648,13 @@ int dqgan_server_aggregate_update(dqgan_handle* h, const void* msgs_all, float* 
     case DQGAN_SQUANT:
     case DQGAN_QSGD: st = dq::launch_squant_server(s, x.params_map, h->stream, &h->launches); break;
     case DQGAN_IDENTITY: st = dq::launch_identity_server(s, h->stream, &h->launches); break;
-    case DQGAN_TOPK: st = dq::launch_topk_server(s, h->scratch, h->stream, &h->launches); break;
+    case DQGAN_TOPK: st = dq::launch_topk_server(s, h->scratch, h->nlocal, h->stream, &h->launches); break;
   }
   if (st != cudaSuccess) return cuda_fail(h, st, "server launch");
+  if (oadam) {
+    st = dq::launch_oadam_update(oadam_args(h, params), h->stream, &h->launches);
+    if (st != cudaSuccess) return cuda_fail(h, st, "optimizer launch");
+  }
   h->t += 1;
   return DQGAN_OK;
 }
@@ -577,8 +741,8 @@ int dqgan_set_step(dqgan_handle* h, int64_t t) {
 
 int64_t dqgan_state_bytes(const dqgan_handle* h) {
   if (!h) return -1;
-  const int64_t rows = (int64_t)h->cfg.M * h->cfg.d * 4;
-  return kHeaderBytes + rows * (h->h ? 2 : 1);
+  const int64_t rows = (int64_t)h->nlocal * h->cfg.d * 4;
+  return kHeaderBytes + rows * (h->h ? 2 : 1) + 4 * opt_state_floats(h);
 }
 
 int dqgan_save_state(dqgan_handle* h, void* host_dst, int64_t bytes) {
@@ -597,16 +761,24 @@ int dqgan_save_state(dqgan_handle* h, void* host_dst, int64_t bytes) {
   hd.bucket = h->cfg.bucket;
   hd.bits = h->cfg.bits;
   hd.flags = h->cfg.flags;
+  hd.server_kind = h->opt_m ? (uint32_t)DQGAN_SERVER_OADAM : (uint32_t)DQGAN_SERVER_OMD;
+  hd.row0 = h->row0;
+  hd.nlocal = h->nlocal;
   memset(dst, 0, kHeaderBytes);
   memcpy(dst, &hd, sizeof hd);
   const size_t row = (size_t)h->cfg.d * 4;
   uint8_t* out = dst + kHeaderBytes;
   for (int which = 0; which < (h->h ? 2 : 1); ++which) {
     float* base = which == 0 ? h->e : h->h;
-    cudaError_t st = cudaMemcpy2DAsync(out, row, base, (size_t)h->ld * 4, row, (size_t)h->cfg.M,
+    cudaError_t st = cudaMemcpy2DAsync(out, row, base, (size_t)h->ld * 4, row, (size_t)h->nlocal,
                                        cudaMemcpyDefault, h->stream);
     if (st != cudaSuccess) return cuda_fail(h, st, "save state copy");
-    out += row * (size_t)h->cfg.M;
+    out += row * (size_t)h->nlocal;
+  }
+  if (h->opt_m) {
+    cudaError_t st = cudaMemcpy2DAsync(out, row, h->opt_m, (size_t)round_up(h->cfg.d, 64) * 4, row, 3,
+                                       cudaMemcpyDefault, h->stream);  // m, v, u_prev rows
+    if (st != cudaSuccess) return cuda_fail(h, st, "save state copy");
   }
   const cudaError_t st = cudaStreamSynchronize(h->stream);
   if (st != cudaSuccess) return cuda_fail(h, st, "save state sync");
@@ -623,20 +795,79 @@ int dqgan_load_state(dqgan_handle* h, const void* host_src, int64_t bytes) {
   memcpy(&hd, src, sizeof hd);
   if (memcmp(hd.magic, "DQGANST1", 8) != 0 || hd.d != h->cfg.d || hd.M != h->cfg.M ||
       hd.compressor != h->cfg.compressor || hd.flags != h->cfg.flags || hd.k != h->cfg.k ||
-      hd.bucket != h->cfg.bucket || hd.bits != h->cfg.bits || hd.t < 1)
+      hd.bucket != h->cfg.bucket || hd.bits != h->cfg.bits || hd.t < 1 ||
+      hd.server_kind != (h->opt_m ? (uint32_t)DQGAN_SERVER_OADAM : (uint32_t)DQGAN_SERVER_OMD) ||
+      hd.row0 != h->row0 || hd.nlocal != h->nlocal)
     return set_error(h, DQGAN_ERR_INVALID_ARG, "state header does not match this handle's config");
   const size_t row = (size_t)h->cfg.d * 4;
   const uint8_t* in = src + kHeaderBytes;
   for (int which = 0; which < (h->h ? 2 : 1); ++which) {
     float* base = which == 0 ? h->e : h->h;
-    cudaError_t st = cudaMemcpy2DAsync(base, (size_t)h->ld * 4, in, row, row, (size_t)h->cfg.M,
+    cudaError_t st = cudaMemcpy2DAsync(base, (size_t)h->ld * 4, in, row, row, (size_t)h->nlocal,
                                        cudaMemcpyDefault, h->stream);
     if (st != cudaSuccess) return cuda_fail(h, st, "load state copy");
-    in += row * (size_t)h->cfg.M;
+    in += row * (size_t)h->nlocal;
+  }
+  if (h->opt_m) {
+    cudaError_t st = cudaMemcpy2DAsync(h->opt_m, (size_t)round_up(h->cfg.d, 64) * 4, in, row, row, 3,
+                                       cudaMemcpyDefault, h->stream);  // m, v, u_prev rows
+    if (st != cudaSuccess) return cuda_fail(h, st, "load state copy");
   }
   const cudaError_t st = cudaStreamSynchronize(h->stream);
   if (st != cudaSuccess) return cuda_fail(h, st, "load state sync");
   h->t = hd.t;
+  h->pow_t = h->t + 1;  // recompute b^t at the next server step
+  return DQGAN_OK;
+}
+
+int dqgan_set_server_optimizer(dqgan_handle* h, const dqgan_server_optimizer* opt) {
+  if (!h) return set_error(nullptr, DQGAN_ERR_INVALID_ARG, "handle is NULL");
+  if (!opt) return set_error(h, DQGAN_ERR_INVALID_ARG, "optimizer is NULL");
+  if (h->t != 1) return set_error(h, DQGAN_ERR_INVALID_ARG, "the server rule must be set before the first step");
+  if (opt->kind != DQGAN_SERVER_OMD && opt->kind != DQGAN_SERVER_OADAM)
+    return set_error(h, DQGAN_ERR_INVALID_ARG, "unknown server rule %d", opt->kind);
+  if (opt->kind == DQGAN_SERVER_OADAM) {
+    if (opt->flags & ~(DQGAN_OADAM_ADAPTIVE | DQGAN_OADAM_BIAS_CORRECTION) || opt->reserved != 0)
+      return set_error(h, DQGAN_ERR_INVALID_ARG, "unknown optimizer flag bits");
+    if (!std::isfinite(opt->alpha) || !std::isfinite(opt->eps) || opt->eps < 0.f)
+      return set_error(h, DQGAN_ERR_INVALID_ARG, "alpha must be finite and eps finite and >= 0");
+    if (!(opt->beta1 >= 0.f && opt->beta1 < 1.f) || !(opt->beta2 >= 0.f && opt->beta2 < 1.f))
+      return set_error(h, DQGAN_ERR_INVALID_ARG, "beta1 and beta2 must lie in [0, 1)");
+    if (h->cfg.compressor == DQGAN_TOPK && h->cfg.M > 64)
+      return set_error(h, DQGAN_ERR_UNSUPPORTED, "Optimistic Adam with top-k messages takes at most 64 workers");
+  }
+  cudaError_t st = cudaStreamSynchronize(h->stream);  // no step in flight
+  if (st != cudaSuccess) return cuda_fail(h, st, "synchronize");
+  if (h->opt_m) cudaFree(h->opt_m);
+  h->opt_m = h->opt_v = h->opt_u = h->opt_q = nullptr;
+  h->opt = *opt;
+  h->pow1 = h->pow2 = 1.f;
+  h->pow_t = 0;
+  if (opt->kind == DQGAN_SERVER_OMD) return DQGAN_OK;
+  const int64_t ld = round_up(h->cfg.d, 64);
+  if ((st = dq_malloc(&h->opt_m, (size_t)(4 * ld) * 4)) != cudaSuccess) {
+    cudaGetLastError();
+    h->opt_m = nullptr;
+    h->opt.kind = DQGAN_SERVER_OMD;
+    return set_error(h, st == cudaErrorMemoryAllocation ? DQGAN_ERR_OOM : DQGAN_ERR_CUDA,
+                     "allocating the optimizer state: %s", cudaGetErrorString(st));
+  }
+  h->opt_v = h->opt_m + ld;
+  h->opt_u = h->opt_v + ld;
+  h->opt_q = h->opt_u + ld;
+  if ((st = cudaMemset(h->opt_m, 0, (size_t)(4 * ld) * 4)) != cudaSuccess)
+    return cuda_fail(h, st, "zeroing the optimizer state");
+  return DQGAN_OK;
+}
+
+int dqgan_get_server_state(dqgan_handle* h, int32_t which, float* dst) {
+  if (!h) return set_error(nullptr, DQGAN_ERR_INVALID_ARG, "handle is NULL");
+  if (!h->opt_m) return set_error(h, DQGAN_ERR_UNSUPPORTED, "the server rule keeps no state");
+  if (which < 0 || which > 2 || !dst) return set_error(h, DQGAN_ERR_INVALID_ARG, "which must be 0, 1 or 2 and dst set");
+  const float* src = which == 0 ? h->opt_m : (which == 1 ? h->opt_v : h->opt_u);
+  cudaError_t st = cudaMemcpyAsync(dst, src, (size_t)h->cfg.d * 4, cudaMemcpyDefault, h->stream);
+  if (st == cudaSuccess) st = cudaStreamSynchronize(h->stream);
+  if (st != cudaSuccess) return cuda_fail(h, st, "copying the optimizer state");
   return DQGAN_OK;
 }
 

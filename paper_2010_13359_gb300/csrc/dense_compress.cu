@@ -131,8 +131,8 @@ sign_compress_kernel(const CompressArgs a) {
   const int row = blockIdx.y;
   const int worker = a.worker0 + row;
   const float* g = a.g + (int64_t)row * a.g_stride;
-  float* e = a.e + (int64_t)worker * a.ld;
-  float* h = KEEP_H ? a.h + (int64_t)worker * a.ld : nullptr;
+  float* e = a.e + (int64_t)(worker - a.row0) * a.ld;
+  float* h = KEEP_H ? a.h + (int64_t)(worker - a.row0) * a.ld : nullptr;
   uint8_t* msg = a.msg + (int64_t)row * a.msg_stride;
 
   // flat buckets: [b n, b n + n) clipped to d; layer buckets (SEG): the table
@@ -245,8 +245,8 @@ squant_compress_kernel(const CompressArgs a) {
   const int row = blockIdx.y;
   const int worker = a.worker0 + row;
   const float* g = a.g + (int64_t)row * a.g_stride;
-  float* e = a.e + (int64_t)worker * a.ld;
-  float* h = KEEP_H ? a.h + (int64_t)worker * a.ld : nullptr;
+  float* e = a.e + (int64_t)(worker - a.row0) * a.ld;
+  float* h = KEEP_H ? a.h + (int64_t)(worker - a.row0) * a.ld : nullptr;
   uint8_t* msg = a.msg + (int64_t)row * a.msg_stride;
 
   // With one warp per bucket the grid is persistent: a warp takes buckets b,
@@ -412,8 +412,8 @@ identity_compress_kernel(const CompressArgs a) {
   const int row = blockIdx.y;
   const int worker = a.worker0 + row;
   const float* g = a.g + (int64_t)row * a.g_stride;
-  float* e = a.e + (int64_t)worker * a.ld;
-  float* h = KEEP_H ? a.h + (int64_t)worker * a.ld : nullptr;
+  float* e = a.e + (int64_t)(worker - a.row0) * a.ld;
+  float* h = KEEP_H ? a.h + (int64_t)(worker - a.row0) * a.ld : nullptr;
   float* vals = reinterpret_cast<float*>(a.msg + (int64_t)row * a.msg_stride);
   const int64_t nchunks = (a.d + 3) >> 2;
   for (int64_t c = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; c < nchunks;

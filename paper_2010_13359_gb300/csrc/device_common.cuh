@@ -186,6 +186,13 @@ struct PairwiseAcc {
   }
 };
 
+// What a server kernel stores for a parameter w with averaged update q:
+// Algorithm 2's step w - q, or (under Optimistic Adam, whose own pass
+// follows) q itself.
+__device__ __forceinline__ float server_out(const ServerArgs& s, float w, float q) {
+  return s.store_q ? q : __fsub_rn(w, q);
+}
+
 // ---------------------------------------------------------------------------
 // mbarrier + 1-D TMA bulk copy (cp.async.bulk) primitives.  Every wait is
 // bounded: after kSpinLimit polls (each may sleep up to kSuspendNs) it sets

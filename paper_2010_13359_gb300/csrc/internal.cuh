@@ -37,8 +37,8 @@ int set_thread_error(int code, const char* msg);
 struct CompressArgs {
   const float* g;      // gradient of row y at g + y * g_stride
   int64_t g_stride;    // floats, multiple of 4
-  float* e;            // residual of worker w at e + w * ld (library-owned)
-  float* h;            // lookahead offset of worker w at h + w * ld, or nullptr
+  float* e;            // residual of worker w at e + (w - row0) * ld (library-owned)
+  float* h;            // lookahead offset of worker w at h + (w - row0) * ld, or nullptr
   int64_t ld;          // floats, multiple of 64
   uint8_t* msg;        // message of row y at msg + y * msg_stride
   int64_t msg_stride;  // bytes
@@ -51,9 +51,28 @@ struct CompressArgs {
   int32_t bits;
   int32_t worker0;
   int32_t nworkers;
+  int32_t row0;        // the worker whose residual is row 0 (the handle's first local worker)
   uint32_t seed_lo, seed_hi;
   uint32_t step;
   uint32_t* err;       // device error word (bit 0: a bounded wait timed out)
+};
+
+// Optimistic Adam on the server's averaged update (Daskalakis et al., the
+// CPOAdam family): one dense pass after the server kernel has written q_hat.
+struct OAdamArgs {
+  const float* q;       // q_hat, d floats
+  float* w;             // parameters, updated in place
+  float* m;             // first moments
+  float* v;             // second moments
+  float* u;             // the previous step's normalised update u_prev
+  int64_t d;
+  float alpha;
+  float beta1, one_m_beta1;  // b1 and fl(1 - b1)
+  float beta2, one_m_beta2;  // b2 and fl(1 - b2)
+  float eps;
+  float c1, c2;         // fl(1 - b1^t), fl(1 - b2^t) at this step (bias correction)
+  int32_t adaptive;     // 1: u = m_hat / (sqrt(v_hat) + eps); 0: u = m_hat
+  int32_t bias_correction;
 };
 
 // Arguments of the server (decode + average + update) kernels.
@@ -73,6 +92,8 @@ struct ServerArgs {
   const uint32_t* word_bucket;  // bucket of each 32-element word (layer segments), or nullptr: j / bucket
   const CUtensorMap* sign_words_map;    // TMA map of the M messages' sign words, or nullptr
   const CUtensorMap* squant_words_map;  // TMA map of the M messages' code words, or nullptr
+  int32_t store_q;      // 1: write q_hat itself where w - q_hat would go (w is then a q_hat buffer,
+                        // dense: top-k writes +0 at the indices nobody sent)
 };
 
 // The sign server's further inputs (kept out of ServerArgs, which every
@@ -112,13 +133,13 @@ cudaError_t launch_squant_compress(const CompressArgs& a, bool keep_h, bool l2_s
 cudaError_t launch_identity_compress(const CompressArgs& a, bool keep_h, cudaStream_t stream,
                                      uint64_t* launches);
 
-// Scratch of the top-k path: one row per worker and the server's
-// record-range table for `nworkers` messages.  A row needs no clearing
+// Scratch of the top-k path: `rows` rows (one per local worker) and the
+// server's record-range table for `nworkers` messages.  A row needs no clearing
 // between calls: every call rewrites its tile counts, tile prefixes and
 // candidates in full.  Only the row's last state word carries over -- the
 // candidate threshold of the worker's previous call (0 before the first),
 // which decides how much work the first pass saves and never a result.
-size_t topk_scratch_bytes(int64_t d, int32_t nworkers);
+size_t topk_scratch_bytes(int64_t d, int32_t rows, int32_t nworkers);
 cudaError_t launch_topk_compress(const CompressArgs& a, int64_t k, bool keep_h, void* scratch,
                                  cudaStream_t stream, uint64_t* launches);
 
@@ -129,12 +150,17 @@ cudaError_t launch_sign_server(const ServerArgs& s, const SignServerExtras& x, c
 cudaError_t launch_squant_server(const ServerArgs& s, const CUtensorMap* params_map, cudaStream_t stream,
                                  uint64_t* launches);
 cudaError_t launch_identity_server(const ServerArgs& s, cudaStream_t stream, uint64_t* launches);
-cudaError_t launch_topk_server(const ServerArgs& s, void* scratch, cudaStream_t stream, uint64_t* launches);
+// scratch: topk_scratch_bytes(d, rows, M); the server's table follows the rows.
+cudaError_t launch_topk_server(const ServerArgs& s, void* scratch, int32_t rows, cudaStream_t stream,
+                               uint64_t* launches);
 
 // Enqueues one kernel that polls an mbarrier nobody arrives on `polls` times
 // and then sets kErrTimeout in *err (the bounded-wait path, on demand).
 cudaError_t launch_wait_selftest(uint32_t polls, uint32_t* err, cudaStream_t stream, uint64_t* launches);
 uint32_t wait_selftest_max_polls();
+
+// Optimistic Adam over all d parameters from q_hat (one dense pass).
+cudaError_t launch_oadam_update(const OAdamArgs& a, cudaStream_t stream, uint64_t* launches);
 
 cudaError_t launch_lookahead(const float* w, const float* h, float* out, int64_t d,
                              cudaStream_t stream, uint64_t* launches);

@@ -34,13 +34,13 @@ __device__ __forceinline__ float average_t(float acc, const ServerArgs& s) {
 __device__ __forceinline__ void apply_chunk(const ServerArgs& s, int64_t j, const float (&acc)[4]) {
   if (j + 3 < s.d) {
     float4 wv = __ldcs(reinterpret_cast<const float4*>(s.w + j));
-    wv.x = __fsub_rn(wv.x, average(acc[0], s));
-    wv.y = __fsub_rn(wv.y, average(acc[1], s));
-    wv.z = __fsub_rn(wv.z, average(acc[2], s));
-    wv.w = __fsub_rn(wv.w, average(acc[3], s));
+    wv.x = server_out(s, wv.x, average(acc[0], s));
+    wv.y = server_out(s, wv.y, average(acc[1], s));
+    wv.z = server_out(s, wv.z, average(acc[2], s));
+    wv.w = server_out(s, wv.w, average(acc[3], s));
     __stcs(reinterpret_cast<float4*>(s.w + j), wv);
   } else {
-    for (int q = 0; q < 4 && j + q < s.d; ++q) s.w[j + q] = __fsub_rn(s.w[j + q], average(acc[q], s));
+    for (int q = 0; q < 4 && j + q < s.d; ++q) s.w[j + q] = server_out(s, s.w[j + q], average(acc[q], s));
   }
 }
 
@@ -240,7 +240,7 @@ __global__ void __launch_bounds__(256) sign_server_shfl_kernel(const ServerArgs 
 #pragma unroll
     for (int k = 0; k < 8; ++k) {
       const int64_t off = 32 * (8 * it + k);
-      if (off < jmax) __stcs(wl + off, __fsub_rn(wv[k], average_t<POW2>(sum[k], s)));
+      if (off < jmax) __stcs(wl + off, server_out(s, wv[k], average_t<POW2>(sum[k], s)));
     }
     if (more) {
 #pragma unroll
@@ -353,7 +353,7 @@ sign_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap t
 #pragma unroll
       for (int k = 0; k < 8; ++k) {
         const int64_t off = 32 * (8 * q + k);
-        if (off < jmax) __stcs(wl + off, __fsub_rn(wv[k], average_t<POW2>(sum[k], s)));
+        if (off < jmax) __stcs(wl + off, server_out(s, wv[k], average_t<POW2>(sum[k], s)));
       }
       if (q < 3) {
 #pragma unroll
@@ -585,8 +585,7 @@ sign_server_col_kernel(const ServerArgs s, const SegSlices seg, const __grid_con
         for (int r = 0; r < 4; ++r) o[r] = (4 * q + r < cnt) ? wg[4 * q + r] : 0.f;
       }
 #pragma unroll
-      for (int r = 0; r < 4; ++r)
-        o[r] = __fsub_rn(o[r], average_t<POW2>(group_sum<NG>(x[4 * q + r], T), s));
+      for (int r = 0; r < 4; ++r) o[r] = server_out(s, o[r], average_t<POW2>(group_sum<NG>(x[4 * q + r], T), s));
       if (direct) {
 #pragma unroll
         for (int r = 0; r < 4; ++r)
@@ -651,7 +650,7 @@ __global__ void __launch_bounds__(256) sign_server_slabs_kernel(const ServerArgs
 #pragma unroll
     for (int k = 0; k < 8; ++k) {
       const int64_t j = 32 * (wbase + 8 * it + k) + lane;
-      if (j < s.d) __stcs(s.w + j, __fsub_rn(__ldcs(s.w + j), average(acc[k].result(), s)));
+      if (j < s.d) __stcs(s.w + j, server_out(s, __ldcs(s.w + j), average(acc[k].result(), s)));
     }
   }
 }
@@ -734,13 +733,14 @@ __global__ void __launch_bounds__(256) squant_server_kernel(const ServerArgs s) 
     for (int q = 0; q < 4; ++q) acc[q] = sum[q].result();
     if (j + 3 < s.d) {
       float4 wv = __ldcs(reinterpret_cast<const float4*>(s.w + j));
-      wv.x = __fsub_rn(wv.x, average_t<POW2>(acc[0], s));
-      wv.y = __fsub_rn(wv.y, average_t<POW2>(acc[1], s));
-      wv.z = __fsub_rn(wv.z, average_t<POW2>(acc[2], s));
-      wv.w = __fsub_rn(wv.w, average_t<POW2>(acc[3], s));
+      wv.x = server_out(s, wv.x, average_t<POW2>(acc[0], s));
+      wv.y = server_out(s, wv.y, average_t<POW2>(acc[1], s));
+      wv.z = server_out(s, wv.z, average_t<POW2>(acc[2], s));
+      wv.w = server_out(s, wv.w, average_t<POW2>(acc[3], s));
       __stcs(reinterpret_cast<float4*>(s.w + j), wv);
     } else {
-      for (int q = 0; q < 4 && j + q < s.d; ++q) s.w[j + q] = __fsub_rn(s.w[j + q], average_t<POW2>(acc[q], s));
+      for (int q = 0; q < 4 && j + q < s.d; ++q)
+        s.w[j + q] = server_out(s, s.w[j + q], average_t<POW2>(acc[q], s));
     }
   }
 }
@@ -802,8 +802,8 @@ __device__ __forceinline__ void build_pair_tables(float my_scale, int lane, int 
   }
 }
 
-// The b = 2 server update of this lane's 16 elements, w_j = fl(w_j - sum_j / M)
-// in wv, with the worker sums by pair tables: the lane's code word of
+// The b = 2 server update of this lane's 16 elements in wv (server_out of
+// sum_j / M), with the worker sums by pair tables: the lane's code word of
 // each worker (16 per set of workers) is transposed so that one register
 // holds one element's codes of 16 workers, whose 4-bit pair fields index the
 // pair tables by shuffle (the lane index is taken mod 32: the tables repeat
@@ -835,7 +835,7 @@ __device__ __forceinline__ void b2_pair_table_update(const uint32_t* words, cons
       const float sum = np >= 8 ? __fadd_rn(a03, __fadd_rn(__fadd_rn(v[4], v[5]), __fadd_rn(v[6], v[7])))
                                 : (np == 4 ? a03 : (np == 2 ? a01 : v[0]));
       acc[e] = set == 0 ? sum : __fadd_rn(acc[e], sum);
-      if (set + 1 == NSET) wv[e] = __fsub_rn(wv[e], average_t<POW2>(acc[e], s));
+      if (set + 1 == NSET) wv[e] = server_out(s, wv[e], average_t<POW2>(acc[e], s));
     }
   }
 }
@@ -1066,31 +1066,27 @@ squant_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap
     if (per_worker) {
       // group value of workers m .. m + 3 into g
       auto group = [&](int m, float (&g)[EPL]) {
+        // the group's code words and scales first (a worker past M is not read)
+        uint32_t wd[4];
+        float sc[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+          const bool here = m + u < s.M;  // warp-uniform
+          wd[u] = here ? words[32 * (m + u)] : 0u;
+          sc[u] = here ? scale_of(m + u) : 0.f;
+        }
         float va[EPL], vb[EPL];
-        decode_worker(words[32 * m], scale_of(m), va);
-        if (m + 1 < s.M) {
-          decode_worker(words[32 * (m + 1)], scale_of(m + 1), vb);
-        } else {
+        decode_worker(wd[0], sc[0], va);
+        decode_worker(wd[1], sc[1], vb);
+        const bool h1 = m + 1 < s.M;
 #pragma unroll
-          for (int e = 0; e < EPL; ++e) vb[e] = 0.f;
-        }
-#pragma unroll
-        for (int e = 0; e < EPL; ++e) g[e] = s.M == 1 ? va[e] : __fadd_rn(va[e], vb[e]);
+        for (int e = 0; e < EPL; ++e) g[e] = s.M == 1 ? va[e] : __fadd_rn(va[e], h1 ? vb[e] : 0.f);
         if (s.M <= 2) return;
-        if (m + 2 < s.M) {
-          decode_worker(words[32 * (m + 2)], scale_of(m + 2), va);
-        } else {
+        decode_worker(wd[2], sc[2], va);
+        decode_worker(wd[3], sc[3], vb);
+        const bool h2 = m + 2 < s.M, h3 = m + 3 < s.M;
 #pragma unroll
-          for (int e = 0; e < EPL; ++e) va[e] = 0.f;
-        }
-        if (m + 3 < s.M) {
-          decode_worker(words[32 * (m + 3)], scale_of(m + 3), vb);
-        } else {
-#pragma unroll
-          for (int e = 0; e < EPL; ++e) vb[e] = 0.f;
-        }
-#pragma unroll
-        for (int e = 0; e < EPL; ++e) g[e] = __fadd_rn(g[e], __fadd_rn(va[e], vb[e]));
+        for (int e = 0; e < EPL; ++e) g[e] = __fadd_rn(g[e], __fadd_rn(h2 ? va[e] : 0.f, h3 ? vb[e] : 0.f));
       };
       // x <- x + (value of groups i, i + 1), the second +0 past M
       auto add_pair = [&](int i, float (&x)[EPL]) {
@@ -1142,7 +1138,7 @@ squant_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap
       float o[4];
 #pragma unroll
       for (int r = 0; r < 4; ++r)
-        o[r] = per_worker ? __fsub_rn(wv[4 * q + r], average_t<POW2>(acc[4 * q + r], s)) : wv[4 * q + r];
+        o[r] = per_worker ? server_out(s, wv[4 * q + r], average_t<POW2>(acc[4 * q + r], s)) : wv[4 * q + r];
       if constexpr (WB) {
         if (boxed)
           *reinterpret_cast<float4*>(prow + (((pc0 + q) ^ (pr & 7)) << 4)) = make_float4(o[0], o[1], o[2], o[3]);
@@ -1219,6 +1215,46 @@ lookahead_kernel(const float* __restrict__ w, const float* __restrict__ h, float
                        __fsub_rn(wv.w, hv.w)));
   } else {
     for (int64_t jj = j; jj < d; ++jj) out[jj] = __fsub_rn(w[jj], h[jj]);
+  }
+}
+
+// Optimistic Adam over all parameters from q_hat (written by the server
+// kernel), every operation rounded once in this order:
+//   m = b1 m + (1 - b1) q;  v = b2 v + ((1 - b2) q) q;
+//   m_hat = m / c1, v_hat = v / c2 (with bias correction);
+//   u = m_hat / (sqrt(v_hat) + eps), 0 where m_hat = 0 (adaptive), else m_hat;
+//   w = w - alpha (2 u - u_prev);  u_prev = u.
+// One thread per 4 parameters, 16-byte streaming loads and stores.
+__device__ __forceinline__ float oadam_element(const OAdamArgs& a, float q, float& m, float& v, float& u, float w) {
+  m = __fadd_rn(__fmul_rn(a.beta1, m), __fmul_rn(a.one_m_beta1, q));
+  v = __fadd_rn(__fmul_rn(a.beta2, v), __fmul_rn(__fmul_rn(a.one_m_beta2, q), q));
+  const float mh = a.bias_correction ? __fdiv_rn(m, a.c1) : m;
+  const float vh = a.bias_correction ? __fdiv_rn(v, a.c2) : v;
+  float un = mh;
+  if (a.adaptive) un = (mh == 0.f) ? 0.f : __fdiv_rn(mh, __fadd_rn(__fsqrt_rn(vh), a.eps));
+  const float step = __fsub_rn(__fmul_rn(2.f, un), u);
+  u = un;
+  return __fsub_rn(w, __fmul_rn(a.alpha, step));
+}
+
+__global__ void __launch_bounds__(256) oadam_update_kernel(const OAdamArgs a) {
+  const int64_t j = 4 * ((int64_t)blockIdx.x * blockDim.x + threadIdx.x);
+  if (j + 3 < a.d) {
+    const float4 q = __ldcs(reinterpret_cast<const float4*>(a.q + j));
+    float4 m = __ldcs(reinterpret_cast<const float4*>(a.m + j));
+    float4 v = __ldcs(reinterpret_cast<const float4*>(a.v + j));
+    float4 u = __ldcs(reinterpret_cast<const float4*>(a.u + j));
+    float4 w = __ldcs(reinterpret_cast<const float4*>(a.w + j));
+    w.x = oadam_element(a, q.x, m.x, v.x, u.x, w.x);
+    w.y = oadam_element(a, q.y, m.y, v.y, u.y, w.y);
+    w.z = oadam_element(a, q.z, m.z, v.z, u.z, w.z);
+    w.w = oadam_element(a, q.w, m.w, v.w, u.w, w.w);
+    __stcs(reinterpret_cast<float4*>(a.m + j), m);
+    __stcs(reinterpret_cast<float4*>(a.v + j), v);
+    __stcs(reinterpret_cast<float4*>(a.u + j), u);
+    __stcs(reinterpret_cast<float4*>(a.w + j), w);
+  } else {
+    for (int64_t jj = j; jj < a.d; ++jj) a.w[jj] = oadam_element(a, a.q[jj], a.m[jj], a.v[jj], a.u[jj], a.w[jj]);
   }
 }
 
@@ -1443,6 +1479,12 @@ cudaError_t launch_identity_server(const ServerArgs& s, cudaStream_t stream, uin
   return cudaGetLastError();
 }
 
+
+cudaError_t launch_oadam_update(const OAdamArgs& a, cudaStream_t stream, uint64_t* launches) {
+  oadam_update_kernel<<<chunk_blocks(a.d, 256), 256, 0, stream>>>(a);
+  *launches += 1;
+  return cudaGetLastError();
+}
 
 cudaError_t launch_lookahead(const float* w, const float* h, float* out, int64_t d,
                              cudaStream_t stream, uint64_t* launches) {

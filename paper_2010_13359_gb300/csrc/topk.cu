@@ -229,9 +229,9 @@ __global__ void __launch_bounds__(kFormThreads, 6) topk_form_kernel(const Compre
   const int row = blockIdx.y;
   const int worker = a.worker0 + row;
   const float* g = a.g + (int64_t)row * a.g_stride;
-  float* e = a.e + (int64_t)worker * a.ld;
-  float* h = KEEP_H ? a.h + (int64_t)worker * a.ld : nullptr;
-  RowScratch rs = row_scratch(scratch, a.d, worker);
+  float* e = a.e + (int64_t)(worker - a.row0) * a.ld;
+  float* h = KEEP_H ? a.h + (int64_t)(worker - a.row0) * a.ld : nullptr;
+  RowScratch rs = row_scratch(scratch, a.d, worker - a.row0);
   const uint32_t tau_word = rs.state[ST_TAU];
   const bool has_tau = (tau_word & kTauValid) != 0;
   const uint32_t tau = tau_word & 0x7FFFFFFFu;
@@ -383,11 +383,11 @@ topk_select_kernel(const CompressArgs a, int64_t k, void* scratch) {
   const int rank = (int)cluster.block_rank();
   const int row = blockIdx.y;
   const int worker = a.worker0 + row;
-  float* e = a.e + (int64_t)worker * a.ld;
-  float* h = KEEP_H ? a.h + (int64_t)worker * a.ld : nullptr;
+  float* e = a.e + (int64_t)(worker - a.row0) * a.ld;
+  float* h = KEEP_H ? a.h + (int64_t)(worker - a.row0) * a.ld : nullptr;
   const float* g = a.g + (int64_t)row * a.g_stride;
   uint2* rec = reinterpret_cast<uint2*>(a.msg + (int64_t)row * a.msg_stride);
-  RowScratch rs = row_scratch(scratch, a.d, worker);
+  RowScratch rs = row_scratch(scratch, a.d, worker - a.row0);
   const int64_t nt = tiles_of(a.d);
   uint32_t* gpre = rs.gpre + (int64_t)rank * (nt + 1);  // this CTA's private prefix array
   const uint32_t tau_word = rs.state[ST_TAU];
@@ -993,20 +993,25 @@ __global__ void __launch_bounds__(kSrvThreads) topk_server_warp_kernel(const Ser
       __syncwarp();
     }
   }
+  // the plain update leaves untouched w_j as they are; with store_q every
+  // index gets its q_hat (+0 where nobody sent it) for the dense pass that
+  // follows
+  const bool dense = s.store_q != 0;
   const uint32_t P = 1u << (nlev - 1);
   constexpr int kPer = kSrvTile / 32;
   constexpr int kHalf = kPer / 2;
 #pragma unroll
   for (int half = 0; half < 2; ++half) {
     float wv[kHalf], sum[kHalf];
+    bool upd[kHalf];
 #pragma unroll
     for (int q = 0; q < kHalf; ++q) {
       const int i = (half * kHalf + q) * 32 + lane;
       const uint32_t n = cnt[i];
-      wv[q] = 0.f;
+      upd[q] = n != 0 || (dense && tile0 + i < s.d);
+      wv[q] = upd[q] ? s.w[tile0 + i] : 0.f;
       sum[q] = 0.f;
       if (n) {
-        wv[q] = s.w[tile0 + i];
         srv_push_zeros(stk, i, n, P);
         sum[q] = stk[(nlev - 1) * kSrvTile + i];
       }
@@ -1014,7 +1019,7 @@ __global__ void __launch_bounds__(kSrvThreads) topk_server_warp_kernel(const Ser
 #pragma unroll
     for (int q = 0; q < kHalf; ++q) {
       const int i = (half * kHalf + q) * 32 + lane;
-      if (cnt[i]) s.w[tile0 + i] = __fsub_rn(wv[q], srv_average<POW2>(sum[q], s));
+      if (upd[q]) s.w[tile0 + i] = server_out(s, wv[q], srv_average<POW2>(sum[q], s));
     }
   }
 }
@@ -1103,9 +1108,9 @@ __global__ void __launch_bounds__(kSrvThreads) topk_server_owner_kernel(const Se
 
 }  // namespace
 
-size_t topk_scratch_bytes(int64_t d, int32_t nworkers) {
+size_t topk_scratch_bytes(int64_t d, int32_t rows, int32_t nworkers) {
   const int64_t server_words = round64((int64_t)nworkers * (srv_tiles(d) + 1));
-  return (size_t)(row_words(d) * nworkers + server_words) * 4u;
+  return (size_t)(row_words(d) * rows + server_words) * 4u;
 }
 
 // Raises a kernel's dynamic shared memory limit when its static plus dynamic
@@ -1153,8 +1158,10 @@ cudaError_t launch_topk_compress(const CompressArgs& a, int64_t k, bool keep_h, 
   return cudaGetLastError();
 }
 
-cudaError_t launch_topk_server(const ServerArgs& s, void* scratch, cudaStream_t stream, uint64_t* launches) {
-  uint32_t* starts = reinterpret_cast<uint32_t*>(scratch) + row_words(s.d) * s.M;
+cudaError_t launch_topk_server(const ServerArgs& s, void* scratch, int32_t rows, cudaStream_t stream,
+                               uint64_t* launches) {
+  if (s.store_q && s.M > kSrvWarpMaxM) return cudaErrorNotSupported;  // the owner kernel is sparse
+  uint32_t* starts = reinterpret_cast<uint32_t*>(scratch) + row_words(s.d) * rows;
   const int64_t n = (int64_t)s.M * s.k;
   topk_server_starts_kernel<<<dim3((unsigned)((s.k + 255) / 256), (unsigned)s.M), 256, 0, stream>>>(s, starts);
   if (s.M <= kSrvWarpMaxM) {

@@ -49,6 +49,31 @@ class Config(ctypes.Structure):
 
 assert ctypes.sizeof(Config) == 56
 
+SERVER_OMD, SERVER_OADAM = 0, 1
+OADAM_ADAPTIVE, OADAM_BIAS_CORRECTION = 1, 2
+
+
+class ServerOptimizer(ctypes.Structure):
+    """Mirror of ``dqgan_server_optimizer`` (28 bytes, no padding)."""
+    _fields_ = [
+        ("kind", ctypes.c_int32),
+        ("flags", ctypes.c_uint32),
+        ("alpha", ctypes.c_float),
+        ("beta1", ctypes.c_float),
+        ("beta2", ctypes.c_float),
+        ("eps", ctypes.c_float),
+        ("reserved", ctypes.c_uint32),
+    ]
+
+
+assert ctypes.sizeof(ServerOptimizer) == 28
+
+
+def oadam(alpha: float, beta1: float, beta2: float, eps: float, adaptive: bool = True,
+          bias_correction: bool = True) -> ServerOptimizer:
+    flags = (OADAM_ADAPTIVE if adaptive else 0) | (OADAM_BIAS_CORRECTION if bias_correction else 0)
+    return ServerOptimizer(kind=SERVER_OADAM, flags=flags, alpha=alpha, beta1=beta1, beta2=beta2, eps=eps)
+
 _lib = None
 
 
@@ -91,6 +116,10 @@ def load_library(path: str = LIBRARY) -> ctypes.CDLL:
         "dqgan_topk_compress_noalloc": (ctypes.c_int, [P, P, P, i64, i64, ctypes.c_float, P]),
         "dqgan_selftest_wait_timeout": (ctypes.c_int, [H, ctypes.c_uint32]),
         "dqgan_set_segments": (ctypes.c_int, [H, ctypes.POINTER(i64), i32]),
+        "dqgan_set_server_optimizer": (ctypes.c_int, [H, ctypes.POINTER(ServerOptimizer)]),
+        "dqgan_workers_compress_range": (ctypes.c_int, [H, i32, i32, P, i64, P]),
+        "dqgan_set_local_workers": (ctypes.c_int, [H, i32, i32]),
+        "dqgan_get_server_state": (ctypes.c_int, [H, i32, P]),
     }
     for name, (res, args) in sig.items():
         fn = getattr(L, name)
@@ -177,6 +206,13 @@ class Handle:
         arr = (ctypes.c_int64 * len(offsets))(*[int(x) for x in offsets])
         _check(load_library().dqgan_set_segments(self._h, arr, len(offsets) - 1), self._h)
 
+    def set_server_optimizer(self, opt: ServerOptimizer) -> None:
+        _check(load_library().dqgan_set_server_optimizer(self._h, ctypes.byref(opt)), self._h)
+
+    def get_server_state(self, which: int, dst) -> None:
+        """which: 0 m, 1 v, 2 u_prev (d fp32 into dst, host or device)."""
+        _check(load_library().dqgan_get_server_state(self._h, which, _ptr(dst)), self._h)
+
     def message_bytes(self) -> int:
         return int(load_library().dqgan_message_bytes(self._h))
 
@@ -186,6 +222,13 @@ class Handle:
     def workers_compress_all(self, g_all, g_stride: int, msgs_all) -> None:
         _check(load_library().dqgan_workers_compress_all(self._h, _ptr(g_all), g_stride, _ptr(msgs_all)),
                self._h)
+
+    def workers_compress_range(self, first: int, count: int, g, g_stride: int, msgs) -> None:
+        _check(load_library().dqgan_workers_compress_range(self._h, first, count, _ptr(g), g_stride, _ptr(msgs)),
+               self._h)
+
+    def set_local_workers(self, first: int, count: int) -> None:
+        _check(load_library().dqgan_set_local_workers(self._h, first, count), self._h)
 
     def server_aggregate_update(self, msgs_all, params) -> None:
         _check(load_library().dqgan_server_aggregate_update(self._h, _ptr(msgs_all), _ptr(params)), self._h)

@@ -127,3 +127,34 @@ def test_missing_library_fails_loudly(P, tmp_path):
             mod.load_library(str(tmp_path / "libdqgan.so"))
     finally:
         mod._lib = saved
+
+
+def test_server_optimizer_struct_layout_matches_header(tmp_path, P):
+    c = tmp_path / "opt.c"
+    c.write_text("""
+#include <stddef.h>
+#include "dqgan.h"
+_Static_assert(sizeof(dqgan_server_optimizer) == 28, "size");
+_Static_assert(offsetof(dqgan_server_optimizer, kind) == 0, "kind");
+_Static_assert(offsetof(dqgan_server_optimizer, flags) == 4, "flags");
+_Static_assert(offsetof(dqgan_server_optimizer, alpha) == 8, "alpha");
+_Static_assert(offsetof(dqgan_server_optimizer, beta1) == 12, "beta1");
+_Static_assert(offsetof(dqgan_server_optimizer, beta2) == 16, "beta2");
+_Static_assert(offsetof(dqgan_server_optimizer, eps) == 20, "eps");
+_Static_assert(DQGAN_SERVER_OMD == 0 && DQGAN_SERVER_OADAM == 1, "kinds");
+_Static_assert(DQGAN_OADAM_ADAPTIVE == 1u && DQGAN_OADAM_BIAS_CORRECTION == 2u, "flags");
+""")
+    subprocess.run(["gcc", "-std=c11", "-fsyntax-only", "-I", os.path.join(ROOT, "include"), str(c)],
+                   check=True)
+    S = P.dqgan.ServerOptimizer
+    for name, off in [("kind", 0), ("flags", 4), ("alpha", 8), ("beta1", 12), ("beta2", 16), ("eps", 20)]:
+        assert getattr(S, name).offset == off
+
+
+def test_server_optimizer_calls_reject_a_null_handle(P):
+    L = P.dqgan.load_library()
+    opt = P.dqgan.oadam(1e-3, 0.5, 0.999, 1e-8)
+    import ctypes
+    assert L.dqgan_set_server_optimizer(None, ctypes.byref(opt)) == P.dqgan.ERR_INVALID_ARG
+    assert L.dqgan_get_server_state(None, 0, None) == P.dqgan.ERR_INVALID_ARG
+    assert b"NULL" in L.dqgan_last_error(None)
