@@ -61,6 +61,7 @@ extern "C" {
 #define DQGAN_ERR_CUDA (-3)        /* a CUDA runtime call or kernel launch failed */
 #define DQGAN_ERR_UNSUPPORTED (-4) /* valid request this build does not provide */
 #define DQGAN_ERR_TIMEOUT (-5)     /* a bounded device-side wait gave up */
+#define DQGAN_ERR_BOUNDS (-6)      /* checked build only: an index check skipped an out-of-range access */
 
 /* Compressors Q (Section 2.4, Section 3.2). */
 #define DQGAN_SIGN 0     /* scaled sign, s_b = ||p_b||_1 / n_b per bucket */
@@ -229,7 +230,11 @@ DQGAN_API int dqgan_worker_lookahead(dqgan_handle* h, int32_t i, const float* pa
  * DQGAN_ERR_TIMEOUT if a bounded device-side wait of an enqueued kernel gave
  * up since the last call (the error word is then cleared, the handle and the
  * CUDA context stay usable, and the results of the steps since the last
- * successful synchronize are undefined). */
+ * successful synchronize are undefined).  In the checked build (compiled
+ * with -DDQGAN_CHECK_BOUNDS, libdqgan_checked.so) also DQGAN_ERR_BOUNDS when
+ * an index check in a kernel skipped an out-of-range access, or when the
+ * guard zones around the top-k scratch were written; the word is cleared
+ * and the guards restored the same way. */
 DQGAN_API int dqgan_synchronize(dqgan_handle* h);
 
 /*

@@ -21,6 +21,11 @@ CSRC = os.path.join(HERE, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 BUILD_DIR = os.path.join(HERE, "_build")
 LIBRARY = os.path.join(HERE, "libdqgan.so")
+# The checked build: the same sources with -DDQGAN_CHECK_BOUNDS (index checks
+# that skip an out-of-range access and report it, guard zones around the
+# top-k scratch), for the tests; the binding loads it when DQGAN_LIBRARY
+# names it.
+CHECKED_LIBRARY = os.path.join(HERE, "libdqgan_checked.so")
 
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ["-O3", "-std=c++17", "-lineinfo", "-fmad=false", "-Xcompiler", "-fPIC",
@@ -43,23 +48,28 @@ def _inputs() -> list[str]:
                                                                   os.path.abspath(__file__)]
 
 
-def up_to_date() -> bool:
-    if not os.path.exists(LIBRARY):
+def up_to_date(library: str = LIBRARY) -> bool:
+    if not os.path.exists(library):
         return False
-    t = os.path.getmtime(LIBRARY)
+    t = os.path.getmtime(library)
     return all(os.path.getmtime(p) <= t for p in _inputs())
 
 
-def build(force: bool = False, verbose: bool = False, ptxas_info: bool = False) -> str:
-    """Compile and link the library if any input changed; return its path."""
-    if not force and up_to_date():
-        return LIBRARY
-    os.makedirs(BUILD_DIR, exist_ok=True)
+def build(force: bool = False, verbose: bool = False, ptxas_info: bool = False, checked: bool = False) -> str:
+    """Compile and link the library (or, with checked=True, the checked
+    build) if any input changed; return its path."""
+    library = CHECKED_LIBRARY if checked else LIBRARY
+    build_dir = BUILD_DIR + ("_checked" if checked else "")
+    if not force and up_to_date(library):
+        return library
+    os.makedirs(build_dir, exist_ok=True)
     exe = nvcc()
     extra = ["-Xptxas", "-v"] if ptxas_info else []
+    if checked:
+        extra.append("-DDQGAN_CHECK_BOUNDS")
 
     def compile_one(src: str) -> tuple[str, str]:
-        obj = os.path.join(BUILD_DIR, os.path.basename(src).replace(".cu", ".o"))
+        obj = os.path.join(build_dir, os.path.basename(src).replace(".cu", ".o"))
         cmd = [exe, *ARCH, *NVCC_FLAGS, *extra, "-I", INCLUDE, "-I", CSRC, "-c", src, "-o", obj]
         res = subprocess.run(cmd, capture_output=True, text=True)
         if res.returncode != 0:
@@ -72,13 +82,13 @@ def build(force: bool = False, verbose: bool = False, ptxas_info: bool = False) 
         for _, log in results:
             if log.strip():
                 print(log)
-    tmp = LIBRARY + f".tmp{os.getpid()}"
+    tmp = library + f".tmp{os.getpid()}"
     cmd = [exe, *ARCH, "-shared", "-o", tmp, *[o for o, _ in results], "-cudart", "static"]
     res = subprocess.run(cmd, capture_output=True, text=True)
     if res.returncode != 0:
         raise RuntimeError(f"nvcc link failed:\n{res.stderr}")
-    os.replace(tmp, LIBRARY)
-    return LIBRARY
+    os.replace(tmp, library)
+    return library
 
 
 if __name__ == "__main__":

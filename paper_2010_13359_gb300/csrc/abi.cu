@@ -109,6 +109,52 @@ cudaError_t dq_malloc(T** p, size_t bytes) {
   return st;
 }
 
+// The top-k scratch.  In the checked build (-DDQGAN_CHECK_BOUNDS) it sits
+// between two guard zones of kScratchGuard bytes of kGuardByte, which
+// dqgan_synchronize checks; otherwise it is a plain allocation.
+#ifdef DQGAN_CHECK_BOUNDS
+constexpr size_t kScratchGuard = 64u << 10;
+#else
+constexpr size_t kScratchGuard = 0;
+#endif
+constexpr unsigned char kGuardByte = 0xA5;
+
+cudaError_t scratch_alloc(void** scratch, size_t bytes) {
+  *scratch = nullptr;
+  void* base = nullptr;
+  cudaError_t st = dq_malloc(&base, bytes + 2 * kScratchGuard);
+  if (st != cudaSuccess) return st;
+  if (kScratchGuard && (st = cudaMemset(base, kGuardByte, bytes + 2 * kScratchGuard)) != cudaSuccess) {
+    cudaFree(base);
+    return st;
+  }
+  *scratch = static_cast<char*>(base) + kScratchGuard;
+  return cudaSuccess;
+}
+
+void scratch_free(void* scratch) {
+  if (scratch) cudaFree(static_cast<char*>(scratch) - kScratchGuard);
+}
+
+// Checked build: whether both guard zones of the scratch still hold
+// kGuardByte (restoring them if not).
+bool scratch_guards_intact(void* scratch, size_t bytes) {
+  if (!kScratchGuard || !scratch) return true;
+  std::vector<unsigned char> host(2 * kScratchGuard);
+  char* lo = static_cast<char*>(scratch) - kScratchGuard;
+  char* hi = static_cast<char*>(scratch) + bytes;
+  if (cudaMemcpy(host.data(), lo, kScratchGuard, cudaMemcpyDeviceToHost) != cudaSuccess ||
+      cudaMemcpy(host.data() + kScratchGuard, hi, kScratchGuard, cudaMemcpyDeviceToHost) != cudaSuccess)
+    return false;
+  for (unsigned char c : host)
+    if (c != kGuardByte) {
+      cudaMemset(lo, kGuardByte, kScratchGuard);
+      cudaMemset(hi, kGuardByte, kScratchGuard);
+      return false;
+    }
+  return true;
+}
+
 bool is_pow2(int64_t x) { return x > 0 && (x & (x - 1)) == 0; }
 bool aligned16(const void* p) { return ((uintptr_t)p & 15u) == 0; }
 
@@ -369,7 +415,7 @@ int dqgan_create(const dqgan_config* cfg, dqgan_handle** out) {
     cudaGetLastError();
     if (h->e) cudaFree(h->e);
     if (h->h) cudaFree(h->h);
-    if (h->scratch) cudaFree(h->scratch);
+    scratch_free(h->scratch);
     if (h->err_word) cudaFree(h->err_word);
     delete h;
     return set_error(nullptr, e == cudaErrorMemoryAllocation ? DQGAN_ERR_OOM : DQGAN_ERR_CUDA,
@@ -382,7 +428,7 @@ int dqgan_create(const dqgan_config* cfg, dqgan_handle** out) {
     if ((st = dq_malloc(&h->h, rows_bytes)) != cudaSuccess) return fail_oom("allocating h", st);
   if (cfg->compressor == DQGAN_TOPK) {
     h->scratch_bytes = dq::topk_scratch_bytes(cfg->d, cfg->M, cfg->M);
-    if ((st = dq_malloc(&h->scratch, h->scratch_bytes)) != cudaSuccess)
+    if ((st = scratch_alloc(&h->scratch, h->scratch_bytes)) != cudaSuccess)
       return fail_oom("allocating top-k scratch", st);
   }
   if ((st = cudaMemsetAsync(h->e, 0, rows_bytes, h->stream)) != cudaSuccess) return fail_oom("zeroing e", st);
@@ -403,7 +449,7 @@ int dqgan_destroy(dqgan_handle* h) {
   cudaStreamSynchronize(h->stream);
   if (h->e) cudaFree(h->e);
   if (h->h) cudaFree(h->h);
-  if (h->scratch) cudaFree(h->scratch);
+  scratch_free(h->scratch);
   if (h->err_word) cudaFree(h->err_word);
   if (h->seg_bstart) cudaFree(h->seg_bstart);
   if (h->seg_wbucket) cudaFree(h->seg_wbucket);
@@ -558,20 +604,20 @@ int dqgan_set_local_workers(dqgan_handle* h, int32_t first, int32_t count) {
     cudaGetLastError();
     if (e) cudaFree(e);
     if (hh) cudaFree(hh);
-    if (scratch) cudaFree(scratch);
+    scratch_free(scratch);
     return set_error(h, err == cudaErrorMemoryAllocation ? DQGAN_ERR_OOM : DQGAN_ERR_CUDA, "%s: %s", what,
                      cudaGetErrorString(err));
   };
   if ((st = dq_malloc(&e, rows_bytes)) != cudaSuccess) return fail("allocating e", st);
   if (h->h && (st = dq_malloc(&hh, rows_bytes)) != cudaSuccess) return fail("allocating h", st);
-  if (scratch_bytes && (st = dq_malloc(&scratch, scratch_bytes)) != cudaSuccess)
+  if (scratch_bytes && (st = scratch_alloc(&scratch, scratch_bytes)) != cudaSuccess)
     return fail("allocating top-k scratch", st);
   if ((st = cudaMemset(e, 0, rows_bytes)) != cudaSuccess || (hh && (st = cudaMemset(hh, 0, rows_bytes)) != cudaSuccess) ||
       (scratch && (st = cudaMemset(scratch, 0, scratch_bytes)) != cudaSuccess))
     return fail("zeroing the worker state", st);
   cudaFree(h->e);
   if (h->h) cudaFree(h->h);
-  if (h->scratch) cudaFree(h->scratch);
+  scratch_free(h->scratch);
   h->e = e;
   h->h = hh;
   h->scratch = scratch;
@@ -682,10 +728,13 @@ int dqgan_synchronize(dqgan_handle* h) {
   uint32_t word = 0;
   st = cudaMemcpy(&word, h->err_word, sizeof word, cudaMemcpyDeviceToHost);
   if (st != cudaSuccess) return cuda_fail(h, st, "reading the error word");
-  if (word != 0) {
-    cudaMemset(h->err_word, 0, sizeof word);
+  if (word != 0) cudaMemset(h->err_word, 0, sizeof word);
+  if (!scratch_guards_intact(h->scratch, h->scratch_bytes))
+    return set_error(h, DQGAN_ERR_BOUNDS, "the guard zones around the top-k scratch were written");
+  if (word & dq::kErrBounds)
+    return set_error(h, DQGAN_ERR_BOUNDS, "an index check skipped an out-of-range access (error word 0x%x)", word);
+  if (word != 0)
     return set_error(h, DQGAN_ERR_TIMEOUT, "a bounded device-side wait gave up (error word 0x%x)", word);
-  }
   return DQGAN_OK;
 }
 

@@ -198,7 +198,20 @@ __device__ __forceinline__ float server_out(const ServerArgs& s, float w, float 
 // bounded: after kSpinLimit polls (each may sleep up to kSuspendNs) it sets
 // kErrTimeout in the launch's error word and returns false.
 // ---------------------------------------------------------------------------
-constexpr uint32_t kErrTimeout = 1u;
+
+// Index checks of the checked build (compiled with -DDQGAN_CHECK_BOUNDS):
+// dq_in_bounds(cond, err) is cond, and when cond is false it also sets
+// kErrBounds in the launch's error word, so that the caller skips the access
+// and dqgan_synchronize reports DQGAN_ERR_BOUNDS.  In the normal build it is
+// cond alone (where cond holds by construction, the compiler drops it).
+__device__ __forceinline__ bool dq_in_bounds(bool cond, uint32_t* err) {
+#ifdef DQGAN_CHECK_BOUNDS
+  if (!cond) atomicOr(err, kErrBounds);
+#else
+  (void)err;
+#endif
+  return cond;
+}
 constexpr uint32_t kSpinLimit = 1u << 21;
 constexpr uint32_t kSuspendNs = 500u;
 

@@ -16,6 +16,9 @@
 namespace dq {
 
 constexpr unsigned kFullMask = 0xffffffffu;
+// Bits of the device error word a handle's kernels share.
+constexpr uint32_t kErrTimeout = 1u;  // a bounded wait gave up
+constexpr uint32_t kErrBounds = 2u;   // checked build: an index check skipped an access
 // Counter word 3 of the Philox4x32-10 draws of the stochastic quantiser.
 constexpr uint32_t kSquantTag = 0x51u;
 

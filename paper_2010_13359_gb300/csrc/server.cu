@@ -840,6 +840,9 @@ __device__ __forceinline__ void b2_pair_table_update(const uint32_t* words, cons
   }
 }
 
+// Passes over a lane's 8 elements in the b = 4 per-worker decode (1 or 2).
+constexpr int kSquant4Parts = 2;
+
 // Whether the squant server stages the parameters by TMA (b = 2 and 4; for
 // b = 8 a lane's 16 bytes of w are contiguous across the warp already).
 constexpr bool sq_params_boxed(int bits) { return bits != 8; }
@@ -1017,16 +1020,22 @@ squant_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap
     }
     const uint32_t* words = reinterpret_cast<const uint32_t*>(buf0 + cur * box_bytes) + lane;
     const float* V8l = V8 + lane;
-    // one worker's decoded values of this lane's EPL elements
-    auto decode_worker = [&](uint32_t word, float sc, float (&v)[EPL]) {
+    // The per-worker decode (b = 4, 8, and b = 2 on slices that span layer
+    // segments) takes the lane's elements in kParts passes of NE (b = 4: two
+    // passes of 4, which halves the live sums at the cost of reading each
+    // code word and scale twice).
+    constexpr int kParts = BITS == 4 ? kSquant4Parts : 1;
+    constexpr int NE = EPL / kParts;
+    // one worker's decoded values of this lane's elements e0 .. e0 + NE - 1
+    auto decode_part = [&](uint32_t word, float sc, int e0, float (&v)[NE]) {
       if constexpr (BITS == 2) {
         // code 0: -s, 1: +0, 2: +s (fl(s * 1) = s): one bit test picks +0,
         // one the sign
         const float nsc = -sc;
 #pragma unroll
-        for (int e = 0; e < EPL; ++e) {
-          const bool zero = (word >> (2 * e)) & 1u;
-          v[e] = zero ? 0.f : (((word >> (2 * e + 1)) & 1u) ? sc : nsc);
+        for (int e = 0; e < NE; ++e) {
+          const bool zero = (word >> (2 * (e0 + e))) & 1u;
+          v[e] = zero ? 0.f : (((word >> (2 * (e0 + e) + 1)) & 1u) ? sc : nsc);
         }
         return;
       }
@@ -1038,12 +1047,12 @@ squant_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap
       // by the lane's own scale instead.)
       const float T4 = (BITS == 4) ? __fmul_rn(mixed ? 1.0f : sc, V4) : 0.f;
 #pragma unroll
-      for (int e = 0; e < EPL; ++e) {
+      for (int e = 0; e < NE; ++e) {
         if constexpr (BITS == 4) {
-          v[e] = __shfl_sync(kFullMask, T4, (int)(word >> (4 * e)));
+          v[e] = __shfl_sync(kFullMask, T4, (int)(word >> (4 * (e0 + e))));
           if (mixed) v[e] = __fmul_rn(sc, v[e]);
         } else {
-          v[e] = __fmul_rn(sc, V8l[__byte_perm(word, 0u, 0x4440u | (uint32_t)e) * 32u]);
+          v[e] = __fmul_rn(sc, V8l[__byte_perm(word, 0u, 0x4440u | (uint32_t)(e0 + e)) * 32u]);
         }
       }
     };
@@ -1057,79 +1066,85 @@ squant_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap
         b2_pair_table_update<NSET, POW2>(words, s, T2, wv);
       }
     }
-    // per-worker decode (b = 4, 8, and b = 2 on slices that span layer
-    // segments): groups of four workers, G = (a + b) + (c + d) with +0 past
-    // M, combined as the padded tree over the next_pow2(ceil(M / 4)) <= 8
-    // groups: G0; G0 + G1; (G0 + G1) + (G2 + G3); then + ((G4 + G5) + (G6 + G7)),
-    // groups past M being +0 (M is warp-uniform, so are the branches)
+    // groups of four workers, G = (a + b) + (c + d) with +0 past M, combined
+    // as the padded tree over the next_pow2(ceil(M / 4)) <= 8 groups: G0;
+    // G0 + G1; (G0 + G1) + (G2 + G3); then + ((G4 + G5) + (G6 + G7)), groups
+    // past M being +0 (M is warp-uniform, so are the branches)
     const bool per_worker = BITS != 2 || (SEG && mixed);
     if (per_worker) {
-      // group value of workers m .. m + 3 into g
-      auto group = [&](int m, float (&g)[EPL]) {
-        // the group's code words and scales first (a worker past M is not read)
-        uint32_t wd[4];
-        float sc[4];
 #pragma unroll
-        for (int u = 0; u < 4; ++u) {
-          const bool here = m + u < s.M;  // warp-uniform
-          wd[u] = here ? words[32 * (m + u)] : 0u;
-          sc[u] = here ? scale_of(m + u) : 0.f;
-        }
-        float va[EPL], vb[EPL];
-        decode_worker(wd[0], sc[0], va);
-        decode_worker(wd[1], sc[1], vb);
-        const bool h1 = m + 1 < s.M;
+      for (int part = 0; part < kParts; ++part) {
+        const int e0 = part * NE;
+        // group value of workers m .. m + 3 into g
+        auto group = [&](int m, float (&g)[NE]) {
+          // the group's code words and scales first (a worker past M is not read)
+          uint32_t wd[4];
+          float sc[4];
 #pragma unroll
-        for (int e = 0; e < EPL; ++e) g[e] = s.M == 1 ? va[e] : __fadd_rn(va[e], h1 ? vb[e] : 0.f);
-        if (s.M <= 2) return;
-        decode_worker(wd[2], sc[2], va);
-        decode_worker(wd[3], sc[3], vb);
-        const bool h2 = m + 2 < s.M, h3 = m + 3 < s.M;
+          for (int u = 0; u < 4; ++u) {
+            const bool here = m + u < s.M;  // warp-uniform
+            wd[u] = here ? words[32 * (m + u)] : 0u;
+            sc[u] = here ? scale_of(m + u) : 0.f;
+          }
+          float va[NE], vb[NE];
+          decode_part(wd[0], sc[0], e0, va);
+          decode_part(wd[1], sc[1], e0, vb);
+          const bool h1 = m + 1 < s.M;
 #pragma unroll
-        for (int e = 0; e < EPL; ++e) g[e] = __fadd_rn(g[e], __fadd_rn(h2 ? va[e] : 0.f, h3 ? vb[e] : 0.f));
-      };
-      // x <- x + (value of groups i, i + 1), the second +0 past M
-      auto add_pair = [&](int i, float (&x)[EPL]) {
-        float t[EPL], g[EPL];
-        group(4 * i, t);
-        if (4 * (i + 1) < s.M) {
-          group(4 * (i + 1), g);
-        } else {
+          for (int e = 0; e < NE; ++e) g[e] = s.M == 1 ? va[e] : __fadd_rn(va[e], h1 ? vb[e] : 0.f);
+          if (s.M <= 2) return;
+          decode_part(wd[2], sc[2], e0, va);
+          decode_part(wd[3], sc[3], e0, vb);
+          const bool h2 = m + 2 < s.M, h3 = m + 3 < s.M;
 #pragma unroll
-          for (int e = 0; e < EPL; ++e) g[e] = 0.f;
-        }
+          for (int e = 0; e < NE; ++e) g[e] = __fadd_rn(g[e], __fadd_rn(h2 ? va[e] : 0.f, h3 ? vb[e] : 0.f));
+        };
+        // x <- x + (value of groups i, i + 1), the second +0 past M
+        auto add_pair = [&](int i, float (&x)[NE]) {
+          float t[NE], g[NE];
+          group(4 * i, t);
+          if (4 * (i + 1) < s.M) {
+            group(4 * (i + 1), g);
+          } else {
 #pragma unroll
-        for (int e = 0; e < EPL; ++e) x[e] = __fadd_rn(x[e], __fadd_rn(t[e], g[e]));
-      };
-      group(0, acc);
-      if (s.M > 4) {
-        float g[EPL];
-        group(4, g);
+            for (int e = 0; e < NE; ++e) g[e] = 0.f;
+          }
 #pragma unroll
-        for (int e = 0; e < EPL; ++e) acc[e] = __fadd_rn(acc[e], g[e]);
-        if (s.M > 8) {
-          add_pair(2, acc);
-          if (s.M > 16) {
-            float h[EPL];
-            group(16, h);
-            if (s.M > 20) {
-              group(20, g);
-            } else {
+          for (int e = 0; e < NE; ++e) x[e] = __fadd_rn(x[e], __fadd_rn(t[e], g[e]));
+        };
+        float r[NE];
+        group(0, r);
+        if (s.M > 4) {
+          float g[NE];
+          group(4, g);
 #pragma unroll
-              for (int e = 0; e < EPL; ++e) g[e] = 0.f;
+          for (int e = 0; e < NE; ++e) r[e] = __fadd_rn(r[e], g[e]);
+          if (s.M > 8) {
+            add_pair(2, r);
+            if (s.M > 16) {
+              float h[NE];
+              group(16, h);
+              if (s.M > 20) {
+                group(20, g);
+              } else {
+#pragma unroll
+                for (int e = 0; e < NE; ++e) g[e] = 0.f;
+              }
+#pragma unroll
+              for (int e = 0; e < NE; ++e) h[e] = __fadd_rn(h[e], g[e]);
+              if (s.M > 24) {
+                add_pair(6, h);
+              } else {
+#pragma unroll
+                for (int e = 0; e < NE; ++e) h[e] = __fadd_rn(h[e], 0.f);
+              }
+#pragma unroll
+              for (int e = 0; e < NE; ++e) r[e] = __fadd_rn(r[e], h[e]);
             }
-#pragma unroll
-            for (int e = 0; e < EPL; ++e) h[e] = __fadd_rn(h[e], g[e]);
-            if (s.M > 24) {
-              add_pair(6, h);
-            } else {
-#pragma unroll
-              for (int e = 0; e < EPL; ++e) h[e] = __fadd_rn(h[e], 0.f);
-            }
-#pragma unroll
-            for (int e = 0; e < EPL; ++e) acc[e] = __fadd_rn(acc[e], h[e]);
           }
         }
+#pragma unroll
+        for (int e = 0; e < NE; ++e) acc[e0 + e] = r[e];
       }
     }
 #pragma unroll

@@ -62,7 +62,7 @@ constexpr int kBatch = 8;                                     // candidate loads
 constexpr int kSrvTile = 256;                                 // indices per server tile
 constexpr int kSrvThreads = 256;
 constexpr int kSrvWarpMaxM = 64;                              // workers the warp-per-tile server takes
-constexpr int kSrvWarpBuf = 512;                              // records a server warp stages at once
+constexpr int kSrvWarpBuf = 128;                              // records a server warp stages at once
 constexpr uint32_t kTauValid = 0x80000000u;                   // flag bit of the carried threshold word
 
 // State words.  ST_TAU (the carried threshold: kTauValid | key, or 0 for
@@ -172,7 +172,8 @@ __device__ void block_select(const uint32_t* hist, uint32_t k_rem, uint32_t* dig
 // `totals` again afterwards).
 template <int NT, int R, bool REUSE>
 __device__ __forceinline__ uint32_t write_tile_candidates(const float (&v)[R][4], const uint32_t (&cmask)[R],
-                                                          int64_t tile0, uint2* slot, uint32_t* totals) {
+                                                          int64_t tile0, uint2* slot, uint32_t* totals,
+                                                          uint32_t* err) {
   static_assert(R <= 4, "four 8-bit row counts per word");
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   uint32_t packed = 0;
@@ -203,7 +204,10 @@ __device__ __forceinline__ uint32_t write_tile_candidates(const float (&v)[R][4]
       const int64_t j = tile0 + 4 * ((int64_t)i * NT + threadIdx.x);
 #pragma unroll
       for (int q = 0; q < 4; ++q)
-        if ((cmask[i] >> q) & 1u) slot[pos++] = make_uint2((uint32_t)(j + q), __float_as_uint(v[i][q]));
+        if ((cmask[i] >> q) & 1u) {
+          if (dq_in_bounds(pos < (uint32_t)kTile, err)) slot[pos] = make_uint2((uint32_t)(j + q), __float_as_uint(v[i][q]));
+          ++pos;
+        }
     }
   }
   if constexpr (REUSE) __syncthreads();
@@ -320,7 +324,9 @@ __global__ void __launch_bounds__(kFormThreads, 6) topk_form_kernel(const Compre
     for (int q = 0; q < 4; ++q) {
       if ((lane_bits >> q) & 1u) {
         const int off = grp * 128 + lane * 4 + q;
-        slot[pos++] = make_uint2((uint32_t)(tile0 + off), __float_as_uint(vstage[off]));
+        if (dq_in_bounds(pos < (uint32_t)kTile, a.err))  // a tile holds at most kTile candidates
+          slot[pos] = make_uint2((uint32_t)(tile0 + off), __float_as_uint(vstage[off]));
+        ++pos;
       }
     }
   }
@@ -525,7 +531,7 @@ topk_select_kernel(const CompressArgs a, int64_t k, void* scratch) {
           }
         }
         const uint32_t n = write_tile_candidates<kSelThreads, kSelRows, true>(v, cmask, tile0,
-                                                                              rs.cand + t * kTile, sm.warp_sums);
+                                                                              rs.cand + t * kTile, sm.warp_sums, a.err);
         if (threadIdx.x == 0) rs.cnt[t] = n;
       }
       __syncthreads();
@@ -756,7 +762,7 @@ topk_select_kernel(const CompressArgs a, int64_t k, void* scratch) {
         const bool is_gt = (gtb[u] >> lane) & 1u, is_tie = (tieb[u] >> lane) & 1u;
         if (is_gt || (is_tie && my_t < need)) {
           const uint32_t pos = my_g + min(my_t, need);
-          if (pos < (uint64_t)k) {  // always true; keeps the write inside the message
+          if (dq_in_bounds(pos < (uint64_t)k, a.err)) {  // always true; keeps the write inside the message
             rec[pos] = c[u];
             keep(c[u]);
           }
@@ -778,7 +784,7 @@ topk_select_kernel(const CompressArgs a, int64_t k, void* scratch) {
       const uint32_t ties = tie_before + (ex >> 16);
       if (is_gt || (is_tie && ties < need)) {
         const uint32_t pos = gt_before + (ex & 0xFFFFu) + min(ties, need);
-        if (pos < (uint64_t)k) {  // always true; keeps the write inside the message
+        if (dq_in_bounds(pos < (uint64_t)k, a.err)) {  // always true; keeps the write inside the message
           rec[pos] = c;
           keep(c);
         }
@@ -984,7 +990,8 @@ __global__ void __launch_bounds__(kSrvThreads) topk_server_warp_kernel(const Ser
       for (uint32_t f = f0 + lane; f < f1; f += 32) {
         const uint2 r = buf[f - b];
         const int64_t off = (int64_t)r.x - tile0;
-        if (off >= 0 && off < kSrvTile && (int64_t)r.x < s.d) {
+        // records come from the compressor: inside the tile and below d
+        if (dq_in_bounds(off >= 0 && off < kSrvTile && (int64_t)r.x < s.d, s.err)) {
           const uint32_t n = srv_push_zeros(stk, (int)off, cnt[off], (uint32_t)m);
           srv_push_block(stk, (int)off, n, 0, __uint_as_float(r.y));
           cnt[off] = (uint8_t)(m + 1);
@@ -1042,7 +1049,7 @@ __global__ void __launch_bounds__(kSrvThreads) topk_server_owner_kernel(const Se
   const int64_t r = id - (int64_t)m * s.k;
   const uint2 mine = reinterpret_cast<const uint2*>(s.msgs + (int64_t)m * s.msg_stride)[r];
   const uint32_t j = mine.x;
-  if ((int64_t)j >= s.d) return;  // records come from the compressor and are < d
+  if (!dq_in_bounds((int64_t)j < s.d, s.err)) return;  // records come from the compressor and are < d
   const int64_t nts = srv_tiles(s.d);
   const int64_t t = j / kSrvTile;
   PairwiseAcc<13> sum;  // M <= 4096

@@ -12,7 +12,9 @@ import ctypes
 import os
 
 HERE = os.path.dirname(os.path.abspath(__file__))
-LIBRARY = os.path.join(HERE, "libdqgan.so")
+# The library to load: libdqgan.so next to this file, or the path the
+# environment variable DQGAN_LIBRARY names (the checked build, for instance).
+LIBRARY = os.environ.get("DQGAN_LIBRARY") or os.path.join(HERE, "libdqgan.so")
 
 OK = 0
 ERR_INVALID_ARG = -1
@@ -20,6 +22,7 @@ ERR_OOM = -2
 ERR_CUDA = -3
 ERR_UNSUPPORTED = -4
 ERR_TIMEOUT = -5
+ERR_BOUNDS = -6
 
 SIGN, TOPK, SQUANT, IDENTITY, QSGD = 0, 1, 2, 3, 4
 KEEP_LOOKAHEAD = 1

@@ -57,14 +57,16 @@ def test_ranges_match_the_single_handle(P, kw, ranks):
     w_rep = [w0.clone() for _ in range(ranks)]
     msgs_ref = torch.zeros((M, mb), dtype=torch.uint8, device=dev)
     msgs = torch.zeros((M, mb), dtype=torch.uint8, device=dev)
+    ld = (d + 3) // 4 * 4  # gradient rows 16-byte aligned
+    g = torch.zeros((M, ld), dtype=torch.float32, device=dev)
     for t in range(4):
-        g = torch.from_numpy((rng.standard_normal((M, d)) * np.exp(rng.uniform(-3, 1, (M, d))))
-                             .astype(np.float32)).to(dev)
-        ref.workers_compress_all(g, d, msgs_ref)
+        g[:, :d] = torch.from_numpy((rng.standard_normal((M, d)) * np.exp(rng.uniform(-3, 1, (M, d))))
+                                    .astype(np.float32)).to(dev)
+        ref.workers_compress_all(g, ld, msgs_ref)
         ref.server_aggregate_update(msgs_ref, w_ref)
         for h, a, b in parts:
             if b > a:
-                h.workers_compress_range(a, b - a, g[a:b], d, msgs[a:b])
+                h.workers_compress_range(a, b - a, g[a:b], ld, msgs[a:b])
         for (h, a, b), w in zip(parts, w_rep):
             h.server_aggregate_update(msgs, w)
         torch.cuda.synchronize(dev)
@@ -81,7 +83,7 @@ def test_ranges_match_the_single_handle(P, kw, ranks):
             with pytest.raises(P.DqganError):  # outside the handle's range
                 h.get_residual(a - 1, np.empty(d, np.float32))
             with pytest.raises(P.DqganError):  # not all workers are local
-                h.workers_compress_all(g, d, msgs)
+                h.workers_compress_all(g, ld, msgs)
         h.destroy()
     ref.destroy()
 
@@ -90,7 +92,7 @@ def test_sharded_step_single_process(P):
     from paper_2010_13359_gb300.sharded import CudaEngine, ShardedStep
     dev = torch.device("cuda:0")
     stream = torch.cuda.current_stream(dev)
-    d, M = 123_457, 4
+    d, M = 123_456, 4
     cfg = P.make_config(d=d, M=M, compressor=P.SIGN, bucket=1024, lr=1e-2, cuda_stream=stream.cuda_stream)
     eng = CudaEngine(cfg, 0, M)
     step = ShardedStep(eng, M, device=dev)
