@@ -841,7 +841,7 @@ __device__ __forceinline__ void b2_pair_table_update(const uint32_t* words, cons
 }
 
 // Passes over a lane's 8 elements in the b = 4 per-worker decode (1 or 2).
-constexpr int kSquant4Parts = 2;
+constexpr int kSquant4Parts = 1;
 
 // Whether the squant server stages the parameters by TMA (b = 2 and 4; for
 // b = 8 a lane's 16 bytes of w are contiguous across the warp already).

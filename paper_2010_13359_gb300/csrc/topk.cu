@@ -900,17 +900,23 @@ __device__ __forceinline__ uint32_t srv_push_zeros(float* stk, int off, uint32_t
 // touched index's sum to P leaves and updates the touched w_j (all loads of
 // w issued before the stores).  Untouched indices sum to +0 and keep w_j.
 // Per-warp shared memory (srv_warp_bytes): the record buffer, then
-// srv_levels(M) rows of per-index blocks, the per-worker record ranges, and
-// one count byte per index.
+// srv_levels(M) rows of per-index blocks, a row of lone values, the
+// per-worker record ranges, and one count byte per index.  An index that
+// only one worker sent (the common case) never touches the blocks: its value
+// waits in the lone-value row, and its tree is that value plus +0.
 __host__ __device__ constexpr int srv_levels(int M) {
   int l = 1;
   while ((1 << (l - 1)) < M) ++l;
   return l;  // log2(next_pow2(M)) + 1
 }
 __host__ __device__ constexpr size_t srv_warp_bytes(int M) {
-  return (size_t)kSrvWarpBuf * 8 + (size_t)srv_levels(M) * kSrvTile * 4 + (kSrvWarpMaxM + kSrvWarpMaxM + 4) * 4 +
-         kSrvTile;
+  return (size_t)kSrvWarpBuf * 8 + (size_t)(srv_levels(M) + 1) * kSrvTile * 4 +
+         (kSrvWarpMaxM + kSrvWarpMaxM + 4) * 4 + kSrvTile;
 }
+// An index's count byte: 0 untouched; kSrvSingle | (m + 1) while worker m's
+// value is the index's only one (kept aside, not yet in the blocks); else
+// the number of workers accounted for in the blocks.
+constexpr uint8_t kSrvSingle = 0x80;
 constexpr int kSrvWarps = kSrvThreads / 32;
 
 template <bool POW2>
@@ -922,7 +928,8 @@ __global__ void __launch_bounds__(kSrvThreads) topk_server_warp_kernel(const Ser
   unsigned char* region = smem_raw + (size_t)warp * srv_warp_bytes(M);
   uint2* buf = reinterpret_cast<uint2*>(region);
   float* stk = reinterpret_cast<float*>(region + (size_t)kSrvWarpBuf * 8);
-  uint32_t* first = reinterpret_cast<uint32_t*>(stk + nlev * kSrvTile);
+  float* single = stk + nlev * kSrvTile;  // an index's value while it is the only one
+  uint32_t* first = reinterpret_cast<uint32_t*>(single + kSrvTile);
   uint32_t* pre = first + kSrvWarpMaxM;
   uint8_t* cnt = reinterpret_cast<uint8_t*>(pre + kSrvWarpMaxM + 4);
   const int64_t nts = srv_tiles(s.d);
@@ -992,9 +999,24 @@ __global__ void __launch_bounds__(kSrvThreads) topk_server_warp_kernel(const Ser
         const int64_t off = (int64_t)r.x - tile0;
         // records come from the compressor: inside the tile and below d
         if (dq_in_bounds(off >= 0 && off < kSrvTile && (int64_t)r.x < s.d, s.err)) {
-          const uint32_t n = srv_push_zeros(stk, (int)off, cnt[off], (uint32_t)m);
-          srv_push_block(stk, (int)off, n, 0, __uint_as_float(r.y));
-          cnt[off] = (uint8_t)(m + 1);
+          const int o = (int)off;
+          const uint8_t c = cnt[o];
+          const float v = __uint_as_float(r.y);
+          if (c == 0) {  // the index's first value: kept aside (most indices get only one)
+            single[o] = v;
+            cnt[o] = (uint8_t)(kSrvSingle | (m + 1));
+          } else {
+            uint32_t n = c;
+            if (c & kSrvSingle) {  // a second value: the first goes into the blocks now
+              const uint32_t m1 = (c & ~kSrvSingle) - 1u;
+              n = srv_push_zeros(stk, o, 0, m1);
+              srv_push_block(stk, o, n, 0, single[o]);
+              n = m1 + 1;
+            }
+            n = srv_push_zeros(stk, o, n, (uint32_t)m);
+            srv_push_block(stk, o, n, 0, v);
+            cnt[o] = (uint8_t)(m + 1);
+          }
         }
       }
       __syncwarp();
@@ -1018,7 +1040,9 @@ __global__ void __launch_bounds__(kSrvThreads) topk_server_warp_kernel(const Ser
       upd[q] = n != 0 || (dense && tile0 + i < s.d);
       wv[q] = upd[q] ? s.w[tile0 + i] : 0.f;
       sum[q] = 0.f;
-      if (n) {
+      if (n & kSrvSingle) {  // one value v among +0 leaves: the tree gives v + 0 (v alone when P = 1)
+        sum[q] = P == 1 ? single[i] : __fadd_rn(single[i], 0.f);
+      } else if (n) {
         srv_push_zeros(stk, i, n, P);
         sum[q] = stk[(nlev - 1) * kSrvTile + i];
       }
