@@ -840,8 +840,10 @@ __device__ __forceinline__ void b2_pair_table_update(const uint32_t* words, cons
   }
 }
 
-// Passes over a lane's 8 elements in the b = 4 per-worker decode (1 or 2).
+// Passes over a lane's 8 elements in the b = 4 per-worker decode (1 or 2),
+// and whether b = 4 with M <= 16 decodes element by element instead.
 constexpr int kSquant4Parts = 1;
+constexpr bool kSquant4ElementOuter = true;
 
 // Whether the squant server stages the parameters by TMA (b = 2 and 4; for
 // b = 8 a lane's 16 bytes of w are contiguous across the warp already).
@@ -873,7 +875,7 @@ constexpr bool sq_params_boxed(int bits) { return bits != 8; }
 // Per warp two buffers of each kind: slice i + 1 loads while slice i is
 // decoded.
 template <int BITS, bool POW2, bool SEG, int NSET>
-__global__ void __launch_bounds__(32 * kTmaWarps)
+__global__ void __launch_bounds__(32 * kTmaWarps, (kSquant4ElementOuter && BITS == 4 && !SEG && NSET == 1) ? 4 : 1)
 squant_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap tmap,
                          const __grid_constant__ CUtensorMap pmap) {
   constexpr int K = (1 << (BITS - 1)) - 1;
@@ -1070,8 +1072,45 @@ squant_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap
     // as the padded tree over the next_pow2(ceil(M / 4)) <= 8 groups: G0;
     // G0 + G1; (G0 + G1) + (G2 + G3); then + ((G4 + G5) + (G6 + G7)), groups
     // past M being +0 (M is warp-uniform, so are the branches)
-    const bool per_worker = BITS != 2 || (SEG && mixed);
-    if (per_worker) {
+    // b = 4 with at most 16 workers and one scale per slice: element by
+    // element instead -- every worker's product fl(s V[c]) (one per lane)
+    // and code word held in registers, and for each element its 16 values
+    // looked up and summed as the padded tree of up to four groups.  The live
+    // set is the 32 held registers and one element's partial sums, not
+    // eight elements' (64 registers instead of 80, four CTAs per SM).
+    // (b = 4 launches with NSET = 1 for M <= 16, 2 above.)
+    constexpr bool ELEMENTWISE = kSquant4ElementOuter && BITS == 4 && !SEG && NSET == 1;
+    const bool per_worker = (BITS != 2 || (SEG && mixed)) && !ELEMENTWISE;
+    if constexpr (ELEMENTWISE) {
+      float T4m[16];
+      uint32_t wm[16];
+#pragma unroll
+      for (int m = 0; m < 16; ++m) {
+        const bool here = m < s.M;  // warp-uniform
+        T4m[m] = here ? __fmul_rn(scale_of(m), V4) : 0.f;
+        wm[m] = here ? words[32 * m] : 0u;
+      }
+#pragma unroll
+      for (int e = 0; e < EPL; ++e) {
+        float G[4];
+#pragma unroll
+        for (int g = 0; g < 4; ++g) {
+          float v[4];
+#pragma unroll
+          for (int u = 0; u < 4; ++u) {
+            const int m = 4 * g + u;
+            v[u] = (4 * g < s.M) ? __shfl_sync(kFullMask, T4m[m], (int)(wm[m] >> (4 * e))) : 0.f;
+            if (m >= s.M) v[u] = 0.f;  // +0 leaves past M
+          }
+          G[g] = group4(v[0], v[1], v[2], v[3], s.M);
+        }
+        // the padded tree over next_pow2(ceil(M / 4)) groups
+        float r = G[0];
+        if (s.M > 4) r = __fadd_rn(r, G[1]);
+        if (s.M > 8) r = __fadd_rn(r, __fadd_rn(G[2], s.M > 12 ? G[3] : 0.f));
+        wv[e] = server_out(s, wv[e], average_t<POW2>(r, s));  // stored as is below
+      }
+    } else if (per_worker) {
 #pragma unroll
       for (int part = 0; part < kParts; ++part) {
         const int e0 = part * NE;
@@ -1465,7 +1504,10 @@ cudaError_t launch_squant_server(const ServerArgs& s, const CUtensorMap* params_
         if (s.M <= 16) DQ_SQ_TMA(2, 1);
         else DQ_SQ_TMA(2, 2);
         break;
-      case 4: DQ_SQ_TMA(4, 1); break;
+      case 4:
+        if (s.M <= 16) DQ_SQ_TMA(4, 1);
+        else DQ_SQ_TMA(4, 2);
+        break;
       case 8: DQ_SQ_TMA(8, 1); break;
     }
 #undef DQ_SQ_TMA

@@ -158,3 +158,18 @@ def test_server_optimizer_calls_reject_a_null_handle(P):
     assert L.dqgan_set_server_optimizer(None, ctypes.byref(opt)) == P.dqgan.ERR_INVALID_ARG
     assert L.dqgan_get_server_state(None, 0, None) == P.dqgan.ERR_INVALID_ARG
     assert b"NULL" in L.dqgan_last_error(None)
+
+
+def test_sharding_calls_reject_a_null_handle(P):
+    L = P.dqgan.load_library()
+    assert L.dqgan_set_local_workers(None, 0, 1) == P.dqgan.ERR_INVALID_ARG
+    assert L.dqgan_workers_compress_range(None, 0, 1, None, 4, None) == P.dqgan.ERR_INVALID_ARG
+    assert b"NULL" in L.dqgan_last_error(None)
+
+
+def test_status_codes_match_the_header(P):
+    hdr = open(os.path.join(ROOT, "include", "dqgan.h")).read()
+    for name in ("OK", "ERR_INVALID_ARG", "ERR_OOM", "ERR_CUDA", "ERR_UNSUPPORTED", "ERR_TIMEOUT", "ERR_BOUNDS"):
+        m = re.search(r"#define DQGAN_%s \(?(-?\d+)\)?" % name, hdr)
+        assert m, name
+        assert int(m.group(1)) == getattr(P.dqgan, name), name
