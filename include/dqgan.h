@@ -205,13 +205,16 @@ DQGAN_API int dqgan_set_local_workers(dqgan_handle* h, int32_t first, int32_t co
 
 /*
  * Server step of Algorithm 2, fused: decode the M messages, average them
- * (q_hat = fl(sum_m Q_m / M); the summation order over m is not specified,
- * except for TOPK and IDENTITY where it is worker order), and update the
- * parameters in place, w = fl(w - q_hat).  Then t <- t + 1.
+ * (q_hat = fl(S / M), S the sum over workers in one fixed order: the M
+ * decoded values, padded with +0 to the next power of two, summed pairwise
+ * -- at every level x_i = fl(x_2i + x_2i+1) -- so the result does not depend
+ * on the kernel that runs), and update the parameters in place,
+ * w = fl(w - q_hat), or apply the server rule dqgan_set_server_optimizer
+ * chose.  Then t <- t + 1.
  * msgs_all: device, M messages back to back (stride dqgan_message_bytes()).
  * params:   device, d fp32, caller-owned, read and written.
  * SIGN with bucket >= 1024 and M <= 32 has two server kernels with the same
- * results up to summation order; the library picks by size.  The environment
+ * results; the library picks by size.  The environment
  * variable DQGAN_SIGN_SERVER, read by dqgan_create, fixes the choice for the
  * handle: "col" (per-lane bit transpose, parameters staged by TMA; needs
  * d >= 32) or "tma" (warp bit transpose).  Any other value: by size.

@@ -840,10 +840,9 @@ __device__ __forceinline__ void b2_pair_table_update(const uint32_t* words, cons
   }
 }
 
-// Passes over a lane's 8 elements in the b = 4 per-worker decode (1 or 2),
-// and whether b = 4 with M <= 16 decodes element by element instead.
+// Passes over a lane's 8 elements in the b = 4 per-worker decode (1 or 2).
 constexpr int kSquant4Parts = 1;
-constexpr bool kSquant4ElementOuter = true;
+
 
 // Whether the squant server stages the parameters by TMA (b = 2 and 4; for
 // b = 8 a lane's 16 bytes of w are contiguous across the warp already).
@@ -873,9 +872,10 @@ constexpr bool sq_params_boxed(int bits) { return bits != 8; }
 // Rows past the map read as zero and are not stored; the partial last row
 // (d mod 32 elements, outside the map) is read and written directly.
 // Per warp two buffers of each kind: slice i + 1 loads while slice i is
-// decoded.
-template <int BITS, bool POW2, bool SEG, int NSET>
-__global__ void __launch_bounds__(32 * kTmaWarps, (kSquant4ElementOuter && BITS == 4 && !SEG && NSET == 1) ? 4 : 1)
+// decoded.  FM > 0 fixes the worker count at compile time (s.M == FM): the
+// per-worker decode then has no tests for workers past M.
+template <int BITS, bool POW2, bool SEG, int NSET, int FM>
+__global__ void __launch_bounds__(32 * kTmaWarps)
 squant_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap tmap,
                          const __grid_constant__ CUtensorMap pmap) {
   constexpr int K = (1 << (BITS - 1)) - 1;
@@ -890,7 +890,8 @@ squant_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap
   __shared__ float V8[BITS == 8 ? 256 * 32 : 1];
   const int lane = threadIdx.x & 31;
   const int warp = threadIdx.x >> 5;
-  const uint32_t box_bytes = (uint32_t)s.M * 128u;
+  const int M = FM > 0 ? FM : s.M;
+  const uint32_t box_bytes = (uint32_t)M * 128u;
   const uint32_t raw = smem_addr(smem_raw);
   // parameter boxes of every warp first (1024-byte aligned), then the word boxes
   uint8_t* const pbuf0 = smem_raw + ((1024u - (raw & 1023u)) & 1023u) + warp * 2 * PBOX;  // + i * PBOX
@@ -931,7 +932,7 @@ squant_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap
   const int32_t x0 = (int32_t)(s.off_payload >> 2);
   const int64_t nrows = s.d >> 5;     // rows of the parameter map
   const int tail = (int)(s.d & 31);   // elements of the partial row nrows
-  const bool active = lane < s.M;
+  const bool active = lane < M;
   // slice sl covers code words [32 sl, 32 sl + 32) and parameter rows
   // [R sl, R sl + R): buckets hold whole slices
   auto issue = [&](int64_t sl_, int i) {
@@ -1072,45 +1073,8 @@ squant_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap
     // as the padded tree over the next_pow2(ceil(M / 4)) <= 8 groups: G0;
     // G0 + G1; (G0 + G1) + (G2 + G3); then + ((G4 + G5) + (G6 + G7)), groups
     // past M being +0 (M is warp-uniform, so are the branches)
-    // b = 4 with at most 16 workers and one scale per slice: element by
-    // element instead -- every worker's product fl(s V[c]) (one per lane)
-    // and code word held in registers, and for each element its 16 values
-    // looked up and summed as the padded tree of up to four groups.  The live
-    // set is the 32 held registers and one element's partial sums, not
-    // eight elements' (64 registers instead of 80, four CTAs per SM).
-    // (b = 4 launches with NSET = 1 for M <= 16, 2 above.)
-    constexpr bool ELEMENTWISE = kSquant4ElementOuter && BITS == 4 && !SEG && NSET == 1;
-    const bool per_worker = (BITS != 2 || (SEG && mixed)) && !ELEMENTWISE;
-    if constexpr (ELEMENTWISE) {
-      float T4m[16];
-      uint32_t wm[16];
-#pragma unroll
-      for (int m = 0; m < 16; ++m) {
-        const bool here = m < s.M;  // warp-uniform
-        T4m[m] = here ? __fmul_rn(scale_of(m), V4) : 0.f;
-        wm[m] = here ? words[32 * m] : 0u;
-      }
-#pragma unroll
-      for (int e = 0; e < EPL; ++e) {
-        float G[4];
-#pragma unroll
-        for (int g = 0; g < 4; ++g) {
-          float v[4];
-#pragma unroll
-          for (int u = 0; u < 4; ++u) {
-            const int m = 4 * g + u;
-            v[u] = (4 * g < s.M) ? __shfl_sync(kFullMask, T4m[m], (int)(wm[m] >> (4 * e))) : 0.f;
-            if (m >= s.M) v[u] = 0.f;  // +0 leaves past M
-          }
-          G[g] = group4(v[0], v[1], v[2], v[3], s.M);
-        }
-        // the padded tree over next_pow2(ceil(M / 4)) groups
-        float r = G[0];
-        if (s.M > 4) r = __fadd_rn(r, G[1]);
-        if (s.M > 8) r = __fadd_rn(r, __fadd_rn(G[2], s.M > 12 ? G[3] : 0.f));
-        wv[e] = server_out(s, wv[e], average_t<POW2>(r, s));  // stored as is below
-      }
-    } else if (per_worker) {
+    const bool per_worker = BITS != 2 || (SEG && mixed);
+    if (per_worker) {
 #pragma unroll
       for (int part = 0; part < kParts; ++part) {
         const int e0 = part * NE;
@@ -1121,20 +1085,20 @@ squant_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap
           float sc[4];
 #pragma unroll
           for (int u = 0; u < 4; ++u) {
-            const bool here = m + u < s.M;  // warp-uniform
+            const bool here = m + u < M;  // warp-uniform
             wd[u] = here ? words[32 * (m + u)] : 0u;
             sc[u] = here ? scale_of(m + u) : 0.f;
           }
           float va[NE], vb[NE];
           decode_part(wd[0], sc[0], e0, va);
           decode_part(wd[1], sc[1], e0, vb);
-          const bool h1 = m + 1 < s.M;
+          const bool h1 = m + 1 < M;
 #pragma unroll
-          for (int e = 0; e < NE; ++e) g[e] = s.M == 1 ? va[e] : __fadd_rn(va[e], h1 ? vb[e] : 0.f);
-          if (s.M <= 2) return;
+          for (int e = 0; e < NE; ++e) g[e] = M == 1 ? va[e] : __fadd_rn(va[e], h1 ? vb[e] : 0.f);
+          if (M <= 2) return;
           decode_part(wd[2], sc[2], e0, va);
           decode_part(wd[3], sc[3], e0, vb);
-          const bool h2 = m + 2 < s.M, h3 = m + 3 < s.M;
+          const bool h2 = m + 2 < M, h3 = m + 3 < M;
 #pragma unroll
           for (int e = 0; e < NE; ++e) g[e] = __fadd_rn(g[e], __fadd_rn(h2 ? va[e] : 0.f, h3 ? vb[e] : 0.f));
         };
@@ -1142,7 +1106,7 @@ squant_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap
         auto add_pair = [&](int i, float (&x)[NE]) {
           float t[NE], g[NE];
           group(4 * i, t);
-          if (4 * (i + 1) < s.M) {
+          if (4 * (i + 1) < M) {
             group(4 * (i + 1), g);
           } else {
 #pragma unroll
@@ -1153,17 +1117,17 @@ squant_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap
         };
         float r[NE];
         group(0, r);
-        if (s.M > 4) {
+        if (M > 4) {
           float g[NE];
           group(4, g);
 #pragma unroll
           for (int e = 0; e < NE; ++e) r[e] = __fadd_rn(r[e], g[e]);
-          if (s.M > 8) {
+          if (M > 8) {
             add_pair(2, r);
-            if (s.M > 16) {
+            if (M > 16) {
               float h[NE];
               group(16, h);
-              if (s.M > 20) {
+              if (M > 20) {
                 group(20, g);
               } else {
 #pragma unroll
@@ -1171,7 +1135,7 @@ squant_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap
               }
 #pragma unroll
               for (int e = 0; e < NE; ++e) h[e] = __fadd_rn(h[e], g[e]);
-              if (s.M > 24) {
+              if (M > 24) {
                 add_pair(6, h);
               } else {
 #pragma unroll
@@ -1379,9 +1343,9 @@ bool sign_col_pays(const ServerArgs& s) {
   return nslices >= 4ll * sms[dev] * kColWarps;
 }
 
-template <int BITS, bool POW2, bool SEG, int NSET>
+template <int BITS, bool POW2, bool SEG, int NSET, int FM = 0>
 cudaError_t launch_squant_tma(const ServerArgs& s, const CUtensorMap* params_map, cudaStream_t stream) {
-  auto kern = squant_server_tma_kernel<BITS, POW2, SEG, NSET>;
+  auto kern = squant_server_tma_kernel<BITS, POW2, SEG, NSET, FM>;
   constexpr int pbox = sq_params_boxed(BITS) ? 32 * (32 / BITS) * 4 : 0;  // bytes of a parameter box
   const int smem = kTmaWarps * 2 * (pbox + s.M * 128) + 1024;  // + alignment slack
   int dev = 0;
@@ -1505,10 +1469,13 @@ cudaError_t launch_squant_server(const ServerArgs& s, const CUtensorMap* params_
         else DQ_SQ_TMA(2, 2);
         break;
       case 4:
-        if (s.M <= 16) DQ_SQ_TMA(4, 1);
-        else DQ_SQ_TMA(4, 2);
+        if (s.M == 16 && !s.word_bucket) st = launch_squant_tma<4, true, false, 1, 16>(s, params_map, stream);
+        else DQ_SQ_TMA(4, 1);
         break;
-      case 8: DQ_SQ_TMA(8, 1); break;
+      case 8:
+        if (s.M == 16 && !s.word_bucket) st = launch_squant_tma<8, true, false, 1, 16>(s, params_map, stream);
+        else DQ_SQ_TMA(8, 1);
+        break;
     }
 #undef DQ_SQ_TMA
     *launches += 1;
