@@ -137,7 +137,10 @@ DQGAN_API int dqgan_validate_config(const dqgan_config* cfg);
  * statement dqgan_create(d, M, compressor, lr, buckets) plus the fields the
  * compressors need).  Allocates on the current device: e (M x d fp32, zero:
  * e_0 = 0), h (M x d fp32, zero, only with DQGAN_KEEP_LOOKAHEAD: F(w_{-1/2})
- * is taken as 0 so that w_{1/2} = w_0), and top-k scratch.  Sets t = 1.
+ * is taken as 0 so that w_{1/2} = w_0), and top-k scratch (per worker row
+ * about 8 bytes per parameter for the candidates; for M <= 64 the server's
+ * per-index worker masks and per-worker value rows, 8 + 4M bytes per
+ * parameter, else a table of record ranges).  Sets t = 1.
  * *out receives the handle; on error *out is NULL and
  * dqgan_last_error(NULL) holds the reason, and nothing stays allocated.
  * Test hook: with the environment variable DQGAN_TEST_FAIL_ALLOC=N set, the

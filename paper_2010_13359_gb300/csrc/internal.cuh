@@ -137,11 +137,13 @@ cudaError_t launch_identity_compress(const CompressArgs& a, bool keep_h, cudaStr
                                      uint64_t* launches);
 
 // Scratch of the top-k path: `rows` rows (one per local worker) and the
-// server's record-range table for `nworkers` messages.  A row needs no clearing
-// between calls: every call rewrites its tile counts, tile prefixes and
-// candidates in full.  Only the row's last state word carries over -- the
+// server's tables for `nworkers` messages (none for 0).  A row needs no
+// clearing between calls: every call rewrites its tile counts, tile prefixes
+// and candidates in full.  Only the row's last state word carries over -- the
 // candidate threshold of the worker's previous call (0 before the first),
-// which decides how much work the first pass saves and never a result.
+// which decides how much work the first pass saves and never a result.  The
+// server's per-index worker masks (up to 64 workers) must be zero when the
+// scratch is created; each server call clears the masks it set.
 size_t topk_scratch_bytes(int64_t d, int32_t rows, int32_t nworkers);
 cudaError_t launch_topk_compress(const CompressArgs& a, int64_t k, bool keep_h, void* scratch,
                                  cudaStream_t stream, uint64_t* launches);

@@ -56,7 +56,7 @@ extern "C" int dqgan_topk_compress_noalloc(const float* g, float* e, void* out_m
   if (((uintptr_t)g | (uintptr_t)e | (uintptr_t)out_msg) & 15u)
     return dq::set_thread_error(DQGAN_ERR_INVALID_ARG,
                                 "gradient, residual and message must be 16-byte aligned");
-  const size_t need = dq::topk_scratch_bytes(d, 1, 1);
+  const size_t need = dq::topk_scratch_bytes(d, 1, 0);  // one row, no server tables
   if (need > dq::kNoAllocScratchBytes)
     return dq::set_thread_error(DQGAN_ERR_INVALID_ARG, "top-k scratch for this d exceeds the fixed array");
 

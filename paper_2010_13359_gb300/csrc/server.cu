@@ -811,10 +811,11 @@ __device__ __forceinline__ void build_pair_tables(float my_scale, int lane, int 
 // values are summed pairwise over the padded tree's next_pow2(ceil(M/2))
 // pairs (one set: 1, 2, 4 or 8 of them, the level picked by M; two sets:
 // the two 8-pair sums added last).
-template <int NSET, bool POW2>
+template <int NSET, bool POW2, int FM>
 __device__ __forceinline__ void b2_pair_table_update(const uint32_t* words, const ServerArgs& s,
                                                      const float (&T)[8 * NSET], float (&wv)[16]) {
-  const int np = next_pow2((s.M + 1) / 2);  // pairs in the padded tree (NSET = 2: 16)
+  const int M = FM > 0 ? FM : s.M;
+  const int np = next_pow2((M + 1) / 2);  // pairs in the padded tree (NSET = 2: 16)
   float acc[16];
 #pragma unroll
   for (int set = 0; set < NSET; ++set) {
@@ -822,7 +823,7 @@ __device__ __forceinline__ void b2_pair_table_update(const uint32_t* words, cons
 #pragma unroll
     for (int r = 0; r < 16; ++r) {
       const int m = 16 * set + r;
-      z[r] = m < s.M ? words[32 * m] : 0x55555555u;  // rows past M: level-0 codes (never read past the box)
+      z[r] = m < M ? words[32 * m] : 0x55555555u;  // rows past M: level-0 codes (never read past the box)
     }
     transpose16x2_regs(z);
 #pragma unroll
@@ -1063,10 +1064,10 @@ squant_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap
     if constexpr (BITS == 2) {
       if (!(SEG && mixed)) {
         if (bkt != t2_bkt) {
-          build_pair_tables<8 * NSET>(my_scale, lane, s.M, T2);
+          build_pair_tables<8 * NSET>(my_scale, lane, M, T2);
           t2_bkt = bkt;
         }
-        b2_pair_table_update<NSET, POW2>(words, s, T2, wv);
+        b2_pair_table_update<NSET, POW2, FM>(words, s, T2, wv);
       }
     }
     // groups of four workers, G = (a + b) + (c + d) with +0 past M, combined
@@ -1465,7 +1466,8 @@ cudaError_t launch_squant_server(const ServerArgs& s, const CUtensorMap* params_
                            : launch_squant_tma<B, false, false, NSET>(s, params_map, stream))
     switch (s.bits) {
       case 2:
-        if (s.M <= 16) DQ_SQ_TMA(2, 1);
+        if (s.M == 16 && !s.word_bucket) st = launch_squant_tma<2, true, false, 1, 16>(s, params_map, stream);
+        else if (s.M <= 16) DQ_SQ_TMA(2, 1);
         else DQ_SQ_TMA(2, 2);
         break;
       case 4:

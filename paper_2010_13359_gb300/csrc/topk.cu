@@ -31,11 +31,13 @@
 //
 // Server: w_j -= (sum over workers of the value recorded for j, absent
 // workers as +0, in the library's pairwise order) / M at the indices some
-// worker sent; elsewhere the sum is +0 and w is unchanged.  A first kernel
-// finds, for each worker and each tile of 256 indices, where the tile's
-// records start; then one warp per tile builds the tile's per-index sums in
-// shared memory, worker by worker, and updates the touched parameters (one
-// thread per record, with searches narrowed to the tile, above 64 workers).
+// worker sent; elsewhere the sum is +0 and w is unchanged.  Up to 64
+// workers, one thread per record in two launches: the records scatter their
+// values into per-worker rows and set their worker's bit in a per-index
+// mask, then the lowest worker of each index sums the index's values and
+// updates w_j.  Above 64 workers, a first kernel finds where each worker's
+// records of each 256-index tile start, and one thread per record searches
+// the other workers' records of its tile.
 #include <atomic>
 
 #include <cooperative_groups.h>
@@ -61,8 +63,6 @@ constexpr int kCacheCap = 20480;                              // candidates a se
 constexpr int kBatch = 8;                                     // candidate loads in flight per thread
 constexpr int kSrvTile = 256;                                 // indices per server tile
 constexpr int kSrvThreads = 256;
-constexpr int kSrvWarpMaxM = 64;                              // workers the warp-per-tile server takes
-constexpr int kSrvWarpBuf = 128;                              // records a server warp stages at once
 constexpr uint32_t kTauValid = 0x80000000u;                   // flag bit of the carried threshold word
 
 // State words.  ST_TAU (the carried threshold: kTauValid | key, or 0 for
@@ -862,197 +862,144 @@ __device__ __forceinline__ float srv_average(float acc, const ServerArgs& s) {
   else return __fdiv_rn(acc, (float)s.M);
 }
 
-// Per index, the server's sum over workers in the library's order (the
-// M values padded with +0 to P = next_pow2(M), summed pairwise), built
-// worker by worker with absent workers as +0 leaves: stk holds the index's
-// complete blocks (level L: the sum of 2^L consecutive workers, column
-// `off` of row L, rows kSrvTile floats apart), n the workers accounted for.
-// Pushes the block of 2^L workers starting at n (n a multiple of 2^L).
-__device__ __forceinline__ void srv_push_block(float* stk, int off, uint32_t n, int L, float v) {
-  float c = v;
-  uint32_t k = n >> L;
-  int l = L;
-  while (k & 1u) {
-    c = __fadd_rn(stk[l * kSrvTile + off], c);
-    k >>= 1;
-    ++l;
-  }
-  stk[l * kSrvTile + off] = c;
-}
+// Per index, the server's sum over workers in the library's order (the M
+// values padded with +0 to P = next_pow2(M), summed pairwise) as a binary
+// counter over complete blocks of leaves: lv[L] holds the sum of the last
+// complete block of 2^L leaves while bit L of n is set, n the leaves
+// accounted for.  Absent workers enter as blocks of +0 leaves of the largest
+// aligned size (a block of +0 leaves sums to +0), so the value is the dense
+// padded tree's at a cost of a few additions per present worker.
+template <int LEV>
+struct SparseTree {
+  float lv[LEV];
+  uint32_t n = 0;
 
-// Accounts for workers n .. t - 1 as +0 leaves, in the largest aligned
-// blocks (a block of +0 leaves sums to +0); returns t.
-__device__ __forceinline__ uint32_t srv_push_zeros(float* stk, int off, uint32_t n, uint32_t t) {
-  while (n < t) {
-    int L = 31 - __clz((int)(t - n));  // the largest block that fits
-    if (n) L = min(L, __ffs((int)n) - 1);  // and that starts on a multiple of its size
-    srv_push_block(stk, off, n, L, 0.f);
+  // Pushes a complete block of 2^L leaves summing to x (n a multiple of 2^L).
+  __device__ __forceinline__ void push_block(int L, float x) {
+    float c = x;
+    bool placed = false;
+#pragma unroll
+    for (int l = 0; l < LEV; ++l) {
+      if (!placed && l >= L) {
+        if ((n >> l) & 1u) {
+          c = __fadd_rn(lv[l], c);  // left sibling + this block
+        } else {
+          lv[l] = c;
+          placed = true;
+        }
+      }
+    }
     n += 1u << L;
   }
-  return n;
+  // Accounts for leaves n .. t - 1 as +0.
+  __device__ __forceinline__ void push_zeros(uint32_t t) {
+    while (n < t) {
+      int L = 31 - __clz((int)(t - n));       // the largest block that fits
+      if (n) L = min(L, __ffs((int)n) - 1);  // and starts on a multiple of its size
+      push_block(L, 0.f);
+    }
+  }
+};
+
+// Server for M <= kSrvMaskMaxM: two launches over the M * k records, with
+// two tables in the scratch -- a worker mask per index (u64; all zero
+// between calls) and a value row per worker (d floats, never cleared).
+//   1. scatter: record (m, r) with index j writes its value to row m at j
+//      and sets bit m of j's mask.
+//   2. reduce: the record of the lowest worker in j's mask owns j.  It sums
+//      the values of the workers in the mask, in worker order with the
+//      absent workers as +0 leaves (the library's pairwise order), updates
+//      w_j and clears j's mask.  The other records of j read its mask
+//      before or after the owner clears it; either way their own bit is not
+//      its lowest, so they do nothing.
+// Indices nobody sent have the sum +0 and keep w_j; with store_q the q_hat
+// buffer is cleared before the scatter.
+constexpr int kSrvMaskMaxM = 64;
+
+constexpr int kSrvLevels = 7;  // log2(64) + 1
+constexpr int kSrvBatch = 8;   // value loads an owner has in flight
+
+struct SrvTables {
+  unsigned long long* mask;  // d masks
+  float* vals;               // row m at vals + m * ldv
+  int64_t ldv;
+};
+
+__host__ __device__ constexpr int64_t srv_mask_table_words(int64_t d, int32_t nworkers) {
+  return 2 * round64(d) + (int64_t)nworkers * round64(d);
 }
 
-// One warp per tile of kSrvTile indices (M <= kSrvWarpMaxM).  The warp
-// stages the tile's records of all workers in shared memory (one flat,
-// worker-ordered batch of loads) and pushes them into the per-index
-// pairwise sums worker by worker -- program order within the warp keeps
-// worker order, so no block barrier is needed -- then completes every
-// touched index's sum to P leaves and updates the touched w_j (all loads of
-// w issued before the stores).  Untouched indices sum to +0 and keep w_j.
-// Per-warp shared memory (srv_warp_bytes): the record buffer, then
-// srv_levels(M) rows of per-index blocks, a row of lone values, the
-// per-worker record ranges, and one count byte per index.  An index that
-// only one worker sent (the common case) never touches the blocks: its value
-// waits in the lone-value row, and its tree is that value plus +0.
-__host__ __device__ constexpr int srv_levels(int M) {
-  int l = 1;
-  while ((1 << (l - 1)) < M) ++l;
-  return l;  // log2(next_pow2(M)) + 1
+inline SrvTables srv_tables(void* scratch, int64_t d, int32_t rows) {
+  uint32_t* base = reinterpret_cast<uint32_t*>(scratch) + row_words(d) * rows;
+  SrvTables t;
+  t.mask = reinterpret_cast<unsigned long long*>(base);
+  t.vals = reinterpret_cast<float*>(base + 2 * round64(d));
+  t.ldv = round64(d);
+  return t;
 }
-__host__ __device__ constexpr size_t srv_warp_bytes(int M) {
-  return (size_t)kSrvWarpBuf * 8 + (size_t)(srv_levels(M) + 1) * kSrvTile * 4 +
-         (kSrvWarpMaxM + kSrvWarpMaxM + 4) * 4 + kSrvTile;
+
+__global__ void __launch_bounds__(kSrvThreads) topk_server_scatter_kernel(const ServerArgs s, SrvTables t) {
+  // the reduce kernel may be scheduled now: it reads its record, then waits
+  // for this grid to finish before it reads the tables
+  asm volatile("griddepcontrol.launch_dependents;");
+  const int m = blockIdx.y;
+  const int64_t r = (int64_t)blockIdx.x * kSrvThreads + threadIdx.x;
+  if (r >= s.k) return;
+  const uint2 rec = reinterpret_cast<const uint2*>(s.msgs + (int64_t)m * s.msg_stride)[r];
+  // records come from the compressor and are below d
+  if (!dq_in_bounds((int64_t)rec.x < s.d, s.err)) return;
+  t.vals[(int64_t)m * t.ldv + rec.x] = __uint_as_float(rec.y);
+  atomicOr(t.mask + rec.x, 1ull << m);
 }
-// An index's count byte: 0 untouched; kSrvSingle | (m + 1) while worker m's
-// value is the index's only one (kept aside, not yet in the blocks); else
-// the number of workers accounted for in the blocks.
-constexpr uint8_t kSrvSingle = 0x80;
-constexpr int kSrvWarps = kSrvThreads / 32;
 
 template <bool POW2>
-__global__ void __launch_bounds__(kSrvThreads) topk_server_warp_kernel(const ServerArgs s, const uint32_t* starts) {
-  extern __shared__ __align__(16) unsigned char smem_raw[];
-  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-  const int M = s.M;
-  const int nlev = srv_levels(M);
-  unsigned char* region = smem_raw + (size_t)warp * srv_warp_bytes(M);
-  uint2* buf = reinterpret_cast<uint2*>(region);
-  float* stk = reinterpret_cast<float*>(region + (size_t)kSrvWarpBuf * 8);
-  float* single = stk + nlev * kSrvTile;  // an index's value while it is the only one
-  uint32_t* first = reinterpret_cast<uint32_t*>(single + kSrvTile);
-  uint32_t* pre = first + kSrvWarpMaxM;
-  uint8_t* cnt = reinterpret_cast<uint8_t*>(pre + kSrvWarpMaxM + 4);
-  const int64_t nts = srv_tiles(s.d);
-  const int64_t t = (int64_t)blockIdx.x * kSrvWarps + warp;
-  if (t >= nts) return;  // the whole warp
-  const int64_t tile0 = t * kSrvTile;
+__global__ void __launch_bounds__(kSrvThreads) topk_server_reduce_kernel(const ServerArgs s, SrvTables t) {
+  const int m = blockIdx.y;
+  const int64_t r = (int64_t)blockIdx.x * kSrvThreads + threadIdx.x;
+  if (r >= s.k) return;
+  const uint2 rec = reinterpret_cast<const uint2*>(s.msgs + (int64_t)m * s.msg_stride)[r];
+  const int64_t j = rec.x;
+  if (j >= s.d) return;  // skipped by the scatter (and reported there by the checked build)
+  // the scatter grid has completed and its writes are visible (a no-op when
+  // this grid was launched in plain stream order)
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+  const unsigned long long mask = t.mask[j];
+  if (mask == 0ull || __ffsll((long long)mask) - 1 != m) return;  // not the owner
+  const uint32_t P = (uint32_t)next_pow2(s.M);
+  const float v = __uint_as_float(rec.y);
+  float sum;
+  if (__popcll(mask) == 1) {
+    sum = P == 1 ? v : __fadd_rn(v, 0.f);  // one value among +0 leaves
+  } else {
+    SparseTree<kSrvLevels> tree;
+    tree.push_zeros((uint32_t)m);
+    tree.push_block(0, v);
+    unsigned long long rest = mask & (mask - 1ull);  // the other workers, lowest first
+    while (rest) {
+      int who[kSrvBatch];
+      float x[kSrvBatch];
 #pragma unroll
-  for (int q = 0; q < kSrvTile / 32; ++q) cnt[q * 32 + lane] = 0;
-  // this tile's record range of every worker, and the flat prefix
-  uint32_t run = 0;
-  for (int base = 0; base < M; base += 32) {
-    const int m = base + lane;
-    uint32_t n = 0;
-    if (m < M) {
-      const uint32_t* st = starts + (int64_t)m * (nts + 1);
-      const uint32_t a0 = (uint32_t)min64(st[t], s.k), a1 = (uint32_t)min64(st[t + 1], s.k);
-      n = a1 > a0 ? a1 - a0 : 0u;
-      first[m] = a0;
-    }
-    uint32_t x = n;
+      for (int u = 0; u < kSrvBatch; ++u) {
+        who[u] = rest ? __ffsll((long long)rest) - 1 : -1;
+        rest &= rest - 1ull;
+        x[u] = who[u] >= 0 ? t.vals[(int64_t)who[u] * t.ldv + j] : 0.f;
+      }
 #pragma unroll
-    for (int off = 1; off < 32; off <<= 1) {
-      const uint32_t y = __shfl_up_sync(kFullMask, x, off);
-      if (lane >= off) x += y;
-    }
-    if (m < M) pre[m] = run + x - n;
-    run += __shfl_sync(kFullMask, x, 31);
-  }
-  if (lane == 0) pre[M] = run;
-  __syncwarp();
-  const uint32_t N = run;
-  for (uint32_t b = 0; b < N; b += kSrvWarpBuf) {
-    const uint32_t nb = (uint32_t)min64(kSrvWarpBuf, N - b);
-    // kStage loads in flight per lane, then their shared-memory stores
-    constexpr int kStage = 8;
-    for (uint32_t i0 = 0; i0 < nb; i0 += 32 * kStage) {
-      uint2 v[kStage];
-#pragma unroll
-      for (int u = 0; u < kStage; ++u) {
-        const uint32_t i = i0 + u * 32 + lane;
-        v[u] = make_uint2(0u, 0u);
-        if (i < nb) {
-          const uint32_t f = b + i;
-          int lo = 0, hi = M;  // pre[lo] <= f < pre[hi]
-          while (hi - lo > 1) {
-            const int mid = (lo + hi) >> 1;
-            if (pre[mid] <= f) lo = mid;
-            else hi = mid;
-          }
-          const uint2* msg = reinterpret_cast<const uint2*>(s.msgs + (int64_t)lo * s.msg_stride);
-          v[u] = msg[first[lo] + (f - pre[lo])];
+      for (int u = 0; u < kSrvBatch; ++u) {
+        if (who[u] >= 0) {
+          tree.push_zeros((uint32_t)who[u]);
+          tree.push_block(0, x[u]);
         }
       }
+    }
+    tree.push_zeros(P);
+    sum = tree.lv[0];
 #pragma unroll
-      for (int u = 0; u < kStage; ++u) {
-        const uint32_t i = i0 + u * 32 + lane;
-        if (i < nb) buf[i] = v[u];
-      }
-    }
-    __syncwarp();
-    for (int m = 0; m < M; ++m) {
-      const uint32_t f0 = max64(pre[m], b), f1 = min64(pre[m + 1], b + nb);
-      // a worker's indices are distinct: its records go to distinct sums,
-      // one per lane at a time
-      for (uint32_t f = f0 + lane; f < f1; f += 32) {
-        const uint2 r = buf[f - b];
-        const int64_t off = (int64_t)r.x - tile0;
-        // records come from the compressor: inside the tile and below d
-        if (dq_in_bounds(off >= 0 && off < kSrvTile && (int64_t)r.x < s.d, s.err)) {
-          const int o = (int)off;
-          const uint8_t c = cnt[o];
-          const float v = __uint_as_float(r.y);
-          if (c == 0) {  // the index's first value: kept aside (most indices get only one)
-            single[o] = v;
-            cnt[o] = (uint8_t)(kSrvSingle | (m + 1));
-          } else {
-            uint32_t n = c;
-            if (c & kSrvSingle) {  // a second value: the first goes into the blocks now
-              const uint32_t m1 = (c & ~kSrvSingle) - 1u;
-              n = srv_push_zeros(stk, o, 0, m1);
-              srv_push_block(stk, o, n, 0, single[o]);
-              n = m1 + 1;
-            }
-            n = srv_push_zeros(stk, o, n, (uint32_t)m);
-            srv_push_block(stk, o, n, 0, v);
-            cnt[o] = (uint8_t)(m + 1);
-          }
-        }
-      }
-      __syncwarp();
-    }
+    for (int l = 1; l < kSrvLevels; ++l)
+      if (P == (1u << l)) sum = tree.lv[l];
   }
-  // the plain update leaves untouched w_j as they are; with store_q every
-  // index gets its q_hat (+0 where nobody sent it) for the dense pass that
-  // follows
-  const bool dense = s.store_q != 0;
-  const uint32_t P = 1u << (nlev - 1);
-  constexpr int kPer = kSrvTile / 32;
-  constexpr int kHalf = kPer / 2;
-#pragma unroll
-  for (int half = 0; half < 2; ++half) {
-    float wv[kHalf], sum[kHalf];
-    bool upd[kHalf];
-#pragma unroll
-    for (int q = 0; q < kHalf; ++q) {
-      const int i = (half * kHalf + q) * 32 + lane;
-      const uint32_t n = cnt[i];
-      upd[q] = n != 0 || (dense && tile0 + i < s.d);
-      wv[q] = upd[q] ? s.w[tile0 + i] : 0.f;
-      sum[q] = 0.f;
-      if (n & kSrvSingle) {  // one value v among +0 leaves: the tree gives v + 0 (v alone when P = 1)
-        sum[q] = P == 1 ? single[i] : __fadd_rn(single[i], 0.f);
-      } else if (n) {
-        srv_push_zeros(stk, i, n, P);
-        sum[q] = stk[(nlev - 1) * kSrvTile + i];
-      }
-    }
-#pragma unroll
-    for (int q = 0; q < kHalf; ++q) {
-      const int i = (half * kHalf + q) * 32 + lane;
-      if (upd[q]) s.w[tile0 + i] = server_out(s, wv[q], srv_average<POW2>(sum[q], s));
-    }
-  }
+  s.w[j] = server_out(s, s.w[j], srv_average<POW2>(sum, s));
+  t.mask[j] = 0ull;
 }
 
 // One thread per record of every worker.  The record of the lowest worker
@@ -1140,7 +1087,11 @@ __global__ void __launch_bounds__(kSrvThreads) topk_server_owner_kernel(const Se
 }  // namespace
 
 size_t topk_scratch_bytes(int64_t d, int32_t rows, int32_t nworkers) {
-  const int64_t server_words = round64((int64_t)nworkers * (srv_tiles(d) + 1));
+  // the server's tables: masks and value rows (M <= kSrvMaskMaxM), or the
+  // record-range table of the owner kernel (more workers); none for 0
+  const int64_t server_words = nworkers <= 0 ? 0
+                               : nworkers <= kSrvMaskMaxM ? srv_mask_table_words(d, nworkers)
+                                                          : round64((int64_t)nworkers * (srv_tiles(d) + 1));
   return (size_t)(row_words(d) * rows + server_words) * 4u;
 }
 
@@ -1190,26 +1141,43 @@ cudaError_t launch_topk_compress(const CompressArgs& a, int64_t k, bool keep_h, 
 }
 
 cudaError_t launch_topk_server(const ServerArgs& s, void* scratch, int32_t rows, cudaStream_t stream,
-                               uint64_t* launches) {
-  if (s.store_q && s.M > kSrvWarpMaxM) return cudaErrorNotSupported;  // the owner kernel is sparse
+                                uint64_t* launches) {
+  if (s.M <= kSrvMaskMaxM) {
+    const SrvTables t = srv_tables(scratch, s.d, rows);
+    const dim3 grid((unsigned)((s.k + kSrvThreads - 1) / kSrvThreads), (unsigned)s.M);
+    if (s.store_q) {  // the dense q_hat buffer: +0 wherever nobody sent an index
+      const cudaError_t st = cudaMemsetAsync(s.w, 0, (size_t)s.d * sizeof(float), stream);
+      if (st != cudaSuccess) return st;
+    }
+    topk_server_scatter_kernel<<<grid, kSrvThreads, 0, stream>>>(s, t);
+    cudaError_t st = cudaGetLastError();
+    if (st != cudaSuccess) return st;
+    // the reduce kernel as a programmatic dependent launch: its blocks may
+    // start (and read their records) while the scatter finishes
+    cudaLaunchConfig_t lc = {};
+    lc.gridDim = grid;
+    lc.blockDim = dim3(kSrvThreads);
+    lc.dynamicSmemBytes = 0;
+    lc.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    lc.attrs = attr;
+    lc.numAttrs = 1;
+    st = s.M_pow2 ? cudaLaunchKernelEx(&lc, topk_server_reduce_kernel<true>, s, t)
+                  : cudaLaunchKernelEx(&lc, topk_server_reduce_kernel<false>, s, t);
+    // (a failure here would leave the scatter's mask bits set; the launch has
+    // the scatter's grid and block, which were just accepted)
+    *launches += st == cudaSuccess ? 2 : 1;
+    return st;
+  }
+  if (s.store_q) return cudaErrorNotSupported;  // the owner kernel is sparse
   uint32_t* starts = reinterpret_cast<uint32_t*>(scratch) + row_words(s.d) * rows;
   const int64_t n = (int64_t)s.M * s.k;
   topk_server_starts_kernel<<<dim3((unsigned)((s.k + 255) / 256), (unsigned)s.M), 256, 0, stream>>>(s, starts);
-  if (s.M <= kSrvWarpMaxM) {
-    static std::atomic<size_t> smem_done[2][kSmemDevices];
-    const size_t smem = srv_warp_bytes(s.M) * kSrvWarps;
-    const unsigned blocks = (unsigned)((srv_tiles(s.d) + kSrvWarps - 1) / kSrvWarps);
-    cudaError_t st;
-    if (s.M_pow2) st = ensure_smem(topk_server_warp_kernel<true>, smem, 0, smem_done[1]);
-    else st = ensure_smem(topk_server_warp_kernel<false>, smem, 0, smem_done[0]);
-    if (st != cudaSuccess) return st;
-    if (s.M_pow2) topk_server_warp_kernel<true><<<blocks, kSrvThreads, smem, stream>>>(s, starts);
-    else topk_server_warp_kernel<false><<<blocks, kSrvThreads, smem, stream>>>(s, starts);
-  } else {
-    const unsigned blocks = (unsigned)((n + kSrvThreads - 1) / kSrvThreads);
-    if (s.M_pow2) topk_server_owner_kernel<true><<<blocks, kSrvThreads, 0, stream>>>(s, starts);
-    else topk_server_owner_kernel<false><<<blocks, kSrvThreads, 0, stream>>>(s, starts);
-  }
+  const unsigned blocks = (unsigned)((n + kSrvThreads - 1) / kSrvThreads);
+  if (s.M_pow2) topk_server_owner_kernel<true><<<blocks, kSrvThreads, 0, stream>>>(s, starts);
+  else topk_server_owner_kernel<false><<<blocks, kSrvThreads, 0, stream>>>(s, starts);
   *launches += 2;
   return cudaGetLastError();
 }
