@@ -862,45 +862,6 @@ __device__ __forceinline__ float srv_average(float acc, const ServerArgs& s) {
   else return __fdiv_rn(acc, (float)s.M);
 }
 
-// Per index, the server's sum over workers in the library's order (the M
-// values padded with +0 to P = next_pow2(M), summed pairwise) as a binary
-// counter over complete blocks of leaves: lv[L] holds the sum of the last
-// complete block of 2^L leaves while bit L of n is set, n the leaves
-// accounted for.  Absent workers enter as blocks of +0 leaves of the largest
-// aligned size (a block of +0 leaves sums to +0), so the value is the dense
-// padded tree's at a cost of a few additions per present worker.
-template <int LEV>
-struct SparseTree {
-  float lv[LEV];
-  uint32_t n = 0;
-
-  // Pushes a complete block of 2^L leaves summing to x (n a multiple of 2^L).
-  __device__ __forceinline__ void push_block(int L, float x) {
-    float c = x;
-    bool placed = false;
-#pragma unroll
-    for (int l = 0; l < LEV; ++l) {
-      if (!placed && l >= L) {
-        if ((n >> l) & 1u) {
-          c = __fadd_rn(lv[l], c);  // left sibling + this block
-        } else {
-          lv[l] = c;
-          placed = true;
-        }
-      }
-    }
-    n += 1u << L;
-  }
-  // Accounts for leaves n .. t - 1 as +0.
-  __device__ __forceinline__ void push_zeros(uint32_t t) {
-    while (n < t) {
-      int L = 31 - __clz((int)(t - n));       // the largest block that fits
-      if (n) L = min(L, __ffs((int)n) - 1);  // and starts on a multiple of its size
-      push_block(L, 0.f);
-    }
-  }
-};
-
 // Server for M <= kSrvMaskMaxM: two launches over the M * k records, with
 // two tables in the scratch -- a worker mask per index (u64; all zero
 // between calls) and a value row per worker (d floats, never cleared).
@@ -916,8 +877,6 @@ struct SparseTree {
 // buffer is cleared before the scatter.
 constexpr int kSrvMaskMaxM = 64;
 
-constexpr int kSrvLevels = 7;  // log2(64) + 1
-constexpr int kSrvBatch = 8;   // value loads an owner has in flight
 
 struct SrvTables {
   unsigned long long* mask;  // d masks
@@ -952,7 +911,7 @@ __global__ void __launch_bounds__(kSrvThreads) topk_server_scatter_kernel(const 
   atomicOr(t.mask + rec.x, 1ull << m);
 }
 
-template <bool POW2>
+template <bool POW2, int P>
 __global__ void __launch_bounds__(kSrvThreads) topk_server_reduce_kernel(const ServerArgs s, SrvTables t) {
   const int m = blockIdx.y;
   const int64_t r = (int64_t)blockIdx.x * kSrvThreads + threadIdx.x;
@@ -964,39 +923,39 @@ __global__ void __launch_bounds__(kSrvThreads) topk_server_reduce_kernel(const S
   // this grid was launched in plain stream order)
   asm volatile("griddepcontrol.wait;" ::: "memory");
   const unsigned long long mask = t.mask[j];
-  if (mask == 0ull || __ffsll((long long)mask) - 1 != m) return;  // not the owner
-  const uint32_t P = (uint32_t)next_pow2(s.M);
+  // the owner: bit m set and no bit below it
+  if (!((mask >> m) & 1ull) || (mask & ((1ull << m) - 1ull))) return;
   const float v = __uint_as_float(rec.y);
   float sum;
-  if (__popcll(mask) == 1) {
+  if ((mask & (mask - 1ull)) == 0ull) {
     sum = P == 1 ? v : __fadd_rn(v, 0.f);  // one value among +0 leaves
   } else {
-    SparseTree<kSrvLevels> tree;
-    tree.push_zeros((uint32_t)m);
-    tree.push_block(0, v);
-    unsigned long long rest = mask & (mask - 1ull);  // the other workers, lowest first
-    while (rest) {
-      int who[kSrvBatch];
-      float x[kSrvBatch];
+    // the padded tree itself: chunks of C leaves (workers), each summed
+    // pairwise from its values (+0 where a worker is absent), then the
+    // P / C chunk sums pairwise -- the chunks are the tree's subtrees
+    constexpr int C = P < 16 ? P : 16;
+    float part[P / C];
 #pragma unroll
-      for (int u = 0; u < kSrvBatch; ++u) {
-        who[u] = rest ? __ffsll((long long)rest) - 1 : -1;
-        rest &= rest - 1ull;
-        x[u] = who[u] >= 0 ? t.vals[(int64_t)who[u] * t.ldv + j] : 0.f;
+    for (int c = 0; c < P / C; ++c) {
+      const uint32_t bits = (uint32_t)(mask >> (C * c)) & (uint32_t)((1ull << C) - 1ull);
+      float x[C];
+#pragma unroll
+      for (int u = 0; u < C; ++u) {
+        const int who = C * c + u;
+        x[u] = 0.f;
+        if ((bits >> u) & 1u) x[u] = who == m ? v : t.vals[(int64_t)who * t.ldv + j];
       }
 #pragma unroll
-      for (int u = 0; u < kSrvBatch; ++u) {
-        if (who[u] >= 0) {
-          tree.push_zeros((uint32_t)who[u]);
-          tree.push_block(0, x[u]);
-        }
-      }
+      for (int width = C / 2; width >= 1; width /= 2)
+#pragma unroll
+        for (int i = 0; i < width; ++i) x[i] = __fadd_rn(x[2 * i], x[2 * i + 1]);
+      part[c] = x[0];
     }
-    tree.push_zeros(P);
-    sum = tree.lv[0];
 #pragma unroll
-    for (int l = 1; l < kSrvLevels; ++l)
-      if (P == (1u << l)) sum = tree.lv[l];
+    for (int width = P / C / 2; width >= 1; width /= 2)
+#pragma unroll
+      for (int i = 0; i < width; ++i) part[i] = __fadd_rn(part[2 * i], part[2 * i + 1]);
+    sum = part[0];
   }
   s.w[j] = server_out(s, s.w[j], srv_average<POW2>(sum, s));
   t.mask[j] = 0ull;
@@ -1164,8 +1123,17 @@ cudaError_t launch_topk_server(const ServerArgs& s, void* scratch, int32_t rows,
     attr[0].val.programmaticStreamSerializationAllowed = 1;
     lc.attrs = attr;
     lc.numAttrs = 1;
-    st = s.M_pow2 ? cudaLaunchKernelEx(&lc, topk_server_reduce_kernel<true>, s, t)
-                  : cudaLaunchKernelEx(&lc, topk_server_reduce_kernel<false>, s, t);
+    st = cudaErrorInvalidValue;
+    switch (next_pow2(s.M)) {
+#define DQ_TOPK_REDUCE(P)                                                                             \
+  case P:                                                                                             \
+    st = s.M_pow2 ? cudaLaunchKernelEx(&lc, topk_server_reduce_kernel<true, P>, s, t)                 \
+                  : cudaLaunchKernelEx(&lc, topk_server_reduce_kernel<false, P>, s, t);               \
+    break;
+      DQ_TOPK_REDUCE(1) DQ_TOPK_REDUCE(2) DQ_TOPK_REDUCE(4) DQ_TOPK_REDUCE(8) DQ_TOPK_REDUCE(16)
+      DQ_TOPK_REDUCE(32) DQ_TOPK_REDUCE(64)
+#undef DQ_TOPK_REDUCE
+    }
     // (a failure here would leave the scatter's mask bits set; the launch has
     // the scatter's grid and block, which were just accepted)
     *launches += st == cudaSuccess ? 2 : 1;
