@@ -962,8 +962,11 @@ squant_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap
     return (sl_ < nslices && j < s.d) ? (int64_t)__ldg(s.word_bucket + (j >> 5)) : -1;
   };
   int64_t wb_next = SEG ? word_bucket_of(sl) : 0;
-  // flat buckets (b = 4, 8): this lane's worker's scale, and (b = 8) the
-  // lane's four parameters, loaded one slice ahead
+  // (b = 4, 8: two slices ahead, so that the scale can be loaded one ahead)
+  int64_t wb_next2 = (SEG && kSqPrefetch) ? word_bucket_of(sl + stride) : 0;
+  // b = 4, 8: this lane's worker's scale of the slice's bucket (the bucket
+  // of lane 0's word), and (b = 8) the lane's four parameters, loaded one
+  // slice ahead
   const float* const lane_scales =
       reinterpret_cast<const float*>(s.msgs + (int64_t)(active ? lane : 0) * s.msg_stride);
   auto load_w4 = [&](int64_t sl_) -> float4 {
@@ -976,7 +979,11 @@ squant_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap
     if (j + 2 < s.d) x.z = s.w[j + 2];
     return x;
   };
-  float scale_nx = (kSqPrefetch && !SEG && active && sl < nslices) ? __ldg(lane_scales + sl / spb) : 0.f;
+  float scale_nx = 0.f;
+  if constexpr (kSqPrefetch) {
+    const int64_t b0 = SEG ? (int64_t)__shfl_sync(kFullMask, wb_next, 0) : sl / spb;
+    scale_nx = (active && sl < nslices && b0 >= 0) ? __ldg(lane_scales + b0) : 0.f;
+  }
   float4 w_nx = (kSqPrefetch && !WB) ? load_w4(sl) : make_float4(0.f, 0.f, 0.f, 0.f);
   uint32_t it = 0;
   bool ok = true;
@@ -991,7 +998,12 @@ squant_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap
       issue(nxt, cur ^ 1);
     }
     const int64_t wb_cur = wb_next;
-    if constexpr (SEG) wb_next = word_bucket_of(nxt);
+    if constexpr (SEG && kSqPrefetch) {
+      wb_next = wb_next2;
+      wb_next2 = word_bucket_of(nxt + stride);
+    } else if constexpr (SEG) {
+      wb_next = word_bucket_of(nxt);
+    }
     const int64_t b = sl / spb;
     const int64_t j0 = SLICE * sl + EPL * lane;  // this lane's first element
     // the lane's parameters: row pr of the box, 16-byte chunks pc0 ..
@@ -1028,15 +1040,42 @@ squant_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap
       mixed = !__all_sync(kFullMask, my_bkt == bkt);
     }
     float my_scale;
-    if constexpr (kSqPrefetch && !SEG) {
+    if constexpr (kSqPrefetch) {
       my_scale = scale_nx;
-      scale_nx = (active && nxt < nslices) ? __ldg(lane_scales + nxt / spb) : 0.f;
+      const int64_t bn = SEG ? (int64_t)__shfl_sync(kFullMask, wb_next, 0) : nxt / spb;
+      scale_nx = (active && nxt < nslices && bn >= 0) ? __ldg(lane_scales + bn) : 0.f;
     } else {
       my_scale = active ? __ldg(reinterpret_cast<const float*>(s.msgs + (int64_t)lane * s.msg_stride) + bkt) : 0.f;
     }
-    // worker m's scale for this lane's elements
-    auto scale_of = [&](int m) -> float {
-      if (SEG && mixed) return __ldg(reinterpret_cast<const float*>(s.msgs + (int64_t)m * s.msg_stride) + my_bkt);
+    // A slice that spans buckets holds consecutive ones, bkt .. bkt + nbk - 1
+    // (one per 32-element word at most).  Up to four: lane m loads worker m's
+    // scales of all of them and each lane picks its own bucket's by shuffle;
+    // more (short partial buckets): each lane loads the scales it needs.
+    int rel = 0, nbk = 1;
+    float sc4[4] = {my_scale, 0.f, 0.f, 0.f};
+    if (SEG && mixed) {
+      rel = (int)(my_bkt - bkt);
+      nbk = __reduce_max_sync(kFullMask, (unsigned)rel) + 1;
+      if (nbk <= 4) {
+#pragma unroll
+        for (int k = 1; k < 4; ++k) sc4[k] = (active && k < nbk) ? __ldg(lane_scales + bkt + k) : 0.f;
+      }
+    }
+    // worker m's scale for this lane's elements (mx: the slice spans buckets;
+    // every call passes a constant)
+    auto scale_of = [&](bool mx, int m) -> float {
+      if (mx) {
+        if (nbk > 4) return __ldg(reinterpret_cast<const float*>(s.msgs + (int64_t)m * s.msg_stride) + my_bkt);
+        float r = __shfl_sync(kFullMask, sc4[0], m);
+#pragma unroll
+        for (int k = 1; k < 4; ++k) {
+          if (k < nbk) {  // warp-uniform
+            const float t = __shfl_sync(kFullMask, sc4[k], m);
+            if (rel == k) r = t;
+          }
+        }
+        return r;
+      }
       return __shfl_sync(kFullMask, my_scale, m);
     };
     ok = mbar_wait_bounded(&bar[cur], (it >> 1) & 1u, s.err);
@@ -1066,7 +1105,7 @@ squant_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap
     constexpr int kParts = BITS == 4 ? kSquant4Parts : 1;
     constexpr int NE = EPL / kParts;
     // one worker's decoded values of this lane's elements e0 .. e0 + NE - 1
-    auto decode_part = [&](uint32_t word, float sc, int e0, float (&v)[NE]) {
+    auto decode_part = [&](bool MX, uint32_t word, float sc, int e0, float (&v)[NE]) {
       if constexpr (BITS == 2) {
         // code 0: -s, 1: +0, 2: +s (fl(s * 1) = s): one bit test picks +0,
         // one the sign
@@ -1084,12 +1123,12 @@ squant_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap
       // 16..31, so the bits above the element's code need no mask).  (With
       // layer segments the lanes' scales may differ: look up V[c] and multiply
       // by the lane's own scale instead.)
-      const float T4 = (BITS == 4) ? __fmul_rn(mixed ? 1.0f : sc, V4) : 0.f;
+      const float T4 = (BITS == 4) ? __fmul_rn(MX ? 1.0f : sc, V4) : 0.f;
 #pragma unroll
       for (int e = 0; e < NE; ++e) {
         if constexpr (BITS == 4) {
           v[e] = __shfl_sync(kFullMask, T4, (int)(word >> (4 * (e0 + e))));
-          if (mixed) v[e] = __fmul_rn(sc, v[e]);
+          if (MX) v[e] = __fmul_rn(sc, v[e]);
         } else {
           v[e] = __fmul_rn(sc, V8l[__byte_perm(word, 0u, 0x4440u | (uint32_t)(e0 + e)) * 32u]);
         }
@@ -1110,7 +1149,9 @@ squant_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap
     // G0 + G1; (G0 + G1) + (G2 + G3); then + ((G4 + G5) + (G6 + G7)), groups
     // past M being +0 (M is warp-uniform, so are the branches)
     const bool per_worker = BITS != 2 || (SEG && mixed);
-    if (per_worker) {
+    // (slices that span buckets take their own instance of the decode, so
+    // that the common one carries none of their scale handling)
+    auto per_worker_sums = [&](bool mx) {
 #pragma unroll
       for (int part = 0; part < kParts; ++part) {
         const int e0 = part * NE;
@@ -1123,17 +1164,17 @@ squant_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap
           for (int u = 0; u < 4; ++u) {
             const bool here = m + u < M;  // warp-uniform
             wd[u] = here ? words[32 * (m + u)] : 0u;
-            sc[u] = here ? scale_of(m + u) : 0.f;
+            sc[u] = here ? scale_of(mx, m + u) : 0.f;
           }
           float va[NE], vb[NE];
-          decode_part(wd[0], sc[0], e0, va);
-          decode_part(wd[1], sc[1], e0, vb);
+          decode_part(mx, wd[0], sc[0], e0, va);
+          decode_part(mx, wd[1], sc[1], e0, vb);
           const bool h1 = m + 1 < M;
 #pragma unroll
           for (int e = 0; e < NE; ++e) g[e] = M == 1 ? va[e] : __fadd_rn(va[e], h1 ? vb[e] : 0.f);
           if (M <= 2) return;
-          decode_part(wd[2], sc[2], e0, va);
-          decode_part(wd[3], sc[3], e0, vb);
+          decode_part(mx, wd[2], sc[2], e0, va);
+          decode_part(mx, wd[3], sc[3], e0, vb);
           const bool h2 = m + 2 < M, h3 = m + 3 < M;
 #pragma unroll
           for (int e = 0; e < NE; ++e) g[e] = __fadd_rn(g[e], __fadd_rn(h2 ? va[e] : 0.f, h3 ? vb[e] : 0.f));
@@ -1184,6 +1225,14 @@ squant_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap
         }
 #pragma unroll
         for (int e = 0; e < NE; ++e) acc[e0 + e] = r[e];
+      }
+    };
+    if (per_worker) {
+      if constexpr (SEG) {
+        if (mixed) per_worker_sums(true);
+        else per_worker_sums(false);
+      } else {
+        per_worker_sums(false);
       }
     }
 #pragma unroll
@@ -1517,7 +1566,9 @@ cudaError_t launch_squant_server(const ServerArgs& s, const CUtensorMap* params_
         else DQ_SQ_TMA(4, 1);
         break;
       case 8:
-        if (s.M == 16 && !s.word_bucket) st = launch_squant_tma<8, true, false, 1, 16>(s, params_map, stream);
+        if (s.M == 16)
+          st = s.word_bucket ? launch_squant_tma<8, true, true, 1, 16>(s, params_map, stream)
+                             : launch_squant_tma<8, true, false, 1, 16>(s, params_map, stream);
         else DQ_SQ_TMA(8, 1);
         break;
     }

@@ -101,6 +101,16 @@ __device__ __forceinline__ RowScratch row_scratch(void* base, int64_t d, int row
 __device__ __forceinline__ uint32_t key_of(float v) { return __float_as_uint(v) & 0x7FFFFFFFu; }
 __device__ __forceinline__ uint32_t key_bits(uint32_t bits) { return bits & 0x7FFFFFFFu; }
 
+// hist[bin] += 1 for each lane of `mask` (the lanes that call it together)
+// with `valid`: lanes with the same bin are counted by one atomic.  (The
+// candidates of a call lie within a few binades above the carried threshold,
+// so their top digits fall into a few bins, and plain per-lane atomics on
+// them serialise.)
+__device__ __forceinline__ void warp_hist_add(uint32_t* hist, uint32_t bin, bool valid, unsigned mask) {
+  const unsigned peers = __match_any_sync(mask, valid ? bin : 0xFFFFFFFFu);
+  if (valid && (int)(threadIdx.x & 31) == __ffs(peers) - 1) atomicAdd(hist + bin, (uint32_t)__popc(peers));
+}
+
 // Block-wide exclusive scan of one value per thread; *total gets the sum.
 // `warp_sums` is shared memory of NT/32 words.  Two barriers.
 template <int NT>
@@ -226,6 +236,9 @@ __device__ __forceinline__ uint32_t write_tile_candidates(const float (&v)[R][4]
 // ---------------------------------------------------------------------------
 template <bool KEEP_H>
 __global__ void __launch_bounds__(kFormThreads, 6) topk_form_kernel(const CompressArgs a, void* scratch) {
+  // the select kernel may be scheduled once every block of this grid has
+  // started; it waits for this grid's completion before reading anything
+  asm volatile("griddepcontrol.launch_dependents;");
   constexpr int kGroups = kTile / 128;
   __shared__ float vstage[kTile];
   __shared__ uint32_t flags[kTile / 32];
@@ -345,7 +358,9 @@ struct SelectSmem {
   uint32_t tpre[kChunkTiles + 1];   // candidate prefix at the chunk's tiles
   uint32_t warp_sums[kSelThreads / 32];
   uint32_t sel[6];
-  uint32_t cta_tot[2];              // keys > T and == T in this CTA's share (read by the cluster)
+  uint32_t pre_t[kBins0];           // the same three histograms summed over the CTAs of lower rank
+  uint32_t pre_a[kBins1];
+  uint32_t pre_b[kBins1];
   uint32_t span[2];                 // first and last tile overlapping this CTA's share
   uint2 cache[kCacheCap];           // this CTA's share of the candidates, when it fits
 };
@@ -353,29 +368,47 @@ struct SelectSmem {
 // Tile counts a select thread holds in registers (all tiles, when nt fits).
 constexpr int kRegTiles = 4;
 
+// The tile of candidate f: the largest i < n with tpre[i] <= f (tpre
+// non-decreasing, tpre[0] <= f < tpre[n]; an empty tile repeats its
+// successor's prefix, so the tile found holds f).  A fixed number of halving
+// steps (n <= kChunkTiles), so that the searches of several candidates
+// interleave.
+__device__ __forceinline__ int tile_of(const uint32_t* tpre, int n, uint32_t f) {
+  int lo = 0;
+#pragma unroll
+  for (int step = kChunkTiles / 2; step >= 1; step >>= 1) {
+    const int mid = lo + step;
+    if (mid < n && tpre[mid] <= f) lo = mid;
+  }
+  return lo;
+}
+
 // Candidate f (prefix coordinates of tpre) of the chunk starting at tile tc0.
 __device__ __forceinline__ uint2 chunk_candidate(const uint2* cand, const uint32_t* tpre, int n, int64_t tc0,
                                                  uint32_t f) {
-  int lo = 0, hi = n;  // tpre[lo] <= f < tpre[hi]
-  while (hi - lo > 1) {
-    const int mid = (lo + hi) >> 1;
-    if (tpre[mid] <= f) lo = mid;
-    else hi = mid;
-  }
-  return cand[(tc0 + lo) * kTile + (f - tpre[lo])];
+  const int i = tile_of(tpre, n, f);
+  return cand[(tc0 + i) * kTile + (f - tpre[i])];
 }
 
-// Sums the cluster's copies of one histogram into sm.full[0, BINS).  The
-// cluster barrier publishes every CTA's counts; each histogram buffer is
-// written once per selection round, so no barrier is needed after the reads.
+// Sums the cluster's copies of one histogram into sm.full[0, BINS), and
+// those of the CTAs of lower rank than this one into pre[0, BINS) (from which
+// the CTA's first record position follows).  The cluster barrier publishes
+// every CTA's counts; each histogram buffer is written once per selection
+// round, so no barrier is needed after the reads.
 template <int BINS>
-__device__ __forceinline__ void cluster_sum(cg::cluster_group& cluster, uint32_t* local, SelectSmem& sm) {
+__device__ __forceinline__ void cluster_sum(cg::cluster_group& cluster, uint32_t* local, uint32_t* pre,
+                                            int rank, SelectSmem& sm) {
   cluster.sync();
   for (int i = threadIdx.x; i < BINS; i += kSelThreads) {
-    uint32_t s = 0;
+    uint32_t s = 0, below = 0;
 #pragma unroll
-    for (int r = 0; r < kCluster; ++r) s += cluster.map_shared_rank(local, r)[i];
+    for (int r = 0; r < kCluster; ++r) {
+      const uint32_t x = cluster.map_shared_rank(local, r)[i];
+      if (r < rank) below += x;
+      s += x;
+    }
     sm.full[i] = s;
+    pre[i] = below;
   }
   __syncthreads();
 }
@@ -383,6 +416,9 @@ __device__ __forceinline__ void cluster_sum(cg::cluster_group& cluster, uint32_t
 template <bool KEEP_H>
 __global__ void __cluster_dims__(kCluster, 1, 1) __launch_bounds__(kSelThreads, 1)
 topk_select_kernel(const CompressArgs a, int64_t k, void* scratch) {
+  // launched as a programmatic dependent of the form kernel: its tile counts,
+  // candidates and p are complete and visible after this wait
+  asm volatile("griddepcontrol.wait;" ::: "memory");
   extern __shared__ __align__(16) unsigned char smem_raw[];
   SelectSmem& sm = *reinterpret_cast<SelectSmem*>(smem_raw);
   cg::cluster_group cluster = cg::this_cluster();
@@ -568,7 +604,73 @@ topk_select_kernel(const CompressArgs a, int64_t k, void* scratch) {
   // (body(candidate, valid) is called by every thread of the block the same
   // number of times, so it may use warp collectives.)
   auto for_each = [&](auto&& body, bool fill) {
-    if (cached && !fill) {
+    if (fill) {
+      // The share becomes the on-chip copy (cached: one chunk of tiles
+      // [ta, tb), candidates [lo1, hi1)).  First every candidate slot gets
+      // its tile: each tile with candidates in the share marks its first
+      // slot with its number, and a block-wide running maximum over the
+      // slots carries each mark forward (the marks grow with the slot).  The
+      // cost does not depend on how the candidates spread over the tiles,
+      // and the loads below need no search.
+      const int n = (int)(tb - ta);
+      const uint32_t S = hi1 - lo1;
+      for (uint32_t f = threadIdx.x; f < S; f += kSelThreads) sm.cache[f].x = 0u;
+      __syncthreads();
+      for (int i = threadIdx.x; i < n; i += kSelThreads) {
+        const uint32_t a0 = sm.tpre[i], a1 = sm.tpre[i + 1];
+        if (a0 < a1 && a1 > lo1 && a0 < hi1) sm.cache[max(a0, lo1) - lo1].x = (uint32_t)i;
+      }
+      __syncthreads();
+      const uint32_t per = (S + kSelThreads - 1) / kSelThreads;
+      const uint32_t g0 = min(threadIdx.x * per, S), g1 = min(g0 + per, S);
+      uint32_t run = 0;
+      for (uint32_t f = g0; f < g1; ++f) run = max(run, sm.cache[f].x);
+      // exclusive running maximum over the threads' runs
+      {
+        const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+        uint32_t x = run;
+#pragma unroll
+        for (int off = 1; off < 32; off <<= 1) {
+          const uint32_t y = __shfl_up_sync(kFullMask, x, off);
+          if (lane >= off) x = max(x, y);
+        }
+        if (lane == 31) sm.warp_sums[warp] = x;
+        __syncthreads();
+        uint32_t before = 0;
+#pragma unroll
+        for (int w = 0; w < kSelThreads / 32; ++w)
+          if (w < warp) before = max(before, sm.warp_sums[w]);
+        const uint32_t up = __shfl_up_sync(kFullMask, x, 1);
+        run = max(before, lane > 0 ? up : 0u);
+        __syncthreads();
+      }
+      for (uint32_t f = g0; f < g1; ++f) {
+        run = max(run, sm.cache[f].x);
+        sm.cache[f].x = run;
+      }
+      __syncthreads();
+      for (uint32_t base = lo1; base < hi1; base += kSelThreads * kBatch) {
+        uint2 c[kBatch];
+#pragma unroll
+        for (int u = 0; u < kBatch; ++u) {
+          const uint32_t f = base + u * kSelThreads + threadIdx.x;
+          c[u] = make_uint2(0u, 0u);
+          if (f < hi1) {
+            const uint32_t i = sm.cache[f - lo1].x;
+            c[u] = rs.cand[(ta + i) * kTile + (f - sm.tpre[i])];
+          }
+        }
+#pragma unroll
+        for (int u = 0; u < kBatch; ++u) {
+          const uint32_t f = base + u * kSelThreads + threadIdx.x;
+          if (f < hi1) sm.cache[f - lo1] = c[u];
+          body(c[u], f < hi1);
+        }
+      }
+      __syncthreads();
+      return;
+    }
+    if (cached) {
       for (uint32_t base = lo1; base < hi1; base += kSelThreads) {
         const uint32_t f = base + threadIdx.x;
         body(f < hi1 ? sm.cache[f - lo1] : make_uint2(0u, 0u), f < hi1);
@@ -595,7 +697,6 @@ topk_select_kernel(const CompressArgs a, int64_t k, void* scratch) {
       }
       if (!one_chunk) __syncthreads();  // sm.tpre is reloaded for the next chunk
     }
-    if (fill) __syncthreads();
   };
 
   // Histogram of the top digit over all of p in this CTA's tiles.
@@ -604,15 +705,18 @@ topk_select_kernel(const CompressArgs a, int64_t k, void* scratch) {
 #pragma unroll
       for (int i = 0; i < kSelRows; ++i) {
         const int64_t j = t * kTile + 4 * ((int64_t)i * kSelThreads + threadIdx.x);
+        float4 x = make_float4(0.f, 0.f, 0.f, 0.f);
         if (j + 3 < a.d) {
-          const float4 x = *reinterpret_cast<const float4*>(e + j);
-          atomicAdd(&sm.hist_t[key_of(x.x) >> 20], 1u);
-          atomicAdd(&sm.hist_t[key_of(x.y) >> 20], 1u);
-          atomicAdd(&sm.hist_t[key_of(x.z) >> 20], 1u);
-          atomicAdd(&sm.hist_t[key_of(x.w) >> 20], 1u);
+          x = *reinterpret_cast<const float4*>(e + j);
         } else {
-          for (int64_t jj = j; jj < a.d && jj < j + 4; ++jj) atomicAdd(&sm.hist_t[key_of(e[jj]) >> 20], 1u);
+          if (j < a.d) x.x = e[j];
+          if (j + 1 < a.d) x.y = e[j + 1];
+          if (j + 2 < a.d) x.z = e[j + 2];
         }
+        warp_hist_add(sm.hist_t, key_of(x.x) >> 20, j < a.d, kFullMask);
+        warp_hist_add(sm.hist_t, key_of(x.y) >> 20, j + 1 < a.d, kFullMask);
+        warp_hist_add(sm.hist_t, key_of(x.z) >> 20, j + 2 < a.d, kFullMask);
+        warp_hist_add(sm.hist_t, key_of(x.w) >> 20, j + 3 < a.d, kFullMask);
       }
     }
     __syncthreads();
@@ -633,14 +737,14 @@ topk_select_kernel(const CompressArgs a, int64_t k, void* scratch) {
       set_up();
       for_each(
           [&](uint2 c, bool valid) {
-            if (valid) atomicAdd(&sm.hist_t[key_bits(c.y) >> 20], 1u);
+            warp_hist_add(sm.hist_t, key_bits(c.y) >> 20, valid, kFullMask);
           },
           cached);
       filled = cached;
     } else {
       histogram_p();
     }
-    cluster_sum<kBins0>(cluster, sm.hist_t, sm);
+    cluster_sum<kBins0>(cluster, sm.hist_t, sm.pre_t, rank, sm);
     if (threadIdx.x == 0) {
       sm.sel[0] = 0;
       sm.sel[1] = (uint32_t)k;
@@ -657,7 +761,7 @@ topk_select_kernel(const CompressArgs a, int64_t k, void* scratch) {
           if (valid && (key >> 20) == b0) atomicAdd(&sm.hist_a[(key >> 10) & 1023u], 1u);
         },
         cached && !filled);
-    cluster_sum<kBins1>(cluster, sm.hist_a, sm);
+    cluster_sum<kBins1>(cluster, sm.hist_a, sm.pre_a, rank, sm);
     if (threadIdx.x == 0) {
       sm.sel[2] = 0;
       sm.sel[3] = krem0;
@@ -673,7 +777,7 @@ topk_select_kernel(const CompressArgs a, int64_t k, void* scratch) {
           if (valid && (key >> 10) == hi21) atomicAdd(&sm.hist_b[key & 1023u], 1u);
         },
         false);
-    cluster_sum<kBins1>(cluster, sm.hist_b, sm);
+    cluster_sum<kBins1>(cluster, sm.hist_b, sm.pre_b, rank, sm);
     if (threadIdx.x == 0) {
       sm.sel[4] = 0;
       sm.sel[5] = krem1;
@@ -688,31 +792,27 @@ topk_select_kernel(const CompressArgs a, int64_t k, void* scratch) {
     fast = false;
   }
 
-  // Keys above and equal to T in this CTA's share, from its own histograms:
-  // top digit above b0, or middle digit above T's, or low digit above T's.
+  // Every read of another CTA's shared memory is done: arrive at the
+  // cluster barrier now, wait for the others only before leaving (no CTA
+  // leaves while another may still read its shared memory).
+  asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
+
+  // Keys above and equal to T in the shares of the CTAs before this one, from
+  // the histogram sums over them: top digit above b0, or middle digit above
+  // T's, or low digit above T's; and keys equal to T.
+  uint32_t gt_before = 0, tie_before = 0;
   {
     const uint32_t b1 = (T >> 10) & 1023u, b2 = T & 1023u;
     uint32_t part = 0;
     for (int i = threadIdx.x; i < kBins0; i += kSelThreads)
-      if ((uint32_t)i > b0) part += sm.hist_t[i];
+      if ((uint32_t)i > b0) part += sm.pre_t[i];
     for (int i = threadIdx.x; i < kBins1; i += kSelThreads) {
-      if ((uint32_t)i > b1) part += sm.hist_a[i];
-      if ((uint32_t)i > b2) part += sm.hist_b[i];
+      if ((uint32_t)i > b1) part += sm.pre_a[i];
+      if ((uint32_t)i > b2) part += sm.pre_b[i];
     }
-    const uint32_t cta_gt = block_sum<kSelThreads>(part, sm.warp_sums);
-    if (threadIdx.x == 0) {
-      sm.cta_tot[0] = cta_gt;
-      sm.cta_tot[1] = sm.hist_b[b2];
-    }
+    gt_before = block_sum<kSelThreads>(part, sm.warp_sums);
+    tie_before = sm.pre_b[b2];
   }
-  cluster.sync();
-  uint32_t gt_before = 0, tie_before = 0;
-  for (int r = 0; r < rank; ++r) {
-    const uint32_t* tot = cluster.map_shared_rank(sm.cta_tot, r);
-    gt_before += tot[0];
-    tie_before += tot[1];
-  }
-  cluster.sync();  // no CTA leaves while another may still read its shared memory
 
   // Kept records: position = (keys > T before) + min(keys == T before, need).
   auto keep = [&](uint2 c) {
@@ -815,6 +915,7 @@ topk_select_kernel(const CompressArgs a, int64_t k, void* scratch) {
     const float t_next = __fmul_rn(__uint_as_float(T), 0.9375f);
     rs.state[ST_TAU] = kTauValid | key_of(t_next);
   }
+  asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
 }
 
 // ---------------------------------------------------------------------------
@@ -1086,17 +1187,30 @@ cudaError_t launch_topk_compress(const CompressArgs& a, int64_t k, bool keep_h, 
   const dim3 clusters(kCluster, rows);
   const size_t smem = sizeof(SelectSmem);
   cudaError_t st;
+  // the select kernel as a programmatic dependent launch of the form kernel
+  cudaLaunchConfig_t lc = {};
+  lc.gridDim = clusters;
+  lc.blockDim = dim3(kSelThreads);
+  lc.dynamicSmemBytes = smem;
+  lc.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  lc.attrs = attr;
+  lc.numAttrs = 1;
   if (keep_h) {
     if ((st = ensure_smem(topk_select_kernel<true>, smem, 0, smem_done[1])) != cudaSuccess) return st;
     topk_form_kernel<true><<<tiles, kFormThreads, 0, stream>>>(a, scratch);
-    topk_select_kernel<true><<<clusters, kSelThreads, smem, stream>>>(a, k, scratch);
+    if ((st = cudaGetLastError()) != cudaSuccess) return st;
+    st = cudaLaunchKernelEx(&lc, topk_select_kernel<true>, a, k, scratch);
   } else {
     if ((st = ensure_smem(topk_select_kernel<false>, smem, 0, smem_done[0])) != cudaSuccess) return st;
     topk_form_kernel<false><<<tiles, kFormThreads, 0, stream>>>(a, scratch);
-    topk_select_kernel<false><<<clusters, kSelThreads, smem, stream>>>(a, k, scratch);
+    if ((st = cudaGetLastError()) != cudaSuccess) return st;
+    st = cudaLaunchKernelEx(&lc, topk_select_kernel<false>, a, k, scratch);
   }
-  *launches += 2;
-  return cudaGetLastError();
+  *launches += st == cudaSuccess ? 2 : 1;
+  return st;
 }
 
 cudaError_t launch_topk_server(const ServerArgs& s, void* scratch, int32_t rows, cudaStream_t stream,
