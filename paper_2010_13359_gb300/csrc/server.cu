@@ -260,13 +260,28 @@ __global__ void __launch_bounds__(256) sign_server_shfl_kernel(const ServerArgs 
 // with conflict-free 128-bit shared loads.  Each warp owns two box buffers
 // and one mbarrier per buffer: while it decodes slice i it has the copy of
 // slice i + 1 in flight.  Waits are bounded (error word on time-out).
+// With layer segments (SEG) the slices come from a host-built table in
+// which every slice lies inside one bucket (runs of up to 32 words); the
+// word box starts at the 16-byte boundary at or before the slice (36 words
+// wide, no swizzle) and each lane realigns its worker's 32 words by the
+// slice's word offset; the words of a short slice past its rows are read
+// but their elements are not stored.
 constexpr int kTmaWarps = 8;
 constexpr int kTmaBoxBytes = 32 * 32 * 4;
-constexpr int kTmaSmemBytes = kTmaWarps * 2 * kTmaBoxBytes + 1024;  // + alignment slack
+constexpr int kTmaSegBoxBytes = 32 * kSignSegBoxWords * 4;
+template <bool SEG>
+constexpr int tma_sign_smem_bytes() { return kTmaWarps * 2 * (SEG ? kTmaSegBoxBytes : kTmaBoxBytes) + 1024; }
 
-template <int NG, bool POW2>
+struct SegSlices {
+  const uint32_t* slices;  // per slice {first word, bucket | (rows - 1) << 27}
+  int64_t n;
+};
+
+template <int NG, bool POW2, bool SEG>
 __global__ void __launch_bounds__(32 * kTmaWarps)
-sign_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap tmap) {
+sign_server_tma_kernel(const ServerArgs s, const SegSlices seg, const __grid_constant__ CUtensorMap tmap) {
+  constexpr int BOX = SEG ? kTmaSegBoxBytes : kTmaBoxBytes;
+  constexpr int PITCH = SEG ? 4 * kSignSegBoxWords : 128;  // bytes of a box row
   extern __shared__ uint8_t smem_raw[];
   __shared__ uint64_t bars[kTmaWarps][2];
   const int lane = threadIdx.x & 31;
@@ -274,7 +289,7 @@ sign_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap t
   // 1024-byte aligned buffers (required by the 128-byte swizzle)
   const uint32_t raw = smem_addr(smem_raw);
   uint8_t* base = smem_raw + ((1024u - (raw & 1023u)) & 1023u);
-  uint8_t* const buf0 = base + warp * 2 * kTmaBoxBytes;  // buffer i at buf0 + i * kTmaBoxBytes
+  uint8_t* const buf0 = base + warp * 2 * BOX;  // buffer i at buf0 + i * BOX
   uint64_t* bar = bars[warp];
   if (lane == 0) {
     mbar_init(&bar[0], 1);
@@ -286,36 +301,54 @@ sign_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap t
   const int words_per_bucket = s.bucket >> 5;  // 32..128
   const int spb = words_per_bucket >> 5;       // 32-word slices per bucket
   const int64_t nb = (s.d + s.bucket - 1) / s.bucket;
-  const int64_t nslices = nb * spb;
+  const int64_t nslices = SEG ? seg.n : nb * spb;
   const int64_t stride = (int64_t)gridDim.x * kTmaWarps;
   const int32_t x0 = (int32_t)(s.off_payload >> 2);
-  const uint32_t box_bytes = (uint32_t)(s.M < 32 ? s.M : 32) * 128u;
+  const uint32_t box_bytes = (uint32_t)(s.M < 32 ? s.M : 32) * (uint32_t)PITCH;
   const bool active = lane < s.M;
   const TransposeLane tl(lane);
 
   int64_t sl = (int64_t)blockIdx.x * kTmaWarps + warp;
-  auto wbase_of = [&](int64_t slice) {
-    const int64_t b = slice / spb;
-    return b * words_per_bucket + (slice - b * spb) * 32;
+  struct Slice {
+    int64_t word;    // first message word
+    int64_t bucket;
+    int rows;        // words in the slice, 1..32
   };
+  auto slice_of = [&](int64_t slice) -> Slice {
+    if constexpr (SEG) {
+      const uint2 e = __ldg(reinterpret_cast<const uint2*>(seg.slices) + slice);
+      return Slice{(int64_t)e.x, (int64_t)(e.y & 0x7FFFFFFu), (int)(e.y >> 27) + 1};
+    } else {
+      const int64_t b = slice / spb;
+      return Slice{b * words_per_bucket + (slice - b * spb) * 32, b, 32};
+    }
+  };
+  auto box_x = [&](const Slice& c) {
+    const int32_t x = x0 + (int32_t)c.word;
+    return SEG ? (x & ~3) : x;  // x0 is a multiple of 64 words
+  };
+  Slice c = sl < nslices ? slice_of(sl) : Slice{0, 0, 0};
   if (sl < nslices && lane == 0) {
     mbar_arrive_expect_tx(&bar[0], box_bytes);
-    tma_load_2d(buf0, &tmap, x0 + (int32_t)wbase_of(sl), 0, &bar[0]);
+    tma_load_2d(buf0, &tmap, box_x(c), 0, &bar[0]);
   }
   uint32_t it = 0;
   bool ok = true;
   for (; sl < nslices; sl += stride, ++it) {
     const int cur = (int)(it & 1u);
     const int64_t nxt = sl + stride;
+    const Slice cn = nxt < nslices ? slice_of(nxt) : Slice{0, 0, 0};
     if (nxt < nslices && lane == 0) {
       fence_proxy_async_shared();  // this warp's reads of that buffer came before
       mbar_arrive_expect_tx(&bar[cur ^ 1], box_bytes);
-      tma_load_2d(buf0 + (cur ^ 1) * kTmaBoxBytes, &tmap, x0 + (int32_t)wbase_of(nxt), 0, &bar[cur ^ 1]);
+      tma_load_2d(buf0 + (cur ^ 1) * BOX, &tmap, box_x(cn), 0, &bar[cur ^ 1]);
     }
-    const int64_t b = sl / spb;
-    const int64_t wbase = wbase_of(sl);
+    const int64_t b = c.bucket;
+    const int64_t wbase = c.word;
+    const int woff = SEG ? (int)((x0 + wbase) & 3) : 0;  // the slice's first word in the box rows
     float* wl = s.w + 32 * wbase + lane;
-    const int64_t jmax = s.d - 32 * wbase - lane;  // wl[32 i] is a parameter iff 32 i < jmax
+    // wl[32 i] is a parameter of this slice iff 32 i < jmax
+    const int64_t jmax = min64(s.d - 32 * wbase - lane, 32 * (int64_t)c.rows);
     float wv[8];
 #pragma unroll
     for (int k = 0; k < 8; ++k) wv[k] = (32 * k < jmax) ? __ldcs(wl + 32 * k) : 0.f;
@@ -326,12 +359,24 @@ sign_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap t
     ok = mbar_wait_bounded(&bar[cur], (it >> 1) & 1u, s.err);
     ok = __all_sync(kFullMask, ok);
     if (!ok) break;
-    const uint8_t* row = buf0 + cur * kTmaBoxBytes + lane * 128;
+    const uint8_t* row = buf0 + cur * BOX + lane * PITCH;
     const int sw = lane & 7;
 #pragma unroll
     for (int q = 0; q < 4; ++q) {
       uint32_t wd[8];
-      if (active) {
+      if (active && SEG) {
+        // words 8q .. 8q + 11 of the row (16-byte aligned), then the 8 from woff
+        const uint4 a = *reinterpret_cast<const uint4*>(row + 32 * q);
+        const uint4 bb = *reinterpret_cast<const uint4*>(row + 32 * q + 16);
+        const uint4 cc = *reinterpret_cast<const uint4*>(row + 32 * q + 32);
+        const uint32_t r[12] = {a.x, a.y, a.z, a.w, bb.x, bb.y, bb.z, bb.w, cc.x, cc.y, cc.z, cc.w};
+#pragma unroll
+        for (int k = 0; k < 8; ++k) {
+          const uint32_t u01 = (woff & 1) ? r[k + 1] : r[k];
+          const uint32_t u23 = (woff & 1) ? r[k + 3] : r[k + 2];
+          wd[k] = (woff & 2) ? u23 : u01;
+        }
+      } else if (active) {
         const uint4 lo = *reinterpret_cast<const uint4*>(row + (((2 * q) ^ sw) << 4));
         const uint4 hi = *reinterpret_cast<const uint4*>(row + (((2 * q + 1) ^ sw) << 4));
         wd[0] = lo.x; wd[1] = lo.y; wd[2] = lo.z; wd[3] = lo.w;
@@ -361,6 +406,7 @@ sign_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap t
       }
     }
     __syncwarp();
+    c = cn;
   }
   // after a time-out the copy of the next slice may still be in flight
   if (!ok && lane == 0 && sl + stride < nslices)
@@ -437,11 +483,6 @@ __device__ __forceinline__ void transpose32_regs(uint32_t (&a)[32]) {
 }
 
 // The slice table of the layer-segmented form.
-struct SegSlices {
-  const uint32_t* slices;  // per slice {first word, bucket | (rows - 1) << 27}
-  int64_t n;
-};
-
 template <int NG, bool POW2, bool SEG>
 __global__ void __launch_bounds__(32 * kColWarps, 1)
 sign_server_col_kernel(const ServerArgs s, const SegSlices seg, const __grid_constant__ CUtensorMap wmap,
@@ -1368,30 +1409,29 @@ __global__ void __launch_bounds__(256) oadam_update_kernel(const OAdamArgs a) {
   }
 }
 
-template <int NG, bool POW2>
-cudaError_t launch_sign_tma(const ServerArgs& s, cudaStream_t stream) {
-  auto kern = sign_server_tma_kernel<NG, POW2>;
+template <int NG, bool POW2, bool SEG>
+cudaError_t launch_sign_tma(const ServerArgs& s, const SignServerExtras& x, cudaStream_t stream) {
+  auto kern = sign_server_tma_kernel<NG, POW2, SEG>;
+  constexpr int smem = tma_sign_smem_bytes<SEG>();
   int dev = 0;
   cudaError_t st = cudaGetDevice(&dev);
   if (st != cudaSuccess) return st;
   static int blocks_for[64] = {0};
   if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
   if (blocks_for[dev] == 0) {
-    if ((st = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kTmaSmemBytes)) !=
-        cudaSuccess)
+    if ((st = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem)) != cudaSuccess)
       return st;
     int sms = 0, per_sm = 0;
     if ((st = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return st;
-    if ((st = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, 32 * kTmaWarps, kTmaSmemBytes)) !=
-        cudaSuccess)
+    if ((st = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, 32 * kTmaWarps, smem)) != cudaSuccess)
       return st;
     blocks_for[dev] = sms * (per_sm > 0 ? per_sm : 1);
   }
-  const int64_t nb = (s.d + s.bucket - 1) / s.bucket;
-  const int64_t warps = nb * (s.bucket / 1024);
+  const int64_t warps = SEG ? x.seg_nslices : ((s.d + s.bucket - 1) / s.bucket) * (s.bucket / 1024);
   const int64_t need = (warps + kTmaWarps - 1) / kTmaWarps;
   const unsigned blocks = (unsigned)(need < blocks_for[dev] ? need : blocks_for[dev]);
-  kern<<<blocks, 32 * kTmaWarps, kTmaSmemBytes, stream>>>(s, *s.sign_words_map);
+  if (blocks == 0) return cudaSuccess;
+  kern<<<blocks, 32 * kTmaWarps, smem, stream>>>(s, SegSlices{x.seg_slices, x.seg_nslices}, *s.sign_words_map);
   return cudaGetLastError();
 }
 
@@ -1425,13 +1465,12 @@ cudaError_t launch_sign_col(const ServerArgs& s, const SignServerExtras& x, cuda
 // The column kernel pays once every resident warp has several slices: with
 // one or two the latency of a slice's chain (copies in, transpose, store)
 // shows and the bit-transpose kernel is as fast or faster.
-bool sign_col_pays(const ServerArgs& s) {
+bool sign_col_pays(int64_t nslices) {
   static int sms[64] = {0};
   int dev = 0;
   if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return false;
   if (sms[dev] == 0 && cudaDeviceGetAttribute(&sms[dev], cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
     return false;
-  const int64_t nslices = ((s.d + s.bucket - 1) / s.bucket) * (s.bucket / 1024);
   return nslices >= 4ll * sms[dev] * kColWarps;
 }
 
@@ -1468,11 +1507,15 @@ unsigned chunk_blocks(int64_t d, int threads) {
 cudaError_t launch_sign_server(const ServerArgs& s, const SignServerExtras& x, cudaStream_t stream,
                                uint64_t* launches) {
   if (s.word_bucket) {  // buckets restart at layer segments
-    if (x.seg_slices && s.sign_words_map && x.params_map && s.bucket >= 1024 && s.M <= 32) {
+    if (x.seg_slices && s.sign_words_map && s.bucket >= 1024 && s.M <= 32) {
       const bool p2 = s.M_pow2 != 0;
+      // the column kernel where it pays (as for flat buckets), else the
+      // warp-transpose kernel; DQGAN_SIGN_SERVER fixes the choice
+      const bool col = x.params_map != nullptr && (x.path == 1 || (x.path == 0 && sign_col_pays(x.seg_nslices)));
       cudaError_t st;
-#define DQ_SIGN_SEG(NG) \
-  st = (p2 ? launch_sign_col<NG, true, true>(s, x, stream) : launch_sign_col<NG, false, true>(s, x, stream))
+#define DQ_SIGN_SEG(NG)                                                                                     \
+  st = col ? (p2 ? launch_sign_col<NG, true, true>(s, x, stream) : launch_sign_col<NG, false, true>(s, x, stream)) \
+           : (p2 ? launch_sign_tma<NG, true, true>(s, x, stream) : launch_sign_tma<NG, false, true>(s, x, stream))
       switch ((s.M + 3) / 4) {
         case 1: DQ_SIGN_SEG(1); break;
         case 2: DQ_SIGN_SEG(2); break;
@@ -1493,11 +1536,12 @@ cudaError_t launch_sign_server(const ServerArgs& s, const SignServerExtras& x, c
   }
   if (s.bucket >= 1024 && s.M <= 32 && s.sign_words_map != nullptr) {
     const bool p2 = s.M_pow2 != 0;
-    const bool col = x.params_map != nullptr && (x.path == 1 || (x.path == 0 && sign_col_pays(s)));
+    const bool col = x.params_map != nullptr &&
+                     (x.path == 1 || (x.path == 0 && sign_col_pays(((s.d + s.bucket - 1) / s.bucket) * (s.bucket / 1024))));
     cudaError_t st;
 #define DQ_SIGN_TMA(NG)                                                                           \
   st = col ? (p2 ? launch_sign_col<NG, true, false>(s, x, stream) : launch_sign_col<NG, false, false>(s, x, stream)) \
-           : (p2 ? launch_sign_tma<NG, true>(s, stream) : launch_sign_tma<NG, false>(s, stream))
+           : (p2 ? launch_sign_tma<NG, true, false>(s, x, stream) : launch_sign_tma<NG, false, false>(s, x, stream))
     switch ((s.M + 3) / 4) {
       case 1: DQ_SIGN_TMA(1); break;
       case 2: DQ_SIGN_TMA(2); break;

@@ -713,10 +713,11 @@ topk_select_kernel(const CompressArgs a, int64_t k, void* scratch) {
           if (j + 1 < a.d) x.y = e[j + 1];
           if (j + 2 < a.d) x.z = e[j + 2];
         }
-        warp_hist_add(sm.hist_t, key_of(x.x) >> 20, j < a.d, kFullMask);
-        warp_hist_add(sm.hist_t, key_of(x.y) >> 20, j + 1 < a.d, kFullMask);
-        warp_hist_add(sm.hist_t, key_of(x.z) >> 20, j + 2 < a.d, kFullMask);
-        warp_hist_add(sm.hist_t, key_of(x.w) >> 20, j + 3 < a.d, kFullMask);
+        // (all of p: its top digits spread over many bins, so plain atomics)
+        if (j < a.d) atomicAdd(&sm.hist_t[key_of(x.x) >> 20], 1u);
+        if (j + 1 < a.d) atomicAdd(&sm.hist_t[key_of(x.y) >> 20], 1u);
+        if (j + 2 < a.d) atomicAdd(&sm.hist_t[key_of(x.z) >> 20], 1u);
+        if (j + 3 < a.d) atomicAdd(&sm.hist_t[key_of(x.w) >> 20], 1u);
       }
     }
     __syncthreads();

@@ -3,13 +3,14 @@ select its TMA paths: buckets of 1024..4096 with M <= 32, where the message
 words and the parameters are staged by TMA and each lane transposes a
 32 x 32 bit block in registers.
 
-Both kernels run on every shape (forced by DQGAN_SIGN_SERVER, read when a
-handle is created), and once more with the choice by size.
+Both kernels run on every shape, with flat buckets and with layer
+segments (forced by DQGAN_SIGN_SERVER, read when a handle is created), and
+once more with the choice by size.
 
 The messages come from the GPU compress step and are checked bit for bit
 against the oracle's; the oracle's server then runs on the same messages and
-the parameters must agree within the step tolerance (the sign server's
-summation order over workers is not worker order).  Parameters past d must
+the parameters must agree within the step tolerance and then bit for bit
+(both sum over workers in the library's pairwise order).  Parameters past d must
 stay untouched: the vector sits inside a larger buffer whose tail holds
 sentinels.  Sizes cover d < 32 (no parameter map), d a multiple of 32, a
 partial last row, a partial row that starts a slice of its own (floor(d/32)
@@ -125,10 +126,17 @@ SEG_CASES = [
 ]
 
 
+@pytest.mark.parametrize("path", ["col", "tma", "auto"])
 @pytest.mark.parametrize("d,M,bucket,kind", SEG_CASES, ids=[f"d{d}-M{M}-b{b}-{k}" for d, M, b, k in SEG_CASES])
-def test_sign_server_segments(P, d, M, bucket, kind):
-    """Layer segments: every slice of the column kernel lies inside one
-    bucket; short slices update their rows with plain stores."""
+def test_sign_server_segments(P, d, M, bucket, kind, path, monkeypatch):
+    """Layer segments, both kernels (forced, and chosen by size): every slice
+    lies inside one bucket; the column kernel updates short slices with
+    plain stores, the warp-transpose kernel realigns each slice's words in
+    its box and stores only the slice's own rows."""
+    if path == "auto":
+        monkeypatch.delenv("DQGAN_SIGN_SERVER", raising=False)
+    else:
+        monkeypatch.setenv("DQGAN_SIGN_SERVER", path)
     dev = torch.device("cuda:0")
     stream = torch.cuda.current_stream(dev)
     rng = np.random.default_rng(d + bucket)
