@@ -24,7 +24,7 @@ namespace dq {
 namespace {
 
 // Largest d the fixed scratch supports, and the scratch itself (8.75 MiB;
-// one worker's top-k scratch at that d needs just under 8.02 MiB).  Both
+// the one scratch row of a top-k worker at that d takes 8.01 MiB).  Both
 // numbers are the ones dqgan.h states.
 constexpr int64_t kNoAllocMaxD = DQGAN_NOALLOC_MAX_D;
 constexpr size_t kNoAllocScratchBytes = (size_t)DQGAN_NOALLOC_SCRATCH_BYTES;
