@@ -116,6 +116,7 @@ __device__ __forceinline__ void store_chunk(const CompressArgs& a, const float* 
 template <int CPT, int WPB, bool KEEP_H, bool SEG>
 __global__ void __launch_bounds__(32 * WPB * (WPB < 4 ? 4 / WPB : 1))
 sign_compress_kernel(const CompressArgs a) {
+  dq_pdl_enter();
   constexpr bool HOLD = KEEP_H && CPT <= 8;
   constexpr int BPC = WPB < 4 ? 4 / WPB : 1;  // buckets per CTA (CTA = max(4, WPB) warps)
   constexpr int CHAIN = 32 * CPT * WPB;
@@ -222,6 +223,7 @@ sign_compress_kernel(const CompressArgs a) {
 template <int CPT, int WPB, int BITS, bool KEEP_H, bool L2, bool SEG>
 __global__ void __launch_bounds__(32 * WPB * (WPB < 4 ? 4 / WPB : 1))
 squant_compress_kernel(const CompressArgs a) {
+  dq_pdl_enter();
   constexpr int K = (1 << (BITS - 1)) - 1;
   constexpr bool HOLD = KEEP_H && CPT <= 8;
   constexpr int BPC = WPB < 4 ? 4 / WPB : 1;  // buckets per CTA (CTA = max(4, WPB) warps)
@@ -409,6 +411,7 @@ squant_compress_kernel(const CompressArgs a) {
 template <bool KEEP_H>
 __global__ void __launch_bounds__(256)
 identity_compress_kernel(const CompressArgs a) {
+  dq_pdl_enter();
   const int row = blockIdx.y;
   const int worker = a.worker0 + row;
   const float* g = a.g + (int64_t)row * a.g_stride;
@@ -455,11 +458,11 @@ cudaError_t sign_dispatch_keep(const CompressArgs& a, bool keep_h, cudaStream_t 
   const dim3 grid((unsigned)((a.nb + BPC - 1) / BPC), (unsigned)a.nworkers);
   const bool seg = a.bstart != nullptr;
   if (keep_h) {
-    if (seg) sign_compress_kernel<CPT, WPB, true, true><<<grid, THREADS, 0, stream>>>(a);
-    else sign_compress_kernel<CPT, WPB, true, false><<<grid, THREADS, 0, stream>>>(a);
+    if (seg) launch_pdl(sign_compress_kernel<CPT, WPB, true, true>, grid, dim3(THREADS), 0, stream, a);
+    else launch_pdl(sign_compress_kernel<CPT, WPB, true, false>, grid, dim3(THREADS), 0, stream, a);
   } else {
-    if (seg) sign_compress_kernel<CPT, WPB, false, true><<<grid, THREADS, 0, stream>>>(a);
-    else sign_compress_kernel<CPT, WPB, false, false><<<grid, THREADS, 0, stream>>>(a);
+    if (seg) launch_pdl(sign_compress_kernel<CPT, WPB, false, true>, grid, dim3(THREADS), 0, stream, a);
+    else launch_pdl(sign_compress_kernel<CPT, WPB, false, false>, grid, dim3(THREADS), 0, stream, a);
   }
   return cudaGetLastError();
 }
@@ -485,11 +488,11 @@ cudaError_t squant_dispatch_keep(const CompressArgs& a, bool keep_h, cudaStream_
   }
   const dim3 grid((unsigned)gx, (unsigned)a.nworkers);
   if (keep_h) {
-    if (seg) squant_compress_kernel<CPT, WPB, BITS, true, L2, true><<<grid, THREADS, 0, stream>>>(a);
-    else squant_compress_kernel<CPT, WPB, BITS, true, L2, false><<<grid, THREADS, 0, stream>>>(a);
+    if (seg) launch_pdl(squant_compress_kernel<CPT, WPB, BITS, true, L2, true>, grid, dim3(THREADS), 0, stream, a);
+    else launch_pdl(squant_compress_kernel<CPT, WPB, BITS, true, L2, false>, grid, dim3(THREADS), 0, stream, a);
   } else {
-    if (seg) squant_compress_kernel<CPT, WPB, BITS, false, L2, true><<<grid, THREADS, 0, stream>>>(a);
-    else squant_compress_kernel<CPT, WPB, BITS, false, L2, false><<<grid, THREADS, 0, stream>>>(a);
+    if (seg) launch_pdl(squant_compress_kernel<CPT, WPB, BITS, false, L2, true>, grid, dim3(THREADS), 0, stream, a);
+    else launch_pdl(squant_compress_kernel<CPT, WPB, BITS, false, L2, false>, grid, dim3(THREADS), 0, stream, a);
   }
   return cudaGetLastError();
 }
@@ -546,8 +549,8 @@ cudaError_t launch_identity_compress(const CompressArgs& a, bool keep_h, cudaStr
   const int64_t nchunks = (a.d + 3) / 4;
   const int64_t blocks = min64((nchunks + 255) / 256, 152 * 8);
   const dim3 grid((unsigned)max64(blocks, 1), (unsigned)a.nworkers);
-  if (keep_h) identity_compress_kernel<true><<<grid, 256, 0, stream>>>(a);
-  else identity_compress_kernel<false><<<grid, 256, 0, stream>>>(a);
+  if (keep_h) launch_pdl(identity_compress_kernel<true>, grid, dim3(256), 0, stream, a);
+  else launch_pdl(identity_compress_kernel<false>, grid, dim3(256), 0, stream, a);
   *launches += 1;
   return cudaGetLastError();
 }

@@ -11,6 +11,8 @@
 
 #include <cuda.h>
 
+#include <utility>
+
 #include "dqgan.h"
 
 namespace dq {
@@ -125,6 +127,25 @@ constexpr int kSignSegBoxWords = 36;
 // b-bit quantiser's server at b = 2, 4), 128-byte swizzle, zero fill.  Needs
 // d >= 32 and w 16-byte aligned.
 bool encode_params_map(float* w, int64_t d, int32_t box_rows, CUtensorMap* out);
+
+// Launches `kern` as a programmatic dependent launch (see dq_pdl_enter in
+// device_common.cuh: every kernel launched this way waits for its
+// predecessor's grid before touching memory).  Returns the launch status.
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem, cudaStream_t stream,
+                              Args&&... args) {
+  cudaLaunchConfig_t lc = {};
+  lc.gridDim = grid;
+  lc.blockDim = block;
+  lc.dynamicSmemBytes = smem;
+  lc.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  lc.attrs = attr;
+  lc.numAttrs = 1;
+  return cudaLaunchKernelEx(&lc, kern, std::forward<Args>(args)...);
+}
 
 // Kernel launchers: each enqueues its kernels on `stream`, adds the number of
 // kernels it launched to *launches and returns the launch status.

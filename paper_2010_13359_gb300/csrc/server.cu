@@ -49,6 +49,7 @@ __device__ __forceinline__ void apply_chunk(const ServerArgs& s, int64_t j, cons
 constexpr int kSumLevels = 11;  // group counts up to 1024 (M <= 4096)
 
 __global__ void __launch_bounds__(256) sign_server_kernel(const ServerArgs s) {
+  dq_pdl_enter();
   const int64_t c = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   const int64_t j = 4 * c;
   if (j >= s.d) return;
@@ -197,6 +198,7 @@ __device__ __forceinline__ void sums8(const uint32_t (&wd)[8], const float (&T)[
 // decoded.
 template <int NG, bool POW2>
 __global__ void __launch_bounds__(256) sign_server_shfl_kernel(const ServerArgs s) {
+  dq_pdl_enter();
   const int lane = threadIdx.x & 31;
   const int64_t gw = (int64_t)blockIdx.x * 8 + (threadIdx.x >> 5);
   const int words_per_bucket = s.bucket >> 5;
@@ -280,6 +282,7 @@ struct SegSlices {
 template <int NG, bool POW2, bool SEG>
 __global__ void __launch_bounds__(32 * kTmaWarps)
 sign_server_tma_kernel(const ServerArgs s, const SegSlices seg, const __grid_constant__ CUtensorMap tmap) {
+  dq_pdl_enter();
   constexpr int BOX = SEG ? kTmaSegBoxBytes : kTmaBoxBytes;
   constexpr int PITCH = SEG ? 4 * kSignSegBoxWords : 128;  // bytes of a box row
   extern __shared__ uint8_t smem_raw[];
@@ -487,6 +490,7 @@ template <int NG, bool POW2, bool SEG>
 __global__ void __launch_bounds__(32 * kColWarps, 1)
 sign_server_col_kernel(const ServerArgs s, const SegSlices seg, const __grid_constant__ CUtensorMap wmap,
                        const __grid_constant__ CUtensorMap pmap) {
+  dq_pdl_enter();
   using L = ColLayout<SEG>;
   constexpr int ROWS = 4 * NG < 32 ? 4 * NG : 32;  // message rows that can hold a worker
   extern __shared__ uint8_t smem_raw[];
@@ -660,6 +664,7 @@ sign_server_col_kernel(const ServerArgs s, const SegSlices seg, const __grid_con
 constexpr int kSlabLevels = 8;  // up to 128 slabs (M <= 4096)
 
 __global__ void __launch_bounds__(256) sign_server_slabs_kernel(const ServerArgs s) {
+  dq_pdl_enter();
   const int lane = threadIdx.x & 31;
   const int64_t gw = (int64_t)blockIdx.x * 8 + (threadIdx.x >> 5);
   const int words_per_bucket = s.bucket >> 5;
@@ -706,6 +711,7 @@ __global__ void __launch_bounds__(256) sign_server_slabs_kernel(const ServerArgs
 // b = 2 (V in {-1, 0, +1}) the value is a select.
 template <int BITS, bool POW2>
 __global__ void __launch_bounds__(256) squant_server_kernel(const ServerArgs s) {
+  dq_pdl_enter();
   constexpr int K = (1 << (BITS - 1)) - 1;
   constexpr uint32_t MASK = (1u << BITS) - 1u;
   constexpr int CODES = (BITS == 2) ? 1 : (1 << BITS);
@@ -929,6 +935,7 @@ template <int BITS, bool POW2, bool SEG, int NSET, int FM>
 __global__ void __launch_bounds__(32 * kTmaWarps)
 squant_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap tmap,
                          const __grid_constant__ CUtensorMap pmap) {
+  dq_pdl_enter();
   constexpr int K = (1 << (BITS - 1)) - 1;
   constexpr int EPL = 32 / BITS;  // elements per lane (one code word)
   constexpr int SLICE = 32 * EPL; // elements per slice
@@ -1321,6 +1328,7 @@ squant_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap
 // Identity: the messages are the p vectors themselves, summed in groups of
 // four workers in the library's pairwise order.
 __global__ void __launch_bounds__(256) identity_server_kernel(const ServerArgs s) {
+  dq_pdl_enter();
   const int64_t c = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   const int64_t j = 4 * c;
   if (j >= s.d) return;
@@ -1356,6 +1364,7 @@ __global__ void __launch_bounds__(256) identity_server_kernel(const ServerArgs s
 __global__ void __launch_bounds__(256)
 lookahead_kernel(const float* __restrict__ w, const float* __restrict__ h, float* __restrict__ out,
                  int64_t d) {
+  dq_pdl_enter();
   const int64_t c = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   const int64_t j = 4 * c;
   if (j + 3 < d) {
@@ -1389,6 +1398,7 @@ __device__ __forceinline__ float oadam_element(const OAdamArgs& a, float q, floa
 }
 
 __global__ void __launch_bounds__(256) oadam_update_kernel(const OAdamArgs a) {
+  dq_pdl_enter();
   const int64_t j = 4 * ((int64_t)blockIdx.x * blockDim.x + threadIdx.x);
   if (j + 3 < a.d) {
     const float4 q = __ldcs(reinterpret_cast<const float4*>(a.q + j));
@@ -1431,7 +1441,8 @@ cudaError_t launch_sign_tma(const ServerArgs& s, const SignServerExtras& x, cuda
   const int64_t need = (warps + kTmaWarps - 1) / kTmaWarps;
   const unsigned blocks = (unsigned)(need < blocks_for[dev] ? need : blocks_for[dev]);
   if (blocks == 0) return cudaSuccess;
-  kern<<<blocks, 32 * kTmaWarps, smem, stream>>>(s, SegSlices{x.seg_slices, x.seg_nslices}, *s.sign_words_map);
+  launch_pdl(kern, dim3(blocks), dim3(32 * kTmaWarps), smem, stream, s, SegSlices{x.seg_slices, x.seg_nslices},
+             *s.sign_words_map);
   return cudaGetLastError();
 }
 
@@ -1457,7 +1468,7 @@ cudaError_t launch_sign_col(const ServerArgs& s, const SignServerExtras& x, cuda
   const int64_t need = (nslices + kColWarps - 1) / kColWarps;
   const unsigned blocks = (unsigned)(need < blocks_for[dev] ? need : blocks_for[dev]);
   if (blocks == 0) return cudaSuccess;
-  kern<<<blocks, 32 * kColWarps, smem, stream>>>(s, SegSlices{x.seg_slices, x.seg_nslices}, *s.sign_words_map,
+  launch_pdl(kern, dim3(blocks), dim3(32 * kColWarps), smem, stream, s, SegSlices{x.seg_slices, x.seg_nslices}, *s.sign_words_map,
                                                   *x.params_map);
   return cudaGetLastError();
 }
@@ -1492,7 +1503,7 @@ cudaError_t launch_squant_tma(const ServerArgs& s, const CUtensorMap* params_map
   const int64_t need = (nslices + kTmaWarps - 1) / kTmaWarps;
   const int64_t cap = (int64_t)sms * (per_sm > 0 ? per_sm : 1);
   // (b = 8 takes no parameter map: the word map stands in for the unused argument)
-  kern<<<(unsigned)(need < cap ? need : cap), 32 * kTmaWarps, smem, stream>>>(
+  launch_pdl(kern, dim3((unsigned)(need < cap ? need : cap)), dim3(32 * kTmaWarps), smem, stream,
       s, *s.squant_words_map, sq_params_boxed(BITS) ? *params_map : *s.squant_words_map);
   return cudaGetLastError();
 }
@@ -1530,7 +1541,7 @@ cudaError_t launch_sign_server(const ServerArgs& s, const SignServerExtras& x, c
       *launches += 1;
       return st;
     }
-    sign_server_kernel<<<chunk_blocks(s.d, 256), 256, 0, stream>>>(s);  // per-element scale lookup
+    launch_pdl(sign_server_kernel, dim3(chunk_blocks(s.d, 256)), dim3(256), 0, stream, s);  // per-element scale lookup
     *launches += 1;
     return cudaGetLastError();
   }
@@ -1562,13 +1573,13 @@ cudaError_t launch_sign_server(const ServerArgs& s, const SignServerExtras& x, c
     const int64_t warps = nb * wpb;
     const unsigned blocks = (unsigned)((warps + 7) / 8);
     if (s.M > 32) {
-      sign_server_slabs_kernel<<<blocks, 256, 0, stream>>>(s);
+      launch_pdl(sign_server_slabs_kernel, dim3(blocks), dim3(256), 0, stream, s);
     } else {
       const int ng = (s.M + 3) / 4;
       const bool p2 = s.M_pow2 != 0;
 #define DQ_SIGN_SERVER(NG) \
-      (p2 ? sign_server_shfl_kernel<NG, true><<<blocks, 256, 0, stream>>>(s) \
-          : sign_server_shfl_kernel<NG, false><<<blocks, 256, 0, stream>>>(s))
+      (p2 ? launch_pdl(sign_server_shfl_kernel<NG, true>, dim3(blocks), dim3(256), 0, stream, s) \
+          : launch_pdl(sign_server_shfl_kernel<NG, false>, dim3(blocks), dim3(256), 0, stream, s))
       switch (ng) {
         case 1: DQ_SIGN_SERVER(1); break;
         case 2: DQ_SIGN_SERVER(2); break;
@@ -1582,7 +1593,7 @@ cudaError_t launch_sign_server(const ServerArgs& s, const SignServerExtras& x, c
 #undef DQ_SIGN_SERVER
     }
   } else {
-    sign_server_kernel<<<chunk_blocks(s.d, 256), 256, 0, stream>>>(s);
+    launch_pdl(sign_server_kernel, dim3(chunk_blocks(s.d, 256)), dim3(256), 0, stream, s);
   }
   *launches += 1;
   return cudaGetLastError();
@@ -1624,12 +1635,12 @@ cudaError_t launch_squant_server(const ServerArgs& s, const CUtensorMap* params_
   const unsigned blocks = chunk_grid < 152u * 6u ? chunk_grid : 152u * 6u;  // V is built once per block
   const bool p2 = s.M_pow2 != 0;
   switch (s.bits) {
-    case 2: p2 ? squant_server_kernel<2, true><<<blocks, 256, 0, stream>>>(s)
-               : squant_server_kernel<2, false><<<blocks, 256, 0, stream>>>(s); break;
-    case 4: p2 ? squant_server_kernel<4, true><<<blocks, 256, 0, stream>>>(s)
-               : squant_server_kernel<4, false><<<blocks, 256, 0, stream>>>(s); break;
-    case 8: p2 ? squant_server_kernel<8, true><<<blocks, 256, 0, stream>>>(s)
-               : squant_server_kernel<8, false><<<blocks, 256, 0, stream>>>(s); break;
+    case 2: p2 ? launch_pdl(squant_server_kernel<2, true>, dim3(blocks), dim3(256), 0, stream, s)
+               : launch_pdl(squant_server_kernel<2, false>, dim3(blocks), dim3(256), 0, stream, s); break;
+    case 4: p2 ? launch_pdl(squant_server_kernel<4, true>, dim3(blocks), dim3(256), 0, stream, s)
+               : launch_pdl(squant_server_kernel<4, false>, dim3(blocks), dim3(256), 0, stream, s); break;
+    case 8: p2 ? launch_pdl(squant_server_kernel<8, true>, dim3(blocks), dim3(256), 0, stream, s)
+               : launch_pdl(squant_server_kernel<8, false>, dim3(blocks), dim3(256), 0, stream, s); break;
     default: return cudaErrorInvalidValue;
   }
   *launches += 1;
@@ -1637,21 +1648,21 @@ cudaError_t launch_squant_server(const ServerArgs& s, const CUtensorMap* params_
 }
 
 cudaError_t launch_identity_server(const ServerArgs& s, cudaStream_t stream, uint64_t* launches) {
-  identity_server_kernel<<<chunk_blocks(s.d, 256), 256, 0, stream>>>(s);
+  launch_pdl(identity_server_kernel, dim3(chunk_blocks(s.d, 256)), dim3(256), 0, stream, s);
   *launches += 1;
   return cudaGetLastError();
 }
 
 
 cudaError_t launch_oadam_update(const OAdamArgs& a, cudaStream_t stream, uint64_t* launches) {
-  oadam_update_kernel<<<chunk_blocks(a.d, 256), 256, 0, stream>>>(a);
+  launch_pdl(oadam_update_kernel, dim3(chunk_blocks(a.d, 256)), dim3(256), 0, stream, a);
   *launches += 1;
   return cudaGetLastError();
 }
 
 cudaError_t launch_lookahead(const float* w, const float* h, float* out, int64_t d,
                              cudaStream_t stream, uint64_t* launches) {
-  lookahead_kernel<<<chunk_blocks(d, 256), 256, 0, stream>>>(w, h, out, d);
+  launch_pdl(lookahead_kernel, dim3(chunk_blocks(d, 256)), dim3(256), 0, stream, w, h, out, d);
   *launches += 1;
   return cudaGetLastError();
 }

@@ -236,9 +236,7 @@ __device__ __forceinline__ uint32_t write_tile_candidates(const float (&v)[R][4]
 // ---------------------------------------------------------------------------
 template <bool KEEP_H>
 __global__ void __launch_bounds__(kFormThreads, 6) topk_form_kernel(const CompressArgs a, void* scratch) {
-  // the select kernel may be scheduled once every block of this grid has
-  // started; it waits for this grid's completion before reading anything
-  asm volatile("griddepcontrol.launch_dependents;");
+  dq_pdl_enter();
   constexpr int kGroups = kTile / 128;
   __shared__ float vstage[kTile];
   __shared__ uint32_t flags[kTile / 32];
@@ -418,7 +416,7 @@ __global__ void __cluster_dims__(kCluster, 1, 1) __launch_bounds__(kSelThreads, 
 topk_select_kernel(const CompressArgs a, int64_t k, void* scratch) {
   // launched as a programmatic dependent of the form kernel: its tile counts,
   // candidates and p are complete and visible after this wait
-  asm volatile("griddepcontrol.wait;" ::: "memory");
+  dq_pdl_enter();
   extern __shared__ __align__(16) unsigned char smem_raw[];
   SelectSmem& sm = *reinterpret_cast<SelectSmem*>(smem_raw);
   cg::cluster_group cluster = cg::this_cluster();
@@ -925,6 +923,7 @@ topk_select_kernel(const CompressArgs a, int64_t k, void* scratch) {
 // and the last record also (tile(k-1), nts].
 // ---------------------------------------------------------------------------
 __global__ void __launch_bounds__(256) topk_server_starts_kernel(const ServerArgs s, uint32_t* starts) {
+  dq_pdl_enter();
   const int m = blockIdx.y;
   const int64_t r = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
   const int lane = threadIdx.x & 31;
@@ -1000,9 +999,7 @@ inline SrvTables srv_tables(void* scratch, int64_t d, int32_t rows) {
 }
 
 __global__ void __launch_bounds__(kSrvThreads) topk_server_scatter_kernel(const ServerArgs s, SrvTables t) {
-  // the reduce kernel may be scheduled now: it reads its record, then waits
-  // for this grid to finish before it reads the tables
-  asm volatile("griddepcontrol.launch_dependents;");
+  dq_pdl_enter();
   const int m = blockIdx.y;
   const int64_t r = (int64_t)blockIdx.x * kSrvThreads + threadIdx.x;
   if (r >= s.k) return;
@@ -1021,9 +1018,9 @@ __global__ void __launch_bounds__(kSrvThreads) topk_server_reduce_kernel(const S
   const uint2 rec = reinterpret_cast<const uint2*>(s.msgs + (int64_t)m * s.msg_stride)[r];
   const int64_t j = rec.x;
   if (j >= s.d) return;  // skipped by the scatter (and reported there by the checked build)
-  // the scatter grid has completed and its writes are visible (a no-op when
-  // this grid was launched in plain stream order)
-  asm volatile("griddepcontrol.wait;" ::: "memory");
+  // the scatter grid has completed and its writes are visible (the record
+  // was complete before the scatter ran)
+  dq_pdl_enter();
   const unsigned long long mask = t.mask[j];
   // the owner: bit m set and no bit below it
   if (!((mask >> m) & 1ull) || (mask & ((1ull << m) - 1ull))) return;
@@ -1075,6 +1072,7 @@ constexpr int kSrvGroup = 8;
 
 template <bool POW2>
 __global__ void __launch_bounds__(kSrvThreads) topk_server_owner_kernel(const ServerArgs s, const uint32_t* starts) {
+  dq_pdl_enter();
   const int64_t id = (int64_t)blockIdx.x * kSrvThreads + threadIdx.x;
   if (id >= (int64_t)s.M * s.k) return;
   const int m = (int)(id / s.k);
@@ -1188,27 +1186,16 @@ cudaError_t launch_topk_compress(const CompressArgs& a, int64_t k, bool keep_h, 
   const dim3 clusters(kCluster, rows);
   const size_t smem = sizeof(SelectSmem);
   cudaError_t st;
-  // the select kernel as a programmatic dependent launch of the form kernel
-  cudaLaunchConfig_t lc = {};
-  lc.gridDim = clusters;
-  lc.blockDim = dim3(kSelThreads);
-  lc.dynamicSmemBytes = smem;
-  lc.stream = stream;
-  cudaLaunchAttribute attr[1];
-  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  attr[0].val.programmaticStreamSerializationAllowed = 1;
-  lc.attrs = attr;
-  lc.numAttrs = 1;
   if (keep_h) {
     if ((st = ensure_smem(topk_select_kernel<true>, smem, 0, smem_done[1])) != cudaSuccess) return st;
-    topk_form_kernel<true><<<tiles, kFormThreads, 0, stream>>>(a, scratch);
+    launch_pdl(topk_form_kernel<true>, tiles, dim3(kFormThreads), 0, stream, a, scratch);
     if ((st = cudaGetLastError()) != cudaSuccess) return st;
-    st = cudaLaunchKernelEx(&lc, topk_select_kernel<true>, a, k, scratch);
+    st = launch_pdl(topk_select_kernel<true>, clusters, dim3(kSelThreads), smem, stream, a, k, scratch);
   } else {
     if ((st = ensure_smem(topk_select_kernel<false>, smem, 0, smem_done[0])) != cudaSuccess) return st;
-    topk_form_kernel<false><<<tiles, kFormThreads, 0, stream>>>(a, scratch);
+    launch_pdl(topk_form_kernel<false>, tiles, dim3(kFormThreads), 0, stream, a, scratch);
     if ((st = cudaGetLastError()) != cudaSuccess) return st;
-    st = cudaLaunchKernelEx(&lc, topk_select_kernel<false>, a, k, scratch);
+    st = launch_pdl(topk_select_kernel<false>, clusters, dim3(kSelThreads), smem, stream, a, k, scratch);
   }
   *launches += st == cudaSuccess ? 2 : 1;
   return st;
@@ -1223,27 +1210,17 @@ cudaError_t launch_topk_server(const ServerArgs& s, void* scratch, int32_t rows,
       const cudaError_t st = cudaMemsetAsync(s.w, 0, (size_t)s.d * sizeof(float), stream);
       if (st != cudaSuccess) return st;
     }
-    topk_server_scatter_kernel<<<grid, kSrvThreads, 0, stream>>>(s, t);
+    launch_pdl(topk_server_scatter_kernel, grid, dim3(kSrvThreads), 0, stream, s, t);
     cudaError_t st = cudaGetLastError();
     if (st != cudaSuccess) return st;
-    // the reduce kernel as a programmatic dependent launch: its blocks may
-    // start (and read their records) while the scatter finishes
-    cudaLaunchConfig_t lc = {};
-    lc.gridDim = grid;
-    lc.blockDim = dim3(kSrvThreads);
-    lc.dynamicSmemBytes = 0;
-    lc.stream = stream;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[0].val.programmaticStreamSerializationAllowed = 1;
-    lc.attrs = attr;
-    lc.numAttrs = 1;
+    // the reduce kernel's blocks read their records while the scatter's last
+    // blocks finish, then wait for the scatter grid
     st = cudaErrorInvalidValue;
     switch (next_pow2(s.M)) {
 #define DQ_TOPK_REDUCE(P)                                                                             \
   case P:                                                                                             \
-    st = s.M_pow2 ? cudaLaunchKernelEx(&lc, topk_server_reduce_kernel<true, P>, s, t)                 \
-                  : cudaLaunchKernelEx(&lc, topk_server_reduce_kernel<false, P>, s, t);               \
+    st = s.M_pow2 ? launch_pdl(topk_server_reduce_kernel<true, P>, grid, dim3(kSrvThreads), 0, stream, s, t) \
+                  : launch_pdl(topk_server_reduce_kernel<false, P>, grid, dim3(kSrvThreads), 0, stream, s, t); \
     break;
       DQ_TOPK_REDUCE(1) DQ_TOPK_REDUCE(2) DQ_TOPK_REDUCE(4) DQ_TOPK_REDUCE(8) DQ_TOPK_REDUCE(16)
       DQ_TOPK_REDUCE(32) DQ_TOPK_REDUCE(64)
@@ -1257,10 +1234,10 @@ cudaError_t launch_topk_server(const ServerArgs& s, void* scratch, int32_t rows,
   if (s.store_q) return cudaErrorNotSupported;  // the owner kernel is sparse
   uint32_t* starts = reinterpret_cast<uint32_t*>(scratch) + row_words(s.d) * rows;
   const int64_t n = (int64_t)s.M * s.k;
-  topk_server_starts_kernel<<<dim3((unsigned)((s.k + 255) / 256), (unsigned)s.M), 256, 0, stream>>>(s, starts);
+  launch_pdl(topk_server_starts_kernel, dim3((unsigned)((s.k + 255) / 256), (unsigned)s.M), dim3(256), 0, stream, s, starts);
   const unsigned blocks = (unsigned)((n + kSrvThreads - 1) / kSrvThreads);
-  if (s.M_pow2) topk_server_owner_kernel<true><<<blocks, kSrvThreads, 0, stream>>>(s, starts);
-  else topk_server_owner_kernel<false><<<blocks, kSrvThreads, 0, stream>>>(s, starts);
+  if (s.M_pow2) launch_pdl(topk_server_owner_kernel<true>, dim3(blocks), dim3(kSrvThreads), 0, stream, s, starts);
+  else launch_pdl(topk_server_owner_kernel<false>, dim3(blocks), dim3(kSrvThreads), 0, stream, s, starts);
   *launches += 2;
   return cudaGetLastError();
 }
