@@ -10,8 +10,8 @@ a call takes, the records and residuals must be the oracle's bit for bit:
   (many candidates), land inside big groups of equal keys, and sit on an
   all-zero p;
 * more candidates than a select CTA keeps on chip (k = d/2);
-* server paths for up to 64 workers (a warp per index tile) and beyond
-  (a thread per record);
+* server paths for up to 64 workers (per-index worker masks, one owner
+  per index) and beyond (a thread per record);
 * at d = 7e7 the CTAs' tiles no longer fit one chunk of tile counts; there
   the selection is checked by the properties that define it uniquely
   (k records in index order holding p_j, no dropped key above the smallest
@@ -138,7 +138,9 @@ def test_many_tiles_per_cta_properties(P):
 
 @pytest.mark.parametrize("M", [33, 64, 65, 70])
 def test_server_worker_counts(P, M):
-    """Up to 64 workers the server runs one warp per index tile; above, one
-    thread per record.  Both sum in worker order, so w matches bit for bit."""
+    """Up to 64 workers the server scatters into per-index worker masks and
+    the lowest worker of each index sums it; above, one thread per record
+    searches the other workers' records.  Both sum in the library's pairwise
+    order, so w matches bit for bit."""
     ocfg = oracle_config(50_003, M, oracle.TOPK, lr=0.5, k=777, seed=M, keep=False)
     run_free(P, ocfg, [1.0, 1.0, "ties"], seed=M)
