@@ -29,7 +29,7 @@ struct dqgan_handle {
   uint32_t* err_word = nullptr;  // device error word written by bounded waits
   int64_t* seg_bstart = nullptr;     // layer segments: nb + 1 bucket starts (device)
   uint32_t* seg_wbucket = nullptr;   // layer segments: bucket of every 32-element word (device)
-  uint32_t* seg_slices = nullptr;    // layer segments, sign: {first word, bucket | (rows - 1) << 27} per slice
+  uint32_t* seg_slices = nullptr;    // layer segments, sign and 8-bit codes: {first word, bucket | (rows - 1) << 27} per slice
   int64_t seg_nslices = 0;
   CUtensorMap words_map;         // TMA map of the last message buffer the server saw
   const void* words_map_msgs = nullptr;
@@ -516,6 +516,18 @@ int dqgan_set_segments(dqgan_handle* h, const int64_t* offsets, int32_t nseg) {
         slices.push_back((uint32_t)b | (uint32_t)(rows - 1) << 27);
       }
     }
+  // 8-bit codes with 16 workers (four codes per word; buckets start on
+  // multiples of 32 elements): the quantiser server's slices, each bucket's
+  // code words in runs of up to 32, so that no slice spans two buckets
+  if ((c.compressor == DQGAN_SQUANT || c.compressor == DQGAN_QSGD) && c.bits == 8 && c.M == 16)
+    for (int64_t b = 0; b < nb; ++b) {
+      const int64_t we = (starts[b + 1] + 3) / 4;
+      for (int64_t w = starts[b] / 4; w < we; w += 32) {
+        const int64_t rows = we - w < 32 ? we - w : 32;
+        slices.push_back((uint32_t)w);
+        slices.push_back((uint32_t)b | (uint32_t)(rows - 1) << 27);
+      }
+    }
   if ((st = dq_malloc(&h->seg_bstart, starts.size() * sizeof(int64_t))) != cudaSuccess ||
       (st = dq_malloc(&h->seg_wbucket, wb.size() * sizeof(uint32_t))) != cudaSuccess ||
       (!slices.empty() && (st = dq_malloc(&h->seg_slices, slices.size() * sizeof(uint32_t))) != cudaSuccess)) {
@@ -667,8 +679,11 @@ int dqgan_server_aggregate_update(dqgan_handle* h, const void* msgs_all, float* 
   if (tma_sign || tma_squant) {
     if (h->words_map_msgs != msgs_all) {
       const int64_t payload_words = tma_sign ? (s.d + 31) / 32 : (s.d * s.bits + 31) / 32;
+      // 36-word boxes wherever slices come from a table (layer segments:
+      // the sign server, and the quantiser server with 8-bit codes)
+      const bool table = !flat && h->seg_slices != nullptr;
       h->words_map_ok = dq::encode_words_map(s.msgs, s.msg_stride, s.off_payload, payload_words, s.M,
-                                             tma_sign && flat, tma_sign && !flat ? dq::kSignSegBoxWords : 32, &h->words_map);
+                                             tma_sign && flat, table ? dq::kSignSegBoxWords : 32, &h->words_map);
       h->words_map_msgs = msgs_all;
     }
     if (h->words_map_ok) (tma_sign ? s.sign_words_map : s.squant_words_map) = &h->words_map;
@@ -692,7 +707,7 @@ int dqgan_server_aggregate_update(dqgan_handle* h, const void* msgs_all, float* 
   switch (h->cfg.compressor) {
     case DQGAN_SIGN: st = dq::launch_sign_server(s, x, h->stream, &h->launches); break;
     case DQGAN_SQUANT:
-    case DQGAN_QSGD: st = dq::launch_squant_server(s, x.params_map, h->stream, &h->launches); break;
+    case DQGAN_QSGD: st = dq::launch_squant_server(s, x, h->stream, &h->launches); break;
     case DQGAN_IDENTITY: st = dq::launch_identity_server(s, h->stream, &h->launches); break;
     case DQGAN_TOPK: st = dq::launch_topk_server(s, h->scratch, h->nlocal, h->stream, &h->launches); break;
   }

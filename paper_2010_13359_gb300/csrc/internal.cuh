@@ -101,8 +101,9 @@ struct ServerArgs {
                         // dense: top-k writes +0 at the indices nobody sent)
 };
 
-// The sign server's further inputs (kept out of ServerArgs, which every
-// server kernel takes as its parameter block).
+// The sign server's further inputs, also the quantiser server's slice table
+// (kept out of ServerArgs, which every server kernel takes as its parameter
+// block).
 struct SignServerExtras {
   const CUtensorMap* params_map;  // TMA map of w as rows of 32 floats, or nullptr
   int32_t path;                   // buckets >= 1024, M <= 32: 0 by size, 1 column kernel, 2 bit-transpose kernel
@@ -171,9 +172,11 @@ cudaError_t launch_topk_compress(const CompressArgs& a, int64_t k, bool keep_h, 
 
 cudaError_t launch_sign_server(const ServerArgs& s, const SignServerExtras& x, cudaStream_t stream,
                                uint64_t* launches);
-// params_map: encode_params_map(w, d, 32 * (32 / bits) / 32) for bits 2 and 4,
-// or nullptr (then those widths take the kernel without TMA).
-cudaError_t launch_squant_server(const ServerArgs& s, const CUtensorMap* params_map, cudaStream_t stream,
+// x.params_map: encode_params_map(w, d, 32 * (32 / bits) / 32) for bits 2 and
+// 4, or nullptr (then those widths take the kernel without TMA); with layer
+// segments and 8-bit codes, x.seg_slices lists each bucket's code words in
+// runs of up to 32 (and the words map has 36-word boxes).
+cudaError_t launch_squant_server(const ServerArgs& s, const SignServerExtras& x, cudaStream_t stream,
                                  uint64_t* launches);
 cudaError_t launch_identity_server(const ServerArgs& s, cudaStream_t stream, uint64_t* launches);
 // scratch: topk_scratch_bytes(d, rows, M); the server's table follows the rows.

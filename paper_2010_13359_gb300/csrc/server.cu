@@ -1325,6 +1325,154 @@ squant_server_tma_kernel(const ServerArgs s, const __grid_constant__ CUtensorMap
   }
 }
 
+// 8-bit codes with layer segments and 16 workers: the slices come from a
+// host-built table of each bucket's code words in runs of up to 32, so no
+// slice spans two buckets (the per-lane bucket lookups and the mixed-slice
+// decode of the kernel above are not needed).  The word box starts at the
+// 16-byte boundary at or before the slice (36 words wide, no swizzle); lane l
+// takes word first + l of every worker when l < rows.  The decode and the
+// sum over workers are the b = 8 ones above: level table replicated per
+// shared-memory bank, groups of four workers (a + b) + (c + d), the four
+// group values added pairwise.  The slice's scale, the next slice's table
+// entry and the lane's four parameters are loaded one slice ahead.
+template <bool POW2>
+__global__ void __launch_bounds__(32 * kTmaWarps)
+squant8_server_table_kernel(const ServerArgs s, const SegSlices seg, const __grid_constant__ CUtensorMap tmap) {
+  dq_pdl_enter();
+  constexpr int K = 127;
+  constexpr int M = 16;
+  constexpr int RW = kSignSegBoxWords;                       // words per box row
+  constexpr uint32_t kBoxBytes = (uint32_t)M * RW * 4u;      // 2304: a multiple of 128
+  extern __shared__ uint8_t smem_raw[];
+  __shared__ uint64_t bars[kTmaWarps][2];
+  __shared__ float V8[256 * 32];
+  const int lane = threadIdx.x & 31;
+  const int warp = threadIdx.x >> 5;
+  const uint32_t raw = smem_addr(smem_raw);
+  uint8_t* const buf0 = smem_raw + ((128u - (raw & 127u)) & 127u) + warp * 2 * kBoxBytes;  // + i * kBoxBytes
+  uint64_t* bar = bars[warp];
+  for (int t = threadIdx.x; t < 256 * 32; t += blockDim.x) {
+    const int code = t >> 5;
+    const int level = code - K;
+    float v = 0.f;
+    if (code <= 2 * K && level != 0) {
+      const float mag = __fdiv_rn((float)(level < 0 ? -level : level), (float)K);
+      v = level < 0 ? -mag : mag;
+    }
+    V8[t] = v;
+  }
+  if (lane == 0) {
+    mbar_init(&bar[0], 1);
+    mbar_init(&bar[1], 1);
+    mbar_fence_init();
+  }
+  __syncthreads();
+
+  const int64_t nslices = seg.n;
+  const int64_t stride = (int64_t)gridDim.x * kTmaWarps;
+  const int32_t x0 = (int32_t)(s.off_payload >> 2);  // a multiple of 64 words
+  const bool active = lane < M;
+  struct Slice {
+    int64_t word;    // first code word
+    int64_t bucket;
+    int rows;        // code words in the slice, 1..32 (0: none)
+  };
+  auto slice_of = [&](int64_t sl_) -> Slice {
+    if (sl_ >= nslices) return Slice{0, 0, 0};
+    const uint2 e = __ldg(reinterpret_cast<const uint2*>(seg.slices) + sl_);
+    return Slice{(int64_t)e.x, (int64_t)(e.y & 0x7FFFFFFu), (int)(e.y >> 27) + 1};
+  };
+  auto issue = [&](const Slice& c, int i) {
+    mbar_arrive_expect_tx(&bar[i], kBoxBytes);
+    tma_load_2d(buf0 + i * kBoxBytes, &tmap, (x0 + (int32_t)c.word) & ~3, 0, &bar[i]);
+  };
+  const float* const lane_scales =
+      reinterpret_cast<const float*>(s.msgs + (int64_t)(active ? lane : 0) * s.msg_stride);
+  // the lane's four parameters of slice c (none past its rows or past d)
+  auto load_w4 = [&](const Slice& c) -> float4 {
+    float4 x = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (lane >= c.rows) return x;
+    const int64_t j = 4 * (c.word + lane);
+    if (j + 3 < s.d) return __ldcs(reinterpret_cast<const float4*>(s.w + j));
+    if (j < s.d) x.x = s.w[j];
+    if (j + 1 < s.d) x.y = s.w[j + 1];
+    if (j + 2 < s.d) x.z = s.w[j + 2];
+    return x;
+  };
+  int64_t sl = (int64_t)blockIdx.x * kTmaWarps + warp;
+  Slice c = slice_of(sl);
+  Slice cn = slice_of(sl + stride);
+  if (sl < nslices && lane == 0) issue(c, 0);
+  float scale_nx = (active && sl < nslices) ? __ldg(lane_scales + c.bucket) : 0.f;
+  float4 w_nx = load_w4(c);
+  uint32_t it = 0;
+  bool ok = true;
+  for (; sl < nslices; sl += stride, ++it) {
+    const int cur = (int)(it & 1u);
+    const int64_t nxt = sl + stride;
+    const Slice cnn = slice_of(nxt + stride);  // the table entry one slice further
+    if (nxt < nslices && lane == 0) {
+      fence_proxy_async_shared();  // this warp's reads of that buffer came before
+      issue(cn, cur ^ 1);
+    }
+    const float my_scale = scale_nx;
+    scale_nx = (active && nxt < nslices) ? __ldg(lane_scales + cn.bucket) : 0.f;
+    const float wv[4] = {w_nx.x, w_nx.y, w_nx.z, w_nx.w};
+    w_nx = load_w4(cn);
+    ok = mbar_wait_bounded(&bar[cur], (it >> 1) & 1u, s.err);
+    ok = __all_sync(kFullMask, ok);
+    if (!ok) break;
+    const uint32_t* words = reinterpret_cast<const uint32_t*>(buf0 + cur * kBoxBytes) + (int)((x0 + c.word) & 3) + lane;
+    const float* V8l = V8 + lane;
+    // group value of workers m .. m + 3: (a + b) + (c + d)
+    auto group = [&](int m, float (&g)[4]) {
+      uint32_t wd[4];
+      float sc[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        wd[u] = words[RW * (m + u)];
+        sc[u] = __shfl_sync(kFullMask, my_scale, m + u);
+      }
+      float v[4][4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u)
+#pragma unroll
+        for (int e = 0; e < 4; ++e)
+          v[u][e] = __fmul_rn(sc[u], V8l[__byte_perm(wd[u], 0u, 0x4440u | (uint32_t)e) * 32u]);
+#pragma unroll
+      for (int e = 0; e < 4; ++e) g[e] = __fadd_rn(__fadd_rn(v[0][e], v[1][e]), __fadd_rn(v[2][e], v[3][e]));
+    };
+    float g0[4], g1[4], r[4];
+    group(0, g0);
+    group(4, g1);
+#pragma unroll
+    for (int e = 0; e < 4; ++e) r[e] = __fadd_rn(g0[e], g1[e]);
+    group(8, g0);
+    group(12, g1);
+#pragma unroll
+    for (int e = 0; e < 4; ++e) r[e] = __fadd_rn(r[e], __fadd_rn(g0[e], g1[e]));
+    if (lane < c.rows) {
+      const int64_t j = 4 * (c.word + lane);
+      float o[4];
+#pragma unroll
+      for (int e = 0; e < 4; ++e) o[e] = server_out(s, wv[e], average_t<POW2>(r[e], s));
+      if (j + 3 < s.d) {
+        __stcs(reinterpret_cast<float4*>(s.w + j), make_float4(o[0], o[1], o[2], o[3]));
+      } else {
+#pragma unroll
+        for (int e = 0; e < 4; ++e)
+          if (j + e < s.d) s.w[j + e] = o[e];
+      }
+    }
+    __syncwarp();
+    c = cn;
+    cn = cnn;
+  }
+  // after a time-out, the copy of the next slice may still be in flight
+  if (!ok && lane == 0 && sl + stride < nslices)
+    mbar_wait_bounded(&bar[(it & 1u) ^ 1u], ((it + 1) >> 1) & 1u, s.err);
+}
+
 // Identity: the messages are the p vectors themselves, summed in groups of
 // four workers in the library's pairwise order.
 __global__ void __launch_bounds__(256) identity_server_kernel(const ServerArgs s) {
@@ -1508,6 +1656,31 @@ cudaError_t launch_squant_tma(const ServerArgs& s, const CUtensorMap* params_map
   return cudaGetLastError();
 }
 
+cudaError_t launch_squant8_table(const ServerArgs& s, const SignServerExtras& x, cudaStream_t stream) {
+  auto kern = squant8_server_table_kernel<true>;
+  constexpr int smem = kTmaWarps * 2 * 16 * kSignSegBoxWords * 4 + 128;  // + alignment slack
+  int dev = 0;
+  cudaError_t st = cudaGetDevice(&dev);
+  if (st != cudaSuccess) return st;
+  static int blocks_for[64] = {0};
+  if (dev < 0 || dev >= 64) return cudaErrorInvalidDevice;
+  if (blocks_for[dev] == 0) {
+    if ((st = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem)) != cudaSuccess)
+      return st;
+    int sms = 0, per_sm = 0;
+    if ((st = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return st;
+    if ((st = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, 32 * kTmaWarps, smem)) != cudaSuccess)
+      return st;
+    blocks_for[dev] = sms * (per_sm > 0 ? per_sm : 1);
+  }
+  const int64_t need = (x.seg_nslices + kTmaWarps - 1) / kTmaWarps;
+  const unsigned blocks = (unsigned)(need < blocks_for[dev] ? need : blocks_for[dev]);
+  if (blocks == 0) return cudaSuccess;
+  launch_pdl(kern, dim3(blocks), dim3(32 * kTmaWarps), smem, stream, s, SegSlices{x.seg_slices, x.seg_nslices},
+             *s.squant_words_map);
+  return cudaGetLastError();
+}
+
 unsigned chunk_blocks(int64_t d, int threads) {
   const int64_t chunks = (d + 3) / 4;
   return (unsigned)((chunks + threads - 1) / threads);
@@ -1599,8 +1772,15 @@ cudaError_t launch_sign_server(const ServerArgs& s, const SignServerExtras& x, c
   return cudaGetLastError();
 }
 
-cudaError_t launch_squant_server(const ServerArgs& s, const CUtensorMap* params_map, cudaStream_t stream,
+cudaError_t launch_squant_server(const ServerArgs& s, const SignServerExtras& x, cudaStream_t stream,
                                  uint64_t* launches) {
+  const CUtensorMap* params_map = x.params_map;
+  if (s.word_bucket && x.seg_slices && s.squant_words_map != nullptr && s.bits == 8 && s.M == 16) {
+    // 8-bit codes, layer segments, 16 workers: slices from the per-bucket table
+    const cudaError_t st = launch_squant8_table(s, x, stream);
+    *launches += 1;
+    return st;
+  }
   if (s.squant_words_map != nullptr && s.M <= 32 && s.bucket >= 32 * (32 / s.bits) &&
       (params_map != nullptr || !sq_params_boxed(s.bits))) {
     const bool p2 = s.M_pow2 != 0;

@@ -96,6 +96,25 @@ def test_segmented_matches_oracle(P, case, layout):
     run_segmented(P, ocfg, T=3, seed=len(segs))
 
 
+@pytest.mark.parametrize("comp", [oracle.SQUANT, oracle.QSGD], ids=["squant", "qsgd"])
+@pytest.mark.parametrize("layout", ["random7", "tiny_and_long", "one", "odd_words"])
+def test_segmented_8bit_sixteen_workers(P, comp, layout):
+    """8-bit codes with 16 workers take the server whose slices come from the
+    per-bucket table (no slice spans two buckets; short slices at the end of
+    a layer's last bucket store only their own rows)."""
+    d = 40_011
+    if layout == "random7":
+        segs = random_segments(np.random.default_rng(11), d, 7)
+    elif layout == "tiny_and_long":
+        segs = (0, 32, 64, 96, 5_024, 5_056, d)
+    elif layout == "odd_words":  # layer starts on every residue of 4 code words
+        segs = (0, 96, 224, 384, 544, 9_600, 9_632, d)
+    else:
+        segs = (0, d)
+    ocfg = oracle_config(d, 16, comp, lr=0.05, seed=5, keep=False, segments=segs, bucket=512, bits=8)
+    run_segmented(P, ocfg, T=3, seed=len(segs) + 16)
+
+
 @pytest.mark.parametrize("name", ["dcgan_sign_layers", "resnet_squant_b8_layers"])
 def test_layer_workloads_first_steps(P, name):
     """The per-layer workloads at a reduced size: their own 16 / 64 layer
