@@ -298,9 +298,13 @@ DQGAN_API int dqgan_load_state(dqgan_handle* h, const void* host_src, int64_t by
  * dqgan_message_layout() describes the flat layout).  nseg = 0 with
  * offsets = NULL returns to flat buckets.  Only for DQGAN_SIGN, SQUANT and
  * QSGD (else DQGAN_ERR_UNSUPPORTED), and only before the first step
- * (step counter 1; else DQGAN_ERR_INVALID_ARG).  Synchronous; allocates two
- * small device tables (nb + 1 int64 bucket starts, one u32 per 32 elements).
- * With segments the servers take their per-element scale-lookup paths.
+ * (step counter 1; else DQGAN_ERR_INVALID_ARG).  Synchronous; allocates
+ * small device tables: nb + 1 int64 bucket starts, one u32 per 32 elements,
+ * and for DQGAN_SIGN (and 8-bit codes with 16 workers) a table of each
+ * bucket's message words in runs of up to 32 (8 bytes per run), from which
+ * the servers take slices that never span two buckets; DQGAN_ERR_OOM if an
+ * allocation fails (the handle is then left with flat buckets).  Other widths and
+ * worker counts look up each 32-element word's bucket.
  */
 DQGAN_API int dqgan_set_segments(dqgan_handle* h, const int64_t* offsets, int32_t nseg);
 
