@@ -9,11 +9,15 @@
 // The parameters therefore come out the same bit for bit whichever kernel
 // runs.
 //
-// Stochastic quantiser, identity, and sign with buckets < 512: one thread per
-// 4-element chunk of w walks the M messages in groups of four workers,
-// fetching the message words of 8 workers before using them.  Sign with
-// buckets >= 512: bit-transposed table decode (below).  w is read and
-// written once.
+// Sign with buckets >= 512: bit-transposed table decode (the column and
+// warp-transpose kernels for M <= 32, words staged by TMA; flat buckets or a
+// per-bucket slice table with layer segments).  Stochastic quantiser with
+// M <= 32: code words staged by TMA, per-worker or pair-table decode (and,
+// for 8-bit codes with layer segments and 16 workers, slices from a
+// per-bucket table).  The rest -- identity, sign with buckets < 512, more
+// than 32 workers -- one thread per 4-element chunk of w walks the M
+// messages in groups of four workers.  w is read and written once; every
+// kernel waits for the grid before it (programmatic dependent launch).
 #include "device_common.cuh"
 
 namespace dq {
