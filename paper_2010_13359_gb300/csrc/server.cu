@@ -899,9 +899,9 @@ constexpr int kSquant4Parts = 1;
 // b = 4 and 8 load each slice's scale (b = 8: and the lane's parameters)
 // one slice ahead; b = 4 writes its parameters back with plain stores
 // instead of a TMA store of the box, which frees the box as soon as the
-// lanes have read it.  (Measured at d = 25M, M = 16: b = 8 0.79 -> 0.84 and
-// b = 4 0.68 -> 0.71 of the copy peak.  b = 2 measured slower with either
-// change and keeps the TMA store.)
+// lanes have read it.  (Both measured faster at d = 25M, M = 16; b = 2
+// measured slower with either change and keeps the TMA store and the
+// per-slice scale load.)
 constexpr bool sq_prefetch(int bits) { return bits != 2; }
 constexpr bool sq_direct_store(int bits) { return bits == 4; }
 

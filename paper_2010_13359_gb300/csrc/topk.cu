@@ -368,9 +368,11 @@ constexpr int kRegTiles = 4;
 
 // The tile of candidate f: the largest i < n with tpre[i] <= f (tpre
 // non-decreasing, tpre[0] <= f < tpre[n]; an empty tile repeats its
-// successor's prefix, so the tile found holds f).  A fixed number of halving
-// steps (n <= kChunkTiles), so that the searches of several candidates
-// interleave.
+// successor's prefix, so the tile found holds f), in a fixed number of
+// halving steps (n <= kChunkTiles).  Used where the share is not kept on
+// chip; filling the on-chip copy uses the tile map instead (a search per
+// candidate, with the lanes reading scattered prefixes, conflicts in the
+// shared-memory banks).
 __device__ __forceinline__ int tile_of(const uint32_t* tpre, int n, uint32_t f) {
   int lo = 0;
 #pragma unroll
